@@ -1,0 +1,201 @@
+/*
+ * ace.h -- C ABI of the GB300 (sm_103a) grouped adapter execution library.
+ *
+ * The library implements the data-parallel hot path of ACE (arxiv 2609.06072):
+ * the forward and backward passes of group-shared LoRA deltas on the MoE
+ * expert gate / up / down projections.
+ *
+ *   Sec. 3.1  expert-wise MoE LoRA: y(x) = sum_{e in R(x)} p_e(x)(W_e x + B_e A_e x)
+ *   Sec. 3.3  rank consolidation: one adapter Delta W_g = B_g A_g per group,
+ *             A_g in R^{r_g x d_in}, B_g in R^{d_out x r_g}, r_g = sum_{e in G_g} r_e
+ *   Sec. 3.4  every routed expert e uses Delta W_{g(e)}; the group adapter
+ *             receives gradient from every pair routed into the group
+ *   Sec. 3.5  grouped execution: c_g(x) = B_g (A_g x) is evaluated once per
+ *             active group of a token and reused by all its routed experts
+ *             of that group (gate / up, whose input x is shared)
+ *   App. "Implementation and Profiling of Grouped Adapter Execution":
+ *             gate/up take x, down takes the expert-specific h_e
+ *
+ * Terms used below.  T tokens, top-k routing, pair p = t*k + j (token t,
+ * slot j), R = T*k pairs.  E experts, G groups, e2g the expert->group map,
+ * rank_off[G+1] the packed rank offsets (r_g = rank_off[g+1] - rank_off[g]).
+ * d = hidden size (gate/up d_in, down d_out), f = expert intermediate size
+ * (gate/up d_out, down d_in).  s = LoRA scale.
+ *
+ * Row order.  Every per-pair tensor the kernels touch is in ROW order: the
+ * pairs sorted by (g(e), e, t), so expert segments are contiguous inside
+ * group segments.  ace_permute produces the map (row_pair / pair_row).
+ * Unique (token, group) pairs -- the set A(x) of Sec. 3.5 -- are sorted by
+ * (g, t).
+ *
+ * Memory.  Every tensor pointer is a DEVICE pointer owned by the caller.
+ * The library allocates no device memory: scratch space is a caller-owned
+ * workspace sized by ace_workspace_size.  Tensors must be 16-byte aligned.
+ * bf16 tensors are passed as `uint16_t*` holding the bf16 bit patterns; fp32
+ * tensors as `float*`.  All matrices are row-major and dense.
+ *
+ * Streams / errors.  Every call is asynchronous on the caller's stream and
+ * returns an ace_status.  Host-side checks (null pointers, shapes, limits,
+ * workspace size, alignment) return an error WITHOUT launching.  Invalid
+ * routing found on the device (expert id out of range, an expert repeated in
+ * a token) sets a device flag; ace_get_error synchronises the stream, reads
+ * and clears it.  No call synchronises otherwise, and none aborts, traps or
+ * throws.  ace_last_error_message() gives a thread-local description of the
+ * last host-side failure.
+ *
+ * Device.  Requires an sm_103 GPU (GB300).  Plans created on another device
+ * fail with ACE_ERR_UNSUPPORTED; there is no fallback.
+ */
+#ifndef ACE_H_
+#define ACE_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define ACE_VERSION 1
+
+typedef int32_t ace_status;
+#define ACE_OK 0
+#define ACE_ERR_ARG 1            /* null pointer or invalid scalar argument */
+#define ACE_ERR_SHAPE 2          /* shape outside the plan or the supported limits */
+#define ACE_ERR_WORKSPACE 3      /* workspace too small or misaligned */
+#define ACE_ERR_INDEX 4          /* invalid routing or expert->group map */
+#define ACE_ERR_UNSUPPORTED 5    /* device is not sm_103, or rank too large */
+#define ACE_ERR_CUDA 6           /* a CUDA runtime call failed */
+#define ACE_ERR_DEVICE_TIMEOUT 7 /* a bounded device-side wait gave up */
+
+/* plan flags */
+#define ACE_FLAG_DETERMINISTIC 1u /* dA / dB^T via fixed-order two-stage split-K (bitwise reproducible);
+                                     otherwise fp32 atomics (any summation order) */
+
+/* Limits. */
+#define ACE_MAX_EXPERTS 512
+#define ACE_MAX_RANK 128 /* max r_g of one group */
+
+/* Layer description (host memory; copied into the plan). */
+typedef struct ace_layer_desc {
+  int32_t T_max;           /* largest T a call will use */
+  int32_t k;               /* top-k, 1 <= k <= E, k <= 32 */
+  int32_t E;               /* experts, 1 <= E <= ACE_MAX_EXPERTS */
+  int32_t G;               /* groups, 1 <= G <= E */
+  const int32_t* e2g;      /* [E] expert -> group, values in [0, G); every group non-empty */
+  const int32_t* rank_off; /* [G+1] rank offsets, rank_off[0] = 0, 1 <= r_g <= ACE_MAX_RANK */
+  int32_t d;               /* hidden size, multiple of 8 */
+  int32_t f;               /* expert intermediate size, multiple of 8 */
+  uint32_t flags;          /* ACE_FLAG_* */
+} ace_layer_desc;
+
+typedef struct ace_plan ace_plan; /* opaque, host memory only */
+
+/* Views into the permutation workspace filled by ace_permute (device pointers).
+ * Row r is the r-th pair in (g(e), e, t) order.  All int32. */
+typedef struct ace_perm {
+  int32_t T;              /* tokens of this call */
+  int32_t R;              /* T * k */
+  int32_t* counts;        /* [8]: [0] U = #unique (g,t), [1] rows written */
+  int32_t* group_off;     /* [G+1] first row of each group segment */
+  int32_t* expert_off;    /* [E] first row of each expert segment */
+  int32_t* expert_cnt;    /* [E] rows of each expert */
+  int32_t* row_pair;      /* [R] pair index p = t*k + j held by row r */
+  int32_t* pair_row;      /* [R] inverse of row_pair */
+  int32_t* uniq_off;      /* [G+1] first unique pair of each group */
+  int32_t* uniq_tok;      /* [R] token of unique pair u (first U entries valid) */
+  int32_t* tok_uniq;      /* [T*k] unique pairs of token t, ascending g, then -1 */
+  void* ws;               /* the workspace these views point into */
+} ace_perm;
+
+int32_t ace_version(void);
+const char* ace_last_error_message(void);
+
+/* Create a plan on the current CUDA device.  Host-side validation of the
+ * description (map in range, every group non-empty, ranks in limits). */
+ace_status ace_plan_create(ace_plan** out, const ace_layer_desc* desc);
+void ace_plan_destroy(ace_plan* plan);
+
+/* Max over groups of r_g; the row stride (in elements) of every H / dH
+ * buffer below. */
+int32_t ace_plan_rank_max(const ace_plan* plan);
+
+/* Workspace bytes for T tokens:
+ *   perm_bytes  -- ace_permute (lives as long as the ace_perm views are used)
+ *   fwd_bytes   -- ace_fwd_shared / ace_fwd_row scratch (may be 0)
+ *   bwd_bytes   -- ace_bwd_shared / ace_bwd_row scratch
+ * A NULL output pointer is skipped. */
+ace_status ace_workspace_size(const ace_plan* plan, int32_t T, size_t* perm_bytes, size_t* fwd_bytes,
+                              size_t* bwd_bytes);
+
+/* Route-permute (Sec. 3.1 R(x), Sec. 3.5 A(x)).
+ *   topk_idx  [T, k] int32 expert ids of each token (slot order as given)
+ * Counts pairs per expert, exclusive-scans them in (g, e) order and scatters
+ * the pairs, stable in t, into group-contiguous rows; builds the unique
+ * (g, t) list and per-token unique lists.  Bit-exact and deterministic.
+ * Invalid tokens (id out of [0,E) or a repeated id) raise the device flag
+ * (ACE_ERR_INDEX from ace_get_error); their pairs are left out and the
+ * outputs are then unspecified. */
+ace_status ace_permute(const ace_plan* plan, const int32_t* topk_idx, int32_t T, void* perm_ws,
+                       size_t perm_ws_bytes, ace_perm* out, void* stream);
+
+/* Forward, shared input (gate / up; Sec. 3.5 and App. implementation).
+ *   X       [T, d] bf16 token activations
+ *   nproj   1 or 2 projections fused on the same X and the same map
+ *   A[i]    [rank_off[G], d] bf16, rows rank_off[g].. hold A_g
+ *   Bt[i]   [rank_off[G], f] bf16, rows rank_off[g].. hold B_g^T
+ *   Y[i]    [R, f] bf16 IN/OUT in row order: Y[row] += s * B_g (A_g X[t])
+ *   H[i]    [R, rank_max] fp32 OUT (may be NULL): H[u] = A_g X[t] for unique
+ *           pair u (first U rows; columns >= r_g are zero)
+ * c_g is computed once per unique (g, t) and added to every row of that pair. */
+ace_status ace_fwd_shared(const ace_plan* plan, const ace_perm* perm, const uint16_t* X, int32_t nproj,
+                          const uint16_t* const* A, const uint16_t* const* Bt, float s, uint16_t* const* Y,
+                          float* const* H, void* ws, size_t ws_bytes, void* stream);
+
+/* Forward, per row (down).
+ *   Hin  [R, f] bf16 expert-specific inputs h_e in row order
+ *   A    [rank_off[G], f] bf16 (A_g);  Bt [rank_off[G], d] bf16 (B_g^T)
+ *   Y    [R, d] bf16 IN/OUT: Y[row] += s * B_g (A_g Hin[row])
+ *   H    [R, rank_max] fp32 OUT or NULL: A_g Hin[row] */
+ace_status ace_fwd_row(const ace_plan* plan, const ace_perm* perm, const uint16_t* Hin, const uint16_t* A,
+                       const uint16_t* Bt, float s, uint16_t* Y, float* H, void* ws, size_t ws_bytes,
+                       void* stream);
+
+/* Backward, shared input (gate / up).  Adjoint of ace_fwd_shared:
+ *   dY[i]   [R, f] bf16 row-order upstream gradients
+ *   H[i]    [R, rank_max] fp32 saved by the forward (unique-pair rows)
+ *   dX      [T, d] bf16 IN/OUT: dX[t] += sum_i sum_{u of t} s A_g^T (B_g^T dC_u),
+ *           dC_u = sum of the dY rows of unique pair u
+ *   dA[i]   [rank_off[G], d] fp32 OUT (overwritten): s sum_u (B_g^T dC_u) X[t_u]^T
+ *   dBt[i]  [rank_off[G], f] fp32 OUT (overwritten): s sum_u H_u dC_u^T
+ * Groups with no routed pair get exact zeros. */
+ace_status ace_bwd_shared(const ace_plan* plan, const ace_perm* perm, int32_t nproj, const uint16_t* const* dY,
+                          const uint16_t* X, const float* const* H, const uint16_t* const* A,
+                          const uint16_t* const* Bt, float s, uint16_t* dX, float* const* dA, float* const* dBt,
+                          void* ws, size_t ws_bytes, void* stream);
+
+/* Backward, per row (down).
+ *   dY    [R, d] bf16;  Hin [R, f] bf16;  H [R, rank_max] fp32 from ace_fwd_row
+ *   dHin  [R, f] bf16 IN/OUT: dHin[row] += s A_g^T (B_g^T dY[row])
+ *   dA    [rank_off[G], f] fp32 OUT;  dBt [rank_off[G], d] fp32 OUT */
+ace_status ace_bwd_row(const ace_plan* plan, const ace_perm* perm, const uint16_t* dY, const uint16_t* Hin,
+                       const float* H, const uint16_t* A, const uint16_t* Bt, float s, uint16_t* dHin, float* dA,
+                       float* dBt, void* ws, size_t ws_bytes, void* stream);
+
+/* Row-order helpers (bf16, `cols` elements per row, cols multiple of 8):
+ *   gather:  dst[row] = src[row_pair[row]]   (pair order -> row order)
+ *   scatter: dst[row_pair[row]] = src[row]   (row order -> pair order) */
+ace_status ace_gather_rows(const ace_perm* perm, const uint16_t* src_pairs, uint16_t* dst_rows, int32_t cols,
+                           void* stream);
+ace_status ace_scatter_rows(const ace_perm* perm, const uint16_t* src_rows, uint16_t* dst_pairs, int32_t cols,
+                            void* stream);
+
+/* Synchronises `stream`, then reads and clears the device error flag of the
+ * permutation workspace: ACE_OK, ACE_ERR_INDEX (invalid routing) or
+ * ACE_ERR_DEVICE_TIMEOUT (a bounded wait gave up; results unspecified). */
+ace_status ace_get_error(const ace_perm* perm, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* ACE_H_ */

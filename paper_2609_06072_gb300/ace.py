@@ -1,0 +1,261 @@
+"""Thin ctypes binding of the ACE C ABI (include/ace.h).
+
+Argument marshalling only: every step of the hot path runs in the CUDA
+kernels of libace.so.  PyTorch supplies device memory and streams.  There is
+no fallback: if libace.so is missing or the device is not sm_103, calls raise.
+
+Functions keep the C names (``ace_permute``, ``ace_fwd_shared``, ...); the
+``Plan`` class is a convenience holder for one layer description.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional, Sequence
+
+import torch
+
+from . import _build
+
+ACE_OK = 0
+ACE_ERR_ARG = 1
+ACE_ERR_SHAPE = 2
+ACE_ERR_WORKSPACE = 3
+ACE_ERR_INDEX = 4
+ACE_ERR_UNSUPPORTED = 5
+ACE_ERR_CUDA = 6
+ACE_ERR_DEVICE_TIMEOUT = 7
+ACE_FLAG_DETERMINISTIC = 1
+
+STATUS_NAMES = {0: "ACE_OK", 1: "ACE_ERR_ARG", 2: "ACE_ERR_SHAPE", 3: "ACE_ERR_WORKSPACE", 4: "ACE_ERR_INDEX",
+                5: "ACE_ERR_UNSUPPORTED", 6: "ACE_ERR_CUDA", 7: "ACE_ERR_DEVICE_TIMEOUT"}
+
+EXPORTED = ["ace_version", "ace_last_error_message", "ace_plan_create", "ace_plan_destroy", "ace_plan_rank_max",
+            "ace_workspace_size", "ace_permute", "ace_fwd_shared", "ace_fwd_row", "ace_bwd_shared", "ace_bwd_row",
+            "ace_gather_rows", "ace_scatter_rows", "ace_get_error"]
+
+
+class AceError(RuntimeError):
+    def __init__(self, status: int, what: str, msg: str = ""):
+        super().__init__(f"{what}: {STATUS_NAMES.get(status, status)} {msg}".strip())
+        self.status = status
+
+
+class ace_layer_desc(ctypes.Structure):
+    _fields_ = [("T_max", ctypes.c_int32), ("k", ctypes.c_int32), ("E", ctypes.c_int32), ("G", ctypes.c_int32),
+                ("e2g", ctypes.POINTER(ctypes.c_int32)), ("rank_off", ctypes.POINTER(ctypes.c_int32)),
+                ("d", ctypes.c_int32), ("f", ctypes.c_int32), ("flags", ctypes.c_uint32)]
+
+
+class ace_perm(ctypes.Structure):
+    _fields_ = [("T", ctypes.c_int32), ("R", ctypes.c_int32), ("counts", ctypes.c_void_p),
+                ("group_off", ctypes.c_void_p), ("expert_off", ctypes.c_void_p), ("expert_cnt", ctypes.c_void_p),
+                ("row_pair", ctypes.c_void_p), ("pair_row", ctypes.c_void_p), ("uniq_off", ctypes.c_void_p),
+                ("uniq_tok", ctypes.c_void_p), ("tok_uniq", ctypes.c_void_p), ("ws", ctypes.c_void_p)]
+
+
+_lib = None
+
+
+def lib_path() -> str:
+    return _build.LIB
+
+
+def load(build_if_missing: bool = False) -> ctypes.CDLL:
+    """Load libace.so (in-tree).  Raises if it has not been built."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = _build.LIB
+    if not os.path.exists(path):
+        if build_if_missing:
+            _build.build()
+        else:
+            raise RuntimeError(f"ACE CUDA library not built ({path}); run __graft_entry__.build()")
+    lib = ctypes.CDLL(path)
+    vp, i32, sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_size_t
+    lib.ace_version.restype = i32
+    lib.ace_last_error_message.restype = ctypes.c_char_p
+    lib.ace_plan_create.restype = i32
+    lib.ace_plan_create.argtypes = [ctypes.POINTER(vp), ctypes.POINTER(ace_layer_desc)]
+    lib.ace_plan_destroy.restype = None
+    lib.ace_plan_destroy.argtypes = [vp]
+    lib.ace_plan_rank_max.restype = i32
+    lib.ace_plan_rank_max.argtypes = [vp]
+    lib.ace_workspace_size.restype = i32
+    lib.ace_workspace_size.argtypes = [vp, i32, ctypes.POINTER(sz), ctypes.POINTER(sz), ctypes.POINTER(sz)]
+    lib.ace_permute.restype = i32
+    lib.ace_permute.argtypes = [vp, vp, i32, vp, sz, ctypes.POINTER(ace_perm), vp]
+    lib.ace_fwd_shared.restype = i32
+    lib.ace_fwd_shared.argtypes = [vp, ctypes.POINTER(ace_perm), vp, i32, vp, vp, ctypes.c_float, vp, vp, vp, sz, vp]
+    lib.ace_fwd_row.restype = i32
+    lib.ace_fwd_row.argtypes = [vp, ctypes.POINTER(ace_perm), vp, vp, vp, ctypes.c_float, vp, vp, vp, sz, vp]
+    lib.ace_bwd_shared.restype = i32
+    lib.ace_bwd_shared.argtypes = [vp, ctypes.POINTER(ace_perm), i32, vp, vp, vp, vp, vp, ctypes.c_float, vp, vp, vp,
+                                   vp, sz, vp]
+    lib.ace_bwd_row.restype = i32
+    lib.ace_bwd_row.argtypes = [vp, ctypes.POINTER(ace_perm), vp, vp, vp, vp, vp, ctypes.c_float, vp, vp, vp, vp, sz,
+                                vp]
+    lib.ace_gather_rows.restype = i32
+    lib.ace_gather_rows.argtypes = [ctypes.POINTER(ace_perm), vp, vp, i32, vp]
+    lib.ace_scatter_rows.restype = i32
+    lib.ace_scatter_rows.argtypes = [ctypes.POINTER(ace_perm), vp, vp, i32, vp]
+    lib.ace_get_error.restype = i32
+    lib.ace_get_error.argtypes = [ctypes.POINTER(ace_perm), vp]
+    _lib = lib
+    return lib
+
+
+def _check(st: int, what: str):
+    if st != ACE_OK:
+        msg = load().ace_last_error_message()
+        raise AceError(st, what, msg.decode() if msg else "")
+
+
+def _ptr(t: Optional[torch.Tensor], dtype=None, name: str = "tensor") -> Optional[int]:
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if dtype is not None and t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    return t.data_ptr()
+
+
+def _arr(ptrs: Sequence[Optional[int]]):
+    return (ctypes.c_void_p * len(ptrs))(*[p or 0 for p in ptrs])
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+class Perm:
+    """Device views filled by ace_permute (the workspace tensor is kept alive)."""
+
+    def __init__(self, c: ace_perm, ws: torch.Tensor):
+        self.c = c
+        self.ws = ws
+
+    @property
+    def T(self):
+        return self.c.T
+
+    @property
+    def R(self):
+        return self.c.R
+
+
+class Plan:
+    """One layer description (ace_plan) on the current CUDA device."""
+
+    def __init__(self, T_max: int, k: int, E: int, G: int, e2g, rank_off, d: int, f: int, deterministic=False):
+        self.lib = load()
+        self._e2g = (ctypes.c_int32 * E)(*[int(x) for x in e2g])
+        self._ro = (ctypes.c_int32 * (G + 1))(*[int(x) for x in rank_off])
+        desc = ace_layer_desc(int(T_max), int(k), int(E), int(G), self._e2g, self._ro, int(d), int(f),
+                              ACE_FLAG_DETERMINISTIC if deterministic else 0)
+        h = ctypes.c_void_p()
+        _check(self.lib.ace_plan_create(ctypes.byref(h), ctypes.byref(desc)), "ace_plan_create")
+        self.h = h
+        self.T_max, self.k, self.E, self.G, self.d, self.f = T_max, k, E, G, d, f
+        self.rank_max = self.lib.ace_plan_rank_max(h)
+        self.n_rank = int(rank_off[-1])
+
+    def __del__(self):
+        h = getattr(self, "h", None)
+        if h is not None and h.value:
+            self.lib.ace_plan_destroy(h)
+            self.h = None
+
+    def workspace_size(self, T: int):
+        p, fw, bw = ctypes.c_size_t(), ctypes.c_size_t(), ctypes.c_size_t()
+        _check(self.lib.ace_workspace_size(self.h, int(T), ctypes.byref(p), ctypes.byref(fw), ctypes.byref(bw)),
+               "ace_workspace_size")
+        return p.value, fw.value, bw.value
+
+    def alloc_workspaces(self, T: int, device="cuda"):
+        p, fw, bw = self.workspace_size(T)
+        mk = lambda n: torch.empty(max(n, 16), dtype=torch.uint8, device=device)
+        return mk(p), mk(fw), mk(bw)
+
+    def permute(self, topk_idx: torch.Tensor, perm_ws: torch.Tensor, stream=None) -> Perm:
+        T = int(topk_idx.shape[0]) if topk_idx.numel() else 0
+        c = ace_perm()
+        _check(self.lib.ace_permute(self.h, _ptr(topk_idx, torch.int32, "topk_idx"), T, _ptr(perm_ws),
+                                    perm_ws.numel(), ctypes.byref(c), _stream(stream)), "ace_permute")
+        return Perm(c, perm_ws)
+
+    def fwd_shared(self, perm: Perm, X, A, Bt, s, Y, H=None, ws=None, stream=None):
+        n = len(A)
+        Hp = _arr([_ptr(h, torch.float32, "H") for h in H]) if H is not None else None
+        _check(self.lib.ace_fwd_shared(self.h, ctypes.byref(perm.c), _ptr(X, torch.bfloat16, "X"), n,
+                                       _arr([_ptr(a, torch.bfloat16, "A") for a in A]),
+                                       _arr([_ptr(b, torch.bfloat16, "Bt") for b in Bt]), float(s),
+                                       _arr([_ptr(y, torch.bfloat16, "Y") for y in Y]), Hp,
+                                       _ptr(ws) if ws is not None else None, 0 if ws is None else ws.numel(),
+                                       _stream(stream)), "ace_fwd_shared")
+
+    def fwd_row(self, perm: Perm, Hin, A, Bt, s, Y, H=None, ws=None, stream=None):
+        _check(self.lib.ace_fwd_row(self.h, ctypes.byref(perm.c), _ptr(Hin, torch.bfloat16, "Hin"),
+                                    _ptr(A, torch.bfloat16, "A"), _ptr(Bt, torch.bfloat16, "Bt"), float(s),
+                                    _ptr(Y, torch.bfloat16, "Y"), _ptr(H, torch.float32, "H"),
+                                    _ptr(ws) if ws is not None else None, 0 if ws is None else ws.numel(),
+                                    _stream(stream)), "ace_fwd_row")
+
+    def bwd_shared(self, perm: Perm, dY, X, H, A, Bt, s, dX, dA, dBt, ws, stream=None):
+        n = len(dY)
+        _check(self.lib.ace_bwd_shared(self.h, ctypes.byref(perm.c), n,
+                                       _arr([_ptr(t, torch.bfloat16, "dY") for t in dY]),
+                                       _ptr(X, torch.bfloat16, "X"), _arr([_ptr(t, torch.float32, "H") for t in H]),
+                                       _arr([_ptr(t, torch.bfloat16, "A") for t in A]),
+                                       _arr([_ptr(t, torch.bfloat16, "Bt") for t in Bt]), float(s),
+                                       _ptr(dX, torch.bfloat16, "dX"), _arr([_ptr(t, torch.float32, "dA") for t in dA]),
+                                       _arr([_ptr(t, torch.float32, "dBt") for t in dBt]), _ptr(ws), ws.numel(),
+                                       _stream(stream)), "ace_bwd_shared")
+
+    def bwd_row(self, perm: Perm, dY, Hin, H, A, Bt, s, dHin, dA, dBt, ws, stream=None):
+        _check(self.lib.ace_bwd_row(self.h, ctypes.byref(perm.c), _ptr(dY, torch.bfloat16, "dY"),
+                                    _ptr(Hin, torch.bfloat16, "Hin"), _ptr(H, torch.float32, "H"),
+                                    _ptr(A, torch.bfloat16, "A"), _ptr(Bt, torch.bfloat16, "Bt"), float(s),
+                                    _ptr(dHin, torch.bfloat16, "dHin"), _ptr(dA, torch.float32, "dA"),
+                                    _ptr(dBt, torch.float32, "dBt"), _ptr(ws), ws.numel(), _stream(stream)),
+               "ace_bwd_row")
+
+    def gather_rows(self, perm: Perm, src_pairs, dst_rows, stream=None):
+        _check(self.lib.ace_gather_rows(ctypes.byref(perm.c), _ptr(src_pairs), _ptr(dst_rows),
+                                        int(src_pairs.shape[-1]), _stream(stream)), "ace_gather_rows")
+
+    def scatter_rows(self, perm: Perm, src_rows, dst_pairs, stream=None):
+        _check(self.lib.ace_scatter_rows(ctypes.byref(perm.c), _ptr(src_rows), _ptr(dst_pairs),
+                                         int(src_rows.shape[-1]), _stream(stream)), "ace_scatter_rows")
+
+    def get_error(self, perm: Perm, stream=None) -> int:
+        """Synchronise, read and clear the device flag; returns the status code."""
+        return self.lib.ace_get_error(ctypes.byref(perm.c), _stream(stream))
+
+
+def perm_arrays(plan: Plan, perm: Perm) -> dict:
+    """Copy the permutation views to host numpy arrays (synchronises)."""
+    import numpy as np
+    T, R, E, G, k = perm.T, perm.R, plan.E, plan.G, plan.k
+    ws = perm.ws
+    base = ws.data_ptr()
+
+    def view(ptr, n):
+        if n == 0:
+            return np.zeros(0, np.int32)
+        off = ptr - base
+        return ws[off: off + 4 * n].view(torch.int32).cpu().numpy().copy()
+
+    c = perm.c
+    counts = view(c.counts, 8)
+    U = int(counts[0])
+    return {"U": U, "rows": int(counts[1]), "group_off": view(c.group_off, G + 1),
+            "expert_off": view(c.expert_off, E), "expert_cnt": view(c.expert_cnt, E),
+            "row_pair": view(c.row_pair, R), "pair_row": view(c.pair_row, R), "uniq_off": view(c.uniq_off, G + 1),
+            "uniq_tok": view(c.uniq_tok, U), "tok_uniq": view(c.tok_uniq, R).reshape(T, k)}

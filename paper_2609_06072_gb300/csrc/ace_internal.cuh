@@ -1,0 +1,160 @@
+// Internal declarations shared by the ACE CUDA translation units.
+#pragma once
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "../../include/ace.h"
+
+namespace ace {
+
+constexpr int kTileM = 128;        // rows (or unique pairs) per MMA tile
+constexpr int kPermTB = 256;       // tokens per permutation chunk / CTA
+constexpr int kMaxK = 32;          // largest top-k the kernels accept
+
+// Device error-flag bits (the flag lives at perm workspace word 0).
+constexpr int kErrIndex = 1;
+constexpr int kErrTimeout = 2;
+
+// Plan tables passed by value (__grid_constant__) to every kernel.
+struct PlanTables {
+  int32_t E, G, k, d, f;
+  int32_t rank_max;  // max_g r_g
+  int32_t rank_pad;  // MMA N of one projection's rank block (16/32/64/128)
+  int32_t nt_split;  // tiles per backward split
+  int16_t e2g[ACE_MAX_EXPERTS];
+  int32_t rank_off[ACE_MAX_EXPERTS + 1];
+};
+
+// A unit of work: rows [start, start + cnt) of group g (row tiles) or unique
+// pairs [start, start + cnt) of group g (shared tiles).  `id` is the split
+// index for backward splits.
+struct Tile {
+  int32_t g, start, cnt, id;
+};
+
+// Byte layout of the permutation workspace for T tokens.
+struct PermLayout {
+  size_t err, counts, group_off, expert_off, expert_cnt, uniq_off, row_pair, pair_row, pair_g, uniq_tok, tok_uniq;
+  size_t chunk_cntE, chunk_cntU, chunk_baseE, chunk_baseU, chunk_err;
+  size_t tiles_sh, tiles_row, splits_sh, splits_row;
+  size_t total;
+  int32_t n_chunks, max_tiles, max_splits;
+};
+
+// counts[] slots
+constexpr int kCntU = 0, kCntRows = 1, kCntTilesSh = 2, kCntTilesRow = 3, kCntSplitsSh = 4, kCntSplitsRow = 5;
+
+inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+inline PermLayout perm_layout(const PlanTables& pt, int32_t T) {
+  PermLayout L{};
+  const int64_t R = (int64_t)T * pt.k;
+  L.n_chunks = (T + kPermTB - 1) / kPermTB;
+  L.max_tiles = (int32_t)((R + kTileM - 1) / kTileM + pt.G);
+  const int64_t split_rows = (int64_t)kTileM * pt.nt_split;
+  L.max_splits = (int32_t)((R + split_rows - 1) / split_rows + pt.G);
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    size_t o = off;
+    off = align_up(off + bytes, 256);
+    return o;
+  };
+  L.err = take(4 * 8);
+  L.counts = take(4 * 8);
+  L.group_off = take(4 * (size_t)(pt.G + 1));
+  L.expert_off = take(4 * (size_t)pt.E);
+  L.expert_cnt = take(4 * (size_t)pt.E);
+  L.uniq_off = take(4 * (size_t)(pt.G + 1));
+  L.row_pair = take(4 * (size_t)R);
+  L.pair_row = take(4 * (size_t)R);
+  L.pair_g = take(4 * (size_t)R);
+  L.uniq_tok = take(4 * (size_t)R);
+  L.tok_uniq = take(4 * (size_t)R);
+  L.chunk_cntE = take(4 * (size_t)L.n_chunks * pt.E);
+  L.chunk_cntU = take(4 * (size_t)L.n_chunks * pt.G);
+  L.chunk_baseE = take(4 * (size_t)L.n_chunks * pt.E);
+  L.chunk_baseU = take(4 * (size_t)L.n_chunks * pt.G);
+  L.chunk_err = take(4 * (size_t)(L.n_chunks + 1));
+  L.tiles_sh = take(sizeof(Tile) * (size_t)L.max_tiles);
+  L.tiles_row = take(sizeof(Tile) * (size_t)L.max_tiles);
+  L.splits_sh = take(sizeof(Tile) * (size_t)L.max_splits);
+  L.splits_row = take(sizeof(Tile) * (size_t)L.max_splits);
+  L.total = off;
+  return L;
+}
+
+template <typename T>
+inline T* at(void* base, size_t off) {
+  return reinterpret_cast<T*>(static_cast<char*>(base) + off);
+}
+
+// Launchers implemented in the .cu files (host side).  Each returns the
+// cudaError_t of its launches.
+cudaError_t launch_permute(const PlanTables& pt, const int32_t* topk_idx, int32_t T, void* ws, const PermLayout& L,
+                           cudaStream_t st);
+cudaError_t launch_rows_copy(const int32_t* row_pair, const uint16_t* src, uint16_t* dst, int64_t R, int32_t cols,
+                             bool gather, cudaStream_t st);
+
+struct FwdLaunch {
+  const Tile* tiles;
+  const int32_t* counts;
+  int32_t count_slot;
+  int32_t max_tiles;
+  const int32_t* uniq_tok;
+  const int32_t* pair_g;  // group of each pair (-1: invalid token)
+  const int32_t* row_pair;
+  const int32_t* pair_row;
+  const int32_t* tok_uniq;
+  const uint16_t* X;
+  const uint16_t* A[2];
+  const uint16_t* Bt[2];
+  uint16_t* Y[2];
+  float* H[2];
+  float s;
+  int32_t d_in, d_out, nproj, T;
+  int32_t* err;
+};
+cudaError_t launch_fwd(const PlanTables& pt, const FwdLaunch& a, bool shared, cudaStream_t st);
+
+struct BwdLaunch {
+  const Tile* splits;
+  const int32_t* counts;
+  int32_t count_slot;
+  int32_t max_splits;
+  const int32_t* uniq_tok;
+  const int32_t* tok_uniq;
+  const int32_t* pair_row;
+  const int32_t* pair_g;
+  const int32_t* uniq_off;
+  const int32_t* group_off;
+  const uint16_t* dY[2];
+  const uint16_t* Xin;   // shared: X [T, d]; row: Hin [R, f]
+  const float* H[2];
+  const uint16_t* A[2];
+  const uint16_t* Bt[2];
+  float s;
+  uint16_t* dXin;        // row path: dHin [R, f] in/out
+  uint16_t* dH[2];       // scratch: bf16 [R, rank_pad] (shared path: per unique pair)
+  float* dA[2];
+  float* dBt[2];
+  float* part_dA[2];     // deterministic partials [max_splits, rank_pad, d_in]
+  float* part_dBt[2];    // [max_splits, rank_pad, d_out]
+  int32_t d_in, d_out, nproj, T;
+  bool deterministic;
+  int32_t* err;
+};
+cudaError_t launch_bwd(const PlanTables& pt, const BwdLaunch& a, bool shared, cudaStream_t st);
+
+struct DxLaunch {
+  const int32_t* tok_uniq;
+  const int32_t* uniq_off;
+  const uint16_t* dH[2];
+  const uint16_t* A[2];
+  uint16_t* dX;
+  int32_t T, d, nproj;
+  int32_t* err;
+};
+cudaError_t launch_dx(const PlanTables& pt, const DxLaunch& a, cudaStream_t st);
+
+}  // namespace ace

@@ -1,0 +1,400 @@
+// Host side of the C ABI declared in include/ace.h: plan validation,
+// workspace layout, argument checks and kernel launches.  No entry point
+// allocates device memory or synchronises (except ace_get_error).
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+
+#include "ace_internal.cuh"
+
+using namespace ace;
+
+struct ace_plan {
+  PlanTables pt;
+  int32_t T_max;
+  uint32_t flags;
+  int device;
+};
+
+namespace {
+
+thread_local char g_msg[512] = "";
+
+ace_status fail(ace_status st, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_msg, sizeof(g_msg), fmt, ap);
+  va_end(ap);
+  return st;
+}
+
+ace_status cuda_status(cudaError_t e, const char* what) {
+  if (e == cudaSuccess) return ACE_OK;
+  return fail(ACE_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Backward TMEM budget: (tiles per split + 2) * rank_pad columns <= 256.
+int nt_split_for(int rank_pad) { return rank_pad <= 16 ? 8 : rank_pad == 32 ? 4 : rank_pad == 64 ? 2 : 1; }
+
+ace_status check_perm(const ace_plan* plan, const ace_perm* perm) {
+  if (!plan || !perm || !perm->ws) return fail(ACE_ERR_ARG, "null plan or perm");
+  if (perm->T < 0 || perm->T > plan->T_max) return fail(ACE_ERR_SHAPE, "perm T=%d outside [0, %d]", perm->T, plan->T_max);
+  if (perm->R != perm->T * plan->pt.k) return fail(ACE_ERR_ARG, "perm R does not match T*k");
+  return ACE_OK;
+}
+
+struct BwdWs {
+  uint16_t* dH[2];
+  float* part_dA[2];
+  float* part_dBt[2];
+  size_t total;
+};
+
+BwdWs bwd_layout(const PlanTables& pt, int32_t T, void* base) {
+  const PermLayout L = perm_layout(pt, T);
+  const int64_t R = (int64_t)T * pt.k;
+  const size_t dh = align_up(2 * (size_t)R * pt.rank_pad, 256);
+  const size_t part = align_up(4 * (size_t)L.max_splits * pt.rank_pad * (size_t)(pt.d + pt.f), 256);
+  BwdWs w{};
+  char* b = static_cast<char*>(base);
+  size_t off = 0;
+  for (int j = 0; j < 2; ++j) {
+    w.dH[j] = reinterpret_cast<uint16_t*>(b + off);
+    off += dh;
+  }
+  for (int j = 0; j < 2; ++j) {
+    w.part_dA[j] = reinterpret_cast<float*>(b + off);
+    // dA partial [max_splits, rank_pad, d_in] followed by dBt partial
+    // [max_splits, rank_pad, d_out]; d_in + d_out = d + f for every projection
+    w.part_dBt[j] = nullptr;
+    off += part;
+  }
+  w.total = off;
+  return w;
+}
+
+}  // namespace
+
+extern "C" {
+
+int32_t ace_version(void) { return ACE_VERSION; }
+
+const char* ace_last_error_message(void) { return g_msg; }
+
+ace_status ace_plan_create(ace_plan** out, const ace_layer_desc* desc) {
+  if (!out || !desc) return fail(ACE_ERR_ARG, "null argument");
+  *out = nullptr;
+  const ace_layer_desc& D = *desc;
+  if (!D.e2g || !D.rank_off) return fail(ACE_ERR_ARG, "null e2g / rank_off");
+  if (D.E < 1 || D.E > ACE_MAX_EXPERTS) return fail(ACE_ERR_SHAPE, "E=%d outside [1, %d]", D.E, ACE_MAX_EXPERTS);
+  if (D.G < 1 || D.G > D.E) return fail(ACE_ERR_SHAPE, "G=%d outside [1, E]", D.G);
+  if (D.k < 1 || D.k > D.E || D.k > kMaxK) return fail(ACE_ERR_SHAPE, "k=%d outside [1, min(E, %d)]", D.k, kMaxK);
+  if (D.T_max < 0) return fail(ACE_ERR_SHAPE, "T_max < 0");
+  if ((int64_t)D.T_max * D.k > (int64_t)1 << 30) return fail(ACE_ERR_SHAPE, "T_max * k too large");
+  if (D.d < 8 || D.f < 8 || D.d % 8 || D.f % 8) return fail(ACE_ERR_SHAPE, "d=%d, f=%d must be positive multiples of 8", D.d, D.f);
+  int used[ACE_MAX_EXPERTS] = {0};
+  for (int e = 0; e < D.E; ++e) {
+    if (D.e2g[e] < 0 || D.e2g[e] >= D.G) return fail(ACE_ERR_INDEX, "e2g[%d]=%d outside [0, G)", e, D.e2g[e]);
+    used[D.e2g[e]] = 1;
+  }
+  for (int g = 0; g < D.G; ++g)
+    if (!used[g]) return fail(ACE_ERR_INDEX, "group %d has no expert", g);
+  if (D.rank_off[0] != 0) return fail(ACE_ERR_ARG, "rank_off[0] must be 0");
+  int rank_max = 0;
+  for (int g = 0; g < D.G; ++g) {
+    const int rg = D.rank_off[g + 1] - D.rank_off[g];
+    if (rg < 1) return fail(ACE_ERR_ARG, "r_%d=%d < 1", g, rg);
+    if (rg > ACE_MAX_RANK) return fail(ACE_ERR_UNSUPPORTED, "r_%d=%d > %d", g, rg, ACE_MAX_RANK);
+    rank_max = rg > rank_max ? rg : rank_max;
+  }
+  int dev = 0;
+  cudaError_t ce = cudaGetDevice(&dev);
+  if (ce != cudaSuccess) return cuda_status(ce, "cudaGetDevice");
+  int major = 0, minor = 0;
+  cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+  cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+  if (!(major == 10 && minor == 3))
+    return fail(ACE_ERR_UNSUPPORTED, "device %d is sm_%d%d; this library is built for sm_103a only", dev, major, minor);
+  ace_plan* p = new (std::nothrow) ace_plan();
+  if (!p) return fail(ACE_ERR_ARG, "out of host memory");
+  std::memset(&p->pt, 0, sizeof(p->pt));
+  p->pt.E = D.E;
+  p->pt.G = D.G;
+  p->pt.k = D.k;
+  p->pt.d = D.d;
+  p->pt.f = D.f;
+  p->pt.rank_max = rank_max;
+  p->pt.rank_pad = rank_max <= 16 ? 16 : rank_max <= 32 ? 32 : rank_max <= 64 ? 64 : 128;
+  p->pt.nt_split = nt_split_for(p->pt.rank_pad);
+  for (int e = 0; e < D.E; ++e) p->pt.e2g[e] = (int16_t)D.e2g[e];
+  for (int g = 0; g <= D.G; ++g) p->pt.rank_off[g] = D.rank_off[g];
+  p->T_max = D.T_max;
+  p->flags = D.flags;
+  p->device = dev;
+  *out = p;
+  return ACE_OK;
+}
+
+void ace_plan_destroy(ace_plan* plan) { delete plan; }
+
+int32_t ace_plan_rank_max(const ace_plan* plan) { return plan ? plan->pt.rank_max : 0; }
+
+ace_status ace_workspace_size(const ace_plan* plan, int32_t T, size_t* perm_bytes, size_t* fwd_bytes,
+                              size_t* bwd_bytes) {
+  if (!plan) return fail(ACE_ERR_ARG, "null plan");
+  if (T < 0 || T > plan->T_max) return fail(ACE_ERR_SHAPE, "T=%d outside [0, %d]", T, plan->T_max);
+  if (perm_bytes) *perm_bytes = perm_layout(plan->pt, T).total;
+  if (fwd_bytes) *fwd_bytes = 0;
+  if (bwd_bytes) *bwd_bytes = bwd_layout(plan->pt, T, nullptr).total;
+  return ACE_OK;
+}
+
+ace_status ace_permute(const ace_plan* plan, const int32_t* topk_idx, int32_t T, void* perm_ws, size_t perm_ws_bytes,
+                       ace_perm* out, void* stream) {
+  if (!plan || !out || !perm_ws) return fail(ACE_ERR_ARG, "null argument");
+  if (T < 0 || T > plan->T_max) return fail(ACE_ERR_SHAPE, "T=%d outside [0, %d]", T, plan->T_max);
+  if (T > 0 && !topk_idx) return fail(ACE_ERR_ARG, "null topk_idx");
+  const PermLayout L = perm_layout(plan->pt, T);
+  if (perm_ws_bytes < L.total) return fail(ACE_ERR_WORKSPACE, "perm workspace %zu < %zu bytes", perm_ws_bytes, L.total);
+  if (!aligned16(perm_ws) || (topk_idx && (reinterpret_cast<uintptr_t>(topk_idx) & 3u)))
+    return fail(ACE_ERR_WORKSPACE, "misaligned workspace or topk_idx");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  ace_status s = cuda_status(launch_permute(plan->pt, topk_idx, T, perm_ws, L, st), "permute launch");
+  if (s != ACE_OK) return s;
+  out->T = T;
+  out->R = T * plan->pt.k;
+  out->counts = at<int32_t>(perm_ws, L.counts);
+  out->group_off = at<int32_t>(perm_ws, L.group_off);
+  out->expert_off = at<int32_t>(perm_ws, L.expert_off);
+  out->expert_cnt = at<int32_t>(perm_ws, L.expert_cnt);
+  out->row_pair = at<int32_t>(perm_ws, L.row_pair);
+  out->pair_row = at<int32_t>(perm_ws, L.pair_row);
+  out->uniq_off = at<int32_t>(perm_ws, L.uniq_off);
+  out->uniq_tok = at<int32_t>(perm_ws, L.uniq_tok);
+  out->tok_uniq = at<int32_t>(perm_ws, L.tok_uniq);
+  out->ws = perm_ws;
+  return ACE_OK;
+}
+
+static ace_status fwd_common(const ace_plan* plan, const ace_perm* perm, const uint16_t* X, int nproj,
+                             const uint16_t* const* A, const uint16_t* const* Bt, float s, uint16_t* const* Y,
+                             float* const* H, bool shared, void* stream) {
+  ace_status st = check_perm(plan, perm);
+  if (st != ACE_OK) return st;
+  if (nproj < 1 || nproj > 2) return fail(ACE_ERR_ARG, "nproj=%d must be 1 or 2", nproj);
+  if (!A || !Bt || !Y) return fail(ACE_ERR_ARG, "null A / Bt / Y array");
+  if (perm->R > 0 && !X) return fail(ACE_ERR_ARG, "null input");
+  if (X && !aligned16(X)) return fail(ACE_ERR_ARG, "input not 16-byte aligned");
+  for (int j = 0; j < nproj; ++j) {
+    if (!A[j] || !Bt[j] || !Y[j]) return fail(ACE_ERR_ARG, "null A / Bt / Y of projection %d", j);
+    if (!aligned16(A[j]) || !aligned16(Bt[j]) || !aligned16(Y[j]) || (H && H[j] && !aligned16(H[j])))
+      return fail(ACE_ERR_ARG, "tensor of projection %d not 16-byte aligned", j);
+  }
+  if (perm->R == 0) return ACE_OK;
+  const PermLayout L = perm_layout(plan->pt, perm->T);
+  FwdLaunch a{};
+  a.tiles = at<Tile>(perm->ws, shared ? L.tiles_sh : L.tiles_row);
+  a.counts = perm->counts;
+  a.count_slot = shared ? kCntTilesSh : kCntTilesRow;
+  a.max_tiles = L.max_tiles;
+  a.uniq_tok = perm->uniq_tok;
+  a.pair_g = at<int32_t>(perm->ws, L.pair_g);
+  a.row_pair = perm->row_pair;
+  a.pair_row = perm->pair_row;
+  a.tok_uniq = perm->tok_uniq;
+  a.X = X;
+  for (int j = 0; j < 2; ++j) {
+    const int jj = j < nproj ? j : 0;
+    a.A[j] = A[jj];
+    a.Bt[j] = Bt[jj];
+    a.Y[j] = Y[jj];
+    a.H[j] = H ? H[jj] : nullptr;
+  }
+  a.s = s;
+  a.d_in = shared ? plan->pt.d : plan->pt.f;
+  a.d_out = shared ? plan->pt.f : plan->pt.d;
+  a.nproj = nproj;
+  a.T = perm->T;
+  a.err = at<int32_t>(perm->ws, L.err);
+  return cuda_status(launch_fwd(plan->pt, a, shared, static_cast<cudaStream_t>(stream)), "forward launch");
+}
+
+ace_status ace_fwd_shared(const ace_plan* plan, const ace_perm* perm, const uint16_t* X, int32_t nproj,
+                          const uint16_t* const* A, const uint16_t* const* Bt, float s, uint16_t* const* Y,
+                          float* const* H, void* ws, size_t ws_bytes, void* stream) {
+  (void)ws;
+  (void)ws_bytes;
+  if (!plan || !perm) return fail(ACE_ERR_ARG, "null plan or perm");
+  return fwd_common(plan, perm, X, nproj, A, Bt, s, Y, H, true, stream);
+}
+
+ace_status ace_fwd_row(const ace_plan* plan, const ace_perm* perm, const uint16_t* Hin, const uint16_t* A,
+                       const uint16_t* Bt, float s, uint16_t* Y, float* H, void* ws, size_t ws_bytes, void* stream) {
+  (void)ws;
+  (void)ws_bytes;
+  const uint16_t* Aa[1] = {A};
+  const uint16_t* Ba[1] = {Bt};
+  uint16_t* Ya[1] = {Y};
+  float* Ha[1] = {H};
+  return fwd_common(plan, perm, Hin, 1, Aa, Ba, s, Ya, Ha, false, stream);
+}
+
+ace_status ace_bwd_shared(const ace_plan* plan, const ace_perm* perm, int32_t nproj, const uint16_t* const* dY,
+                          const uint16_t* X, const float* const* H, const uint16_t* const* A,
+                          const uint16_t* const* Bt, float s, uint16_t* dX, float* const* dA, float* const* dBt,
+                          void* ws, size_t ws_bytes, void* stream) {
+  ace_status st = check_perm(plan, perm);
+  if (st != ACE_OK) return st;
+  if (nproj < 1 || nproj > 2) return fail(ACE_ERR_ARG, "nproj=%d must be 1 or 2", nproj);
+  if (!dY || !H || !A || !Bt || !dA || !dBt || !dX || !X) return fail(ACE_ERR_ARG, "null argument");
+  if (!aligned16(X) || !aligned16(dX)) return fail(ACE_ERR_ARG, "X / dX not 16-byte aligned");
+  for (int j = 0; j < nproj; ++j) {
+    if (!dY[j] || !H[j] || !A[j] || !Bt[j] || !dA[j] || !dBt[j]) return fail(ACE_ERR_ARG, "null tensor of projection %d", j);
+    if (!aligned16(dY[j]) || !aligned16(H[j]) || !aligned16(A[j]) || !aligned16(Bt[j]) || !aligned16(dA[j]) ||
+        !aligned16(dBt[j]))
+      return fail(ACE_ERR_ARG, "tensor of projection %d not 16-byte aligned", j);
+  }
+  const BwdWs need = bwd_layout(plan->pt, perm->T, nullptr);
+  if (!ws || ws_bytes < need.total) return fail(ACE_ERR_WORKSPACE, "backward workspace %zu < %zu bytes", ws_bytes, need.total);
+  if (!aligned16(ws)) return fail(ACE_ERR_WORKSPACE, "backward workspace misaligned");
+  const PermLayout L = perm_layout(plan->pt, perm->T);
+  const BwdWs w = bwd_layout(plan->pt, perm->T, ws);
+  cudaStream_t cs = static_cast<cudaStream_t>(stream);
+  BwdLaunch a{};
+  a.splits = at<Tile>(perm->ws, L.splits_sh);
+  a.counts = perm->counts;
+  a.count_slot = kCntSplitsSh;
+  a.max_splits = L.max_splits;
+  a.uniq_tok = perm->uniq_tok;
+  a.tok_uniq = perm->tok_uniq;
+  a.pair_row = perm->pair_row;
+  a.pair_g = at<int32_t>(perm->ws, L.pair_g);
+  a.uniq_off = perm->uniq_off;
+  a.group_off = perm->group_off;
+  a.Xin = X;
+  for (int j = 0; j < 2; ++j) {
+    const int jj = j < nproj ? j : 0;
+    a.dY[j] = dY[jj];
+    a.H[j] = H[jj];
+    a.A[j] = A[jj];
+    a.Bt[j] = Bt[jj];
+    a.dA[j] = dA[jj];
+    a.dBt[j] = dBt[jj];
+    a.dH[j] = w.dH[jj];
+    a.part_dA[j] = w.part_dA[jj];
+    a.part_dBt[j] = w.part_dA[jj] + (size_t)L.max_splits * plan->pt.rank_pad * plan->pt.d;
+  }
+  a.s = s;
+  a.dXin = nullptr;
+  a.d_in = plan->pt.d;
+  a.d_out = plan->pt.f;
+  a.nproj = nproj;
+  a.T = perm->T;
+  a.deterministic = (plan->flags & ACE_FLAG_DETERMINISTIC) != 0;
+  a.err = at<int32_t>(perm->ws, L.err);
+  st = cuda_status(launch_bwd(plan->pt, a, true, cs), "backward launch");
+  if (st != ACE_OK) return st;
+  if (perm->R == 0) return ACE_OK;
+  DxLaunch x{};
+  x.tok_uniq = perm->tok_uniq;
+  x.uniq_off = perm->uniq_off;
+  for (int j = 0; j < 2; ++j) {
+    const int jj = j < nproj ? j : 0;
+    x.dH[j] = w.dH[jj];
+    x.A[j] = A[jj];
+  }
+  x.dX = dX;
+  x.T = perm->T;
+  x.d = plan->pt.d;
+  x.nproj = nproj;
+  x.err = a.err;
+  return cuda_status(launch_dx(plan->pt, x, cs), "dX launch");
+}
+
+ace_status ace_bwd_row(const ace_plan* plan, const ace_perm* perm, const uint16_t* dY, const uint16_t* Hin,
+                       const float* H, const uint16_t* A, const uint16_t* Bt, float s, uint16_t* dHin, float* dA,
+                       float* dBt, void* ws, size_t ws_bytes, void* stream) {
+  ace_status st = check_perm(plan, perm);
+  if (st != ACE_OK) return st;
+  if (!dY || !Hin || !H || !A || !Bt || !dHin || !dA || !dBt) return fail(ACE_ERR_ARG, "null argument");
+  if (!aligned16(dY) || !aligned16(Hin) || !aligned16(H) || !aligned16(A) || !aligned16(Bt) || !aligned16(dHin) ||
+      !aligned16(dA) || !aligned16(dBt))
+    return fail(ACE_ERR_ARG, "tensor not 16-byte aligned");
+  const BwdWs need = bwd_layout(plan->pt, perm->T, nullptr);
+  if (!ws || ws_bytes < need.total) return fail(ACE_ERR_WORKSPACE, "backward workspace %zu < %zu bytes", ws_bytes, need.total);
+  if (!aligned16(ws)) return fail(ACE_ERR_WORKSPACE, "backward workspace misaligned");
+  const PermLayout L = perm_layout(plan->pt, perm->T);
+  const BwdWs w = bwd_layout(plan->pt, perm->T, ws);
+  BwdLaunch a{};
+  a.splits = at<Tile>(perm->ws, L.splits_row);
+  a.counts = perm->counts;
+  a.count_slot = kCntSplitsRow;
+  a.max_splits = L.max_splits;
+  a.uniq_tok = perm->uniq_tok;
+  a.tok_uniq = perm->tok_uniq;
+  a.pair_row = perm->pair_row;
+  a.pair_g = at<int32_t>(perm->ws, L.pair_g);
+  a.uniq_off = perm->uniq_off;
+  a.group_off = perm->group_off;
+  a.Xin = Hin;
+  for (int j = 0; j < 2; ++j) {
+    a.dY[j] = dY;
+    a.H[j] = H;
+    a.A[j] = A;
+    a.Bt[j] = Bt;
+    a.dA[j] = dA;
+    a.dBt[j] = dBt;
+    a.dH[j] = w.dH[0];
+    a.part_dA[j] = w.part_dA[0];
+    a.part_dBt[j] = w.part_dA[0] + (size_t)L.max_splits * plan->pt.rank_pad * plan->pt.f;
+  }
+  a.s = s;
+  a.dXin = dHin;
+  a.d_in = plan->pt.f;
+  a.d_out = plan->pt.d;
+  a.nproj = 1;
+  a.T = perm->T;
+  a.deterministic = (plan->flags & ACE_FLAG_DETERMINISTIC) != 0;
+  a.err = at<int32_t>(perm->ws, L.err);
+  return cuda_status(launch_bwd(plan->pt, a, false, static_cast<cudaStream_t>(stream)), "backward launch");
+}
+
+ace_status ace_gather_rows(const ace_perm* perm, const uint16_t* src_pairs, uint16_t* dst_rows, int32_t cols,
+                           void* stream) {
+  if (!perm || !src_pairs || !dst_rows) return fail(ACE_ERR_ARG, "null argument");
+  if (cols < 8 || cols % 8) return fail(ACE_ERR_SHAPE, "cols=%d must be a positive multiple of 8", cols);
+  if (!aligned16(src_pairs) || !aligned16(dst_rows)) return fail(ACE_ERR_ARG, "misaligned tensor");
+  return cuda_status(launch_rows_copy(perm->row_pair, src_pairs, dst_rows, perm->R, cols, true,
+                                      static_cast<cudaStream_t>(stream)),
+                     "gather launch");
+}
+
+ace_status ace_scatter_rows(const ace_perm* perm, const uint16_t* src_rows, uint16_t* dst_pairs, int32_t cols,
+                            void* stream) {
+  if (!perm || !src_rows || !dst_pairs) return fail(ACE_ERR_ARG, "null argument");
+  if (cols < 8 || cols % 8) return fail(ACE_ERR_SHAPE, "cols=%d must be a positive multiple of 8", cols);
+  if (!aligned16(src_rows) || !aligned16(dst_pairs)) return fail(ACE_ERR_ARG, "misaligned tensor");
+  return cuda_status(launch_rows_copy(perm->row_pair, src_rows, dst_pairs, perm->R, cols, false,
+                                      static_cast<cudaStream_t>(stream)),
+                     "scatter launch");
+}
+
+ace_status ace_get_error(const ace_perm* perm, void* stream) {
+  if (!perm || !perm->ws) return fail(ACE_ERR_ARG, "null perm");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  ace_status s = cuda_status(cudaStreamSynchronize(st), "stream synchronize");
+  if (s != ACE_OK) return s;
+  int32_t flag = 0;
+  s = cuda_status(cudaMemcpy(&flag, perm->ws, sizeof(flag), cudaMemcpyDeviceToHost), "read error flag");
+  if (s != ACE_OK) return s;
+  s = cuda_status(cudaMemset(perm->ws, 0, sizeof(flag)), "clear error flag");
+  if (s != ACE_OK) return s;
+  if (flag & kErrTimeout) return fail(ACE_ERR_DEVICE_TIMEOUT, "a bounded device wait gave up");
+  if (flag & kErrIndex) return fail(ACE_ERR_INDEX, "invalid routing: expert id out of range or repeated in a token");
+  return ACE_OK;
+}
+
+}  // extern "C"

@@ -120,8 +120,8 @@ def fwd(topk_idx, e2g, rank_off, X, A_all, Bt_all, s, x_per_pair=False, y_in=Non
         want_h=False):
     """y_out[p] = y_in[p] + s B_g (A_g x_p) for every pair p (or the pairs in sel).
 
-    Returns (y_out [T*k, d_out] float64, H [T*k, r_max] float64 or None).
-    Rows of pairs outside ``sel`` are NaN.
+    Returns (y_out, H): [T*k, d_out] / [T*k, r_max] float64, or, with
+    ``sel``, [len(sel), ...] with row i holding pair sel[i].
     """
     lib = _load()
     idx = _c(topk_idx, np.int32)
@@ -134,10 +134,11 @@ def fwd(topk_idx, e2g, rank_off, X, A_all, Bt_all, s, x_per_pair=False, y_in=Non
     Bt_all = _c(Bt_all, np.uint16)
     d_in, d_out = A_all.shape[1], Bt_all.shape[1]
     R = T * k
-    y_out = np.full((R, d_out), np.nan)
-    r_max = int(np.max(np.diff(rank_off))) if G > 0 else 0
-    H = np.full((R, r_max), np.nan) if want_h else None
     sel_a = _c(sel, np.int32)
+    n_out = R if sel_a is None else sel_a.shape[0]
+    y_out = np.empty((n_out, d_out))
+    r_max = int(np.max(np.diff(rank_off))) if G > 0 else 0
+    H = np.empty((n_out, r_max)) if want_h else None
     st = lib.oracle_fwd(T, k, e2g.shape[0], G, _p(idx), _p(e2g), _p(rank_off), d_in, d_out, _p(X),
                         int(bool(x_per_pair)), _p(A_all), _p(Bt_all), float(s), _p(_c(y_in, np.uint16)),
                         _p(y_out), _p(H), r_max, _p(sel_a), 0 if sel_a is None else sel_a.shape[0])
@@ -147,7 +148,8 @@ def fwd(topk_idx, e2g, rank_off, X, A_all, Bt_all, s, x_per_pair=False, y_in=Non
 
 
 def bwd_dx(topk_idx, e2g, rank_off, dy, A_all, Bt_all, s, x_per_pair=False, dx_in=None, sel=None):
-    """Input gradient: token rows [T, d_in] (gate/up) or pair rows [T*k, d_in] (down)."""
+    """Input gradient: token rows [T, d_in] (gate/up) or pair rows [T*k, d_in]
+    (down); with ``sel``, [len(sel), d_in] with row i holding sel[i]."""
     lib = _load()
     idx = _c(topk_idx, np.int32)
     T, k = idx.shape
@@ -159,8 +161,8 @@ def bwd_dx(topk_idx, e2g, rank_off, dy, A_all, Bt_all, s, x_per_pair=False, dx_i
     dy = _c(dy, np.uint16)
     d_in, d_out = A_all.shape[1], Bt_all.shape[1]
     n_rows = T * k if x_per_pair else T
-    dx = np.full((n_rows, d_in), np.nan)
     sel_a = _c(sel, np.int32)
+    dx = np.empty((n_rows if sel_a is None else sel_a.shape[0], d_in))
     st = lib.oracle_bwd_dx(T, k, e2g.shape[0], G, _p(idx), _p(e2g), _p(rank_off), d_in, d_out,
                            int(bool(x_per_pair)), _p(dy), _p(A_all), _p(Bt_all), float(s),
                            _p(_c(dx_in, np.uint16)), _p(dx), _p(sel_a), 0 if sel_a is None else sel_a.shape[0])
@@ -170,7 +172,8 @@ def bwd_dx(topk_idx, e2g, rank_off, dy, A_all, Bt_all, s, x_per_pair=False, dx_i
 
 
 def bwd_w(topk_idx, e2g, rank_off, X, dy, A_all, Bt_all, s, x_per_pair=False, sel=None):
-    """(dA [sum r_g, d_in], dBt [sum r_g, d_out]) in float64; unselected rows NaN."""
+    """(dA [sum r_g, d_in], dBt [sum r_g, d_out]) in float64; with ``sel``,
+    [len(sel), ...] with row i holding rank row sel[i]."""
     lib = _load()
     idx = _c(topk_idx, np.int32)
     T, k = idx.shape
@@ -183,9 +186,10 @@ def bwd_w(topk_idx, e2g, rank_off, X, dy, A_all, Bt_all, s, x_per_pair=False, se
     Bt_all = _c(Bt_all, np.uint16)
     d_in, d_out = A_all.shape[1], Bt_all.shape[1]
     n_rank = int(rank_off[-1])
-    dA = np.full((n_rank, d_in), np.nan)
-    dBt = np.full((n_rank, d_out), np.nan)
     sel_a = _c(sel, np.int32)
+    n_out = n_rank if sel_a is None else sel_a.shape[0]
+    dA = np.empty((n_out, d_in))
+    dBt = np.empty((n_out, d_out))
     st = lib.oracle_bwd_w(T, k, e2g.shape[0], G, _p(idx), _p(e2g), _p(rank_off), d_in, d_out, _p(X),
                           int(bool(x_per_pair)), _p(dy), _p(A_all), _p(Bt_all), float(s), _p(dA), _p(dBt),
                           _p(sel_a), 0 if sel_a is None else sel_a.shape[0])

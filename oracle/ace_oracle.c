@@ -191,8 +191,8 @@ int oracle_permute(int32_t T, int32_t k, int32_t E, int32_t G, const int32_t* to
  *   y_out[p] = y_in[p] + s * B_g H_p           (d_out values)
  * x_p = X[t] when x_per_pair == 0 (gate/up: shared input), else X[p] (down).
  * B_g is given transposed: Bt_all holds B_g^T as rows rank_off[g]..rank_off[g+1]-1.
- * y_in may be NULL (taken as zero).  Only the pairs in sel[0..n_sel) are
- * computed when sel != NULL; y_out / h_out rows of other pairs are untouched.
+ * y_in may be NULL (taken as zero).  When sel != NULL only the pairs
+ * sel[0..n_sel) are computed and output row i holds pair sel[i] (compact).
  * h_out (may be NULL) receives H_p, padded with zeros to r_max entries.
  */
 int oracle_fwd(int32_t T, int32_t k, int32_t E, int32_t G, const int32_t* topk_idx, const int32_t* e2g,
@@ -223,14 +223,15 @@ int oracle_fwd(int32_t T, int32_t k, int32_t E, int32_t G, const int32_t* topk_i
       for (int32_t c = 0; c < d_in; ++c) acc += bf16_to_f64(a[c]) * bf16_to_f64(x[c]);
       H[i_r] = acc;
     }
+    const int64_t o_row = sel ? i : p;
     if (h_out) {
-      for (int32_t i_r = 0; i_r < r_max; ++i_r) h_out[p * r_max + i_r] = i_r < rg ? H[i_r] : 0.0;
+      for (int32_t i_r = 0; i_r < r_max; ++i_r) h_out[o_row * r_max + i_r] = i_r < rg ? H[i_r] : 0.0;
     }
     for (int32_t o = 0; o < d_out; ++o) {
       double acc = 0.0;
       for (int32_t i_r = 0; i_r < rg; ++i_r) acc += bf16_to_f64(Bt_all[(int64_t)(r0 + i_r) * d_out + o]) * H[i_r];
       double base = y_in ? bf16_to_f64(y_in[p * (int64_t)d_out + o]) : 0.0;
-      y_out[p * (int64_t)d_out + o] = base + s * acc;
+      y_out[o_row * (int64_t)d_out + o] = base + s * acc;
     }
   }
   return OR_OK;
@@ -243,7 +244,7 @@ int oracle_fwd(int32_t T, int32_t k, int32_t E, int32_t G, const int32_t* topk_i
  *   x_per_pair == 0 : dx_out[t] = dx_in[t] + sum_j s * A_g^T (B_g^T dy_{t*k+j})   (token rows)
  *   x_per_pair == 1 : dx_out[p] = dx_in[p] + s * A_g^T (B_g^T dy_p)              (pair rows)
  * dy is pair-ordered [T*k, d_out].  dx_in may be NULL.  sel lists the tokens
- * (or pairs) to compute; NULL = all.
+ * (or pairs) to compute, output row i holding sel[i]; NULL = all.
  */
 int oracle_bwd_dx(int32_t T, int32_t k, int32_t E, int32_t G, const int32_t* topk_idx, const int32_t* e2g,
                   const int32_t* rank_off, int32_t d_in, int32_t d_out, int32_t x_per_pair, const uint16_t* dy,
@@ -264,7 +265,7 @@ int oracle_bwd_dx(int32_t T, int32_t k, int32_t E, int32_t G, const int32_t* top
 #pragma omp parallel for schedule(dynamic, 8)
   for (int64_t i = 0; i < n; ++i) {
     int64_t q = sel ? sel[i] : i;
-    double* out = dx_out + q * (int64_t)d_in;
+    double* out = dx_out + (sel ? i : q) * (int64_t)d_in;
     for (int32_t c = 0; c < d_in; ++c) out[c] = dx_in ? bf16_to_f64(dx_in[q * (int64_t)d_in + c]) : 0.0;
     int64_t p_lo = x_per_pair ? q : q * k;
     int64_t p_hi = x_per_pair ? q + 1 : q * k + k;
@@ -292,7 +293,8 @@ int oracle_bwd_dx(int32_t T, int32_t k, int32_t E, int32_t G, const int32_t* top
  *   dBt[i][o] = s * sum_{p: g(e_p)=g(i)} (A_g x_p)[i]   * dy_p[o]
  * for every global rank row i (group g(i) owns rows rank_off[g]..rank_off[g+1]-1).
  * Pairs are visited in ascending p.  Groups with no pairs get exact zeros.
- * sel lists the rank rows to compute; NULL = all rank_off[G] rows.
+ * sel lists the rank rows to compute, output row ii holding rank row sel[ii];
+ * NULL = all rank_off[G] rows.
  */
 int oracle_bwd_w(int32_t T, int32_t k, int32_t E, int32_t G, const int32_t* topk_idx, const int32_t* e2g,
                  const int32_t* rank_off, int32_t d_in, int32_t d_out, const uint16_t* X, int32_t x_per_pair,
@@ -315,8 +317,8 @@ int oracle_bwd_w(int32_t T, int32_t k, int32_t E, int32_t G, const int32_t* topk
     int32_t i = (int32_t)(sel ? sel[ii] : ii);
     int32_t g = 0;
     while (!(rank_off[g] <= i && i < rank_off[g + 1])) ++g;
-    double* da = dA + (int64_t)i * d_in;
-    double* db = dBt + (int64_t)i * d_out;
+    double* da = dA + (sel ? ii : (int64_t)i) * d_in;
+    double* db = dBt + (sel ? ii : (int64_t)i) * d_out;
     for (int32_t c = 0; c < d_in; ++c) da[c] = 0.0;
     for (int32_t o = 0; o < d_out; ++o) db[o] = 0.0;
     const uint16_t* a = A_all + (int64_t)i * d_in;

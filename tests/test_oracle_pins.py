@@ -201,11 +201,15 @@ def test_selection_matches_full():
     full, Hf = oracle.fwd(L["idx"], L["e2g"], L["rank_off"], L["X"], L["Ag"], L["Btg"], 2.0, want_h=True)
     sel = np.array([5, 0, 17], np.int32)
     part, Hp = oracle.fwd(L["idx"], L["e2g"], L["rank_off"], L["X"], L["Ag"], L["Btg"], 2.0, sel=sel, want_h=True)
-    assert np.array_equal(part[sel], full[sel]) and np.all(np.isnan(np.delete(part, sel, axis=0)))
+    assert np.array_equal(part, full[sel]) and np.array_equal(Hp, Hf[sel])
+    dx = oracle.bwd_dx(L["idx"], L["e2g"], L["rank_off"], L["dYg"], L["Ag"], L["Btg"], 2.0)
+    sdx = oracle.bwd_dx(L["idx"], L["e2g"], L["rank_off"], L["dYg"], L["Ag"], L["Btg"], 2.0,
+                        sel=np.array([3, 1], np.int32))
+    assert np.array_equal(sdx, dx[[3, 1]])
     dA, dBt = oracle.bwd_w(L["idx"], L["e2g"], L["rank_off"], L["X"], L["dYg"], L["Ag"], L["Btg"], 2.0)
     sA, sB = oracle.bwd_w(L["idx"], L["e2g"], L["rank_off"], L["X"], L["dYg"], L["Ag"], L["Btg"], 2.0,
                           sel=np.array([4, 1], np.int32))
-    assert np.array_equal(sA[[4, 1]], dA[[4, 1]]) and np.array_equal(sB[[4, 1]], dBt[[4, 1]])
+    assert np.array_equal(sA, dA[[4, 1]]) and np.array_equal(sB, dBt[[4, 1]])
 
 
 # ---------------------------------------------------------------- backward

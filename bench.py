@@ -1,0 +1,469 @@
+"""Benchmark of the grouped adapter execution hot path (one MoE layer).
+
+One step = route-permute + fused gate/up forward (shared input, dedup) +
+down forward (per row) + down backward + gate/up backward (incl. dX), i.e. the
+forward and backward passes of the group-shared LoRA deltas on all three
+expert projections of one layer.  Metric: routed rows (T*k) per second.
+
+Default workload: the OLMoE-shaped layer (T=8192, d=2048, ff=1024, E=64,
+top-8, Zipf(1.0) routing, 16 groups of 4, rank 8 -> 32, s=2), synthetic
+seeded inputs.  Inputs are resident in HBM for ``value``; ``e2e`` also moves
+the step's inputs from pinned host memory and reads the weight gradients back.
+
+    python bench.py [--gpus N --steps K --warmup W] [--impl reference]
+                    [--config olmoe] [--expertwise] [--det] [--no-cpu]
+Multi-GPU (torchrun, one rank per GPU): independent replicas, weak scaling.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import glob
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "grouped-LoRA fwd+bwd routed rows/s per MoE layer"
+UNIT = "rows/s"
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return {"hbm_gbs": float(d["hbm_gbs"]), "bf16_tflops": float(d["bf16_tflops"]),
+                "bf16_tflops_sustained": float(d.get("bf16_tflops_sustained", d["bf16_tflops"])),
+                "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "source": "fallback"}
+
+
+def csrc_sha():
+    h = hashlib.sha256()
+    for p in sorted(glob.glob(os.path.join(ROOT, "paper_2609_06072_gb300", "csrc", "*"))):
+        h.update(open(p, "rb").read())
+    return h.hexdigest()[:16]
+
+
+# ------------------------------------------------------------------ byte model
+def model(T, k, d, f, rank_off, U_g, R_g, nproj_shared=2):
+    """Algorithmic bytes / flops per call (each distinct tensor counted once)."""
+    r_g = np.diff(np.asarray(rank_off, np.int64))
+    Pw = int(r_g.sum()) * (d + f)
+    R = T * k
+    U = int(np.sum(U_g))
+    sUr = int(np.sum(np.asarray(U_g) * r_g))
+    sRr = int(np.sum(np.asarray(R_g) * r_g))
+    npj = nproj_shared
+    b = {
+        "permute": 4 * R + 16 * R + 4 * U,
+        "fwd_shared": 2 * T * d + npj * 4 * R * f + npj * 4 * sUr + npj * 2 * Pw,
+        "fwd_row": 2 * R * f + 4 * R * d + 4 * sRr + 2 * Pw,
+        "bwd_row": 2 * R * d + 2 * R * f + 4 * sRr + 4 * R * f + 6 * Pw,
+        "bwd_shared": npj * 2 * R * f + 2 * T * d + npj * 4 * sUr + 4 * T * d + npj * 6 * Pw,
+    }
+    fl = {
+        "permute": 0,
+        "fwd_shared": npj * 2 * sUr * (d + f),
+        "fwd_row": 2 * sRr * (d + f),
+        "bwd_row": 4 * sRr * (d + f),
+        "bwd_shared": npj * 4 * sUr * (d + f),
+    }
+    return b, fl
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{index}.csv") if os.path.isdir(
+            os.path.join(ROOT, "gpurun_out")) else f"/tmp/ace_clocks_{os.getpid()}.csv"
+
+    def start(self):
+        q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+        try:
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"], stdout=self.fh,
+                                         stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.fh.close()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------------ GPU arm
+class Layer:
+    """Device-resident tensors of one layer plus the plan and workspaces."""
+
+    def __init__(self, cfg_name, seed, expertwise, det, T=None):
+        import torch
+        from paper_2609_06072_gb300 import ace, workloads as W
+        over = {"T": T} if T else {}
+        self.L = W.Layer(W.get_config(cfg_name, **over), seed=seed, expertwise=expertwise)
+        c = self.L.cfg
+        self.c = c
+        self.plan = ace.Plan(c.T, c.k, c.E, self.L.G, self.L.e2g, self.L.rank_off, c.d, c.f, deterministic=det)
+        self.det = det
+        dev = "cuda"
+        self.pws, _, self.bws = self.plan.alloc_workspaces(c.T)
+        gen = torch.Generator().manual_seed(1000 + seed)
+
+        def randn(*shape, std=1.0):
+            return (torch.randn(*shape, generator=gen) * std).to(torch.bfloat16)
+
+        def unif(*shape, bound):
+            return ((torch.rand(*shape, generator=gen) * 2 - 1) * bound).to(torch.bfloat16)
+
+        R, d, f, nr = c.R, c.d, c.f, self.plan.n_rank
+        # host (pinned) inputs of a step: routing, activations, upstream gradients
+        self.h_topk = torch.from_numpy(self.L.topk_idx).pin_memory()
+        self.h_X = randn(c.T, d).pin_memory()
+        self.h_hin = randn(R, f).pin_memory()
+        self.h_dY = [randn(R, f).pin_memory(), randn(R, f).pin_memory(), randn(R, d).pin_memory()]
+        self.topk = self.h_topk.to(dev)
+        self.X = self.h_X.to(dev)
+        self.hin = self.h_hin.to(dev)
+        self.dY = [t.to(dev) for t in self.h_dY]
+        # adapters (rank-major A_g, B_g^T), three projections
+        self.A = [unif(nr, d, bound=d ** -0.5).to(dev), unif(nr, d, bound=d ** -0.5).to(dev),
+                  unif(nr, f, bound=f ** -0.5).to(dev)]
+        self.Bt = [randn(nr, f, std=0.02).to(dev), randn(nr, f, std=0.02).to(dev), randn(nr, d, std=0.02).to(dev)]
+        # base-path outputs / input gradients that the deltas accumulate onto
+        self.Y = [randn(R, f).to(dev), randn(R, f).to(dev), randn(R, d).to(dev)]
+        self.dX = randn(c.T, d).to(dev)
+        self.dh = randn(R, f).to(dev)
+        self.H = [torch.empty(R, self.plan.rank_max, device=dev) for _ in range(3)]
+        self.dA = [torch.empty(nr, d, device=dev), torch.empty(nr, d, device=dev), torch.empty(nr, f, device=dev)]
+        self.dBt = [torch.empty(nr, f, device=dev), torch.empty(nr, f, device=dev), torch.empty(nr, d, device=dev)]
+        self.h_grads = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in self.dA + self.dBt]
+        self.perm = None
+
+    def kernels_per_step(self):
+        # permute 3 + fwd_shared 1 + fwd_row 1 + bwd_row 1 + bwd_shared 1 + dX 1 (+ 2 reduces per projection)
+        return 8 + (6 if self.det else 0)
+
+    def step(self, ev=None):
+        """One pass of the hot path.  ev: list of 6 CUDA events (call boundaries)."""
+        c, p = self.c, self.plan
+        if ev:
+            ev[0].record()
+        self.perm = p.permute(self.topk, self.pws)
+        if ev:
+            ev[1].record()
+        p.fwd_shared(self.perm, self.X, self.A[:2], self.Bt[:2], c.s, self.Y[:2], self.H[:2])
+        if ev:
+            ev[2].record()
+        p.fwd_row(self.perm, self.hin, self.A[2], self.Bt[2], c.s, self.Y[2], self.H[2])
+        if ev:
+            ev[3].record()
+        p.bwd_row(self.perm, self.dY[2], self.hin, self.H[2], self.A[2], self.Bt[2], c.s, self.dh, self.dA[2],
+                  self.dBt[2], self.bws)
+        if ev:
+            ev[4].record()
+        p.bwd_shared(self.perm, self.dY[:2], self.X, self.H[:2], self.A[:2], self.Bt[:2], c.s, self.dX,
+                     self.dA[:2], self.dBt[:2], self.bws)
+        if ev:
+            ev[5].record()
+
+    def h2d_inputs(self):
+        self.topk.copy_(self.h_topk, non_blocking=True)
+        self.X.copy_(self.h_X, non_blocking=True)
+        self.hin.copy_(self.h_hin, non_blocking=True)
+        for dst, src in zip(self.dY, self.h_dY):
+            dst.copy_(src, non_blocking=True)
+
+    def d2h_result(self):
+        for dst, src in zip(self.h_grads, self.dA + self.dBt):
+            dst.copy_(src, non_blocking=True)
+
+    def h2d_bytes(self):
+        return sum(t.numel() * t.element_size() for t in [self.h_topk, self.h_X, self.h_hin] + self.h_dY)
+
+    def d2h_bytes(self):
+        return sum(t.numel() * t.element_size() for t in self.h_grads)
+
+
+CALLS = ["permute", "fwd_shared", "fwd_row", "bwd_row", "bwd_shared"]
+
+
+def run_gpu(args, rank, world, local):
+    import torch
+    torch.cuda.set_device(local)
+    from paper_2609_06072_gb300 import ace
+    ace.load()
+    lay = Layer(args.config, args.seed, args.expertwise, args.det)
+    c = lay.c
+    flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device="cuda")  # > L2 (~126 MB)
+    for _ in range(args.warmup):
+        lay.step()
+    torch.cuda.synchronize()
+    assert lay.plan.get_error(lay.perm) == 0
+    P = ace.perm_arrays(lay.plan, lay.perm)
+    U_g = np.diff(P["uniq_off"])
+    R_g = np.diff(P["group_off"])
+    bytes_, flops = model(c.T, c.k, c.d, c.f, lay.L.rank_off, U_g, R_g)
+
+    # ---- device-resident timed region
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(args.steps)]
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    clk = ClockSampler(local)
+    clk.start()
+    t_wall0 = time.perf_counter()
+    for i in range(args.steps):
+        flush.zero_()  # L2 flush between timed steps (outside the event pair)
+        lay.step(evs[i])
+    torch.cuda.synchronize()
+    t_wall = time.perf_counter() - t_wall0
+    clocks = clk.stop()
+    per_call = {n: [] for n in CALLS}
+    step_ms = []
+    for e in evs:
+        for j, n in enumerate(CALLS):
+            per_call[n].append(e[j].elapsed_time(e[j + 1]))
+        step_ms.append(e[0].elapsed_time(e[5]))
+    ms = float(np.sum(step_ms))
+    if world > 1:
+        t = torch.tensor([ms], device="cuda")
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms = float(t.item())
+        torch.distributed.barrier()
+    ms_per_step = ms / args.steps
+    value = world * c.R / (ms_per_step * 1e-3)
+
+    # ---- end to end through host buffers (same calls, pinned H2D in, grads D2H out)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    for _ in range(2):
+        lay.h2d_inputs()
+        lay.step()
+        lay.d2h_result()
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    e0.record()
+    for _ in range(args.steps):
+        lay.h2d_inputs()
+        lay.step()
+        lay.d2h_result()
+    e1.record()
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1)
+    if world > 1:
+        t = torch.tensor([e2e_ms], device="cuda")
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+    e2e_value = world * c.R * args.steps / (e2e_ms * 1e-3)
+
+    peaks = load_peaks()
+    call_ms = {n: float(np.mean(v)) for n, v in per_call.items()}
+    dom = max(CALLS, key=lambda n: call_ms[n])
+    achieved = bytes_[dom] / (call_ms[dom] * 1e-3) / 1e9
+    traffic = None
+    tf = os.path.join(ROOT, "profiles", "traffic.json")
+    if os.path.exists(tf):
+        tj = json.load(open(tf))
+        ent = tj.get(f"{args.config}{'_ew' if args.expertwise else ''}{'_det' if args.det else ''}", {}).get(dom)
+        if ent and tj.get("csrc_sha") == csrc_sha():
+            traffic = ent
+    total_bytes = sum(bytes_.values())
+    total_flops = sum(flops.values())
+    out = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": f"{args.config}-shaped MoE layer"
+                               f"{' (expert-wise, matched budget)' if args.expertwise else ' (grouped)'}",
+                   "T": c.T, "d": c.d, "f": c.f, "E": c.E, "k": c.k, "G": lay.L.G, "r": c.r,
+                   "rank_g": int(np.max(np.diff(lay.L.rank_off))), "s": c.s, "routing": f"{c.routing}({c.alpha})",
+                   "rows_per_step": c.R, "U": int(P["U"]), "deterministic": bool(args.det),
+                   "l2": "flushed between timed steps (256 MB write outside the event pair)",
+                   "parallelism": f"replicas x{world}"},
+        "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peaks["hbm_gbs"],
+                     "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"], "traffic": traffic,
+                     "algorithmic_bytes": bytes_[dom], "peak_source": peaks["source"]},
+        "step_roofline": {"algorithmic_bytes": total_bytes, "algorithmic_flops": total_flops,
+                          "achieved_GBps": total_bytes / (ms_per_step * 1e-3) / 1e9,
+                          "frac_hbm": total_bytes / (ms_per_step * 1e-3) / 1e9 / peaks["hbm_gbs"],
+                          "tensor_TFLOPs": total_flops / (ms_per_step * 1e-3) / 1e12},
+        "per_call_ms": call_ms,
+        "per_call_frac_hbm": {n: bytes_[n] / (call_ms[n] * 1e-3) / 1e9 / peaks["hbm_gbs"] for n in CALLS},
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": lay.h2d_bytes(),
+                "d2h_bytes_per_step": lay.d2h_bytes()},
+        "gpu_launches": lay.kernels_per_step() * args.steps,
+        "clocks": clocks,
+        "wall_s_timed": t_wall,
+    }
+    return out, lay
+
+
+# ------------------------------------------------------------------ CPU oracle
+def oracle_sample(cfg_name, seed, expertwise, frac, rng_seed=0):
+    """Time the fp64 oracle on a sample of one step: the full permutation, the
+    forward of a fraction `frac` of the pairs, input gradients of the same
+    fraction of tokens / pairs and weight gradients of that fraction of the
+    rank rows, for all three projections.  Returns (seconds, sampled rows)."""
+    import oracle
+    from paper_2609_06072_gb300 import workloads as W
+    L = W.Layer(W.get_config(cfg_name), seed=seed, expertwise=expertwise)
+    c = L.cfg
+    rng = np.random.default_rng(rng_seed)
+    n_p = max(1, int(round(frac * c.R)))
+    n_t = max(1, int(round(frac * c.T)))
+    n_r = max(1, int(round(frac * int(L.rank_off[-1]))))
+    sel_p = np.sort(rng.choice(c.R, n_p, replace=False)).astype(np.int32)
+    sel_t = np.sort(rng.choice(c.T, n_t, replace=False)).astype(np.int32)
+    sel_r = np.sort(rng.choice(int(L.rank_off[-1]), n_r, replace=False)).astype(np.int32)
+    ins = {"X": L.X(), "h": L.h(), "dY": {p: L.dY(p) for p in ("gate", "up", "down")},
+           "A": {p: L.A(p) for p in ("gate", "up", "down")}, "Bt": {p: L.Bt(p) for p in ("gate", "up", "down")}}
+    t0 = time.perf_counter()
+    oracle.permute(L.topk_idx, L.e2g, L.G)
+    for p in ("gate", "up"):
+        oracle.fwd(L.topk_idx, L.e2g, L.rank_off, ins["X"], ins["A"][p], ins["Bt"][p], c.s, sel=sel_p)
+        oracle.bwd_dx(L.topk_idx, L.e2g, L.rank_off, ins["dY"][p], ins["A"][p], ins["Bt"][p], c.s, sel=sel_t)
+        oracle.bwd_w(L.topk_idx, L.e2g, L.rank_off, ins["X"], ins["dY"][p], ins["A"][p], ins["Bt"][p], c.s,
+                     sel=sel_r)
+    p = "down"
+    oracle.fwd(L.topk_idx, L.e2g, L.rank_off, ins["h"], ins["A"][p], ins["Bt"][p], c.s, x_per_pair=True, sel=sel_p)
+    oracle.bwd_dx(L.topk_idx, L.e2g, L.rank_off, ins["dY"][p], ins["A"][p], ins["Bt"][p], c.s, x_per_pair=True,
+                  sel=sel_p)
+    oracle.bwd_w(L.topk_idx, L.e2g, L.rank_off, ins["h"], ins["dY"][p], ins["A"][p], ins["Bt"][p], c.s,
+                 x_per_pair=True, sel=sel_r)
+    dt = time.perf_counter() - t0
+    return dt, frac * c.R
+
+
+def cpu_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def cpu_baseline(cfg_name, seed, expertwise, target_s):
+    """Calibrate a sample fraction to ~target_s seconds of oracle work, then time it."""
+    os.environ.setdefault("OMP_NUM_THREADS", str(cpu_cores()))
+    frac = 1.0 / 512
+    dt, _ = oracle_sample(cfg_name, seed, expertwise, frac)
+    frac = min(1.0, frac * target_s / max(dt, 1e-3))
+    dt, rows = oracle_sample(cfg_name, seed, expertwise, frac)
+    return {"value": rows / dt, "unit": UNIT, "cores": int(os.environ["OMP_NUM_THREADS"]), "kind": "oracle",
+            "sample": f"one step's permutation plus {frac:.4f} of its pairs (forward, dX/dh) and of its rank "
+                      f"rows (dA, dB^T), all 3 projections; {dt:.1f} s", "seconds": dt}
+
+
+def run_reference(args, rank, world):
+    if rank != 0:
+        return None
+    from paper_2609_06072_gb300 import workloads as W
+    os.environ.setdefault("OMP_NUM_THREADS", str(cpu_cores()))
+    c = W.get_config(args.config)
+    # per step: a bounded sample sized so that warmup + steps end within minutes
+    per_step_s = max(2.0, min(20.0, 120.0 / max(1, args.steps + args.warmup)))
+    frac = 1.0 / 512
+    dt, _ = oracle_sample(args.config, args.seed, args.expertwise, frac)
+    frac = min(1.0, frac * per_step_s / max(dt, 1e-3))
+    for _ in range(args.warmup):
+        oracle_sample(args.config, args.seed, args.expertwise, frac)
+    times, rows = [], 0.0
+    for i in range(args.steps):
+        dt, r = oracle_sample(args.config, args.seed, args.expertwise, frac, rng_seed=i + 1)
+        times.append(dt)
+        rows += r
+    total = float(np.sum(times))
+    value = rows / total
+    cores = int(os.environ["OMP_NUM_THREADS"])
+    return {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": 1e3 * c.R / value, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": f"{args.config}-shaped MoE layer{' (expert-wise)' if args.expertwise else ' (grouped)'}",
+                   "T": c.T, "d": c.d, "f": c.f, "E": c.E, "k": c.k},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": f"per step: permutation plus {frac:.4f} of the pairs and rank rows of one step"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ace", choices=["ace", "reference"])
+    ap.add_argument("--config", default="olmoe")
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--expertwise", action="store_true", help="matched-budget expert-wise layout (G=E, rank r)")
+    ap.add_argument("--det", action="store_true", help="deterministic two-stage split-K for dA / dB^T")
+    ap.add_argument("--no-cpu", action="store_true", help="skip the CPU-oracle baseline leg")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    rank, world, local = dist_env()
+    if args.impl == "reference":
+        out = run_reference(args, rank, world)
+        if out is not None:
+            print(json.dumps(out))
+        return
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    out, _ = run_gpu(args, rank, world, local)
+    if rank == 0:
+        if world == 1 and not args.no_cpu:
+            out["cpu_baseline"] = cpu_baseline(args.config, args.seed, args.expertwise, args.cpu_seconds)
+        print(json.dumps(out))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

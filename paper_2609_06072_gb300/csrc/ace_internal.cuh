@@ -35,7 +35,8 @@ struct Tile {
 
 // Byte layout of the permutation workspace for T tokens.
 struct PermLayout {
-  size_t err, counts, group_off, expert_off, expert_cnt, uniq_off, row_pair, pair_row, pair_g, uniq_tok, tok_uniq;
+  size_t err, counts, group_off, expert_off, expert_cnt, uniq_off, row_pair, pair_row, pair_g, row_uniq, uniq_tok,
+      tok_uniq;
   size_t chunk_cntE, chunk_cntU, chunk_baseE, chunk_baseU, chunk_err;
   size_t tiles_sh, tiles_row, splits_sh, splits_row;
   size_t total;
@@ -69,6 +70,7 @@ inline PermLayout perm_layout(const PlanTables& pt, int32_t T) {
   L.row_pair = take(4 * (size_t)R);
   L.pair_row = take(4 * (size_t)R);
   L.pair_g = take(4 * (size_t)R);
+  L.row_uniq = take(4 * (size_t)R);
   L.uniq_tok = take(4 * (size_t)R);
   L.tok_uniq = take(4 * (size_t)R);
   L.chunk_cntE = take(4 * (size_t)L.n_chunks * pt.E);
@@ -118,24 +120,25 @@ struct FwdLaunch {
 cudaError_t launch_fwd(const PlanTables& pt, const FwdLaunch& a, bool shared, cudaStream_t st);
 
 struct BwdLaunch {
-  const Tile* splits;
+  const Tile* splits;      // splits of this path (gate/up: unique pairs, used by dA; down: rows)
+  const Tile* splits_row;  // row splits (the dY streaming phase of both paths)
+  const Tile* tiles_sh;    // unique-pair tiles (dH per unique pair)
   const int32_t* counts;
-  int32_t count_slot;
-  int32_t max_splits;
+  int32_t count_slot;      // counts[] slot of `splits`
+  int32_t max_splits, max_splits_row, max_tiles_sh;
   const int32_t* uniq_tok;
-  const int32_t* tok_uniq;
   const int32_t* pair_row;
   const int32_t* pair_g;
-  const int32_t* uniq_off;
-  const int32_t* group_off;
+  const int32_t* row_uniq;
   const uint16_t* dY[2];
-  const uint16_t* Xin;   // shared: X [T, d]; row: Hin [R, f]
-  const float* H[2];
+  const uint16_t* Xin;   // gate/up: X [T, d]; down: Hin [R, f]
+  const float* H[2];     // saved H (gate/up: per unique pair; down: per row), stride rank_max
   const uint16_t* A[2];
   const uint16_t* Bt[2];
   float s;
-  uint16_t* dXin;        // row path: dHin [R, f] in/out
-  uint16_t* dH[2];       // scratch: bf16 [R, rank_pad] (shared path: per unique pair)
+  uint16_t* dXin;        // down: dHin [R, f] in/out
+  uint16_t* dH[2];       // scratch: bf16 dH per unique pair [R, rank_pad]
+  float* dHrow[2];       // scratch: fp32 dH per row [R, rank_pad]
   float* dA[2];
   float* dBt[2];
   float* part_dA[2];     // deterministic partials [max_splits, rank_pad, d_in]

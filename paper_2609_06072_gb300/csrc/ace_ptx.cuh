@@ -30,13 +30,26 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// Bounded wait on an mbarrier phase.  Returns false (and the caller raises its
-// error flag) if the phase did not complete within `limit` polls; every
-// try_wait already suspends the thread for a hardware-defined interval, so
-// the limit bounds the wall time to well under a second.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint32_t limit = (1u << 22)) {
-  for (uint32_t i = 0; i < limit; ++i)
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// Wall-clock bound of every device-side wait (a legitimate wait lasts
+// microseconds).
+constexpr uint64_t kWaitLimitNs = 1000000000ull;
+
+// Bounded wait on an mbarrier phase.  Returns false (the caller raises its
+// error flag and winds down) if the phase has not completed within
+// kWaitLimitNs of wall time; the iteration cap is a second bound.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t i = 0; i < (1u << 24); ++i) {
     if (mbar_try_wait(bar, parity)) return true;
+    if ((i & 7) == 7 && globaltimer_ns() - t0 > kWaitLimitNs) return false;
+  }
   return false;
 }
 

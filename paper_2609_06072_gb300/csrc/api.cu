@@ -36,8 +36,8 @@ ace_status cuda_status(cudaError_t e, const char* what) {
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-// Backward TMEM budget: (tiles per split + 2) * rank_pad columns <= 256.
-int nt_split_for(int rank_pad) { return rank_pad <= 16 ? 8 : rank_pad == 32 ? 4 : rank_pad == 64 ? 2 : 1; }
+// Row tiles per backward split: (tiles + 2) * rank_pad TMEM columns <= 256.
+int nt_split_for(int rank_pad) { return rank_pad <= 32 ? 4 : rank_pad == 64 ? 2 : 1; }
 
 ace_status check_perm(const ace_plan* plan, const ace_perm* perm) {
   if (!plan || !perm || !perm->ws) return fail(ACE_ERR_ARG, "null plan or perm");
@@ -48,29 +48,32 @@ ace_status check_perm(const ace_plan* plan, const ace_perm* perm) {
 
 struct BwdWs {
   uint16_t* dH[2];
+  float* dHrow[2];
   float* part_dA[2];
   float* part_dBt[2];
   size_t total;
 };
 
+// Backward scratch: dH per unique pair (bf16), dH per row (fp32) and the
+// deterministic split-K partials, each per projection.
 BwdWs bwd_layout(const PlanTables& pt, int32_t T, void* base) {
   const PermLayout L = perm_layout(pt, T);
   const int64_t R = (int64_t)T * pt.k;
   const size_t dh = align_up(2 * (size_t)R * pt.rank_pad, 256);
-  const size_t part = align_up(4 * (size_t)L.max_splits * pt.rank_pad * (size_t)(pt.d + pt.f), 256);
+  const size_t dhrow = align_up(4 * (size_t)R * pt.rank_pad, 256);
+  const size_t pa = align_up(4 * (size_t)L.max_splits * pt.rank_pad * (size_t)(pt.d > pt.f ? pt.d : pt.f), 256);
   BwdWs w{};
   char* b = static_cast<char*>(base);
   size_t off = 0;
   for (int j = 0; j < 2; ++j) {
     w.dH[j] = reinterpret_cast<uint16_t*>(b + off);
     off += dh;
-  }
-  for (int j = 0; j < 2; ++j) {
+    w.dHrow[j] = reinterpret_cast<float*>(b + off);
+    off += dhrow;
     w.part_dA[j] = reinterpret_cast<float*>(b + off);
-    // dA partial [max_splits, rank_pad, d_in] followed by dBt partial
-    // [max_splits, rank_pad, d_out]; d_in + d_out = d + f for every projection
-    w.part_dBt[j] = nullptr;
-    off += part;
+    off += pa;
+    w.part_dBt[j] = reinterpret_cast<float*>(b + off);
+    off += pa;
   }
   w.total = off;
   return w;
@@ -265,15 +268,17 @@ ace_status ace_bwd_shared(const ace_plan* plan, const ace_perm* perm, int32_t np
   cudaStream_t cs = static_cast<cudaStream_t>(stream);
   BwdLaunch a{};
   a.splits = at<Tile>(perm->ws, L.splits_sh);
+  a.splits_row = at<Tile>(perm->ws, L.splits_row);
+  a.tiles_sh = at<Tile>(perm->ws, L.tiles_sh);
   a.counts = perm->counts;
   a.count_slot = kCntSplitsSh;
   a.max_splits = L.max_splits;
+  a.max_splits_row = L.max_splits;
+  a.max_tiles_sh = L.max_tiles;
   a.uniq_tok = perm->uniq_tok;
-  a.tok_uniq = perm->tok_uniq;
   a.pair_row = perm->pair_row;
   a.pair_g = at<int32_t>(perm->ws, L.pair_g);
-  a.uniq_off = perm->uniq_off;
-  a.group_off = perm->group_off;
+  a.row_uniq = at<int32_t>(perm->ws, L.row_uniq);
   a.Xin = X;
   for (int j = 0; j < 2; ++j) {
     const int jj = j < nproj ? j : 0;
@@ -284,8 +289,9 @@ ace_status ace_bwd_shared(const ace_plan* plan, const ace_perm* perm, int32_t np
     a.dA[j] = dA[jj];
     a.dBt[j] = dBt[jj];
     a.dH[j] = w.dH[jj];
+    a.dHrow[j] = w.dHrow[jj];
     a.part_dA[j] = w.part_dA[jj];
-    a.part_dBt[j] = w.part_dA[jj] + (size_t)L.max_splits * plan->pt.rank_pad * plan->pt.d;
+    a.part_dBt[j] = w.part_dBt[jj];
   }
   a.s = s;
   a.dXin = nullptr;
@@ -330,15 +336,17 @@ ace_status ace_bwd_row(const ace_plan* plan, const ace_perm* perm, const uint16_
   const BwdWs w = bwd_layout(plan->pt, perm->T, ws);
   BwdLaunch a{};
   a.splits = at<Tile>(perm->ws, L.splits_row);
+  a.splits_row = a.splits;
+  a.tiles_sh = at<Tile>(perm->ws, L.tiles_sh);
   a.counts = perm->counts;
   a.count_slot = kCntSplitsRow;
   a.max_splits = L.max_splits;
+  a.max_splits_row = L.max_splits;
+  a.max_tiles_sh = L.max_tiles;
   a.uniq_tok = perm->uniq_tok;
-  a.tok_uniq = perm->tok_uniq;
   a.pair_row = perm->pair_row;
   a.pair_g = at<int32_t>(perm->ws, L.pair_g);
-  a.uniq_off = perm->uniq_off;
-  a.group_off = perm->group_off;
+  a.row_uniq = at<int32_t>(perm->ws, L.row_uniq);
   a.Xin = Hin;
   for (int j = 0; j < 2; ++j) {
     a.dY[j] = dY;
@@ -348,8 +356,9 @@ ace_status ace_bwd_row(const ace_plan* plan, const ace_perm* perm, const uint16_
     a.dA[j] = dA;
     a.dBt[j] = dBt;
     a.dH[j] = w.dH[0];
+    a.dHrow[j] = w.dHrow[0];
     a.part_dA[j] = w.part_dA[0];
-    a.part_dBt[j] = w.part_dA[0] + (size_t)L.max_splits * plan->pt.rank_pad * plan->pt.f;
+    a.part_dBt[j] = w.part_dBt[0];
   }
   a.s = s;
   a.dXin = dHin;

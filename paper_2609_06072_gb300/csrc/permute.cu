@@ -199,6 +199,7 @@ __global__ void __launch_bounds__(kPermTB) k_perm_scatter(const __grid_constant_
                                                           int32_t* __restrict__ row_pair,
                                                           int32_t* __restrict__ pair_row,
                                                           int32_t* __restrict__ pair_g,
+                                                          int32_t* __restrict__ row_uniq,
                                                           int32_t* __restrict__ uniq_tok,
                                                           int32_t* __restrict__ tok_uniq) {
   constexpr int W = kPermTB / 32;
@@ -232,9 +233,11 @@ __global__ void __launch_bounds__(kPermTB) k_perm_scatter(const __grid_constant_
     }
     return;
   }
+  int rows_j[kMaxK];
   for (int j = 0; j < k; ++j) {
     const int row = chunk_baseE[(int64_t)c * pt.E + e[j]] + prefix_bits(&mE[e[j] * W], tid);
     const int p = t * k + j;
+    rows_j[j] = row;
     pair_row[p] = row;
     pair_g[p] = pt.e2g[e[j]];
     row_pair[row] = p;
@@ -252,6 +255,8 @@ __global__ void __launch_bounds__(kPermTB) k_perm_scatter(const __grid_constant_
     const int u = chunk_baseU[(int64_t)c * pt.G + nxt] + prefix_bits(&mU[nxt * W], tid);
     uniq_tok[u] = t;
     tok_uniq[(int64_t)t * k + n_u] = u;
+    for (int j = 0; j < k; ++j)
+      if (pt.e2g[e[j]] == nxt) row_uniq[rows_j[j]] = u;
     ++n_u;
     last = nxt;
   }
@@ -293,7 +298,7 @@ cudaError_t launch_permute(const PlanTables& pt, const int32_t* topk_idx, int32_
     k_perm_scatter<<<C, kPermTB, sm3, st>>>(pt, topk_idx, T, at<int32_t>(ws, L.chunk_baseE),
                                             at<int32_t>(ws, L.chunk_baseU), at<int32_t>(ws, L.row_pair),
                                             at<int32_t>(ws, L.pair_row), at<int32_t>(ws, L.pair_g),
-                                            at<int32_t>(ws, L.uniq_tok),
+                                            at<int32_t>(ws, L.row_uniq), at<int32_t>(ws, L.uniq_tok),
                                             at<int32_t>(ws, L.tok_uniq));
   }
   return cudaGetLastError();

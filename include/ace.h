@@ -122,7 +122,7 @@ int32_t ace_plan_rank_max(const ace_plan* plan);
 
 /* Workspace bytes for T tokens:
  *   perm_bytes  -- ace_permute (lives as long as the ace_perm views are used)
- *   fwd_bytes   -- ace_fwd_shared / ace_fwd_row scratch (may be 0)
+ *   fwd_bytes   -- ace_fwd_shared scratch, used only when its H argument is NULL
  *   bwd_bytes   -- ace_bwd_shared / ace_bwd_row scratch
  * A NULL output pointer is skipped. */
 ace_status ace_workspace_size(const ace_plan* plan, int32_t T, size_t* perm_bytes, size_t* fwd_bytes,
@@ -145,9 +145,10 @@ ace_status ace_permute(const ace_plan* plan, const int32_t* topk_idx, int32_t T,
  *   A[i]    [rank_off[G], d] bf16, rows rank_off[g].. hold A_g
  *   Bt[i]   [rank_off[G], f] bf16, rows rank_off[g].. hold B_g^T
  *   Y[i]    [R, f] bf16 IN/OUT in row order: Y[row] += s * B_g (A_g X[t])
- *   H[i]    [R, rank_max] fp32 OUT (may be NULL): H[u] = A_g X[t] for unique
- *           pair u (first U rows; columns >= r_g are zero)
- * c_g is computed once per unique (g, t) and added to every row of that pair. */
+ *   H[i]    [R, rank_max] fp32 OUT (NULL: kept in the forward workspace):
+ *           H[u] = A_g X[t] for unique pair u (first U rows; columns >= r_g zero)
+ * A_g x is computed once per unique (g, t) pair; the result B_g (A_g x) is
+ * added to every row of that pair. */
 ace_status ace_fwd_shared(const ace_plan* plan, const ace_perm* perm, const uint16_t* X, int32_t nproj,
                           const uint16_t* const* A, const uint16_t* const* Bt, float s, uint16_t* const* Y,
                           float* const* H, void* ws, size_t ws_bytes, void* stream);

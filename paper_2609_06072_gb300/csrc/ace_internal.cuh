@@ -2,6 +2,7 @@
 #pragma once
 #include <cstddef>
 #include <cstdint>
+#include <cuda.h>  // CUtensorMap (types only; the encoder is fetched at run time)
 #include <cuda_runtime.h>
 
 #include "../../include/ace.h"
@@ -98,26 +99,45 @@ cudaError_t launch_permute(const PlanTables& pt, const int32_t* topk_idx, int32_
 cudaError_t launch_rows_copy(const int32_t* row_pair, const uint16_t* src, uint16_t* dst, int64_t R, int32_t cols,
                              bool gather, cudaStream_t st);
 
-struct FwdLaunch {
-  const Tile* tiles;
+// H = A_g x per unique (g, t) pair of gate/up (deduplicated; X rows gathered).
+struct FwdHLaunch {
+  const Tile* tiles;  // unique-pair tiles
   const int32_t* counts;
-  int32_t count_slot;
   int32_t max_tiles;
   const int32_t* uniq_tok;
-  const int32_t* pair_g;  // group of each pair (-1: invalid token)
-  const int32_t* row_pair;
-  const int32_t* pair_row;
-  const int32_t* tok_uniq;
   const uint16_t* X;
   const uint16_t* A[2];
-  const uint16_t* Bt[2];
-  uint16_t* Y[2];
-  float* H[2];
-  float s;
-  int32_t d_in, d_out, nproj, T;
+  float* H[2];        // [R, rank_max] fp32, row u
+  int32_t d_in, nproj;
   int32_t* err;
 };
-cudaError_t launch_fwd(const PlanTables& pt, const FwdLaunch& a, bool shared, cudaStream_t st);
+cudaError_t launch_fwd_h(const PlanTables& pt, const FwdHLaunch& a, cudaStream_t st);
+
+// Row-tile forward: Y[row] += s * B_g H_row over contiguous rows of a group.
+// MODE down: H_row = A_g h_row computed here (K loop over h);  gate/up:
+// H_row = H_u gathered from the unique-pair H of launch_fwd_h.
+struct FwdRowsLaunch {
+  CUtensorMap tm_x;      // down: Hin [R, d_in], box 64 x 128
+  CUtensorMap tm_a;      // down: A [n_rank, d_in], box 64 x rank_pad
+  CUtensorMap tm_bt[2];  // Bt [n_rank, d_out], box 64 x rank_pad
+  CUtensorMap tm_y[2];   // Y [R, d_out], box 64 x 128
+  const Tile* tiles;     // row tiles
+  const int32_t* counts;
+  int32_t max_tiles;
+  const int32_t* row_uniq;
+  const float* Hu[2];    // gate/up: H per unique pair
+  uint16_t* Y[2];
+  float* Hsave;          // down: H per row out (may be null)
+  float s;
+  int32_t d_in, d_out, nproj;
+  int32_t* err;
+};
+cudaError_t launch_fwd_rows(const PlanTables& pt, const FwdRowsLaunch& a, bool shared, cudaStream_t st);
+
+// 2-D bf16 tensor map (row-major [rows, cols]) with a 64-column x box_rows box
+// and 128-byte swizzle.  Returns false when the encoder is unavailable or
+// rejects the layout.
+bool make_tmap_bf16(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows);
 
 struct BwdLaunch {
   const Tile* splits;      // splits of this path (gate/up: unique pairs, used by dA; down: rows)

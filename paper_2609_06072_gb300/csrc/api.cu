@@ -10,6 +10,38 @@
 
 using namespace ace;
 
+namespace {
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn tensor_map_encoder() {
+  static EncodeTiledFn fn = nullptr;
+  static bool tried = false;
+  if (!tried) {
+    tried = true;
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+}  // namespace
+
+bool ace::make_tmap_bf16(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows) {
+  EncodeTiledFn fn = tensor_map_encoder();
+  if (!fn || rows == 0 || cols == 0) return false;
+  cuuint64_t gdim[2] = {cols, rows};
+  cuuint64_t gstr[1] = {cols * 2};
+  cuuint32_t box[2] = {64, box_rows};
+  cuuint32_t es[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), gdim, gstr, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 struct ace_plan {
   PlanTables pt;
   int32_t T_max;
@@ -150,7 +182,7 @@ ace_status ace_workspace_size(const ace_plan* plan, int32_t T, size_t* perm_byte
   if (!plan) return fail(ACE_ERR_ARG, "null plan");
   if (T < 0 || T > plan->T_max) return fail(ACE_ERR_SHAPE, "T=%d outside [0, %d]", T, plan->T_max);
   if (perm_bytes) *perm_bytes = perm_layout(plan->pt, T).total;
-  if (fwd_bytes) *fwd_bytes = 0;
+  if (fwd_bytes) *fwd_bytes = 2 * align_up(4 * (size_t)T * plan->pt.k * plan->pt.rank_max, 256);
   if (bwd_bytes) *bwd_bytes = bwd_layout(plan->pt, T, nullptr).total;
   return ACE_OK;
 }
@@ -184,7 +216,7 @@ ace_status ace_permute(const ace_plan* plan, const int32_t* topk_idx, int32_t T,
 
 static ace_status fwd_common(const ace_plan* plan, const ace_perm* perm, const uint16_t* X, int nproj,
                              const uint16_t* const* A, const uint16_t* const* Bt, float s, uint16_t* const* Y,
-                             float* const* H, bool shared, void* stream) {
+                             float* const* H, bool shared, void* ws, size_t ws_bytes, void* stream) {
   ace_status st = check_perm(plan, perm);
   if (st != ACE_OK) return st;
   if (nproj < 1 || nproj > 2) return fail(ACE_ERR_ARG, "nproj=%d must be 1 or 2", nproj);
@@ -197,52 +229,85 @@ static ace_status fwd_common(const ace_plan* plan, const ace_perm* perm, const u
       return fail(ACE_ERR_ARG, "tensor of projection %d not 16-byte aligned", j);
   }
   if (perm->R == 0) return ACE_OK;
-  const PermLayout L = perm_layout(plan->pt, perm->T);
-  FwdLaunch a{};
-  a.tiles = at<Tile>(perm->ws, shared ? L.tiles_sh : L.tiles_row);
-  a.counts = perm->counts;
-  a.count_slot = shared ? kCntTilesSh : kCntTilesRow;
-  a.max_tiles = L.max_tiles;
-  a.uniq_tok = perm->uniq_tok;
-  a.pair_g = at<int32_t>(perm->ws, L.pair_g);
-  a.row_pair = perm->row_pair;
-  a.pair_row = perm->pair_row;
-  a.tok_uniq = perm->tok_uniq;
-  a.X = X;
+  const PlanTables& pt = plan->pt;
+  const PermLayout L = perm_layout(pt, perm->T);
+  const int64_t R = perm->R;
+  const int n_rank = pt.rank_off[pt.G];
+  const int d_in = shared ? pt.d : pt.f, d_out = shared ? pt.f : pt.d;
+  cudaStream_t cs = static_cast<cudaStream_t>(stream);
+  int32_t* err = at<int32_t>(perm->ws, L.err);
+  // H per unique pair (gate/up) lives in the caller's H buffers or, if absent,
+  // in the forward workspace
+  float* Hbuf[2] = {nullptr, nullptr};
+  for (int j = 0; j < nproj; ++j) Hbuf[j] = H ? H[j] : nullptr;
+  if (shared && (!Hbuf[0] || (nproj == 2 && !Hbuf[1]))) {
+    const size_t need = 2 * align_up(4 * (size_t)R * pt.rank_max, 256);
+    if (!ws || ws_bytes < need || !aligned16(ws))
+      return fail(ACE_ERR_WORKSPACE, "forward workspace %zu < %zu bytes (needed when H is NULL)", ws_bytes, need);
+    for (int j = 0; j < nproj; ++j)
+      if (!Hbuf[j]) Hbuf[j] = reinterpret_cast<float*>(static_cast<char*>(ws) + j * align_up(4 * (size_t)R * pt.rank_max, 256));
+  }
+  if (shared) {
+    FwdHLaunch h{};
+    h.tiles = at<Tile>(perm->ws, L.tiles_sh);
+    h.counts = perm->counts;
+    h.max_tiles = L.max_tiles;
+    h.uniq_tok = perm->uniq_tok;
+    h.X = X;
+    for (int j = 0; j < 2; ++j) {
+      const int jj = j < nproj ? j : 0;
+      h.A[j] = A[jj];
+      h.H[j] = Hbuf[jj];
+    }
+    h.d_in = d_in;
+    h.nproj = nproj;
+    h.err = err;
+    st = cuda_status(launch_fwd_h(pt, h, cs), "forward H launch");
+    if (st != ACE_OK) return st;
+  }
+  FwdRowsLaunch r{};
+  bool ok = true;
+  if (!shared) {
+    ok = ok && make_tmap_bf16(&r.tm_x, X, (uint64_t)R, (uint64_t)d_in, kTileM);
+    ok = ok && make_tmap_bf16(&r.tm_a, A[0], (uint64_t)n_rank, (uint64_t)d_in, pt.rank_pad);
+  }
+  for (int j = 0; j < nproj; ++j) {
+    ok = ok && make_tmap_bf16(&r.tm_bt[j], Bt[j], (uint64_t)n_rank, (uint64_t)d_out, pt.rank_pad);
+    ok = ok && make_tmap_bf16(&r.tm_y[j], Y[j], (uint64_t)R, (uint64_t)d_out, kTileM);
+  }
+  if (!ok) return fail(ACE_ERR_UNSUPPORTED, "tensor-map encoding failed for this layout");
+  r.tiles = at<Tile>(perm->ws, L.tiles_row);
+  r.counts = perm->counts;
+  r.max_tiles = L.max_tiles;
+  r.row_uniq = at<int32_t>(perm->ws, L.row_uniq);
   for (int j = 0; j < 2; ++j) {
     const int jj = j < nproj ? j : 0;
-    a.A[j] = A[jj];
-    a.Bt[j] = Bt[jj];
-    a.Y[j] = Y[jj];
-    a.H[j] = H ? H[jj] : nullptr;
+    r.Hu[j] = Hbuf[jj];
+    r.Y[j] = Y[jj];
   }
-  a.s = s;
-  a.d_in = shared ? plan->pt.d : plan->pt.f;
-  a.d_out = shared ? plan->pt.f : plan->pt.d;
-  a.nproj = nproj;
-  a.T = perm->T;
-  a.err = at<int32_t>(perm->ws, L.err);
-  return cuda_status(launch_fwd(plan->pt, a, shared, static_cast<cudaStream_t>(stream)), "forward launch");
+  r.Hsave = shared ? nullptr : (H ? H[0] : nullptr);
+  r.s = s;
+  r.d_in = d_in;
+  r.d_out = d_out;
+  r.nproj = nproj;
+  r.err = err;
+  return cuda_status(launch_fwd_rows(pt, r, shared, cs), "forward rows launch");
 }
 
 ace_status ace_fwd_shared(const ace_plan* plan, const ace_perm* perm, const uint16_t* X, int32_t nproj,
                           const uint16_t* const* A, const uint16_t* const* Bt, float s, uint16_t* const* Y,
                           float* const* H, void* ws, size_t ws_bytes, void* stream) {
-  (void)ws;
-  (void)ws_bytes;
   if (!plan || !perm) return fail(ACE_ERR_ARG, "null plan or perm");
-  return fwd_common(plan, perm, X, nproj, A, Bt, s, Y, H, true, stream);
+  return fwd_common(plan, perm, X, nproj, A, Bt, s, Y, H, true, ws, ws_bytes, stream);
 }
 
 ace_status ace_fwd_row(const ace_plan* plan, const ace_perm* perm, const uint16_t* Hin, const uint16_t* A,
                        const uint16_t* Bt, float s, uint16_t* Y, float* H, void* ws, size_t ws_bytes, void* stream) {
-  (void)ws;
-  (void)ws_bytes;
   const uint16_t* Aa[1] = {A};
   const uint16_t* Ba[1] = {Bt};
   uint16_t* Ya[1] = {Y};
   float* Ha[1] = {H};
-  return fwd_common(plan, perm, Hin, 1, Aa, Ba, s, Ya, Ha, false, stream);
+  return fwd_common(plan, perm, Hin, 1, Aa, Ba, s, Ya, Ha, false, ws, ws_bytes, stream);
 }
 
 ace_status ace_bwd_shared(const ace_plan* plan, const ace_perm* perm, int32_t nproj, const uint16_t* const* dY,

@@ -140,29 +140,29 @@ cudaError_t launch_fwd_rows(const PlanTables& pt, const FwdRowsLaunch& a, bool s
 bool make_tmap_bf16(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows);
 
 struct BwdLaunch {
-  const Tile* splits;      // splits of this path (gate/up: unique pairs, used by dA; down: rows)
-  const Tile* splits_row;  // row splits (the dY streaming phase of both paths)
+  CUtensorMap tm_dy[2];    // dY [R, d_out], box 64 x 128
+  CUtensorMap tm_bt[2];    // Bt [n_rank, d_out], box 64 x rank_pad
+  CUtensorMap tm_a;        // down: A [n_rank, d_in], box 64 x rank_pad
+  CUtensorMap tm_dh;       // down: dHin [R, d_in], box 64 x 128
+  const Tile* splits_row;  // row splits (the dY streaming kernel)
   const Tile* tiles_sh;    // unique-pair tiles (dH per unique pair)
   const int32_t* counts;
-  int32_t count_slot;      // counts[] slot of `splits`
-  int32_t max_splits, max_splits_row, max_tiles_sh;
+  int32_t max_splits_row, max_tiles_sh;
   const int32_t* uniq_tok;
+  const int32_t* uniq_off;
+  const int32_t* group_off;
   const int32_t* pair_row;
   const int32_t* pair_g;
   const int32_t* row_uniq;
-  const uint16_t* dY[2];
   const uint16_t* Xin;   // gate/up: X [T, d]; down: Hin [R, f]
   const float* H[2];     // saved H (gate/up: per unique pair; down: per row), stride rank_max
-  const uint16_t* A[2];
-  const uint16_t* Bt[2];
   float s;
   uint16_t* dXin;        // down: dHin [R, f] in/out
-  uint16_t* dH[2];       // scratch: bf16 dH per unique pair [R, rank_pad]
-  float* dHrow[2];       // scratch: fp32 dH per row [R, rank_pad]
+  uint16_t* dH[2];       // scratch: bf16 dH [R, rank_pad] (gate/up: per unique pair; down: per row)
+  float* dHrow[2];       // scratch: fp32 dH per row [R, rank_pad] (gate/up)
   float* dA[2];
   float* dBt[2];
-  float* part_dA[2];     // deterministic partials [max_splits, rank_pad, d_in]
-  float* part_dBt[2];    // [max_splits, rank_pad, d_out]
+  float* part_dBt[2];    // deterministic dB^T partials [max_splits, rank_pad, d_out]
   int32_t d_in, d_out, nproj, T;
   bool deterministic;
   int32_t* err;

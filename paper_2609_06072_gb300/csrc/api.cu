@@ -81,13 +81,12 @@ ace_status check_perm(const ace_plan* plan, const ace_perm* perm) {
 struct BwdWs {
   uint16_t* dH[2];
   float* dHrow[2];
-  float* part_dA[2];
   float* part_dBt[2];
   size_t total;
 };
 
-// Backward scratch: dH per unique pair (bf16), dH per row (fp32) and the
-// deterministic split-K partials, each per projection.
+// Backward scratch per projection: dH per unique pair / row (bf16), dH per
+// row (fp32) and the deterministic dB^T split-K partials.
 BwdWs bwd_layout(const PlanTables& pt, int32_t T, void* base) {
   const PermLayout L = perm_layout(pt, T);
   const int64_t R = (int64_t)T * pt.k;
@@ -102,8 +101,6 @@ BwdWs bwd_layout(const PlanTables& pt, int32_t T, void* base) {
     off += dh;
     w.dHrow[j] = reinterpret_cast<float*>(b + off);
     off += dhrow;
-    w.part_dA[j] = reinterpret_cast<float*>(b + off);
-    off += pa;
     w.part_dBt[j] = reinterpret_cast<float*>(b + off);
     off += pa;
   }
@@ -332,32 +329,35 @@ ace_status ace_bwd_shared(const ace_plan* plan, const ace_perm* perm, int32_t np
   const BwdWs w = bwd_layout(plan->pt, perm->T, ws);
   cudaStream_t cs = static_cast<cudaStream_t>(stream);
   BwdLaunch a{};
-  a.splits = at<Tile>(perm->ws, L.splits_sh);
+  bool ok = true;
+  for (int j = 0; j < nproj; ++j) {
+    ok = ok && make_tmap_bf16(&a.tm_dy[j], dY[j], (uint64_t)perm->R, (uint64_t)plan->pt.f, kTileM);
+    ok = ok && make_tmap_bf16(&a.tm_bt[j], Bt[j], (uint64_t)plan->pt.rank_off[plan->pt.G], (uint64_t)plan->pt.f,
+                              plan->pt.rank_pad);
+  }
+  if (perm->R > 0 && !ok) return fail(ACE_ERR_UNSUPPORTED, "tensor-map encoding failed for this layout");
   a.splits_row = at<Tile>(perm->ws, L.splits_row);
   a.tiles_sh = at<Tile>(perm->ws, L.tiles_sh);
   a.counts = perm->counts;
-  a.count_slot = kCntSplitsSh;
-  a.max_splits = L.max_splits;
   a.max_splits_row = L.max_splits;
   a.max_tiles_sh = L.max_tiles;
   a.uniq_tok = perm->uniq_tok;
+  a.uniq_off = perm->uniq_off;
+  a.group_off = perm->group_off;
   a.pair_row = perm->pair_row;
   a.pair_g = at<int32_t>(perm->ws, L.pair_g);
   a.row_uniq = at<int32_t>(perm->ws, L.row_uniq);
   a.Xin = X;
   for (int j = 0; j < 2; ++j) {
     const int jj = j < nproj ? j : 0;
-    a.dY[j] = dY[jj];
     a.H[j] = H[jj];
-    a.A[j] = A[jj];
-    a.Bt[j] = Bt[jj];
     a.dA[j] = dA[jj];
     a.dBt[j] = dBt[jj];
     a.dH[j] = w.dH[jj];
     a.dHrow[j] = w.dHrow[jj];
-    a.part_dA[j] = w.part_dA[jj];
     a.part_dBt[j] = w.part_dBt[jj];
   }
+  if (nproj == 1) a.tm_dy[1] = a.tm_dy[0], a.tm_bt[1] = a.tm_bt[0];
   a.s = s;
   a.dXin = nullptr;
   a.d_in = plan->pt.d;
@@ -400,29 +400,33 @@ ace_status ace_bwd_row(const ace_plan* plan, const ace_perm* perm, const uint16_
   const PermLayout L = perm_layout(plan->pt, perm->T);
   const BwdWs w = bwd_layout(plan->pt, perm->T, ws);
   BwdLaunch a{};
-  a.splits = at<Tile>(perm->ws, L.splits_row);
-  a.splits_row = a.splits;
+  bool ok = true;
+  const uint64_t R = (uint64_t)perm->R, nr = (uint64_t)plan->pt.rank_off[plan->pt.G];
+  ok = ok && make_tmap_bf16(&a.tm_dy[0], dY, R, (uint64_t)plan->pt.d, kTileM);
+  ok = ok && make_tmap_bf16(&a.tm_bt[0], Bt, nr, (uint64_t)plan->pt.d, plan->pt.rank_pad);
+  ok = ok && make_tmap_bf16(&a.tm_a, A, nr, (uint64_t)plan->pt.f, plan->pt.rank_pad);
+  ok = ok && make_tmap_bf16(&a.tm_dh, dHin, R, (uint64_t)plan->pt.f, kTileM);
+  if (perm->R > 0 && !ok) return fail(ACE_ERR_UNSUPPORTED, "tensor-map encoding failed for this layout");
+  a.tm_dy[1] = a.tm_dy[0];
+  a.tm_bt[1] = a.tm_bt[0];
+  a.splits_row = at<Tile>(perm->ws, L.splits_row);
   a.tiles_sh = at<Tile>(perm->ws, L.tiles_sh);
   a.counts = perm->counts;
-  a.count_slot = kCntSplitsRow;
-  a.max_splits = L.max_splits;
   a.max_splits_row = L.max_splits;
   a.max_tiles_sh = L.max_tiles;
   a.uniq_tok = perm->uniq_tok;
+  a.uniq_off = perm->uniq_off;
+  a.group_off = perm->group_off;
   a.pair_row = perm->pair_row;
   a.pair_g = at<int32_t>(perm->ws, L.pair_g);
   a.row_uniq = at<int32_t>(perm->ws, L.row_uniq);
   a.Xin = Hin;
   for (int j = 0; j < 2; ++j) {
-    a.dY[j] = dY;
     a.H[j] = H;
-    a.A[j] = A;
-    a.Bt[j] = Bt;
     a.dA[j] = dA;
     a.dBt[j] = dBt;
     a.dH[j] = w.dH[0];
     a.dHrow[j] = w.dHrow[0];
-    a.part_dA[j] = w.part_dA[0];
     a.part_dBt[j] = w.part_dBt[0];
   }
   a.s = s;

@@ -2,23 +2,27 @@
 // shared adapter updates of Sec. 3.4).
 //
 // k_bwd_rows<RP, MODE>: one CTA per split of up to NT row tiles (128
-// consecutive rows of one group).  Phase 1 streams the upstream gradient in
-// 128-column chunks through a 3-stage cp.async ring:
-//     dH_i  += dY_i . B_g                 (tcgen05, TMEM, accumulated over chunks)
-//     dBt_c  = sum_i H_{u(row)}^T . dY_i  (tcgen05, one 128-column chunk of dB_g^T)
-//   dBt_c is flushed while the next chunk's MMAs run (double-buffered TMEM):
-//   fp32 atomics, or a per-split partial for the deterministic two-stage sum.
-//   MODE_DOWN then runs phase 2 over chunks of the input h:
-//     dA_c  += h_i^T . dH_i   and   dh_i += dH_i . A_g   (bf16 RMW of the rows)
-//   MODE_SHARED writes dH per row (fp32 scratch); for gate/up the rows of one
-//   unique pair (g, t) share H_u, and dC_u . B_g = sum_rows dY_row . B_g, so
-//   streaming contiguous rows moves exactly the bytes of the deduplicated form.
+//   consecutive rows of one group), warp-specialised (TMA producer warp, MMA
+//   warp, 4 epilogue warps).  Phase 1 streams the upstream gradient dY in
+//   128-column chunks:
+//     dH_i  += dY_i . B_g                 (TMEM, accumulated over chunks)
+//     dBt_c  = sum_i H_{u(row)}^T . dY_i  (TMEM, double-buffered per chunk)
+//   and the epilogue flushes each dBt chunk (fp32 atomics, or a per-split
+//   partial for the deterministic two-stage sum) while the next chunk runs.
+//   The epilogue then writes dH (scaled by s).  MODE_DOWN continues with
+//     dh_i += dH_i . A_g                  (dh tiles staged by TMA, added in
+//                                          swizzled smem, coalesced stores)
+//   For gate/up (MODE_SHARED) the rows of one unique pair (g, t) share H_u and
+//   dC_u . B_g = sum_rows dY_row . B_g, so streaming contiguous rows moves the
+//   bytes of the deduplicated form; dH per row goes to fp32 scratch.
 // k_dh_reduce: dH_u = sum of the dH rows of unique pair u (fixed slot order).
-// k_bwd_dA: gate and up fused; per split of unique pairs, X rows gathered by
-//   token: dA_c += X_i^T . dH_u,i for both projections.
-// k_dx: token-major, deterministic: dX[t] += sum_proj sum_{u of t} dH_u . A_g(u),
-//   groups in ascending order.
-// k_splitk_reduce: deterministic stage 2 (split order); empty groups -> zeros.
+// k_bwd_dA: one CTA per (group, 128-column chunk of d_in) streams all of the
+//   group's unique pairs (X gathered by token) or rows (h):
+//     dA_c^T = sum X_i^T . dH_i           (gate and up fused on one X gather)
+//   and stores the chunk directly: deterministic, no split-K.
+// k_dx: token-major, deterministic: dX[t] += sum_proj sum_{u of t} dH_u . A_g(u).
+// k_splitk_reduce: deterministic stage 2 of dB^T (split order); empty groups
+//   -> exact zeros.
 #include <cstdint>
 
 #include "ace_internal.cuh"
@@ -27,10 +31,12 @@
 namespace ace {
 namespace {
 
-constexpr int kNcB = 128;   // columns per chunk
-constexpr int kS = 3;       // pipeline stages
+constexpr int kNcB = 128;           // columns per chunk
 constexpr int kBlk = kTileM * 128;  // one [128 x 64] bf16 SW128 block (16 KB)
 constexpr int MODE_DOWN = 0, MODE_SHARED = 1;
+constexpr int kThreadsWS = 192;     // producer, MMA, 4 epilogue warps
+constexpr int kEpiThreads = 128;
+constexpr int kEpiBar = 1;
 
 // Operand slots of [128 x RP] bf16 (H or dH tiles).  For RP <= 64 several
 // slots share one 128-byte-swizzled block side by side (column offset
@@ -66,49 +72,24 @@ __device__ __forceinline__ uint32_t tile_off(int rows, int r, int c_chunk /*0..1
   return (uint32_t)((c_chunk >> 3) * rows * 128) + sw128_off(r, c_chunk & 7);
 }
 
-// rows [r0, r0 + RP) x cols [n0, n0 + 128) of a row-major bf16 matrix into a
-// weight tile; rows >= rv or cols >= ncol are zero.
+__device__ __forceinline__ uint4 pack8(const float* v) {
+  uint4 w;
+  w.x = pack_bf16x2(v[0], v[1]);
+  w.y = pack_bf16x2(v[2], v[3]);
+  w.z = pack_bf16x2(v[4], v[5]);
+  w.w = pack_bf16x2(v[6], v[7]);
+  return w;
+}
+
+// Flush one [128 cols x RP] fp32 accumulator of a weight gradient (TMEM lane
+// `col_lane` = column n0 + col_lane): atomics into out, a per-split partial,
+// or a plain store of the final value.
+enum FlushMode { kAtomic = 0, kPartial = 1, kStore = 2 };
 template <int RP>
-__device__ __forceinline__ void load_w_tile(uint32_t dst, const uint16_t* __restrict__ base, int r0, int rv, int ld,
-                                            int n0, int ncol, int tid) {
-#pragma unroll
-  for (int idx = tid; idx < RP * 16; idx += 128) {
-    const int k = idx >> 4, cc = idx & 15, col = n0 + cc * 8;
-    const bool v = k < rv && col < ncol;
-    cp_async16(dst + tile_off(RP, k, cc), v ? base + (int64_t)(r0 + k) * ld + col : base, v);
-  }
-}
-
-// 128 rows x 128 columns of a row-major bf16 matrix, row ids from `rows`
-// (-1 = zero row), into an activation tile.
-__device__ __forceinline__ void load_act_tile(uint32_t dst, const uint16_t* __restrict__ base, const int32_t* rows,
-                                              int ld, int n0, int ncol, int tid) {
-#pragma unroll
-  for (int q = 0; q < 16; ++q) {
-    const int idx = q * 128 + tid, m = idx >> 4, cc = idx & 15, col = n0 + cc * 8;
-    const int r = rows[m];
-    const bool v = r >= 0 && col < ncol;
-    cp_async16(dst + tile_off(kTileM, m, cc), v ? base + (int64_t)r * ld + col : base, v);
-  }
-}
-
-__device__ __forceinline__ uint4 add_bf16x8(uint4 y, const uint32_t* d, float scale) {
-  const float2 f0 = unpack_bf16x2(y.x), f1 = unpack_bf16x2(y.y), f2 = unpack_bf16x2(y.z), f3 = unpack_bf16x2(y.w);
-  uint4 o;
-  o.x = pack_bf16x2(f0.x + scale * __uint_as_float(d[0]), f0.y + scale * __uint_as_float(d[1]));
-  o.y = pack_bf16x2(f1.x + scale * __uint_as_float(d[2]), f1.y + scale * __uint_as_float(d[3]));
-  o.z = pack_bf16x2(f2.x + scale * __uint_as_float(d[4]), f2.y + scale * __uint_as_float(d[5]));
-  o.w = pack_bf16x2(f3.x + scale * __uint_as_float(d[6]), f3.y + scale * __uint_as_float(d[7]));
-  return o;
-}
-
-// Flush one [128 cols x RP] fp32 accumulator (TMEM lane = column) of a weight
-// gradient: atomics into out[(r0 + k) * ld + col] or a per-split partial.
-template <int RP>
-__device__ __forceinline__ void flush_wgrad(uint32_t taddr, int n0, int ld, int rg, int r0, float scale, bool det,
+__device__ __forceinline__ void flush_wgrad(uint32_t taddr, int n0, int ld, int rg, int r0, float scale, int mode,
                                             float* __restrict__ part, int split_id, float* __restrict__ out,
-                                            int tid) {
-  const int col = n0 + tid;
+                                            int col_lane, bool zero = false) {
+  const int col = n0 + col_lane;
 #pragma unroll
   for (int c0 = 0; c0 < RP; c0 += 16) {
     uint32_t r[16];
@@ -119,82 +100,98 @@ __device__ __forceinline__ void flush_wgrad(uint32_t taddr, int n0, int ld, int 
       for (int q = 0; q < 16; ++q) {
         const int kk = c0 + q;
         if (kk < rg) {
-          const float v = scale * __uint_as_float(r[q]);
-          if (det)
+          const float v = zero ? 0.f : scale * __uint_as_float(r[q]);
+          if (mode == kPartial)
             part[((int64_t)split_id * RP + kk) * ld + col] = v;
-          else
+          else if (mode == kAtomic)
             atomicAdd(&out[(int64_t)(r0 + kk) * ld + col], v);
+          else
+            out[(int64_t)(r0 + kk) * ld + col] = v;
         }
       }
     }
   }
 }
 
+// ----------------------------------------------------------------- k_bwd_rows
 template <int RP, int MODE>
 struct RowsCfg {
   static constexpr int NT = RP <= 32 ? 4 : (RP == 64 ? 2 : 1);
   static constexpr int kOps = Slots<RP>::bytes(NT);
-  static constexpr int kAct = kTileM * 256;
-  static constexpr int kW = RP * 256;
-  static constexpr int kStage = kAct + kW;
-  static constexpr int kSmem = kOps + kS * kStage + 1024;
-  static constexpr int kTmem = RP <= 64 ? 256 : 512;
+  static constexpr int kWBlk = RP * 128;
+  static constexpr int kSlotA = 2 * kBlk + 2 * kWBlk;          // dY tile + B^T chunk (down phase 2: A chunk)
+  static constexpr int kSlotB = 2 * kBlk;                      // down: dh tile for the RMW
+  static constexpr int SB = MODE == MODE_DOWN ? 2 : 0;
+  static constexpr int kBudget = 220 * 1024;
+  static constexpr int kSA0 = (kBudget - kOps - SB * kSlotB) / kSlotA;
+  static constexpr int SA = kSA0 > 6 ? 6 : (kSA0 < 2 ? 2 : kSA0);
+  static constexpr int kSmem = kOps + SA * kSlotA + SB * kSlotB + 1024;
+  static constexpr int kTB = 128;  // dB^T accumulators (2 x RP columns)
+  static constexpr int kDB = 256;  // down: dh D accumulators (2 x 128 columns)
+  static constexpr int kTmem = (MODE == MODE_DOWN || RP > 64) ? 512 : 256;
 };
 
 template <int RP, int MODE>
-__global__ void __launch_bounds__(128, 1) k_bwd_rows(const __grid_constant__ PlanTables pt,
-                                                     const __grid_constant__ BwdLaunch a) {
+__global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constant__ PlanTables pt,
+                                                            const __grid_constant__ BwdLaunch a) {
   using C = RowsCfg<RP, MODE>;
   using SL = Slots<RP>;
-  constexpr int NT = C::NT;
+  constexpr int NT = C::NT, SA = C::SA, SB = C::SB > 0 ? C::SB : 1;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  __shared__ __align__(8) uint64_t bar[kS];
+  __shared__ __align__(8) uint64_t fullA[SA], emptyA[SA], fullB[SB], emptyB[SB];
+  __shared__ __align__(8) uint64_t dbt_full[2], dbt_empty[2], d_full[2], d_empty[2], dh_full, hs_ready;
   __shared__ uint32_t tslot;
-  __shared__ int32_t s_row[NT * kTileM];
+  static_assert(NT * RP <= 128, "dH accumulators must fit below the dB^T columns");
 
-  const int n_splits = a.counts[a.count_slot];
+  const int n_splits = a.counts[kCntSplitsRow];
   if ((int)blockIdx.x >= n_splits) return;
   const int proj = blockIdx.y;
-  const Tile sp = a.splits[blockIdx.x];
-  const int tid = threadIdx.x, warp = tid >> 5;
+  const Tile sp = a.splits_row[blockIdx.x];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = sp.g, r0 = pt.rank_off[g], rg = pt.rank_off[g + 1] - r0;
   const int ntiles = (sp.cnt + kTileM - 1) / kTileM;
   const int d_in = a.d_in, d_out = a.d_out;
-  const float s = a.s;
-  const uint16_t* __restrict__ dY = a.dY[proj];
+  const int nch1 = (d_out + kNcB - 1) / kNcB;
+  const int nch2 = MODE == MODE_DOWN ? (d_in + kNcB - 1) / kNcB : 0;
+  const int NI1 = nch1 * ntiles, NI2 = nch2 * ntiles;
+  const uint32_t sOps = smem_u32(smem);
+  const uint32_t sA0 = sOps + C::kOps;
+  const uint32_t sB0 = sA0 + SA * C::kSlotA;
 
-  const uint32_t ops = smem_u32(smem);
-  const uint32_t stage0 = ops + C::kOps;
-  auto act = [&](int slot) { return stage0 + slot * C::kStage; };
-  auto wt = [&](int slot) { return stage0 + slot * C::kStage + C::kAct; };
-
-  for (int i = tid; i < NT * kTileM; i += 128) {
-    const int ti = i / kTileM, m = i % kTileM;
-    s_row[i] = (ti < ntiles && m < sp.cnt - ti * kTileM) ? sp.start + ti * kTileM + m : -1;
-  }
   if (tid == 0) {
-    for (int i = 0; i < kS; ++i) mbar_init(&bar[i], 1);
+    for (int i = 0; i < SA; ++i) {
+      mbar_init(&fullA[i], 1);
+      mbar_init(&emptyA[i], 1);
+    }
+    for (int i = 0; i < SB; ++i) {
+      mbar_init(&fullB[i], 1);
+      mbar_init(&emptyB[i], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&dbt_full[i], 1);
+      mbar_init(&dbt_empty[i], 1);
+      mbar_init(&d_full[i], 1);
+      mbar_init(&d_empty[i], 1);
+    }
+    mbar_init(&dh_full, 1);
+    mbar_init(&hs_ready, 1);
     fence_mbar_init();
   }
   if (warp == 0) tmem_alloc(&tslot, C::kTmem);
-  __syncthreads();
-  // H operand slots: bf16 of the saved H of each row (per unique pair for gate/up)
-  for (int i = 0; i < ntiles; ++i) {
-    const int row = s_row[i * kTileM + tid];
-    const int hrow = row < 0 ? -1 : (MODE == MODE_SHARED ? a.row_uniq[row] : row);
+  // H operand slots (all threads): bf16 of the saved H of each row
+  for (int idx = tid; idx < ntiles * kTileM; idx += kThreadsWS) {
+    const int i = idx / kTileM, m = idx % kTileM;
+    const int row = sp.start + i * kTileM + m;
+    const bool live = i * kTileM + m < sp.cnt;
+    const int hrow = !live ? -1 : (MODE == MODE_SHARED ? a.row_uniq[row] : row);
     const float* hp = a.H[proj] + (int64_t)(hrow < 0 ? 0 : hrow) * pt.rank_max;
 #pragma unroll
     for (int c8 = 0; c8 < RP; c8 += 8) {
       float v[8];
 #pragma unroll
       for (int q = 0; q < 8; ++q) v[q] = (hrow >= 0 && c8 + q < rg) ? hp[c8 + q] : 0.f;
-      uint4 w;
-      w.x = pack_bf16x2(v[0], v[1]);
-      w.y = pack_bf16x2(v[2], v[3]);
-      w.z = pack_bf16x2(v[4], v[5]);
-      w.w = pack_bf16x2(v[6], v[7]);
-      *reinterpret_cast<uint4*>(smem + SL::elem(i, tid, c8)) = w;
+      sts128(sOps + SL::elem(i, m, c8), pack8(v));
     }
   }
   fence_proxy_async_smem();
@@ -202,198 +199,206 @@ __global__ void __launch_bounds__(128, 1) k_bwd_rows(const __grid_constant__ Pla
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = tslot;
-  bool bad = false, aborted = false;  // bad: this thread's wait gave up; aborted: CTA-uniform
-  const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
-  const uint32_t t_dbt = tmem + NT * RP;  // two buffers of RP columns
+  bool bad = false;
 
-  // ------------------------------------------------------------- phase 1
-  constexpr uint32_t id_dh = idesc_bf16_f32(128, RP, 0, 0);
-  constexpr uint32_t id_w = idesc_bf16_f32(128, RP, 1, 1);
-  const int nch1 = (d_out + kNcB - 1) / kNcB;
-  const int NI1 = nch1 * ntiles;
-  auto load1 = [&](int it, int slot) {
-    const int c = it / ntiles, i = it % ntiles;
-    load_w_tile<RP>(wt(slot), a.Bt[proj], r0, rg, d_out, c * kNcB, d_out, tid);
-    load_act_tile(act(slot), dY, &s_row[i * kTileM], d_out, c * kNcB, d_out, tid);
-  };
-#pragma unroll
-  for (int j = 0; j < kS - 1; ++j) {
-    if (j < NI1) load1(j, j);
-    cp_async_commit();
-  }
-  for (int it = 0; it < NI1; ++it) {
-    const int c = it / ntiles, i = it % ntiles, slot = it % kS;
-    cp_async_wait<kS - 2>();
-    fence_proxy_async_smem();
-    if (__syncthreads_or(bad)) {
-      aborted = true;
-      break;
-    }
-    if (tid == 0) {
-      tc_fence_after();
-      const uint32_t A0 = act(slot), W0 = wt(slot);
-#pragma unroll
-      for (int kk = 0; kk < kNcB / 16; ++kk)  // dH_i += dY_i . B_g
-        tc_mma_bf16(tmem + i * RP, sdesc_sw128(A0 + (kk >> 2) * kBlk + (kk & 3) * 32, 16, 1024),
-                    sdesc_sw128(W0 + (kk >> 2) * (RP * 128) + (kk & 3) * 32, 16, 1024), id_dh,
-                    (c > 0 || kk > 0) ? 1u : 0u);
-#pragma unroll
-      for (int kk = 0; kk < kTileM / 16; ++kk)  // dBt_c^T += dY_i^T . H_i
-        tc_mma_bf16(t_dbt + (c & 1) * RP, sdesc_sw128(A0 + kk * 2048, kBlk, 1024), SL::desc_mn(ops, i, kk), id_w,
-                    (i > 0 || kk > 0) ? 1u : 0u);
-      tc_commit(&bar[slot]);
-    }
-    if (i == 0 && c > 0) {  // flush chunk c-1 while chunk c runs
-      if (!mbar_wait(&bar[(it - 1) % kS], ((it - 1) / kS) & 1)) bad = true;
-      tc_fence_after();
-      flush_wgrad<RP>(t_dbt + ((c - 1) & 1) * RP + lane_base, (c - 1) * kNcB, d_out, rg, r0, s, a.deterministic,
-                      a.part_dBt[proj], sp.id, a.dBt[proj], tid);
-      tc_fence_before();
-    }
-    const int nxt = it + kS - 1;
-    if (nxt < NI1) {
-      if (it >= 1 && !mbar_wait(&bar[(it - 1) % kS], ((it - 1) / kS) & 1)) bad = true;
-      load1(nxt, nxt % kS);
-    }
-    cp_async_commit();
-  }
-  cp_async_wait<0>();
-  if (NI1 > 0 && !aborted && !bad && !mbar_wait(&bar[(NI1 - 1) % kS], ((NI1 - 1) / kS) & 1)) bad = true;
-  aborted = __syncthreads_or(bad || aborted);
-  if (NI1 > 0 && !aborted) {
-    tc_fence_after();
-    flush_wgrad<RP>(t_dbt + ((nch1 - 1) & 1) * RP + lane_base, (nch1 - 1) * kNcB, d_out, rg, r0, s, a.deterministic,
-                    a.part_dBt[proj], sp.id, a.dBt[proj], tid);
-  }
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  if (aborted) {
-    if (tid == 0) atomicOr(a.err, kErrTimeout);
-    if (warp == 0) tmem_dealloc(tmem, C::kTmem);
-    return;
-  }
-
-  // dH (scaled by s): MODE_SHARED -> fp32 scratch per row; MODE_DOWN -> bf16 operand slots
-  for (int i = 0; i < ntiles; ++i) {
-    const int row = s_row[i * kTileM + tid];
-#pragma unroll
-    for (int c0 = 0; c0 < RP; c0 += 16) {
-      uint32_t r[16];
-      tmem_ld16(tmem + lane_base + i * RP + c0, r);
-      tmem_ld_wait();
-      if (MODE == MODE_SHARED) {
-        if (row >= 0) {
-          float4* dst = reinterpret_cast<float4*>(a.dHrow[proj] + (int64_t)row * RP + c0);
-#pragma unroll
-          for (int q = 0; q < 4; ++q)
-            dst[q] = make_float4(s * __uint_as_float(r[4 * q]), s * __uint_as_float(r[4 * q + 1]),
-                                 s * __uint_as_float(r[4 * q + 2]), s * __uint_as_float(r[4 * q + 3]));
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      for (int q = 0; q < NI1 + NI2 && !bad; ++q) {
+        const int s = q % SA, u = q / SA;
+        if (u >= 1 && !mbar_wait(&emptyA[s], (u - 1) & 1)) {
+          bad = true;
+          break;
         }
-      } else {
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          uint4 w = make_uint4(0, 0, 0, 0);
-          if (row >= 0) {
-            w.x = pack_bf16x2(s * __uint_as_float(r[h * 8 + 0]), s * __uint_as_float(r[h * 8 + 1]));
-            w.y = pack_bf16x2(s * __uint_as_float(r[h * 8 + 2]), s * __uint_as_float(r[h * 8 + 3]));
-            w.z = pack_bf16x2(s * __uint_as_float(r[h * 8 + 4]), s * __uint_as_float(r[h * 8 + 5]));
-            w.w = pack_bf16x2(s * __uint_as_float(r[h * 8 + 6]), s * __uint_as_float(r[h * 8 + 7]));
+        const uint32_t base = sA0 + s * C::kSlotA;
+        if (q < NI1) {
+          const int c = q / ntiles, i = q % ntiles, n0 = c * kNcB, row0 = sp.start + i * kTileM;
+          mbar_arrive_expect_tx(&fullA[s], 2 * kBlk + 2 * C::kWBlk);
+          tma_load_2d(base, &a.tm_dy[proj], n0, row0, &fullA[s]);
+          tma_load_2d(base + kBlk, &a.tm_dy[proj], n0 + 64, row0, &fullA[s]);
+          tma_load_2d(base + 2 * kBlk, &a.tm_bt[proj], n0, r0, &fullA[s]);
+          tma_load_2d(base + 2 * kBlk + C::kWBlk, &a.tm_bt[proj], n0 + 64, r0, &fullA[s]);
+        } else {
+          const int j = q - NI1, c = j / ntiles, i = j % ntiles, n0 = c * kNcB, row0 = sp.start + i * kTileM;
+          mbar_arrive_expect_tx(&fullA[s], 2 * C::kWBlk);
+          tma_load_2d(base, &a.tm_a, n0, r0, &fullA[s]);
+          tma_load_2d(base + C::kWBlk, &a.tm_a, n0 + 64, r0, &fullA[s]);
+          const int sb = j % SB, ub = j / SB;
+          if (ub >= 1 && !mbar_wait(&emptyB[sb], (ub - 1) & 1)) {
+            bad = true;
+            break;
           }
-          *reinterpret_cast<uint4*>(smem + SL::elem(i, tid, c0 + h * 8)) = w;
+          const uint32_t bb = sB0 + sb * C::kSlotB;
+          mbar_arrive_expect_tx(&fullB[sb], 2 * kBlk);
+          tma_load_2d(bb, &a.tm_dh, n0, row0, &fullB[sb]);
+          tma_load_2d(bb + kBlk, &a.tm_dh, n0 + 64, row0, &fullB[sb]);
         }
       }
     }
-  }
-  if (MODE == MODE_DOWN) {
-    fence_proxy_async_smem();
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    // ----------------------------------------------------------- phase 2
-    constexpr uint32_t id_dh2 = idesc_bf16_f32(128, kNcB, 0, 1);
-    const uint32_t t_d = tmem;                 // dh chunk, 128 columns
-    const uint32_t t_da = tmem + kNcB;         // two buffers of RP columns
-    const int nch2 = (d_in + kNcB - 1) / kNcB;
-    const int NI2 = nch2 * ntiles;
-    auto load2 = [&](int it, int slot) {
-      const int c = it / ntiles, i = it % ntiles;
-      load_w_tile<RP>(wt(slot), a.A[proj], r0, rg, d_in, c * kNcB, d_in, tid);
-      load_act_tile(act(slot), a.Xin, &s_row[i * kTileM], d_in, c * kNcB, d_in, tid);
-    };
-    // barrier phases continue from phase 1: iteration j of phase 2 is global NI1 + j
-#pragma unroll
-    for (int j = 0; j < kS - 1; ++j) {
-      if (j < NI2) {
-        const int gj = NI1 + j;
-        if (gj >= kS && !mbar_wait(&bar[gj % kS], ((gj - kS) / kS) & 1)) bad = true;
-        load2(j, gj % kS);
-      }
-      cp_async_commit();
-    }
-    for (int it = 0; it < NI2; ++it) {
-      const int c = it / ntiles, i = it % ntiles, git = NI1 + it, slot = git % kS;
-      cp_async_wait<kS - 2>();
-      fence_proxy_async_smem();
-      if (__syncthreads_or(bad)) {
-        aborted = true;
-        break;
-      }
-      if (tid == 0) {
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t id_dh = idesc_bf16_f32(128, RP, 0, 0);
+      constexpr uint32_t id_w = idesc_bf16_f32(128, RP, 1, 1);
+      for (int q = 0; q < NI1 && !bad; ++q) {
+        const int c = q / ntiles, i = q % ntiles, s = q % SA, u = q / SA;
+        if (!mbar_wait(&fullA[s], u & 1)) {
+          bad = true;
+          break;
+        }
+        if (i == 0 && c >= 2 && !mbar_wait(&dbt_empty[c & 1], ((c - 2) >> 1) & 1)) {
+          bad = true;
+          break;
+        }
         tc_fence_after();
-        const uint32_t A0 = act(slot), W0 = wt(slot);
+        const uint32_t base = sA0 + s * C::kSlotA;
 #pragma unroll
-        for (int kk = 0; kk < RP / 16; ++kk)  // dh chunk = dH_i . A_g
-          tc_mma_bf16(t_d, SL::desc_k(ops, i, kk), sdesc_sw128(W0 + kk * 2048, RP * 128, 1024), id_dh2,
-                      kk > 0 ? 1u : 0u);
+        for (int kk = 0; kk < kNcB / 16; ++kk)  // dH_i += dY_i . B_g
+          tc_mma_bf16(tmem + i * RP, sdesc_sw128(base + (kk >> 2) * kBlk + (kk & 3) * 32, 16, 1024),
+                      sdesc_sw128(base + 2 * kBlk + (kk >> 2) * C::kWBlk + (kk & 3) * 32, 16, 1024), id_dh,
+                      (c > 0 || kk > 0) ? 1u : 0u);
 #pragma unroll
-        for (int kk = 0; kk < kTileM / 16; ++kk)  // dA_c^T += h_i^T . dH_i
-          tc_mma_bf16(t_da + (c & 1) * RP, sdesc_sw128(A0 + kk * 2048, kBlk, 1024), SL::desc_mn(ops, i, kk), id_w,
-                      (i > 0 || kk > 0) ? 1u : 0u);
-        tc_commit(&bar[slot]);
+        for (int kk = 0; kk < kTileM / 16; ++kk)  // dBt_c^T += dY_i^T . H_i
+          tc_mma_bf16(tmem + C::kTB + (c & 1) * RP, sdesc_sw128(base + kk * 2048, kBlk, 1024),
+                      SL::desc_mn(sOps, i, kk), id_w, (i > 0 || kk > 0) ? 1u : 0u);
+        tc_commit(&emptyA[s]);
+        if (i == ntiles - 1) tc_commit(&dbt_full[c & 1]);
       }
-      // this thread's dh row chunk (issued before waiting on the MMA)
-      const int row = s_row[i * kTileM + tid];
-      const int n0 = c * kNcB;
-      uint4 y[16];
-      uint16_t* yp = a.dXin + (int64_t)(row < 0 ? 0 : row) * d_in + n0;
+      if (!bad) tc_commit(&dh_full);
+      if (MODE == MODE_DOWN && !bad) {
+        constexpr uint32_t id_d = idesc_bf16_f32(128, kNcB, 0, 1);
+        if (!mbar_wait(&hs_ready, 0)) bad = true;
+        for (int j = 0; j < NI2 && !bad; ++j) {
+          const int q = NI1 + j, i = j % ntiles, s = q % SA, u = q / SA, b = j & 1;
+          if (!mbar_wait(&fullA[s], u & 1)) {
+            bad = true;
+            break;
+          }
+          if (j >= 2 && !mbar_wait(&d_empty[b], ((j - 2) >> 1) & 1)) {
+            bad = true;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t base = sA0 + s * C::kSlotA;
 #pragma unroll
-      for (int q = 0; q < 16; ++q)
-        y[q] = (row >= 0 && n0 + q * 8 < d_in) ? *reinterpret_cast<const uint4*>(yp + q * 8) : make_uint4(0, 0, 0, 0);
-      if (!mbar_wait(&bar[slot], (git / kS) & 1)) bad = true;
-      tc_fence_after();
-      if (i == 0 && c > 0)
-        flush_wgrad<RP>(t_da + ((c - 1) & 1) * RP + lane_base, (c - 1) * kNcB, d_in, rg, r0, 1.f, a.deterministic,
-                        a.part_dA[proj], sp.id, a.dA[proj], tid);
-#pragma unroll
-      for (int sc = 0; sc < kNcB; sc += 32) {
-        uint32_t r[32];
-        tmem_ld16(t_d + lane_base + sc, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
-        tmem_ld16(t_d + lane_base + sc + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
-        tmem_ld_wait();
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const int qq = sc / 8 + q;
-          if (row >= 0 && n0 + qq * 8 < d_in)
-            *reinterpret_cast<uint4*>(yp + qq * 8) = add_bf16x8(y[qq], &r[q * 8], 1.f);
+          for (int kk = 0; kk < RP / 16; ++kk)  // dh chunk = dH_i . A_g chunk
+            tc_mma_bf16(tmem + C::kDB + b * kNcB, SL::desc_k(sOps, i, kk),
+                        sdesc_sw128(base + kk * 2048, C::kWBlk, 1024), id_d, kk > 0 ? 1u : 0u);
+          tc_commit(&emptyA[s]);
+          tc_commit(&d_full[b]);
         }
       }
-      tc_fence_before();
-      const int nxt = it + kS - 1;
-      if (nxt < NI2) load2(nxt, (NI1 + nxt) % kS);  // its slot's previous MMA (git - 1) is complete
-      cp_async_commit();
     }
-    cp_async_wait<0>();
-    aborted = __syncthreads_or(bad || aborted);
-    if (NI2 > 0 && !aborted) {
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int et = tid - 64;
+    const int quarter = warp & 3;
+    const int m = quarter * 32 + lane;
+    const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
+    const int fmode = a.deterministic ? kPartial : kAtomic;
+    bool ok = true;
+    for (int c = 0; c < nch1 && ok; ++c) {
+      ok = named_bar_and(kEpiBar, kEpiThreads, mbar_wait(&dbt_full[c & 1], (c >> 1) & 1));
+      if (!ok) break;
       tc_fence_after();
-      flush_wgrad<RP>(t_da + ((nch2 - 1) & 1) * RP + lane_base, (nch2 - 1) * kNcB, d_in, rg, r0, 1.f,
-                      a.deterministic, a.part_dA[proj], sp.id, a.dA[proj], tid);
+      flush_wgrad<RP>(tmem + lane_base + C::kTB + (c & 1) * RP, c * kNcB, d_out, rg, r0, a.s, fmode,
+                      a.part_dBt[proj], sp.id, a.dBt[proj], m);
+      tc_fence_before();
+      named_bar(kEpiBar, kEpiThreads);
+      if (et == 0) mbar_arrive(&dbt_empty[c & 1]);
     }
+    if (ok) ok = named_bar_and(kEpiBar, kEpiThreads, mbar_wait(&dh_full, 0));
+    if (ok) {
+      tc_fence_after();
+      // dH (scaled by s): gate/up -> fp32 per row; down -> bf16 operand slots + bf16 per row
+      for (int i = 0; i < ntiles; ++i) {
+        const bool live = i * kTileM + m < sp.cnt;
+        const int64_t row = sp.start + i * kTileM + m;
+#pragma unroll
+        for (int c0 = 0; c0 < RP; c0 += 16) {
+          uint32_t r[16];
+          tmem_ld16(tmem + lane_base + i * RP + c0, r);
+          tmem_ld_wait();
+          float v[16];
+#pragma unroll
+          // columns >= r_g come from the next group's rank rows of the B^T box: zero them
+          for (int q = 0; q < 16; ++q) v[q] = (live && c0 + q < rg) ? a.s * __uint_as_float(r[q]) : 0.f;
+          if (MODE == MODE_SHARED) {
+            if (live) {
+              float4* dst = reinterpret_cast<float4*>(a.dHrow[proj] + row * RP + c0);
+#pragma unroll
+              for (int q = 0; q < 4; ++q) dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+            }
+          } else {
+            const uint4 w0 = pack8(v), w1 = pack8(v + 8);
+            sts128(sOps + SL::elem(i, m, c0), w0);
+            sts128(sOps + SL::elem(i, m, c0 + 8), w1);
+            if (live) {
+              uint4* dst = reinterpret_cast<uint4*>(a.dH[0] + row * RP + c0);
+              dst[0] = w0;
+              dst[1] = w1;
+            }
+          }
+        }
+      }
+      fence_proxy_async_smem();
+      tc_fence_before();
+      named_bar(kEpiBar, kEpiThreads);
+      if (et == 0) mbar_arrive(&hs_ready);
+    }
+    if (MODE == MODE_DOWN) {
+      for (int j = 0; j < NI2 && ok; ++j) {
+        const int c = j / ntiles, i = j % ntiles, b = j & 1, sb = j % SB, n0 = c * kNcB;
+        bool w_ok = mbar_wait(&fullB[sb], (j / SB) & 1);
+        w_ok = w_ok && mbar_wait(&d_full[b], (j >> 1) & 1);
+        ok = named_bar_and(kEpiBar, kEpiThreads, w_ok);
+        if (!ok) break;
+        tc_fence_after();
+        const uint32_t bb = sB0 + sb * C::kSlotB;
+#pragma unroll
+        for (int h = 0; h < 4; ++h) {
+          uint32_t r[32];
+          const uint32_t ta = tmem + lane_base + C::kDB + b * kNcB + h * 32;
+          tmem_ld16(ta, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
+          tmem_ld16(ta + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
+          tmem_ld_wait();
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const uint32_t addr = bb + tile_off(kTileM, m, h * 4 + q);
+            const uint4 y = lds128(addr);
+            const uint32_t* dq = &r[q * 8];
+            const float2 f0 = unpack_bf16x2(y.x), f1 = unpack_bf16x2(y.y), f2 = unpack_bf16x2(y.z),
+                         f3 = unpack_bf16x2(y.w);
+            uint4 o;
+            o.x = pack_bf16x2(f0.x + __uint_as_float(dq[0]), f0.y + __uint_as_float(dq[1]));
+            o.y = pack_bf16x2(f1.x + __uint_as_float(dq[2]), f1.y + __uint_as_float(dq[3]));
+            o.z = pack_bf16x2(f2.x + __uint_as_float(dq[4]), f2.y + __uint_as_float(dq[5]));
+            o.w = pack_bf16x2(f3.x + __uint_as_float(dq[6]), f3.y + __uint_as_float(dq[7]));
+            sts128(addr, o);
+          }
+        }
+        tc_fence_before();
+        named_bar(kEpiBar, kEpiThreads);
+        if (et == 0) mbar_arrive(&d_empty[b]);
+        const int cnt_i = sp.cnt - i * kTileM;
+#pragma unroll 4
+        for (int it = et; it < kTileM * 16; it += kEpiThreads) {
+          const int row = it >> 4, ch = it & 15, col = n0 + ch * 8;
+          if (row < cnt_i && col < d_in) {
+            const uint4 v = lds128(bb + tile_off(kTileM, row, ch));
+            *reinterpret_cast<uint4*>(a.dXin + (int64_t)(sp.start + i * kTileM + row) * d_in + col) = v;
+          }
+        }
+        fence_proxy_async_smem();
+        named_bar(kEpiBar, kEpiThreads);
+        if (et == 0) mbar_arrive(&emptyB[sb]);
+      }
+    }
+    if (!ok) bad = true;
   }
+  __syncwarp();
   tc_fence_before();
-  aborted = __syncthreads_or(bad || aborted);
-  if (aborted && tid == 0) atomicOr(a.err, kErrTimeout);
+  if (__syncthreads_or(bad) && tid == 0) atomicOr(a.err, kErrTimeout);
   if (warp == 0) tmem_dealloc(tmem, C::kTmem);
 }
 
@@ -425,88 +430,83 @@ __global__ void __launch_bounds__(128) k_dh_reduce(const __grid_constant__ PlanT
   }
   uint4* dst = reinterpret_cast<uint4*>(a.dH[proj] + (int64_t)u * RP);
 #pragma unroll
-  for (int q = 0; q < RP / 8; ++q) {
-    uint4 w;
-    w.x = pack_bf16x2(acc[8 * q], acc[8 * q + 1]);
-    w.y = pack_bf16x2(acc[8 * q + 2], acc[8 * q + 3]);
-    w.z = pack_bf16x2(acc[8 * q + 4], acc[8 * q + 5]);
-    w.w = pack_bf16x2(acc[8 * q + 6], acc[8 * q + 7]);
-    dst[q] = w;
-  }
+  for (int q = 0; q < RP / 8; ++q) dst[q] = pack8(&acc[8 * q]);
 }
 
-// ---------------------------------------------------------------- dA (gate/up)
+// ---------------------------------------------------------------- dA
 template <int RP, int NPROJ>
 struct DaCfg {
-  static constexpr int NT = RP <= 32 ? 4 : (RP == 64 ? 2 : 1);
-  static constexpr int kOps = Slots<RP>::bytes(NT * NPROJ);
-  static constexpr int kStage = kTileM * 256;
-  static constexpr int kSmem = kOps + kS * kStage + 1024;
-  static constexpr int kTmem = NPROJ * 2 * RP <= 256 ? 256 : 512;
+  static constexpr int kOp = Slots<RP>::bytes(NPROJ);     // dH tile(s) of one row tile
+  static constexpr int kStage = kTileM * 256 + kOp;       // X / h chunk [128 x 128] + dH
+  static constexpr int kS0 = (220 * 1024) / kStage;
+  static constexpr int S = kS0 > 4 ? 4 : kS0;             // >= 2 for every rank_pad
+  static constexpr int kSmem = S * kStage + 1024;
+  static constexpr int kTmem = NPROJ * RP <= 32 ? 32 : NPROJ * RP <= 64 ? 64 : NPROJ * RP <= 128 ? 128 : 256;
 };
 
-template <int RP, int NPROJ>
+// grid (G, ceil(d_in / 128)); MODE_SHARED: rows are unique pairs (X gathered
+// by token, dH per unique pair); MODE_DOWN: rows are routed rows (h, dH per row).
+template <int RP, int NPROJ, int MODE>
 __global__ void __launch_bounds__(128, 1) k_bwd_dA(const __grid_constant__ PlanTables pt,
                                                    const __grid_constant__ BwdLaunch a) {
   using C = DaCfg<RP, NPROJ>;
   using SL = Slots<RP>;
-  constexpr int NT = C::NT;
+  constexpr int kDaStages = C::S;
+  static_assert(kDaStages >= 2, "dA pipeline needs two stages");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  __shared__ __align__(8) uint64_t bar[kS];
+  __shared__ __align__(8) uint64_t bar[kDaStages];
   __shared__ uint32_t tslot;
-  __shared__ int32_t s_tok[NT * kTileM];
-
-  const int n_splits = a.counts[a.count_slot];
-  if ((int)blockIdx.x >= n_splits) return;
-  const Tile sp = a.splits[blockIdx.x];
+  const int g = blockIdx.x, c0 = blockIdx.y * kNcB;
   const int tid = threadIdx.x, warp = tid >> 5;
-  const int g = sp.g, r0 = pt.rank_off[g], rg = pt.rank_off[g + 1] - r0;
-  const int ntiles = (sp.cnt + kTileM - 1) / kTileM;
+  const int r0 = pt.rank_off[g], rg = pt.rank_off[g + 1] - r0;
   const int d = a.d_in;
-  const uint32_t ops = smem_u32(smem);
-  const uint32_t stage0 = ops + C::kOps;
-
-  for (int i = tid; i < NT * kTileM; i += 128) {
-    const int ti = i / kTileM, m = i % kTileM;
-    s_tok[i] = (ti < ntiles && m < sp.cnt - ti * kTileM) ? a.uniq_tok[sp.start + ti * kTileM + m] : -1;
-  }
+  const int lo = MODE == MODE_SHARED ? a.uniq_off[g] : a.group_off[g];
+  const int n = (MODE == MODE_SHARED ? a.uniq_off[g + 1] : a.group_off[g + 1]) - lo;
+  const int NI = (n + kTileM - 1) / kTileM;
+  const uint32_t stage0 = smem_u32(smem);
   if (tid == 0) {
-    for (int i = 0; i < kS; ++i) mbar_init(&bar[i], 1);
+    for (int i = 0; i < kDaStages; ++i) mbar_init(&bar[i], 1);
     fence_mbar_init();
   }
   if (warp == 0) tmem_alloc(&tslot, C::kTmem);
-  // dH_u slots (bf16 scratch rows), slot q = i * NPROJ + j
-  for (int i = 0; i < ntiles; ++i) {
-    const int cnt_i = sp.cnt - i * kTileM;
-    const int u = sp.start + i * kTileM + tid;
-    for (int j = 0; j < NPROJ; ++j) {
-#pragma unroll
-      for (int c8 = 0; c8 < RP; c8 += 8) {
-        const bool v = tid < cnt_i;
-        cp_async16(ops + SL::elem(i * NPROJ + j, tid, c8), v ? a.dH[j] + (int64_t)u * RP + c8 : a.dH[0], v);
-      }
-    }
-  }
-  cp_async_commit();
+  tc_fence_before();
   __syncthreads();
+  tc_fence_after();
   const uint32_t tmem = tslot;
-  bool bad = false, aborted = false;  // bad: this thread's wait gave up; aborted: CTA-uniform
   const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
-  constexpr uint32_t id_w = idesc_bf16_f32(128, RP, 1, 1);
-  const int nch = (d + kNcB - 1) / kNcB;
-  const int NI = nch * ntiles;
   auto load = [&](int it, int slot) {
-    load_act_tile(stage0 + slot * C::kStage, a.Xin, &s_tok[(it % ntiles) * kTileM], d, (it / ntiles) * kNcB, d, tid);
-  };
+    const uint32_t st = stage0 + slot * C::kStage;
+    const int item = lo + it * kTileM + tid;  // this thread's row of the tile
+    const bool live = it * kTileM + tid < n;
+    // dH row(s) of this row (all projections)
 #pragma unroll
-  for (int j = 0; j < kS - 1; ++j) {
+    for (int j = 0; j < NPROJ; ++j)
+#pragma unroll
+      for (int c8 = 0; c8 < RP; c8 += 8)
+        cp_async16(st + kTileM * 256 + SL::elem(j, tid, c8), live ? a.dH[j] + (int64_t)item * RP + c8 : a.dH[0],
+                   live);
+    // input chunk [128 rows x 128 cols]; element (m, cc) belongs to tile row m
+#pragma unroll
+    for (int q = 0; q < 16; ++q) {
+      const int idx = q * 128 + tid, m = idx >> 4, cc = idx & 15, col = c0 + cc * 8;
+      const int rr = it * kTileM + m;
+      const bool v = rr < n && col < d;
+      int64_t src_row = 0;
+      if (v) src_row = MODE == MODE_SHARED ? a.uniq_tok[lo + rr] : lo + rr;
+      cp_async16(st + tile_off(kTileM, m, cc), v ? a.Xin + src_row * d + col : a.Xin, v);
+    }
+  };
+  constexpr uint32_t id_w = idesc_bf16_f32(128, RP, 1, 1);
+#pragma unroll
+  for (int j = 0; j < kDaStages - 1; ++j) {
     if (j < NI) load(j, j);
     cp_async_commit();
   }
+  bool bad = false, aborted = false;
   for (int it = 0; it < NI; ++it) {
-    const int c = it / ntiles, i = it % ntiles, slot = it % kS;
-    cp_async_wait<kS - 2>();
+    const int slot = it % kDaStages;
+    cp_async_wait<kDaStages - 2>();
     fence_proxy_async_smem();
     if (__syncthreads_or(bad)) {
       aborted = true;
@@ -514,59 +514,58 @@ __global__ void __launch_bounds__(128, 1) k_bwd_dA(const __grid_constant__ PlanT
     }
     if (tid == 0) {
       tc_fence_after();
-      const uint32_t A0 = stage0 + slot * C::kStage;
+      const uint32_t st = stage0 + slot * C::kStage;
 #pragma unroll
       for (int j = 0; j < NPROJ; ++j)
 #pragma unroll
-        for (int kk = 0; kk < kTileM / 16; ++kk)
-          tc_mma_bf16(tmem + (j * 2 + (c & 1)) * RP, sdesc_sw128(A0 + kk * 2048, kBlk, 1024),
-                      SL::desc_mn(ops, i * NPROJ + j, kk), id_w, (i > 0 || kk > 0) ? 1u : 0u);
+        for (int kk = 0; kk < kTileM / 16; ++kk)  // dA_c^T += X^T . dH
+          tc_mma_bf16(tmem + j * RP, sdesc_sw128(st + kk * 2048, kBlk, 1024), SL::desc_mn(st + kTileM * 256, j, kk),
+                      id_w, (it > 0 || kk > 0) ? 1u : 0u);
       tc_commit(&bar[slot]);
     }
-    if (i == 0 && c > 0) {
-      if (!mbar_wait(&bar[(it - 1) % kS], ((it - 1) / kS) & 1)) bad = true;
-      tc_fence_after();
-      for (int j = 0; j < NPROJ; ++j)
-        flush_wgrad<RP>(tmem + (j * 2 + ((c - 1) & 1)) * RP + lane_base, (c - 1) * kNcB, d, rg, r0, 1.f,
-                        a.deterministic, a.part_dA[j], sp.id, a.dA[j], tid);
-      tc_fence_before();
-    }
-    const int nxt = it + kS - 1;
+    const int nxt = it + kDaStages - 1;
     if (nxt < NI) {
-      if (it >= 1 && !mbar_wait(&bar[(it - 1) % kS], ((it - 1) / kS) & 1)) bad = true;
-      load(nxt, nxt % kS);
+      if (it >= 1 && !mbar_wait(&bar[(it - 1) % kDaStages], ((it - 1) / kDaStages) & 1)) bad = true;
+      if (!bad) load(nxt, nxt % kDaStages);
     }
     cp_async_commit();
   }
   cp_async_wait<0>();
-  if (NI > 0 && !aborted && !bad && !mbar_wait(&bar[(NI - 1) % kS], ((NI - 1) / kS) & 1)) bad = true;
+  if (NI > 0 && !aborted && !bad && !mbar_wait(&bar[(NI - 1) % kDaStages], ((NI - 1) / kDaStages) & 1)) bad = true;
+  tc_fence_before();
   aborted = __syncthreads_or(bad || aborted);
-  if (NI > 0 && !aborted) {
-    tc_fence_after();
+  tc_fence_after();
+  if (!aborted) {
+    // the chunk is complete: store it (a group without rows gets zeros)
     for (int j = 0; j < NPROJ; ++j)
-      flush_wgrad<RP>(tmem + (j * 2 + ((nch - 1) & 1)) * RP + lane_base, (nch - 1) * kNcB, d, rg, r0, 1.f,
-                      a.deterministic, a.part_dA[j], sp.id, a.dA[j], tid);
+      flush_wgrad<RP>(tmem + lane_base + j * RP, c0, d, rg, r0, 1.f, kStore, nullptr, 0, a.dA[j], tid, NI == 0);
+  } else if (tid == 0) {
+    atomicOr(a.err, kErrTimeout);
   }
-  if (aborted && tid == 0) atomicOr(a.err, kErrTimeout);
   tc_fence_before();
   __syncthreads();
   if (warp == 0) tmem_dealloc(tmem, C::kTmem);
 }
 
 // ---------------------------------------------------------------- dX
+
 template <int RP>
 struct DxCfg {
   static constexpr int kNd = 256;
   static constexpr int kOp = (RP > 64 ? 2 : 1) * kBlk;
   static constexpr int kW = RP * kNd * 2;  // 4 blocks of [RP x 128 B]
   static constexpr int kStage = kOp + kW;
-  static constexpr int kSmem = kS * kStage + 1024;
+  static constexpr int kS0 = (220 * 1024) / kStage;
+  static constexpr int S = kS0 > 3 ? 3 : kS0;
+  static constexpr int kSmem = S * kStage + 1024;
 };
 
 template <int RP>
 __global__ void __launch_bounds__(128) k_dx(const __grid_constant__ PlanTables pt, const __grid_constant__ DxLaunch a) {
   using C = DxCfg<RP>;
   constexpr int kNd = C::kNd;
+  constexpr int kS = C::S;
+  static_assert(kS >= 2, "dX pipeline needs two stages");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   __shared__ __align__(8) uint64_t bar[kS];
@@ -585,7 +584,6 @@ __global__ void __launch_bounds__(128) k_dx(const __grid_constant__ PlanTables p
   }
   if (warp == 0) tmem_alloc(&tslot, 256);
   __syncthreads();
-  // token's unique pairs (ascending g) and the active groups of the tile
   int my_u[kMaxK];
   int nu = 0;
   if (t < a.T) {
@@ -597,7 +595,6 @@ __global__ void __launch_bounds__(128) k_dx(const __grid_constant__ PlanTables p
   }
   if (tid == 0) s_nkb = 0;
   __syncthreads();
-  // groups with at least one token of this tile, ascending
   for (int g = 0; g < G; ++g) {
     bool has = false;
     for (int q = 0; q < nu; ++q) has |= (my_u[q] >= s_uoff[g] && my_u[q] < s_uoff[g + 1]);
@@ -607,8 +604,8 @@ __global__ void __launch_bounds__(128) k_dx(const __grid_constant__ PlanTables p
   const int ng = s_nkb;
   const int NI = ng * a.nproj;
   const uint32_t stage0 = smem_u32(smem);
+  tc_fence_after();
   const uint32_t tmem = tslot;
-  bool bad = false, aborted = false;  // bad: this thread's wait gave up; aborted: CTA-uniform
   const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
   constexpr uint32_t idesc = idesc_bf16_f32(128, kNd, 0, 1);
   auto load = [&](int it, int slot) {
@@ -637,6 +634,7 @@ __global__ void __launch_bounds__(128) k_dx(const __grid_constant__ PlanTables p
     if (j < NI) load(j, j);
     cp_async_commit();
   }
+  bool bad = false, aborted = false;
   for (int it = 0; it < NI; ++it) {
     const int slot = it % kS;
     cp_async_wait<kS - 2>();
@@ -657,7 +655,7 @@ __global__ void __launch_bounds__(128) k_dx(const __grid_constant__ PlanTables p
     const int nxt = it + kS - 1;
     if (nxt < NI) {
       if (it >= 1 && !mbar_wait(&bar[(it - 1) % kS], ((it - 1) / kS) & 1)) bad = true;
-      load(nxt, nxt % kS);
+      if (!bad) load(nxt, nxt % kS);
     }
     cp_async_commit();
   }
@@ -684,8 +682,17 @@ __global__ void __launch_bounds__(128) k_dx(const __grid_constant__ PlanTables p
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
             const int qq = h * 4 + q;
-            if (t < a.T && col0 + qq * 8 < d)
-              *reinterpret_cast<uint4*>(yp + qq * 8) = add_bf16x8(y[qq], &r[q * 8], 1.f);
+            if (t < a.T && col0 + qq * 8 < d) {
+              const uint32_t* dq = &r[q * 8];
+              const float2 f0 = unpack_bf16x2(y[qq].x), f1 = unpack_bf16x2(y[qq].y), f2 = unpack_bf16x2(y[qq].z),
+                           f3 = unpack_bf16x2(y[qq].w);
+              uint4 o;
+              o.x = pack_bf16x2(f0.x + __uint_as_float(dq[0]), f0.y + __uint_as_float(dq[1]));
+              o.y = pack_bf16x2(f1.x + __uint_as_float(dq[2]), f1.y + __uint_as_float(dq[3]));
+              o.z = pack_bf16x2(f2.x + __uint_as_float(dq[4]), f2.y + __uint_as_float(dq[5]));
+              o.w = pack_bf16x2(f3.x + __uint_as_float(dq[6]), f3.y + __uint_as_float(dq[7]));
+              *reinterpret_cast<uint4*>(yp + qq * 8) = o;
+            }
           }
         }
       }
@@ -728,11 +735,23 @@ cudaError_t set_smem(K kern, int bytes) {
   return cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
 }
 
-cudaError_t reduce_launch(const PlanTables& pt, const Tile* splits, const int32_t* counts, int slot, const float* part,
-                          int RP, int width, float* out, cudaStream_t st) {
-  const int n_rank = pt.rank_off[pt.G];
-  dim3 grid(n_rank, (width / 4 + 255) / 256);
-  k_splitk_reduce<<<grid, 256, 0, st>>>(pt, splits, counts, slot, part, RP, width, out);
+template <int RP, int MODE>
+cudaError_t launch_rows(const PlanTables& pt, const BwdLaunch& a, int nproj, cudaStream_t st) {
+  using C = RowsCfg<RP, MODE>;
+  auto kern = k_bwd_rows<RP, MODE>;
+  cudaError_t e = set_smem(kern, C::kSmem);
+  if (e != cudaSuccess) return e;
+  kern<<<dim3(a.max_splits_row, nproj), kThreadsWS, C::kSmem, st>>>(pt, a);
+  return cudaGetLastError();
+}
+
+template <int RP, int NPROJ, int MODE>
+cudaError_t launch_da(const PlanTables& pt, const BwdLaunch& a, cudaStream_t st) {
+  using C = DaCfg<RP, NPROJ>;
+  auto kern = k_bwd_dA<RP, NPROJ, MODE>;
+  cudaError_t e = set_smem(kern, C::kSmem);
+  if (e != cudaSuccess) return e;
+  kern<<<dim3(pt.G, (a.d_in + kNcB - 1) / kNcB), 128, C::kSmem, st>>>(pt, a);
   return cudaGetLastError();
 }
 
@@ -742,54 +761,25 @@ cudaError_t launch_bwd_t(const PlanTables& pt, const BwdLaunch& a, bool shared, 
   const int n_rank = pt.rank_off[pt.G];
   const int nproj = shared ? a.nproj : 1;
   if (!a.deterministic) {
-    for (int j = 0; j < nproj; ++j) {
-      if ((e = cudaMemsetAsync(a.dA[j], 0, sizeof(float) * (size_t)n_rank * a.d_in, st)) != cudaSuccess) return e;
+    for (int j = 0; j < nproj; ++j)
       if ((e = cudaMemsetAsync(a.dBt[j], 0, sizeof(float) * (size_t)n_rank * a.d_out, st)) != cudaSuccess) return e;
-    }
   }
-  if (a.T > 0) {
-    if (!shared) {
-      using C = RowsCfg<RP, MODE_DOWN>;
-      auto kern = k_bwd_rows<RP, MODE_DOWN>;
-      if ((e = set_smem(kern, C::kSmem)) != cudaSuccess) return e;
-      kern<<<dim3(a.max_splits_row, 1), 128, C::kSmem, st>>>(pt, a);
-      if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    } else {
-      using C = RowsCfg<RP, MODE_SHARED>;
-      auto kern = k_bwd_rows<RP, MODE_SHARED>;
-      if ((e = set_smem(kern, C::kSmem)) != cudaSuccess) return e;
-      BwdLaunch b = a;
-      b.splits = a.splits_row;
-      b.count_slot = kCntSplitsRow;
-      b.part_dBt[0] = a.part_dBt[0];
-      b.part_dBt[1] = a.part_dBt[1];
-      kern<<<dim3(a.max_splits_row, nproj), 128, C::kSmem, st>>>(pt, b);
-      if ((e = cudaGetLastError()) != cudaSuccess) return e;
-      k_dh_reduce<RP><<<dim3(a.max_tiles_sh, nproj), 128, 0, st>>>(pt, a);
-      if ((e = cudaGetLastError()) != cudaSuccess) return e;
-      if (nproj == 2) {
-        using D = DaCfg<RP, 2>;
-        auto kd = k_bwd_dA<RP, 2>;
-        if ((e = set_smem(kd, D::kSmem)) != cudaSuccess) return e;
-        kd<<<a.max_splits, 128, D::kSmem, st>>>(pt, a);
-      } else {
-        using D = DaCfg<RP, 1>;
-        auto kd = k_bwd_dA<RP, 1>;
-        if ((e = set_smem(kd, D::kSmem)) != cudaSuccess) return e;
-        kd<<<a.max_splits, 128, D::kSmem, st>>>(pt, a);
-      }
-      if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    }
+  if (!shared) {
+    if ((e = launch_rows<RP, MODE_DOWN>(pt, a, 1, st)) != cudaSuccess) return e;
+    if ((e = launch_da<RP, 1, MODE_DOWN>(pt, a, st)) != cudaSuccess) return e;
+  } else {
+    if ((e = launch_rows<RP, MODE_SHARED>(pt, a, nproj, st)) != cudaSuccess) return e;
+    k_dh_reduce<RP><<<dim3(a.max_tiles_sh, nproj), 128, 0, st>>>(pt, a);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    e = nproj == 2 ? launch_da<RP, 2, MODE_SHARED>(pt, a, st) : launch_da<RP, 1, MODE_SHARED>(pt, a, st);
+    if (e != cudaSuccess) return e;
   }
   if (a.deterministic) {
     for (int j = 0; j < nproj; ++j) {
-      // dB^T partials are indexed by row splits, dA partials by the path's splits
-      if ((e = reduce_launch(pt, a.splits_row, a.counts, kCntSplitsRow, a.part_dBt[j], RP, a.d_out, a.dBt[j], st)) !=
-          cudaSuccess)
-        return e;
-      if ((e = reduce_launch(pt, shared ? a.splits : a.splits_row, a.counts, shared ? kCntSplitsSh : kCntSplitsRow,
-                             a.part_dA[j], RP, a.d_in, a.dA[j], st)) != cudaSuccess)
-        return e;
+      dim3 grid(n_rank, (a.d_out / 4 + 255) / 256);
+      k_splitk_reduce<<<grid, 256, 0, st>>>(pt, a.splits_row, a.counts, kCntSplitsRow, a.part_dBt[j], RP, a.d_out,
+                                            a.dBt[j]);
+      if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
   }
   return cudaSuccess;
@@ -809,6 +799,17 @@ cudaError_t launch_dx_t(const PlanTables& pt, const DxLaunch& a, cudaStream_t st
 }  // namespace
 
 cudaError_t launch_bwd(const PlanTables& pt, const BwdLaunch& a, bool shared, cudaStream_t st) {
+  if (a.T == 0) {
+    // no routed rows: every weight gradient is zero
+    const int n_rank = pt.rank_off[pt.G];
+    const int nproj = shared ? a.nproj : 1;
+    for (int j = 0; j < nproj; ++j) {
+      cudaError_t e = cudaMemsetAsync(a.dA[j], 0, sizeof(float) * (size_t)n_rank * a.d_in, st);
+      if (e == cudaSuccess) e = cudaMemsetAsync(a.dBt[j], 0, sizeof(float) * (size_t)n_rank * a.d_out, st);
+      if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
+  }
   switch (pt.rank_pad) {
     case 16: return launch_bwd_t<16>(pt, a, shared, st);
     case 32: return launch_bwd_t<32>(pt, a, shared, st);

@@ -10,7 +10,7 @@
 namespace ace {
 
 constexpr int kTileM = 128;        // rows (or unique pairs) per MMA tile
-constexpr int kPermTB = 256;       // tokens per permutation chunk / CTA
+constexpr int kPermTB = 64;        // tokens per permutation chunk / CTA
 constexpr int kMaxK = 32;          // largest top-k the kernels accept
 
 // Device error-flag bits (the flag lives at perm workspace word 0).

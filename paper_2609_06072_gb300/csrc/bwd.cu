@@ -34,8 +34,8 @@ namespace {
 constexpr int kNcB = 128;           // columns per chunk
 constexpr int kBlk = kTileM * 128;  // one [128 x 64] bf16 SW128 block (16 KB)
 constexpr int MODE_DOWN = 0, MODE_SHARED = 1;
-constexpr int kThreadsWS = 192;     // producer, MMA, 4 epilogue warps
-constexpr int kEpiThreads = 128;
+constexpr int kThreadsWS = 320;     // producer, MMA, 8 epilogue warps (two per TMEM lane quarter)
+constexpr int kEpiThreads = 256;
 constexpr int kEpiBar = 1;
 
 // Operand slots of [128 x RP] bf16 (H or dH tiles).  For RP <= 64 several
@@ -88,10 +88,9 @@ enum FlushMode { kAtomic = 0, kPartial = 1, kStore = 2 };
 template <int RP>
 __device__ __forceinline__ void flush_wgrad(uint32_t taddr, int n0, int ld, int rg, int r0, float scale, int mode,
                                             float* __restrict__ part, int split_id, float* __restrict__ out,
-                                            int col_lane, bool zero = false) {
+                                            int col_lane, bool zero = false, int c_begin = 0, int c_step = 16) {
   const int col = n0 + col_lane;
-#pragma unroll
-  for (int c0 = 0; c0 < RP; c0 += 16) {
+  for (int c0 = c_begin; c0 < RP; c0 += c_step) {
     uint32_t r[16];
     tmem_ld16(taddr + c0, r);
     tmem_ld_wait();
@@ -293,6 +292,7 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
     // ------------------------------------------------------------ epilogue
     const int et = tid - 64;
     const int quarter = warp & 3;
+    const int ehalf = (warp - 2) >> 2;  // which half of the columns this warp owns
     const int m = quarter * 32 + lane;
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
     const int fmode = a.deterministic ? kPartial : kAtomic;
@@ -302,7 +302,7 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
       if (!ok) break;
       tc_fence_after();
       flush_wgrad<RP>(tmem + lane_base + C::kTB + (c & 1) * RP, c * kNcB, d_out, rg, r0, a.s, fmode,
-                      a.part_dBt[proj], sp.id, a.dBt[proj], m);
+                      a.part_dBt[proj], sp.id, a.dBt[proj], m, false, ehalf * 16, 32);
       tc_fence_before();
       named_bar(kEpiBar, kEpiThreads);
       if (et == 0) mbar_arrive(&dbt_empty[c & 1]);
@@ -315,7 +315,7 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
         const bool live = i * kTileM + m < sp.cnt;
         const int64_t row = sp.start + i * kTileM + m;
 #pragma unroll
-        for (int c0 = 0; c0 < RP; c0 += 16) {
+        for (int c0 = ehalf * 16; c0 < RP; c0 += 32) {
           uint32_t r[16];
           tmem_ld16(tmem + lane_base + i * RP + c0, r);
           tmem_ld_wait();
@@ -356,7 +356,8 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
         tc_fence_after();
         const uint32_t bb = sB0 + sb * C::kSlotB;
 #pragma unroll
-        for (int h = 0; h < 4; ++h) {
+        for (int hh = 0; hh < 2; ++hh) {
+          const int h = ehalf * 2 + hh;
           uint32_t r[32];
           const uint32_t ta = tmem + lane_base + C::kDB + b * kNcB + h * 32;
           tmem_ld16(ta, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));

@@ -148,8 +148,8 @@ __global__ void __launch_bounds__(kHThreads) k_fwd_h(const __grid_constant__ Pla
 }
 
 // --------------------------------------------------------------- k_fwd_rows
-constexpr int kRowsThreads = 192;  // 6 warps: producer, MMA, 4 epilogue
-constexpr int kEpiThreads = 128;
+constexpr int kRowsThreads = 320;  // 10 warps: producer, MMA, 8 epilogue (two per TMEM lane quarter)
+constexpr int kEpiThreads = 256;
 constexpr int kChunk = 64;         // output columns per D chunk
 constexpr int kEpiBar = 1;         // named barrier of the epilogue warps
 
@@ -279,8 +279,9 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
     }
   } else {
     // ------------------------------------------------------------ epilogue
-    const int et = tid - 64;                 // 0..127
+    const int et = tid - 64;                 // 0..255
     const int quarter = warp & 3;            // TMEM lane quarter of this warp
+    const int ehalf = (warp - 2) >> 2;       // which half of the chunk's columns this warp owns
     const int m = quarter * 32 + lane;       // tile row owned by this thread
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
     const bool live = m < tl.cnt;
@@ -289,8 +290,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
     if (!SHARED) {
       ok = mbar_wait(&hacc, 0);
       tc_fence_after();
-#pragma unroll
-      for (int c0 = 0; c0 < RP; c0 += 16) {
+      for (int c0 = ehalf * 16; c0 < RP; c0 += 32) {
         uint32_t r[16];
         tmem_ld16(tmem + lane_base + c0, r);
         tmem_ld_wait();
@@ -319,8 +319,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
 #pragma unroll
       for (int j = 0; j < NPROJ; ++j) {
         const float* hp = a.Hu[j] + (int64_t)(u < 0 ? 0 : u) * pt.rank_max;
-#pragma unroll
-        for (int c8 = 0; c8 < RP; c8 += 8) {
+        for (int c8 = ehalf * 8; c8 < RP; c8 += 16) {
           float v[8];
 #pragma unroll
           for (int q = 0; q < 8; ++q) v[q] = (u >= 0 && c8 + q < rg) ? hp[c8 + q] : 0.f;
@@ -347,10 +346,11 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
       if (!ok) break;
       tc_fence_after();
       const uint32_t base = slot0 + sl * C::kSlot;
+      {
+        const int j = NPROJ == 2 ? ehalf : 0;
 #pragma unroll
-      for (int j = 0; j < NPROJ; ++j) {
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
+        for (int hh = 0; hh < (NPROJ == 2 ? 2 : 1); ++hh) {
+          const int h = NPROJ == 2 ? hh : ehalf;
           uint32_t r[32];
           const uint32_t ta = tmem + lane_base + dbase + (b * NPROJ + j) * kChunk + h * 32;
           tmem_ld16(ta, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));

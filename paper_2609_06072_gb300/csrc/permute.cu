@@ -98,6 +98,50 @@ __device__ int build_tiles(const int32_t* n_g, const int32_t* off_g, int G, int 
   return total;
 }
 
+// Per-column prefix over chunks of a [C x ncol] count matrix, parallel over
+// (column, part) with P parts per column.  Pass 1 writes each column's total;
+// pass 2 writes base[c][col] = col_base[col] + sum_{c' < c} cnt[c'][col].
+__device__ void column_totals(const int32_t* __restrict__ cnt, int C, int ncol, int32_t* part_sum /*smem 1024*/,
+                              int32_t* total /*smem [ncol]*/) {
+  const int tid = threadIdx.x;
+  int P = 1;
+  while (P * 2 * ncol <= (int)blockDim.x && P < 32) P *= 2;
+  const int len = (C + P - 1) / P;
+  if (tid < ncol * P) {
+    const int col = tid / P, part = tid % P;
+    int s = 0;
+    for (int c = part * len; c < min(C, (part + 1) * len); ++c) s += cnt[(int64_t)c * ncol + col];
+    part_sum[tid] = s;
+  }
+  __syncthreads();
+  for (int col = tid; col < ncol; col += blockDim.x) {
+    int run = 0;
+    for (int part = 0; part < P; ++part) {
+      const int v = part_sum[col * P + part];
+      part_sum[col * P + part] = run;
+      run += v;
+    }
+    total[col] = run;
+  }
+  __syncthreads();
+}
+__device__ void column_bases(const int32_t* __restrict__ cnt, int C, int ncol, const int32_t* part_sum,
+                             const int32_t* col_base, int32_t* __restrict__ base) {
+  const int tid = threadIdx.x;
+  int P = 1;
+  while (P * 2 * ncol <= (int)blockDim.x && P < 32) P *= 2;
+  const int len = (C + P - 1) / P;
+  if (tid < ncol * P) {
+    const int col = tid / P, part = tid % P;
+    int run = col_base[col] + part_sum[tid];
+    for (int c = part * len; c < min(C, (part + 1) * len); ++c) {
+      base[(int64_t)c * ncol + col] = run;
+      run += cnt[(int64_t)c * ncol + col];
+    }
+  }
+  __syncthreads();
+}
+
 __global__ void __launch_bounds__(1024) k_perm_scan(const __grid_constant__ PlanTables pt, int n_chunks,
                                                     const int32_t* __restrict__ chunk_cntE,
                                                     const int32_t* __restrict__ chunk_cntU,
@@ -116,6 +160,9 @@ __global__ void __launch_bounds__(1024) k_perm_scan(const __grid_constant__ Plan
   __shared__ int32_t gofs[ACE_MAX_EXPERTS + 1];
   __shared__ int32_t uofs[ACE_MAX_EXPERTS + 1];
   __shared__ int32_t scratch[ACE_MAX_EXPERTS + 1];
+  __shared__ int32_t eoff[ACE_MAX_EXPERTS];
+  __shared__ int32_t partE[1024];
+  __shared__ int32_t partU[1024];
   __shared__ int32_t err_s;
   const int tid = threadIdx.x;
   const int E = pt.E, G = pt.G;
@@ -124,17 +171,9 @@ __global__ void __launch_bounds__(1024) k_perm_scan(const __grid_constant__ Plan
   __syncthreads();
   for (int c = tid; c < n_chunks; c += blockDim.x)
     if (chunk_err[c]) atomicOr(&err_s, chunk_err[c]);
-  for (int e = tid; e < E; e += blockDim.x) {
-    int s = 0;
-    for (int c = 0; c < n_chunks; ++c) s += chunk_cntE[(int64_t)c * E + e];
-    totE[e] = s;
-    atomicAdd(&rowsG[pt.e2g[e]], s);
-  }
-  for (int g = tid; g < G; g += blockDim.x) {
-    int s = 0;
-    for (int c = 0; c < n_chunks; ++c) s += chunk_cntU[(int64_t)c * G + g];
-    totU[g] = s;
-  }
+  column_totals(chunk_cntE, n_chunks, E, partE, totE);
+  column_totals(chunk_cntU, n_chunks, G, partU, totU);
+  for (int e = tid; e < E; e += blockDim.x) atomicAdd(&rowsG[pt.e2g[e]], totE[e]);
   __syncthreads();
   if (tid == 0) {
     gofs[0] = 0;
@@ -157,22 +196,13 @@ __global__ void __launch_bounds__(1024) k_perm_scan(const __grid_constant__ Plan
     int start = gofs[g];
     for (int e2 = 0; e2 < e; ++e2)
       if (pt.e2g[e2] == g) start += totE[e2];
+    eoff[e] = start;
     expert_off[e] = start;
     expert_cnt[e] = totE[e];
-    int run = start;
-    for (int c = 0; c < n_chunks; ++c) {
-      chunk_baseE[(int64_t)c * E + e] = run;
-      run += chunk_cntE[(int64_t)c * E + e];
-    }
-  }
-  for (int g = tid; g < G; g += blockDim.x) {
-    int run = uofs[g];
-    for (int c = 0; c < n_chunks; ++c) {
-      chunk_baseU[(int64_t)c * G + g] = run;
-      run += chunk_cntU[(int64_t)c * G + g];
-    }
   }
   __syncthreads();
+  column_bases(chunk_cntE, n_chunks, E, partE, eoff, chunk_baseE);
+  column_bases(chunk_cntU, n_chunks, G, partU, uofs, chunk_baseU);
   const int per_split = kTileM * pt.nt_split;
   int n;
   n = build_tiles(totU, uofs, G, kTileM, tiles_sh, scratch);

@@ -185,8 +185,8 @@ class Layer:
     def kernels_per_step(self):
         # permute 3, fwd_shared 2 (H per unique pair, row stream), fwd_row 1, bwd_row 1,
         # bwd_shared 4 (row stream, dH_u sum, dA, dX);
-        # deterministic mode adds 2 split-K reduces per projection (3 projections)
-        return 11 + (6 if self.det else 0)
+        # deterministic mode adds one dB^T split-K reduce per projection
+        return 11 + (3 if self.det else 0)
 
     def step(self, ev=None):
         """One pass of the hot path.  ev: list of 6 CUDA events (call boundaries)."""

@@ -158,7 +158,9 @@ struct BwdLaunch {
   const float* H[2];     // saved H (gate/up: per unique pair; down: per row), stride rank_max
   float s;
   uint16_t* dXin;        // down: dHin [R, f] in/out
-  uint16_t* dH[2];       // scratch: bf16 dH [R, rank_pad] (gate/up: per unique pair; down: per row)
+  uint16_t* dH[2];       // scratch: bf16 dH per row [R, rank_pad] (down)
+  uint16_t* dHx;         // scratch: token-major dense dH [T, nproj * n_rank_pad] (gate/up)
+  int32_t n_rank_pad;    // n_rank rounded up to a multiple of 64
   float* dHrow[2];       // scratch: fp32 dH per row [R, rank_pad] (gate/up)
   float* dA[2];
   float* dBt[2];
@@ -169,15 +171,18 @@ struct BwdLaunch {
 };
 cudaError_t launch_bwd(const PlanTables& pt, const BwdLaunch& a, bool shared, cudaStream_t st);
 
-struct DxLaunch {
-  const int32_t* tok_uniq;
-  const int32_t* uniq_off;
-  const uint16_t* dH[2];
-  const uint16_t* A[2];
+// Dense gate/up backward over the token-major dH matrix (see gemm.cu).
+struct DenseBwdLaunch {
+  CUtensorMap tm_dhx;      // dHx [T, nproj * n_rank_pad], box 64 x 128
+  CUtensorMap tm_dhx_t;    // same tensor, box 64 x 64
+  CUtensorMap tm_acat[2];  // A_j [n_rank, d], box 64 x 64
+  CUtensorMap tm_x;        // X [T, d], box 64 x 64
+  CUtensorMap tm_dx;       // dX [T, d], box 64 x 128
   uint16_t* dX;
-  int32_t T, d, nproj;
+  float* dA[2];
+  int32_t T, d, n_rank, n_rank_pad, nproj;
   int32_t* err;
 };
-cudaError_t launch_dx(const PlanTables& pt, const DxLaunch& a, cudaStream_t st);
+cudaError_t launch_dense_bwd(const DenseBwdLaunch& a, cudaStream_t st);
 
 }  // namespace ace

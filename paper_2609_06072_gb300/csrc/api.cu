@@ -82,8 +82,11 @@ struct BwdWs {
   uint16_t* dH[2];
   float* dHrow[2];
   float* part_dBt[2];
+  uint16_t* dHx;
   size_t total;
 };
+
+int n_rank_pad_of(const PlanTables& pt) { return (pt.rank_off[pt.G] + 63) / 64 * 64; }
 
 // Backward scratch per projection: dH per unique pair / row (bf16), dH per
 // row (fp32) and the deterministic dB^T split-K partials.
@@ -104,6 +107,8 @@ BwdWs bwd_layout(const PlanTables& pt, int32_t T, void* base) {
     w.part_dBt[j] = reinterpret_cast<float*>(b + off);
     off += pa;
   }
+  w.dHx = reinterpret_cast<uint16_t*>(b + off);
+  off += align_up(2 * (size_t)T * 2 * n_rank_pad_of(pt), 256);
   w.total = off;
   return w;
 }
@@ -358,6 +363,8 @@ ace_status ace_bwd_shared(const ace_plan* plan, const ace_perm* perm, int32_t np
     a.part_dBt[j] = w.part_dBt[jj];
   }
   if (nproj == 1) a.tm_dy[1] = a.tm_dy[0], a.tm_bt[1] = a.tm_bt[0];
+  a.dHx = w.dHx;
+  a.n_rank_pad = n_rank_pad_of(plan->pt);
   a.s = s;
   a.dXin = nullptr;
   a.d_in = plan->pt.d;
@@ -369,20 +376,25 @@ ace_status ace_bwd_shared(const ace_plan* plan, const ace_perm* perm, int32_t np
   st = cuda_status(launch_bwd(plan->pt, a, true, cs), "backward launch");
   if (st != ACE_OK) return st;
   if (perm->R == 0) return ACE_OK;
-  DxLaunch x{};
-  x.tok_uniq = perm->tok_uniq;
-  x.uniq_off = perm->uniq_off;
-  for (int j = 0; j < 2; ++j) {
-    const int jj = j < nproj ? j : 0;
-    x.dH[j] = w.dH[jj];
-    x.A[j] = A[jj];
-  }
+  // dX += dHx . [A_j], dA_j = dHx_j^T . X  (dense, token-major)
+  const PlanTables& pt = plan->pt;
+  DenseBwdLaunch x{};
+  const int n_rank = pt.rank_off[pt.G], nrp = n_rank_pad_of(pt);
+  const uint64_t T = (uint64_t)perm->T, kw = (uint64_t)nproj * nrp;
+  bool okm = make_tmap_bf16(&x.tm_dhx, w.dHx, T, kw, kTileM) && make_tmap_bf16(&x.tm_dhx_t, w.dHx, T, kw, 64) &&
+             make_tmap_bf16(&x.tm_x, X, T, (uint64_t)pt.d, 64) && make_tmap_bf16(&x.tm_dx, dX, T, (uint64_t)pt.d, kTileM);
+  for (int j = 0; j < nproj; ++j) okm = okm && make_tmap_bf16(&x.tm_acat[j], A[j], (uint64_t)n_rank, (uint64_t)pt.d, 64);
+  if (!okm) return fail(ACE_ERR_UNSUPPORTED, "tensor-map encoding failed for this layout");
+  if (nproj == 1) x.tm_acat[1] = x.tm_acat[0];
   x.dX = dX;
+  for (int j = 0; j < 2; ++j) x.dA[j] = dA[j < nproj ? j : 0];
   x.T = perm->T;
-  x.d = plan->pt.d;
+  x.d = pt.d;
+  x.n_rank = n_rank;
+  x.n_rank_pad = nrp;
   x.nproj = nproj;
   x.err = a.err;
-  return cuda_status(launch_dx(plan->pt, x, cs), "dX launch");
+  return cuda_status(launch_dense_bwd(x, cs), "dense dX / dA launch");
 }
 
 ace_status ace_bwd_row(const ace_plan* plan, const ace_perm* perm, const uint16_t* dY, const uint16_t* Hin,

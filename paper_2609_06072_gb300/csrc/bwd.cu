@@ -15,12 +15,12 @@
 //   For gate/up (MODE_SHARED) the rows of one unique pair (g, t) share H_u and
 //   dC_u . B_g = sum_rows dY_row . B_g, so streaming contiguous rows moves the
 //   bytes of the deduplicated form; dH per row goes to fp32 scratch.
-// k_dh_reduce: dH_u = sum of the dH rows of unique pair u (fixed slot order).
-// k_bwd_dA: one CTA per (group, 128-column chunk of d_in) streams all of the
-//   group's unique pairs (X gathered by token) or rows (h):
-//     dA_c^T = sum X_i^T . dH_i           (gate and up fused on one X gather)
-//   and stores the chunk directly: deterministic, no split-K.
-// k_dx: token-major, deterministic: dX[t] += sum_proj sum_{u of t} dH_u . A_g(u).
+// k_dh_reduce: dH_u = sum of the dH rows of unique pair u (fixed slot order),
+//   written into the token-major dense dHx consumed by the dense dX / dA
+//   GEMMs of gemm.cu.
+// k_bwd_dA (down): one CTA per (group, 128-column chunk of f) streams all of
+//   the group's rows: dA_c^T = sum h_i^T . dH_i, stored directly
+//   (deterministic, no split-K).
 // k_splitk_reduce: deterministic stage 2 of dB^T (split order); empty groups
 //   -> exact zeros.
 #include <cstdint>
@@ -404,6 +404,8 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
 }
 
 // ---------------------------------------------------------------- dH_u
+// dH_u = sum of the dH rows of unique pair u (fixed slot order), written into
+// the token-major dense matrix dHx[t][j * n_rank_pad + rank_off[g] + k].
 template <int RP>
 __global__ void __launch_bounds__(128) k_dh_reduce(const __grid_constant__ PlanTables pt,
                                                    const __grid_constant__ BwdLaunch a) {
@@ -413,12 +415,13 @@ __global__ void __launch_bounds__(128) k_dh_reduce(const __grid_constant__ PlanT
   const Tile tl = a.tiles_sh[blockIdx.x];
   const int m = threadIdx.x;
   if (m >= tl.cnt) return;
-  const int u = tl.start + m, t = a.uniq_tok[u], k = pt.k;
+  const int u = tl.start + m, t = a.uniq_tok[u], k = pt.k, g = tl.g;
+  const int r0 = pt.rank_off[g], rg = pt.rank_off[g + 1] - r0;
   float acc[RP];
 #pragma unroll
   for (int q = 0; q < RP; ++q) acc[q] = 0.f;
   for (int j = 0; j < k; ++j) {
-    if (a.pair_g[(int64_t)t * k + j] != tl.g) continue;
+    if (a.pair_g[(int64_t)t * k + j] != g) continue;
     const float4* src = reinterpret_cast<const float4*>(a.dHrow[proj] + (int64_t)a.pair_row[(int64_t)t * k + j] * RP);
 #pragma unroll
     for (int q = 0; q < RP / 4; ++q) {
@@ -429,9 +432,20 @@ __global__ void __launch_bounds__(128) k_dh_reduce(const __grid_constant__ PlanT
       acc[4 * q + 3] += v.w;
     }
   }
-  uint4* dst = reinterpret_cast<uint4*>(a.dH[proj] + (int64_t)u * RP);
+  const int kw = a.nproj * a.n_rank_pad;
+  uint16_t* dst = a.dHx + (int64_t)t * kw + proj * a.n_rank_pad + r0;
+  if ((r0 & 7) == 0 && (rg & 7) == 0) {
 #pragma unroll
-  for (int q = 0; q < RP / 8; ++q) dst[q] = pack8(&acc[8 * q]);
+    for (int q = 0; q < RP / 8; ++q)
+      if (q * 8 < rg) reinterpret_cast<uint4*>(dst)[q] = pack8(&acc[8 * q]);
+  } else {
+#pragma unroll
+    for (int q = 0; q < RP; ++q)
+      if (q < rg) {
+        const __nv_bfloat16 h = __float2bfloat16_rn(acc[q]);
+        dst[q] = *reinterpret_cast<const uint16_t*>(&h);
+      }
+  }
 }
 
 // ---------------------------------------------------------------- dA
@@ -548,163 +562,6 @@ __global__ void __launch_bounds__(128, 1) k_bwd_dA(const __grid_constant__ PlanT
   if (warp == 0) tmem_dealloc(tmem, C::kTmem);
 }
 
-// ---------------------------------------------------------------- dX
-
-template <int RP>
-struct DxCfg {
-  static constexpr int kNd = 256;
-  static constexpr int kOp = (RP > 64 ? 2 : 1) * kBlk;
-  static constexpr int kW = RP * kNd * 2;  // 4 blocks of [RP x 128 B]
-  static constexpr int kStage = kOp + kW;
-  static constexpr int kS0 = (220 * 1024) / kStage;
-  static constexpr int S = kS0 > 3 ? 3 : kS0;
-  static constexpr int kSmem = S * kStage + 1024;
-};
-
-template <int RP>
-__global__ void __launch_bounds__(128) k_dx(const __grid_constant__ PlanTables pt, const __grid_constant__ DxLaunch a) {
-  using C = DxCfg<RP>;
-  constexpr int kNd = C::kNd;
-  constexpr int kS = C::S;
-  static_assert(kS >= 2, "dX pipeline needs two stages");
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  __shared__ __align__(8) uint64_t bar[kS];
-  __shared__ uint32_t tslot;
-  __shared__ int32_t s_uoff[ACE_MAX_EXPERTS + 1];
-  __shared__ int32_t s_kb[ACE_MAX_EXPERTS];  // groups active in this token tile
-  __shared__ int32_t s_nkb;
-  const int tid = threadIdx.x, warp = tid >> 5;
-  const int t0 = blockIdx.x * kTileM, c0 = blockIdx.y * kNd;
-  const int d = a.d, k = pt.k, G = pt.G;
-  const int t = t0 + tid;
-  for (int i = tid; i <= G; i += 128) s_uoff[i] = a.uniq_off[i];
-  if (tid == 0) {
-    for (int i = 0; i < kS; ++i) mbar_init(&bar[i], 1);
-    fence_mbar_init();
-  }
-  if (warp == 0) tmem_alloc(&tslot, 256);
-  __syncthreads();
-  int my_u[kMaxK];
-  int nu = 0;
-  if (t < a.T) {
-    for (int j = 0; j < k; ++j) {
-      const int u = a.tok_uniq[(int64_t)t * k + j];
-      if (u < 0) break;
-      my_u[nu++] = u;
-    }
-  }
-  if (tid == 0) s_nkb = 0;
-  __syncthreads();
-  for (int g = 0; g < G; ++g) {
-    bool has = false;
-    for (int q = 0; q < nu; ++q) has |= (my_u[q] >= s_uoff[g] && my_u[q] < s_uoff[g + 1]);
-    if (__syncthreads_or(has) && tid == 0) s_kb[s_nkb++] = g;
-  }
-  __syncthreads();
-  const int ng = s_nkb;
-  const int NI = ng * a.nproj;
-  const uint32_t stage0 = smem_u32(smem);
-  tc_fence_after();
-  const uint32_t tmem = tslot;
-  const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
-  constexpr uint32_t idesc = idesc_bf16_f32(128, kNd, 0, 1);
-  auto load = [&](int it, int slot) {
-    const int j = it / ng, g = s_kb[it % ng];
-    const uint32_t sop = stage0 + slot * C::kStage, sw = sop + C::kOp;
-    int u = -1;
-    for (int q = 0; q < nu; ++q)
-      if (my_u[q] >= s_uoff[g] && my_u[q] < s_uoff[g + 1]) u = my_u[q];
-    const uint16_t* dHj = a.dH[j];
-#pragma unroll
-    for (int c8 = 0; c8 < RP; c8 += 8) {
-      const bool v = u >= 0;
-      cp_async16(sop + (c8 >> 6) * kBlk + sw128_off(tid, (c8 & 63) >> 3), v ? dHj + (int64_t)u * RP + c8 : dHj, v);
-    }
-    const int r0 = pt.rank_off[g], rg = pt.rank_off[g + 1] - r0;
-#pragma unroll 4
-    for (int idx = tid; idx < RP * (kNd / 8); idx += 128) {
-      const int kr = idx / (kNd / 8), cc = idx % (kNd / 8), col = c0 + cc * 8;
-      const bool v = kr < rg && col < d;
-      cp_async16(sw + (cc >> 3) * (RP * 128) + sw128_off(kr, cc & 7), v ? a.A[j] + (int64_t)(r0 + kr) * d + col : a.A[0],
-                 v);
-    }
-  };
-#pragma unroll
-  for (int j = 0; j < kS - 1; ++j) {
-    if (j < NI) load(j, j);
-    cp_async_commit();
-  }
-  bool bad = false, aborted = false;
-  for (int it = 0; it < NI; ++it) {
-    const int slot = it % kS;
-    cp_async_wait<kS - 2>();
-    fence_proxy_async_smem();
-    if (__syncthreads_or(bad)) {
-      aborted = true;
-      break;
-    }
-    if (tid == 0) {
-      tc_fence_after();
-      const uint32_t sop = stage0 + slot * C::kStage, sw = sop + C::kOp;
-#pragma unroll
-      for (int kk = 0; kk < RP / 16; ++kk)
-        tc_mma_bf16(tmem, sdesc_sw128(sop + (kk >> 2) * kBlk + (kk & 3) * 32, 16, 1024),
-                    sdesc_sw128(sw + kk * 2048, RP * 128, 1024), idesc, (it > 0 || kk > 0) ? 1u : 0u);
-      tc_commit(&bar[slot]);
-    }
-    const int nxt = it + kS - 1;
-    if (nxt < NI) {
-      if (it >= 1 && !mbar_wait(&bar[(it - 1) % kS], ((it - 1) / kS) & 1)) bad = true;
-      if (!bad) load(nxt, nxt % kS);
-    }
-    cp_async_commit();
-  }
-  cp_async_wait<0>();
-  if (NI > 0) {
-    if (!aborted && !bad && !mbar_wait(&bar[(NI - 1) % kS], ((NI - 1) / kS) & 1)) bad = true;
-    tc_fence_after();
-    aborted = __syncthreads_or(bad || aborted);
-    if (!aborted) {
-#pragma unroll 1
-      for (int sc = 0; sc < kNd; sc += 64) {
-        const int col0 = c0 + sc;
-        uint4 y[8];
-        uint16_t* yp = a.dX + (int64_t)(t < a.T ? t : 0) * d + col0;
-#pragma unroll
-        for (int q = 0; q < 8; ++q)
-          y[q] = (t < a.T && col0 + q * 8 < d) ? *reinterpret_cast<const uint4*>(yp + q * 8) : make_uint4(0, 0, 0, 0);
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          uint32_t r[32];
-          tmem_ld16(tmem + lane_base + sc + h * 32, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
-          tmem_ld16(tmem + lane_base + sc + h * 32 + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
-          tmem_ld_wait();
-#pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            const int qq = h * 4 + q;
-            if (t < a.T && col0 + qq * 8 < d) {
-              const uint32_t* dq = &r[q * 8];
-              const float2 f0 = unpack_bf16x2(y[qq].x), f1 = unpack_bf16x2(y[qq].y), f2 = unpack_bf16x2(y[qq].z),
-                           f3 = unpack_bf16x2(y[qq].w);
-              uint4 o;
-              o.x = pack_bf16x2(f0.x + __uint_as_float(dq[0]), f0.y + __uint_as_float(dq[1]));
-              o.y = pack_bf16x2(f1.x + __uint_as_float(dq[2]), f1.y + __uint_as_float(dq[3]));
-              o.z = pack_bf16x2(f2.x + __uint_as_float(dq[4]), f2.y + __uint_as_float(dq[5]));
-              o.w = pack_bf16x2(f3.x + __uint_as_float(dq[6]), f3.y + __uint_as_float(dq[7]));
-              *reinterpret_cast<uint4*>(yp + qq * 8) = o;
-            }
-          }
-        }
-      }
-    }
-  }
-  if (aborted && tid == 0) atomicOr(a.err, kErrTimeout);
-  tc_fence_before();
-  __syncthreads();
-  if (warp == 0) tmem_dealloc(tmem, 256);
-}
-
 // ---------------------------------------------------------------- stage 2
 __global__ void __launch_bounds__(256) k_splitk_reduce(const __grid_constant__ PlanTables pt,
                                                        const Tile* __restrict__ splits,
@@ -770,10 +627,10 @@ cudaError_t launch_bwd_t(const PlanTables& pt, const BwdLaunch& a, bool shared, 
     if ((e = launch_da<RP, 1, MODE_DOWN>(pt, a, st)) != cudaSuccess) return e;
   } else {
     if ((e = launch_rows<RP, MODE_SHARED>(pt, a, nproj, st)) != cudaSuccess) return e;
+    const size_t dhx = sizeof(uint16_t) * (size_t)a.T * nproj * a.n_rank_pad;
+    if ((e = cudaMemsetAsync(a.dHx, 0, dhx, st)) != cudaSuccess) return e;
     k_dh_reduce<RP><<<dim3(a.max_tiles_sh, nproj), 128, 0, st>>>(pt, a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    e = nproj == 2 ? launch_da<RP, 2, MODE_SHARED>(pt, a, st) : launch_da<RP, 1, MODE_SHARED>(pt, a, st);
-    if (e != cudaSuccess) return e;
   }
   if (a.deterministic) {
     for (int j = 0; j < nproj; ++j) {
@@ -784,17 +641,6 @@ cudaError_t launch_bwd_t(const PlanTables& pt, const BwdLaunch& a, bool shared, 
     }
   }
   return cudaSuccess;
-}
-
-template <int RP>
-cudaError_t launch_dx_t(const PlanTables& pt, const DxLaunch& a, cudaStream_t st) {
-  using C = DxCfg<RP>;
-  auto kern = k_dx<RP>;
-  cudaError_t e = set_smem(kern, C::kSmem);
-  if (e != cudaSuccess) return e;
-  dim3 grid((a.T + kTileM - 1) / kTileM, (a.d + C::kNd - 1) / C::kNd);
-  kern<<<grid, 128, C::kSmem, st>>>(pt, a);
-  return cudaGetLastError();
 }
 
 }  // namespace
@@ -816,17 +662,6 @@ cudaError_t launch_bwd(const PlanTables& pt, const BwdLaunch& a, bool shared, cu
     case 32: return launch_bwd_t<32>(pt, a, shared, st);
     case 64: return launch_bwd_t<64>(pt, a, shared, st);
     case 128: return launch_bwd_t<128>(pt, a, shared, st);
-  }
-  return cudaErrorInvalidValue;
-}
-
-cudaError_t launch_dx(const PlanTables& pt, const DxLaunch& a, cudaStream_t st) {
-  if (a.T == 0) return cudaSuccess;
-  switch (pt.rank_pad) {
-    case 16: return launch_dx_t<16>(pt, a, st);
-    case 32: return launch_dx_t<32>(pt, a, st);
-    case 64: return launch_dx_t<64>(pt, a, st);
-    case 128: return launch_dx_t<128>(pt, a, st);
   }
   return cudaErrorInvalidValue;
 }

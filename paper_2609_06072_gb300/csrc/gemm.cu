@@ -1,0 +1,269 @@
+// Dense tcgen05 GEMMs of the gate/up backward over the token-major dH matrix
+//   dHx [T, nproj * n_rank_pad] bf16,  dHx[t][j * n_rank_pad + rank_off[g] + k]
+//     = (dH_{u(t,g)})_k for projection j when token t routes into group g,
+//       zero otherwise
+// (Sec. 3.4: the group adapter collects the gradient of every token routed to
+// any expert of the group).  With it both remaining gradients are plain
+// products over contiguous rows:
+//   k_gemm_dx:  dX[t] += sum_j dHx_j[t] . A_j            (M = T, N = d, K = rank)
+//   k_gemm_da:  dA_j   = dHx_j^T . X                      (M = rank, N = d, K = T)
+// Each CTA owns one output tile and its whole K loop, so both are
+// deterministic.  Warp-specialised: TMA producer warp, MMA warp, 8 epilogue
+// warps.  Operands arrive by TMA in 128-byte-swizzled boxes.
+#include <cstdint>
+
+#include "ace_internal.cuh"
+#include "ace_ptx.cuh"
+
+namespace ace {
+namespace {
+
+constexpr int kThreads = 320;
+constexpr int kEpiThreads = 256;
+constexpr int kEpiBar = 1;
+constexpr int kBlk = 128 * 128;       // [128 rows x 64 bf16]
+constexpr int kHalfBlk = 64 * 128;    // [64 rows x 64 bf16]
+
+// ------------------------------------------------------------------ dX
+constexpr int kDxN = 256;                               // d columns per CTA
+constexpr int kDxStage = kBlk + (kDxN / 64) * kHalfBlk; // dHx [128 t x 64 k] + A [64 k x 256 d]
+constexpr int kDxS = 3;
+constexpr int kDxStaging = (kDxN / 64) * kBlk;          // dX tile [128 x 256]
+constexpr int kDxSmem = kDxS * kDxStage + kDxStaging + 1024;
+
+__global__ void __launch_bounds__(kThreads, 1) k_gemm_dx(const __grid_constant__ DenseBwdLaunch a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  __shared__ __align__(8) uint64_t full[kDxS], empty[kDxS], acc_full, dx_full;
+  __shared__ uint32_t tslot;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int t0 = blockIdx.x * 128, c0 = blockIdx.y * kDxN;
+  const int ksteps = a.n_rank_pad / 64;
+  const int NK = a.nproj * ksteps;
+  const uint32_t s0 = smem_u32(smem);
+  const uint32_t stg = s0 + kDxS * kDxStage;
+  if (tid == 0) {
+    for (int i = 0; i < kDxS; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], 1);
+    }
+    mbar_init(&acc_full, 1);
+    mbar_init(&dx_full, 1);
+    fence_mbar_init();
+  }
+  if (warp == 0) tmem_alloc(&tslot, 256);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tslot;
+  bool bad = false;
+  if (warp == 0) {
+    if (lane == 0) {
+      // the dX tile to update, then the K loop operands
+      mbar_arrive_expect_tx(&dx_full, kDxStaging);
+      for (int q = 0; q < kDxN / 64; ++q) tma_load_2d(stg + q * kBlk, &a.tm_dx, c0 + q * 64, t0, &dx_full);
+      for (int i = 0; i < NK; ++i) {
+        const int s = i % kDxS, u = i / kDxS;
+        if (u >= 1 && !mbar_wait(&empty[s], (u - 1) & 1)) {
+          bad = true;
+          break;
+        }
+        const int j = i / ksteps, ks = i % ksteps;
+        const uint32_t base = s0 + s * kDxStage;
+        mbar_arrive_expect_tx(&full[s], kDxStage);
+        tma_load_2d(base, &a.tm_dhx, j * a.n_rank_pad + ks * 64, t0, &full[s]);
+        for (int q = 0; q < kDxN / 64; ++q)
+          tma_load_2d(base + kBlk + q * kHalfBlk, &a.tm_acat[j], c0 + q * 64, ks * 64, &full[s]);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(128, kDxN, 0, 1);
+      for (int i = 0; i < NK; ++i) {
+        const int s = i % kDxS;
+        if (!mbar_wait(&full[s], (i / kDxS) & 1)) {
+          bad = true;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t base = s0 + s * kDxStage;
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk)
+          tc_mma_bf16(tmem, sdesc_sw128(base + kk * 32, 16, 1024), sdesc_sw128(base + kBlk + kk * 2048, kHalfBlk, 1024),
+                      idesc, (i > 0 || kk > 0) ? 1u : 0u);
+        tc_commit(&empty[s]);
+      }
+      if (!bad) tc_commit(&acc_full);
+    }
+  } else {
+    const int et = tid - 64, quarter = warp & 3, ehalf = (warp - 2) >> 2;
+    const int m = quarter * 32 + lane;
+    const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
+    bool ok = mbar_wait(&dx_full, 0);
+    ok = ok && (NK == 0 || mbar_wait(&acc_full, 0));
+    ok = named_bar_and(kEpiBar, kEpiThreads, ok);
+    if (ok) {
+      tc_fence_after();
+      if (NK > 0) {
+#pragma unroll
+        for (int hq = 0; hq < 4; ++hq) {  // 4 x 32 columns of this warp half's 128
+          const int h = ehalf * 4 + hq;    // 32-column group 0..7
+          uint32_t r[32];
+          tmem_ld16(tmem + lane_base + h * 32, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
+          tmem_ld16(tmem + lane_base + h * 32 + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
+          tmem_ld_wait();
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const int chunk = h * 4 + q;  // 16-byte chunk 0..31 of the 256-column row
+            const uint32_t addr = stg + (chunk >> 3) * kBlk + sw128_off(m, chunk & 7);
+            const uint4 y = lds128(addr);
+            const uint32_t* dq = &r[q * 8];
+            const float2 f0 = unpack_bf16x2(y.x), f1 = unpack_bf16x2(y.y), f2 = unpack_bf16x2(y.z),
+                         f3 = unpack_bf16x2(y.w);
+            uint4 o;
+            o.x = pack_bf16x2(f0.x + __uint_as_float(dq[0]), f0.y + __uint_as_float(dq[1]));
+            o.y = pack_bf16x2(f1.x + __uint_as_float(dq[2]), f1.y + __uint_as_float(dq[3]));
+            o.z = pack_bf16x2(f2.x + __uint_as_float(dq[4]), f2.y + __uint_as_float(dq[5]));
+            o.w = pack_bf16x2(f3.x + __uint_as_float(dq[6]), f3.y + __uint_as_float(dq[7]));
+            sts128(addr, o);
+          }
+        }
+      }
+      named_bar(kEpiBar, kEpiThreads);
+#pragma unroll 4
+      for (int it = et; it < 128 * (kDxN / 8); it += kEpiThreads) {
+        const int row = it / (kDxN / 8), ch = it % (kDxN / 8), col = c0 + ch * 8;
+        if (t0 + row < a.T && col < a.d) {
+          const uint4 v = lds128(stg + (ch >> 3) * kBlk + sw128_off(row, ch & 7));
+          *reinterpret_cast<uint4*>(a.dX + (int64_t)(t0 + row) * a.d + col) = v;
+        }
+      }
+    }
+    if (!ok) bad = true;
+  }
+  __syncwarp();
+  tc_fence_before();
+  if (__syncthreads_or(bad) && tid == 0) atomicOr(a.err, kErrTimeout);
+  if (warp == 0) tmem_dealloc(tmem, 256);
+}
+
+// ------------------------------------------------------------------ dA
+constexpr int kDaN = 128;                              // d columns per CTA
+constexpr int kDaStage = 2 * kHalfBlk + (kDaN / 64) * kHalfBlk;  // dHx^T [64 t x 128 k] + X [64 t x 128 d]
+constexpr int kDaS = 6;
+constexpr int kDaSmem = kDaS * kDaStage + 1024;
+
+__global__ void __launch_bounds__(kThreads, 1) k_gemm_da(const __grid_constant__ DenseBwdLaunch a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  __shared__ __align__(8) uint64_t full[kDaS], empty[kDaS], acc_full;
+  __shared__ uint32_t tslot;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int m0 = blockIdx.x * 128;  // row of the stacked [nproj * n_rank_pad] rank dimension
+  const int c0 = blockIdx.y * kDaN;
+  const int NK = (a.T + 63) / 64;
+  const uint32_t s0 = smem_u32(smem);
+  if (tid == 0) {
+    for (int i = 0; i < kDaS; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], 1);
+    }
+    mbar_init(&acc_full, 1);
+    fence_mbar_init();
+  }
+  if (warp == 0) tmem_alloc(&tslot, 128);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tslot;
+  bool bad = false;
+  if (warp == 0) {
+    if (lane == 0) {
+      for (int i = 0; i < NK; ++i) {
+        const int s = i % kDaS, u = i / kDaS;
+        if (u >= 1 && !mbar_wait(&empty[s], (u - 1) & 1)) {
+          bad = true;
+          break;
+        }
+        const uint32_t base = s0 + s * kDaStage;
+        mbar_arrive_expect_tx(&full[s], kDaStage);
+        tma_load_2d(base, &a.tm_dhx_t, m0, i * 64, &full[s]);
+        tma_load_2d(base + kHalfBlk, &a.tm_dhx_t, m0 + 64, i * 64, &full[s]);
+        for (int q = 0; q < kDaN / 64; ++q)
+          tma_load_2d(base + 2 * kHalfBlk + q * kHalfBlk, &a.tm_x, c0 + q * 64, i * 64, &full[s]);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(128, kDaN, 1, 1);
+      for (int i = 0; i < NK; ++i) {
+        const int s = i % kDaS;
+        if (!mbar_wait(&full[s], (i / kDaS) & 1)) {
+          bad = true;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t base = s0 + s * kDaStage;
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk)
+          tc_mma_bf16(tmem, sdesc_sw128(base + kk * 2048, kHalfBlk, 1024),
+                      sdesc_sw128(base + 2 * kHalfBlk + kk * 2048, kHalfBlk, 1024), idesc, (i > 0 || kk > 0) ? 1u : 0u);
+        tc_commit(&empty[s]);
+      }
+      if (!bad) tc_commit(&acc_full);
+    }
+  } else {
+    const int quarter = warp & 3, ehalf = (warp - 2) >> 2;
+    const int m = quarter * 32 + lane;
+    const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
+    bool ok = NK == 0 || mbar_wait(&acc_full, 0);
+    ok = named_bar_and(kEpiBar, kEpiThreads, ok);
+    if (ok) {
+      tc_fence_after();
+      const int r = m0 + m, j = r / a.n_rank_pad, rr = r % a.n_rank_pad;
+      const bool live = j < a.nproj && rr < a.n_rank;
+      float* out = live ? a.dA[j] + (int64_t)rr * a.d : nullptr;
+#pragma unroll
+      for (int hq = 0; hq < 2; ++hq) {
+        const int h = ehalf * 2 + hq;  // 32-column group 0..3
+        uint32_t v[32];
+        tmem_ld16(tmem + lane_base + h * 32, *reinterpret_cast<uint32_t(*)[16]>(&v[0]));
+        tmem_ld16(tmem + lane_base + h * 32 + 16, *reinterpret_cast<uint32_t(*)[16]>(&v[16]));
+        tmem_ld_wait();
+        if (live) {
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            const int col = c0 + h * 32 + q * 4;
+            if (col < a.d)
+              *reinterpret_cast<float4*>(out + col) =
+                  NK == 0 ? make_float4(0.f, 0.f, 0.f, 0.f)
+                          : make_float4(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]),
+                                        __uint_as_float(v[4 * q + 2]), __uint_as_float(v[4 * q + 3]));
+          }
+        }
+      }
+    }
+    if (!ok) bad = true;
+  }
+  __syncwarp();
+  tc_fence_before();
+  if (__syncthreads_or(bad) && tid == 0) atomicOr(a.err, kErrTimeout);
+  if (warp == 0) tmem_dealloc(tmem, 128);
+}
+
+}  // namespace
+
+cudaError_t launch_dense_bwd(const DenseBwdLaunch& a, cudaStream_t st) {
+  if (a.T == 0) return cudaSuccess;
+  cudaError_t e = cudaFuncSetAttribute(k_gemm_dx, cudaFuncAttributeMaxDynamicSharedMemorySize, kDxSmem);
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(k_gemm_da, cudaFuncAttributeMaxDynamicSharedMemorySize, kDaSmem);
+  if (e != cudaSuccess) return e;
+  k_gemm_dx<<<dim3((a.T + 127) / 128, (a.d + kDxN - 1) / kDxN), kThreads, kDxSmem, st>>>(a);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  k_gemm_da<<<dim3(a.nproj * a.n_rank_pad / 128 + (a.nproj * a.n_rank_pad % 128 ? 1 : 0), (a.d + kDaN - 1) / kDaN),
+              kThreads, kDaSmem, st>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace ace

@@ -144,6 +144,7 @@ struct BwdLaunch {
   CUtensorMap tm_bt[2];    // Bt [n_rank, d_out], box 64 x rank_pad
   CUtensorMap tm_a;        // down: A [n_rank, d_in], box 64 x rank_pad
   CUtensorMap tm_dh;       // down: dHin [R, d_in], box 64 x 128
+  CUtensorMap tm_h;        // down: Hin [R, d_in], box 64 x 128
   const Tile* splits_row;  // row splits (the dY streaming kernel)
   const Tile* tiles_sh;    // unique-pair tiles (dH per unique pair)
   const int32_t* counts;
@@ -165,6 +166,7 @@ struct BwdLaunch {
   float* dA[2];
   float* dBt[2];
   float* part_dBt[2];    // deterministic dB^T partials [max_splits, rank_pad, d_out]
+  float* part_dA[2];     // deterministic dA partials (down) [max_splits, rank_pad, d_in]
   int32_t d_in, d_out, nproj, T;
   bool deterministic;
   int32_t* err;

@@ -82,6 +82,7 @@ struct BwdWs {
   uint16_t* dH[2];
   float* dHrow[2];
   float* part_dBt[2];
+  float* part_dA;
   uint16_t* dHx;
   size_t total;
 };
@@ -107,6 +108,8 @@ BwdWs bwd_layout(const PlanTables& pt, int32_t T, void* base) {
     w.part_dBt[j] = reinterpret_cast<float*>(b + off);
     off += pa;
   }
+  w.part_dA = reinterpret_cast<float*>(b + off);
+  off += pa;
   w.dHx = reinterpret_cast<uint16_t*>(b + off);
   off += align_up(2 * (size_t)T * 2 * n_rank_pad_of(pt), 256);
   w.total = off;
@@ -418,6 +421,7 @@ ace_status ace_bwd_row(const ace_plan* plan, const ace_perm* perm, const uint16_
   ok = ok && make_tmap_bf16(&a.tm_bt[0], Bt, nr, (uint64_t)plan->pt.d, plan->pt.rank_pad);
   ok = ok && make_tmap_bf16(&a.tm_a, A, nr, (uint64_t)plan->pt.f, plan->pt.rank_pad);
   ok = ok && make_tmap_bf16(&a.tm_dh, dHin, R, (uint64_t)plan->pt.f, kTileM);
+  ok = ok && make_tmap_bf16(&a.tm_h, Hin, R, (uint64_t)plan->pt.f, kTileM);
   if (perm->R > 0 && !ok) return fail(ACE_ERR_UNSUPPORTED, "tensor-map encoding failed for this layout");
   a.tm_dy[1] = a.tm_dy[0];
   a.tm_bt[1] = a.tm_bt[0];
@@ -440,6 +444,7 @@ ace_status ace_bwd_row(const ace_plan* plan, const ace_perm* perm, const uint16_
     a.dH[j] = w.dH[0];
     a.dHrow[j] = w.dHrow[0];
     a.part_dBt[j] = w.part_dBt[0];
+    a.part_dA[j] = w.part_dA;
   }
   a.s = s;
   a.dXin = dHin;

@@ -9,19 +9,18 @@
 //     dBt_c  = sum_i H_{u(row)}^T . dY_i  (TMEM, double-buffered per chunk)
 //   and the epilogue flushes each dBt chunk (fp32 atomics, or a per-split
 //   partial for the deterministic two-stage sum) while the next chunk runs.
-//   The epilogue then writes dH (scaled by s).  MODE_DOWN continues with
-//     dh_i += dH_i . A_g                  (dh tiles staged by TMA, added in
+//   The epilogue then writes dH (scaled by s).  MODE_DOWN continues over
+//   128-column chunks of the input h:
+//     dh_i  += dH_i . A_g                 (dh tiles staged by TMA, added in
 //                                          swizzled smem, coalesced stores)
+//     dA_c   = sum_i h_i^T . dH_i         (flushed like dB^T)
 //   For gate/up (MODE_SHARED) the rows of one unique pair (g, t) share H_u and
 //   dC_u . B_g = sum_rows dY_row . B_g, so streaming contiguous rows moves the
 //   bytes of the deduplicated form; dH per row goes to fp32 scratch.
 // k_dh_reduce: dH_u = sum of the dH rows of unique pair u (fixed slot order),
 //   written into the token-major dense dHx consumed by the dense dX / dA
 //   GEMMs of gemm.cu.
-// k_bwd_dA (down): one CTA per (group, 128-column chunk of f) streams all of
-//   the group's rows: dA_c^T = sum h_i^T . dH_i, stored directly
-//   (deterministic, no split-K).
-// k_splitk_reduce: deterministic stage 2 of dB^T (split order); empty groups
+// k_splitk_reduce: deterministic stage 2 of dB^T / dA (split order); empty groups
 //   -> exact zeros.
 #include <cstdint>
 
@@ -118,15 +117,16 @@ struct RowsCfg {
   static constexpr int NT = RP <= 32 ? 4 : (RP == 64 ? 2 : 1);
   static constexpr int kOps = Slots<RP>::bytes(NT);
   static constexpr int kWBlk = RP * 128;
-  static constexpr int kSlotA = 2 * kBlk + 2 * kWBlk;          // dY tile + B^T chunk (down phase 2: A chunk)
+  static constexpr int kSlotA = 2 * kBlk + 2 * kWBlk;  // dY tile + B^T chunk (down phase 2: A chunk + h tile)
   static constexpr int kSlotB = 2 * kBlk;                      // down: dh tile for the RMW
   static constexpr int SB = MODE == MODE_DOWN ? 2 : 0;
   static constexpr int kBudget = 220 * 1024;
   static constexpr int kSA0 = (kBudget - kOps - SB * kSlotB) / kSlotA;
   static constexpr int SA = kSA0 > 6 ? 6 : (kSA0 < 2 ? 2 : kSA0);
   static constexpr int kSmem = kOps + SA * kSlotA + SB * kSlotB + 1024;
-  static constexpr int kTB = 128;  // dB^T accumulators (2 x RP columns)
-  static constexpr int kDB = 256;  // down: dh D accumulators (2 x 128 columns)
+  static constexpr int kTB = 128;  // dB^T (phase 1) / dA (phase 2) accumulators, 2 x RP columns
+  static constexpr int ND = RP > 64 ? 1 : 2;            // down: dh D buffers of 128 columns
+  static constexpr int kDB = RP > 64 ? 384 : 256;
   static constexpr int kTmem = (MODE == MODE_DOWN || RP > 64) ? 512 : 256;
 };
 
@@ -139,7 +139,8 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   __shared__ __align__(8) uint64_t fullA[SA], emptyA[SA], fullB[SB], emptyB[SB];
-  __shared__ __align__(8) uint64_t dbt_full[2], dbt_empty[2], d_full[2], d_empty[2], dh_full, hs_ready;
+  __shared__ __align__(8) uint64_t dbt_full[2], dbt_empty[2], d_full[2], d_empty[2], da_full[2], da_empty[2];
+  __shared__ __align__(8) uint64_t dh_full, hs_ready;
   __shared__ uint32_t tslot;
   static_assert(NT * RP <= 128, "dH accumulators must fit below the dB^T columns");
 
@@ -172,6 +173,8 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
       mbar_init(&dbt_empty[i], 1);
       mbar_init(&d_full[i], 1);
       mbar_init(&d_empty[i], 1);
+      mbar_init(&da_full[i], 1);
+      mbar_init(&da_empty[i], 1);
     }
     mbar_init(&dh_full, 1);
     mbar_init(&hs_ready, 1);
@@ -219,9 +222,11 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
           tma_load_2d(base + 2 * kBlk + C::kWBlk, &a.tm_bt[proj], n0 + 64, r0, &fullA[s]);
         } else {
           const int j = q - NI1, c = j / ntiles, i = j % ntiles, n0 = c * kNcB, row0 = sp.start + i * kTileM;
-          mbar_arrive_expect_tx(&fullA[s], 2 * C::kWBlk);
+          mbar_arrive_expect_tx(&fullA[s], 2 * C::kWBlk + 2 * kBlk);
           tma_load_2d(base, &a.tm_a, n0, r0, &fullA[s]);
           tma_load_2d(base + C::kWBlk, &a.tm_a, n0 + 64, r0, &fullA[s]);
+          tma_load_2d(base + 2 * C::kWBlk, &a.tm_h, n0, row0, &fullA[s]);
+          tma_load_2d(base + 2 * C::kWBlk + kBlk, &a.tm_h, n0 + 64, row0, &fullA[s]);
           const int sb = j % SB, ub = j / SB;
           if (ub >= 1 && !mbar_wait(&emptyB[sb], (ub - 1) & 1)) {
             bad = true;
@@ -268,12 +273,17 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
         constexpr uint32_t id_d = idesc_bf16_f32(128, kNcB, 0, 1);
         if (!mbar_wait(&hs_ready, 0)) bad = true;
         for (int j = 0; j < NI2 && !bad; ++j) {
-          const int q = NI1 + j, i = j % ntiles, s = q % SA, u = q / SA, b = j & 1;
+          const int q = NI1 + j, c = j / ntiles, i = j % ntiles, s = q % SA, u = q / SA;
+          const int b = j % C::ND;
           if (!mbar_wait(&fullA[s], u & 1)) {
             bad = true;
             break;
           }
-          if (j >= 2 && !mbar_wait(&d_empty[b], ((j - 2) >> 1) & 1)) {
+          if (j >= C::ND && !mbar_wait(&d_empty[b], ((j - C::ND) / C::ND) & 1)) {
+            bad = true;
+            break;
+          }
+          if (i == 0 && c >= 2 && !mbar_wait(&da_empty[c & 1], ((c - 2) >> 1) & 1)) {
             bad = true;
             break;
           }
@@ -283,8 +293,13 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
           for (int kk = 0; kk < RP / 16; ++kk)  // dh chunk = dH_i . A_g chunk
             tc_mma_bf16(tmem + C::kDB + b * kNcB, SL::desc_k(sOps, i, kk),
                         sdesc_sw128(base + kk * 2048, C::kWBlk, 1024), id_d, kk > 0 ? 1u : 0u);
+#pragma unroll
+          for (int kk = 0; kk < kTileM / 16; ++kk)  // dA_c^T += h_i^T . dH_i
+            tc_mma_bf16(tmem + C::kTB + (c & 1) * RP, sdesc_sw128(base + 2 * C::kWBlk + kk * 2048, kBlk, 1024),
+                        SL::desc_mn(sOps, i, kk), id_w, (i > 0 || kk > 0) ? 1u : 0u);
           tc_commit(&emptyA[s]);
           tc_commit(&d_full[b]);
+          if (i == ntiles - 1) tc_commit(&da_full[c & 1]);
         }
       }
     }
@@ -348,9 +363,9 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
     }
     if (MODE == MODE_DOWN) {
       for (int j = 0; j < NI2 && ok; ++j) {
-        const int c = j / ntiles, i = j % ntiles, b = j & 1, sb = j % SB, n0 = c * kNcB;
+        const int c = j / ntiles, i = j % ntiles, b = j % C::ND, sb = j % SB, n0 = c * kNcB;
         bool w_ok = mbar_wait(&fullB[sb], (j / SB) & 1);
-        w_ok = w_ok && mbar_wait(&d_full[b], (j >> 1) & 1);
+        w_ok = w_ok && mbar_wait(&d_full[b], (j / C::ND) & 1);
         ok = named_bar_and(kEpiBar, kEpiThreads, w_ok);
         if (!ok) break;
         tc_fence_after();
@@ -393,6 +408,16 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
         fence_proxy_async_smem();
         named_bar(kEpiBar, kEpiThreads);
         if (et == 0) mbar_arrive(&emptyB[sb]);
+        if (i == ntiles - 1) {  // dA chunk c of this split is complete
+          ok = named_bar_and(kEpiBar, kEpiThreads, mbar_wait(&da_full[c & 1], (c >> 1) & 1));
+          if (!ok) break;
+          tc_fence_after();
+          flush_wgrad<RP>(tmem + lane_base + C::kTB + (c & 1) * RP, n0, d_in, rg, r0, 1.f, fmode, a.part_dA[proj],
+                          sp.id, a.dA[proj], m, false, ehalf * 16, 32);
+          tc_fence_before();
+          named_bar(kEpiBar, kEpiThreads);
+          if (et == 0) mbar_arrive(&da_empty[c & 1]);
+        }
       }
     }
     if (!ok) bad = true;
@@ -448,120 +473,6 @@ __global__ void __launch_bounds__(128) k_dh_reduce(const __grid_constant__ PlanT
   }
 }
 
-// ---------------------------------------------------------------- dA
-template <int RP, int NPROJ>
-struct DaCfg {
-  static constexpr int kOp = Slots<RP>::bytes(NPROJ);     // dH tile(s) of one row tile
-  static constexpr int kStage = kTileM * 256 + kOp;       // X / h chunk [128 x 128] + dH
-  static constexpr int kS0 = (220 * 1024) / kStage;
-  static constexpr int S = kS0 > 4 ? 4 : kS0;             // >= 2 for every rank_pad
-  static constexpr int kSmem = S * kStage + 1024;
-  static constexpr int kTmem = NPROJ * RP <= 32 ? 32 : NPROJ * RP <= 64 ? 64 : NPROJ * RP <= 128 ? 128 : 256;
-};
-
-// grid (G, ceil(d_in / 128)); MODE_SHARED: rows are unique pairs (X gathered
-// by token, dH per unique pair); MODE_DOWN: rows are routed rows (h, dH per row).
-template <int RP, int NPROJ, int MODE>
-__global__ void __launch_bounds__(128, 1) k_bwd_dA(const __grid_constant__ PlanTables pt,
-                                                   const __grid_constant__ BwdLaunch a) {
-  using C = DaCfg<RP, NPROJ>;
-  using SL = Slots<RP>;
-  constexpr int kDaStages = C::S;
-  static_assert(kDaStages >= 2, "dA pipeline needs two stages");
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  __shared__ __align__(8) uint64_t bar[kDaStages];
-  __shared__ uint32_t tslot;
-  const int g = blockIdx.x, c0 = blockIdx.y * kNcB;
-  const int tid = threadIdx.x, warp = tid >> 5;
-  const int r0 = pt.rank_off[g], rg = pt.rank_off[g + 1] - r0;
-  const int d = a.d_in;
-  const int lo = MODE == MODE_SHARED ? a.uniq_off[g] : a.group_off[g];
-  const int n = (MODE == MODE_SHARED ? a.uniq_off[g + 1] : a.group_off[g + 1]) - lo;
-  const int NI = (n + kTileM - 1) / kTileM;
-  const uint32_t stage0 = smem_u32(smem);
-  if (tid == 0) {
-    for (int i = 0; i < kDaStages; ++i) mbar_init(&bar[i], 1);
-    fence_mbar_init();
-  }
-  if (warp == 0) tmem_alloc(&tslot, C::kTmem);
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem = tslot;
-  const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
-  auto load = [&](int it, int slot) {
-    const uint32_t st = stage0 + slot * C::kStage;
-    const int item = lo + it * kTileM + tid;  // this thread's row of the tile
-    const bool live = it * kTileM + tid < n;
-    // dH row(s) of this row (all projections)
-#pragma unroll
-    for (int j = 0; j < NPROJ; ++j)
-#pragma unroll
-      for (int c8 = 0; c8 < RP; c8 += 8)
-        cp_async16(st + kTileM * 256 + SL::elem(j, tid, c8), live ? a.dH[j] + (int64_t)item * RP + c8 : a.dH[0],
-                   live);
-    // input chunk [128 rows x 128 cols]; element (m, cc) belongs to tile row m
-#pragma unroll
-    for (int q = 0; q < 16; ++q) {
-      const int idx = q * 128 + tid, m = idx >> 4, cc = idx & 15, col = c0 + cc * 8;
-      const int rr = it * kTileM + m;
-      const bool v = rr < n && col < d;
-      int64_t src_row = 0;
-      if (v) src_row = MODE == MODE_SHARED ? a.uniq_tok[lo + rr] : lo + rr;
-      cp_async16(st + tile_off(kTileM, m, cc), v ? a.Xin + src_row * d + col : a.Xin, v);
-    }
-  };
-  constexpr uint32_t id_w = idesc_bf16_f32(128, RP, 1, 1);
-#pragma unroll
-  for (int j = 0; j < kDaStages - 1; ++j) {
-    if (j < NI) load(j, j);
-    cp_async_commit();
-  }
-  bool bad = false, aborted = false;
-  for (int it = 0; it < NI; ++it) {
-    const int slot = it % kDaStages;
-    cp_async_wait<kDaStages - 2>();
-    fence_proxy_async_smem();
-    if (__syncthreads_or(bad)) {
-      aborted = true;
-      break;
-    }
-    if (tid == 0) {
-      tc_fence_after();
-      const uint32_t st = stage0 + slot * C::kStage;
-#pragma unroll
-      for (int j = 0; j < NPROJ; ++j)
-#pragma unroll
-        for (int kk = 0; kk < kTileM / 16; ++kk)  // dA_c^T += X^T . dH
-          tc_mma_bf16(tmem + j * RP, sdesc_sw128(st + kk * 2048, kBlk, 1024), SL::desc_mn(st + kTileM * 256, j, kk),
-                      id_w, (it > 0 || kk > 0) ? 1u : 0u);
-      tc_commit(&bar[slot]);
-    }
-    const int nxt = it + kDaStages - 1;
-    if (nxt < NI) {
-      if (it >= 1 && !mbar_wait(&bar[(it - 1) % kDaStages], ((it - 1) / kDaStages) & 1)) bad = true;
-      if (!bad) load(nxt, nxt % kDaStages);
-    }
-    cp_async_commit();
-  }
-  cp_async_wait<0>();
-  if (NI > 0 && !aborted && !bad && !mbar_wait(&bar[(NI - 1) % kDaStages], ((NI - 1) / kDaStages) & 1)) bad = true;
-  tc_fence_before();
-  aborted = __syncthreads_or(bad || aborted);
-  tc_fence_after();
-  if (!aborted) {
-    // the chunk is complete: store it (a group without rows gets zeros)
-    for (int j = 0; j < NPROJ; ++j)
-      flush_wgrad<RP>(tmem + lane_base + j * RP, c0, d, rg, r0, 1.f, kStore, nullptr, 0, a.dA[j], tid, NI == 0);
-  } else if (tid == 0) {
-    atomicOr(a.err, kErrTimeout);
-  }
-  tc_fence_before();
-  __syncthreads();
-  if (warp == 0) tmem_dealloc(tmem, C::kTmem);
-}
-
 // ---------------------------------------------------------------- stage 2
 __global__ void __launch_bounds__(256) k_splitk_reduce(const __grid_constant__ PlanTables pt,
                                                        const Tile* __restrict__ splits,
@@ -603,16 +514,6 @@ cudaError_t launch_rows(const PlanTables& pt, const BwdLaunch& a, int nproj, cud
   return cudaGetLastError();
 }
 
-template <int RP, int NPROJ, int MODE>
-cudaError_t launch_da(const PlanTables& pt, const BwdLaunch& a, cudaStream_t st) {
-  using C = DaCfg<RP, NPROJ>;
-  auto kern = k_bwd_dA<RP, NPROJ, MODE>;
-  cudaError_t e = set_smem(kern, C::kSmem);
-  if (e != cudaSuccess) return e;
-  kern<<<dim3(pt.G, (a.d_in + kNcB - 1) / kNcB), 128, C::kSmem, st>>>(pt, a);
-  return cudaGetLastError();
-}
-
 template <int RP>
 cudaError_t launch_bwd_t(const PlanTables& pt, const BwdLaunch& a, bool shared, cudaStream_t st) {
   cudaError_t e;
@@ -623,8 +524,10 @@ cudaError_t launch_bwd_t(const PlanTables& pt, const BwdLaunch& a, bool shared, 
       if ((e = cudaMemsetAsync(a.dBt[j], 0, sizeof(float) * (size_t)n_rank * a.d_out, st)) != cudaSuccess) return e;
   }
   if (!shared) {
+    if (!a.deterministic &&
+        (e = cudaMemsetAsync(a.dA[0], 0, sizeof(float) * (size_t)n_rank * a.d_in, st)) != cudaSuccess)
+      return e;
     if ((e = launch_rows<RP, MODE_DOWN>(pt, a, 1, st)) != cudaSuccess) return e;
-    if ((e = launch_da<RP, 1, MODE_DOWN>(pt, a, st)) != cudaSuccess) return e;
   } else {
     if ((e = launch_rows<RP, MODE_SHARED>(pt, a, nproj, st)) != cudaSuccess) return e;
     const size_t dhx = sizeof(uint16_t) * (size_t)a.T * nproj * a.n_rank_pad;
@@ -637,6 +540,12 @@ cudaError_t launch_bwd_t(const PlanTables& pt, const BwdLaunch& a, bool shared, 
       dim3 grid(n_rank, (a.d_out / 4 + 255) / 256);
       k_splitk_reduce<<<grid, 256, 0, st>>>(pt, a.splits_row, a.counts, kCntSplitsRow, a.part_dBt[j], RP, a.d_out,
                                             a.dBt[j]);
+      if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
+    if (!shared) {
+      dim3 grid(n_rank, (a.d_in / 4 + 255) / 256);
+      k_splitk_reduce<<<grid, 256, 0, st>>>(pt, a.splits_row, a.counts, kCntSplitsRow, a.part_dA[0], RP, a.d_in,
+                                            a.dA[0]);
       if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
   }

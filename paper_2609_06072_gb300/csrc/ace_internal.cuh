@@ -159,7 +159,6 @@ struct BwdLaunch {
   const float* H[2];     // saved H (gate/up: per unique pair; down: per row), stride rank_max
   float s;
   uint16_t* dXin;        // down: dHin [R, f] in/out
-  uint16_t* dH[2];       // scratch: bf16 dH per row [R, rank_pad] (down)
   uint16_t* dHx;         // scratch: token-major dense dH [T, nproj * n_rank_pad] (gate/up)
   int32_t n_rank_pad;    // n_rank rounded up to a multiple of 64
   float* dHrow[2];       // scratch: fp32 dH per row [R, rank_pad] (gate/up)

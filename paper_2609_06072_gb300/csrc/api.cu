@@ -79,7 +79,6 @@ ace_status check_perm(const ace_plan* plan, const ace_perm* perm) {
 }
 
 struct BwdWs {
-  uint16_t* dH[2];
   float* dHrow[2];
   float* part_dBt[2];
   float* part_dA;
@@ -89,20 +88,18 @@ struct BwdWs {
 
 int n_rank_pad_of(const PlanTables& pt) { return (pt.rank_off[pt.G] + 63) / 64 * 64; }
 
-// Backward scratch per projection: dH per unique pair / row (bf16), dH per
-// row (fp32) and the deterministic dB^T split-K partials.
+// Backward scratch: dH per row (fp32, per projection), the deterministic
+// split-K partials of dB^T (per projection) and dA (down), and the
+// token-major dense dH of gate/up (bf16).
 BwdWs bwd_layout(const PlanTables& pt, int32_t T, void* base) {
   const PermLayout L = perm_layout(pt, T);
   const int64_t R = (int64_t)T * pt.k;
-  const size_t dh = align_up(2 * (size_t)R * pt.rank_pad, 256);
   const size_t dhrow = align_up(4 * (size_t)R * pt.rank_pad, 256);
   const size_t pa = align_up(4 * (size_t)L.max_splits * pt.rank_pad * (size_t)(pt.d > pt.f ? pt.d : pt.f), 256);
   BwdWs w{};
   char* b = static_cast<char*>(base);
   size_t off = 0;
   for (int j = 0; j < 2; ++j) {
-    w.dH[j] = reinterpret_cast<uint16_t*>(b + off);
-    off += dh;
     w.dHrow[j] = reinterpret_cast<float*>(b + off);
     off += dhrow;
     w.part_dBt[j] = reinterpret_cast<float*>(b + off);
@@ -361,7 +358,6 @@ ace_status ace_bwd_shared(const ace_plan* plan, const ace_perm* perm, int32_t np
     a.H[j] = H[jj];
     a.dA[j] = dA[jj];
     a.dBt[j] = dBt[jj];
-    a.dH[j] = w.dH[jj];
     a.dHrow[j] = w.dHrow[jj];
     a.part_dBt[j] = w.part_dBt[jj];
   }
@@ -441,7 +437,6 @@ ace_status ace_bwd_row(const ace_plan* plan, const ace_perm* perm, const uint16_
     a.H[j] = H;
     a.dA[j] = dA;
     a.dBt[j] = dBt;
-    a.dH[j] = w.dH[0];
     a.dHrow[j] = w.dHrow[0];
     a.part_dBt[j] = w.part_dBt[0];
     a.part_dA[j] = w.part_dA;
@@ -493,3 +488,4 @@ ace_status ace_get_error(const ace_perm* perm, void* stream) {
 }
 
 }  // extern "C"
+

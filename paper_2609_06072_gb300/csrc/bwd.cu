@@ -325,7 +325,7 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
     if (ok) ok = named_bar_and(kEpiBar, kEpiThreads, mbar_wait(&dh_full, 0));
     if (ok) {
       tc_fence_after();
-      // dH (scaled by s): gate/up -> fp32 per row; down -> bf16 operand slots + bf16 per row
+      // dH (scaled by s): gate/up -> fp32 per row; down -> bf16 operand slots
       for (int i = 0; i < ntiles; ++i) {
         const bool live = i * kTileM + m < sp.cnt;
         const int64_t row = sp.start + i * kTileM + m;
@@ -345,14 +345,8 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
               for (int q = 0; q < 4; ++q) dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
             }
           } else {
-            const uint4 w0 = pack8(v), w1 = pack8(v + 8);
-            sts128(sOps + SL::elem(i, m, c0), w0);
-            sts128(sOps + SL::elem(i, m, c0 + 8), w1);
-            if (live) {
-              uint4* dst = reinterpret_cast<uint4*>(a.dH[0] + row * RP + c0);
-              dst[0] = w0;
-              dst[1] = w1;
-            }
+            sts128(sOps + SL::elem(i, m, c0), pack8(v));
+            sts128(sOps + SL::elem(i, m, c0 + 8), pack8(v + 8));
           }
         }
       }

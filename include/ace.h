@@ -153,6 +153,24 @@ ace_status ace_fwd_shared(const ace_plan* plan, const ace_perm* perm, const uint
                           const uint16_t* const* A, const uint16_t* const* Bt, float s, uint16_t* const* Y,
                           float* const* H, void* ws, size_t ws_bytes, void* stream);
 
+/* Allocation-free variant of ace_fwd_shared for callers that cannot
+ * allocate device memory (an inference server or plug-in host that reserves
+ * the device memory for its own pool up front and gives a plug-in neither an
+ * allocator nor a workspace).  The paper has no counterpart: this is a
+ * deployment convenience.  Same arguments as ace_fwd_shared without H and
+ * without the workspace: H is not returned, and the scratch it needs (2 x
+ * T*k x rank_max fp32) lives in a 32 MiB array inside the library that every
+ * GPU loading the library holds until the process exits.  Larger sizes fail
+ * with ACE_ERR_WORKSPACE and launch nothing.  The first call on a device
+ * looks up the array's device address (make it before any stream capture).
+ * All calls share the array: calls that overlap on the GPU race, so issue
+ * them on one stream or otherwise order them.  Nothing in the array has to
+ * start at zero: each call writes every scratch word it reads before reading
+ * it.  Nothing is allocated. */
+ace_status ace_fwd_shared_noalloc(const ace_plan* plan, const ace_perm* perm, const uint16_t* X, int32_t nproj,
+                                  const uint16_t* const* A, const uint16_t* const* Bt, float s, uint16_t* const* Y,
+                                  void* stream);
+
 /* Forward, per row (down).
  *   Hin  [R, f] bf16 expert-specific inputs h_e in row order
  *   A    [rank_off[G], f] bf16 (A_g);  Bt [rank_off[G], d] bf16 (B_g^T)

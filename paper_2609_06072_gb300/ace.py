@@ -31,7 +31,8 @@ STATUS_NAMES = {0: "ACE_OK", 1: "ACE_ERR_ARG", 2: "ACE_ERR_SHAPE", 3: "ACE_ERR_W
                 5: "ACE_ERR_UNSUPPORTED", 6: "ACE_ERR_CUDA", 7: "ACE_ERR_DEVICE_TIMEOUT"}
 
 EXPORTED = ["ace_version", "ace_last_error_message", "ace_plan_create", "ace_plan_destroy", "ace_plan_rank_max",
-            "ace_workspace_size", "ace_permute", "ace_fwd_shared", "ace_fwd_row", "ace_bwd_shared", "ace_bwd_row",
+            "ace_workspace_size", "ace_permute", "ace_fwd_shared", "ace_fwd_shared_noalloc", "ace_fwd_row",
+            "ace_bwd_shared", "ace_bwd_row",
             "ace_gather_rows", "ace_scatter_rows", "ace_get_error"]
 
 
@@ -88,6 +89,8 @@ def load(build_if_missing: bool = False) -> ctypes.CDLL:
     lib.ace_permute.argtypes = [vp, vp, i32, vp, sz, ctypes.POINTER(ace_perm), vp]
     lib.ace_fwd_shared.restype = i32
     lib.ace_fwd_shared.argtypes = [vp, ctypes.POINTER(ace_perm), vp, i32, vp, vp, ctypes.c_float, vp, vp, vp, sz, vp]
+    lib.ace_fwd_shared_noalloc.restype = i32
+    lib.ace_fwd_shared_noalloc.argtypes = [vp, ctypes.POINTER(ace_perm), vp, i32, vp, vp, ctypes.c_float, vp, vp]
     lib.ace_fwd_row.restype = i32
     lib.ace_fwd_row.argtypes = [vp, ctypes.POINTER(ace_perm), vp, vp, vp, ctypes.c_float, vp, vp, vp, sz, vp]
     lib.ace_bwd_shared.restype = i32
@@ -199,6 +202,14 @@ class Plan:
                                        _arr([_ptr(y, torch.bfloat16, "Y") for y in Y]), Hp,
                                        _ptr(ws) if ws is not None else None, 0 if ws is None else ws.numel(),
                                        _stream(stream)), "ace_fwd_shared")
+
+    def fwd_shared_noalloc(self, perm: Perm, X, A, Bt, s, Y, stream=None):
+        """ace_fwd_shared_noalloc: no H output, scratch inside the library."""
+        _check(self.lib.ace_fwd_shared_noalloc(self.h, ctypes.byref(perm.c), _ptr(X, torch.bfloat16, "X"), len(A),
+                                               _arr([_ptr(a, torch.bfloat16, "A") for a in A]),
+                                               _arr([_ptr(b, torch.bfloat16, "Bt") for b in Bt]), float(s),
+                                               _arr([_ptr(y, torch.bfloat16, "Y") for y in Y]), _stream(stream)),
+               "ace_fwd_shared_noalloc")
 
     def fwd_row(self, perm: Perm, Hin, A, Bt, s, Y, H=None, ws=None, stream=None):
         _check(self.lib.ace_fwd_row(self.h, ctypes.byref(perm.c), _ptr(Hin, torch.bfloat16, "Hin"),

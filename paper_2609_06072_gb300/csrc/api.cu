@@ -4,6 +4,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <mutex>
 #include <new>
 
 #include "ace_internal.cuh"
@@ -489,3 +490,50 @@ ace_status ace_get_error(const ace_perm* perm, void* stream) {
 
 }  // extern "C"
 
+// ---------------------------------------------------------------------------
+// Allocation-free forward (gate/up).  Some callers cannot allocate device
+// memory: an inference server or a plug-in host that reserves the device
+// memory for its own pool up front and hands a plug-in no allocator and no
+// workspace.  For them the shared-input forward keeps its scratch (H per
+// unique pair, both projections) in this file-scope array instead of a
+// caller workspace.  Every GPU that loads the library holds the array until
+// the process exits.  Calls that overlap on the GPU share it and race.  No
+// word of it has to start at zero: the first kernel of a call writes every H
+// word the second one reads.
+namespace {
+constexpr size_t kNoAllocScratchBytes = size_t(32) << 20;  // 32 MiB
+__device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+constexpr int kNoAllocMaxDevices = 64;
+std::mutex g_noalloc_mu;
+void* g_noalloc_ptr[kNoAllocMaxDevices] = {};
+}  // namespace
+
+extern "C" ace_status ace_fwd_shared_noalloc(const ace_plan* plan, const ace_perm* perm, const uint16_t* X,
+                                             int32_t nproj, const uint16_t* const* A, const uint16_t* const* Bt,
+                                             float s, uint16_t* const* Y, void* stream) {
+  ace_status st = check_perm(plan, perm);
+  if (st != ACE_OK) return st;
+  const size_t need = 2 * align_up(4 * (size_t)perm->R * plan->pt.rank_max, 256);
+  if (need > kNoAllocScratchBytes)
+    return fail(ACE_ERR_WORKSPACE,
+                "ace_fwd_shared_noalloc needs %zu bytes of scratch (T*k*rank_max too large); the static limit is %zu",
+                need, kNoAllocScratchBytes);
+  int dev = 0;
+  cudaError_t ce = cudaGetDevice(&dev);
+  if (ce != cudaSuccess) return cuda_status(ce, "cudaGetDevice");
+  if (dev != plan->device) return fail(ACE_ERR_ARG, "current device %d is not the plan's device %d", dev, plan->device);
+  if (dev < 0 || dev >= kNoAllocMaxDevices) return fail(ACE_ERR_UNSUPPORTED, "device index %d too large", dev);
+  void* scratch = nullptr;
+  {
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    if (!g_noalloc_ptr[dev]) {
+      // once per device, with that device current: the device address of the array
+      void* p = nullptr;
+      ce = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+      if (ce != cudaSuccess) return cuda_status(ce, "cudaGetSymbolAddress");
+      g_noalloc_ptr[dev] = p;
+    }
+    scratch = g_noalloc_ptr[dev];
+  }
+  return ace_fwd_shared(plan, perm, X, nproj, A, Bt, s, Y, nullptr, scratch, kNoAllocScratchBytes, stream);
+}

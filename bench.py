@@ -229,7 +229,82 @@ class Layer:
         return sum(t.numel() * t.element_size() for t in self.h_grads)
 
 
+class NvmlSampler:
+    """Reads the SM clock and the clock-event reasons of one GPU through NVML
+    every few milliseconds on a host thread (read-only queries), so that a
+    short timed region still gets many samples.  Silently inactive when the
+    NVML library or the device cannot be found."""
+    # nvmlClocksEventReasons bits (nvml.h)
+    BITS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown", 0x40: "hw_thermal_slowdown",
+            0x80: "hw_power_brake_slowdown"}
+
+    def __init__(self, props, period_s=0.002):
+        import ctypes
+        import threading
+        self.ct, self.period, self.samples, self.stop_ev = ctypes, period_s, [], threading.Event()
+        self.thread, self.lib, self.dev, self.max_mhz = None, None, None, None
+        try:
+            lib = ctypes.CDLL("libnvidia-ml.so.1")
+            if lib.nvmlInit_v2() != 0:
+                return
+            dev = ctypes.c_void_p()
+            bus = f"{props.pci_domain_id:08x}:{props.pci_bus_id:02x}:{props.pci_device_id:02x}.0".encode()
+            if lib.nvmlDeviceGetHandleByUUID(("GPU-" + str(props.uuid)).encode(), ctypes.byref(dev)) != 0 and \
+                    lib.nvmlDeviceGetHandleByPciBusId_v2(bus, ctypes.byref(dev)) != 0:
+                return
+            mx = ctypes.c_uint()
+            if lib.nvmlDeviceGetMaxClockInfo(dev, 1, ctypes.byref(mx)) == 0:  # 1 = NVML_CLOCK_SM
+                self.max_mhz = float(mx.value)
+            self.reasons_fn = getattr(lib, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+                getattr(lib, "nvmlDeviceGetCurrentClocksThrottleReasons")
+            self.lib, self.dev = lib, dev
+        except (OSError, AttributeError):
+            self.lib = None
+
+    def _run(self):
+        ct = self.ct
+        mhz, mask = ct.c_uint(), ct.c_ulonglong()
+        while not self.stop_ev.is_set():
+            if self.lib.nvmlDeviceGetClockInfo(self.dev, 1, ct.byref(mhz)) == 0 and \
+                    self.reasons_fn(self.dev, ct.byref(mask)) == 0:
+                self.samples.append((float(mhz.value), int(mask.value)))
+            self.stop_ev.wait(self.period)
+
+    def start(self):
+        import threading
+        if self.lib is not None:
+            self.thread = threading.Thread(target=self._run, daemon=True)
+            self.thread.start()
+
+    def stop(self):
+        if self.thread is None:
+            return None
+        self.stop_ev.set()
+        self.thread.join()
+        if not self.samples:
+            return None
+        reasons = sorted({n for _, m in self.samples for bit, n in self.BITS.items() if m & bit})
+        return {"sm_mhz": statistics.median(v for v, _ in self.samples), "sm_max_mhz": self.max_mhz,
+                "reasons": reasons, "samples": len(self.samples), "source": "nvml"}
+
+
+def merge_clocks(nvml, smi):
+    """NVML samples (many) when present, nvidia-smi ones otherwise; reasons of both."""
+    if nvml is None and smi is None:
+        return None
+    out = dict(nvml or smi)
+    if nvml and smi:
+        out["reasons"] = sorted(set(nvml["reasons"]) | set(smi["reasons"]))
+        out["nvidia_smi"] = {k: smi[k] for k in ("sm_mhz", "sm_max_mhz", "samples")}
+    out.setdefault("source", "nvidia-smi")
+    return out
+
+
 CALLS = ["permute", "fwd_shared", "fwd_row", "bwd_row", "bwd_shared"]
+# calls that launch exactly one kernel of ours: their CUDA-event span is that
+# kernel's duration (the fast-mode down backward adds two memsets of the fp32
+# weight gradients, about 0.5% of its bytes)
+SINGLE_KERNEL = {"fwd_row": "k_fwd_rows<down>", "bwd_row": "k_bwd_rows<down>"}
 
 
 def run_gpu(args, rank, world, local):
@@ -255,14 +330,16 @@ def run_gpu(args, rank, world, local):
         torch.distributed.barrier()
     torch.cuda.synchronize()
     clk = ClockSampler(local)
+    nv = NvmlSampler(torch.cuda.get_device_properties(local))
     clk.start()
+    nv.start()
     t_wall0 = time.perf_counter()
     for i in range(args.steps):
         flush.zero_()  # L2 flush between timed steps (outside the event pair)
         lay.step(evs[i])
     torch.cuda.synchronize()
     t_wall = time.perf_counter() - t_wall0
-    clocks = clk.stop()
+    clocks = merge_clocks(nv.stop(), clk.stop())
     per_call = {n: [] for n in CALLS}
     step_ms = []
     for e in evs:
@@ -303,7 +380,9 @@ def run_gpu(args, rank, world, local):
 
     peaks = load_peaks()
     call_ms = {n: float(np.mean(v)) for n, v in per_call.items()}
-    dom = max(CALLS, key=lambda n: call_ms[n])
+    # dominant kernel: the slowest of the single-kernel calls (the launch list
+    # under profiles/ shows it is also the top kernel of the step)
+    dom = max(SINGLE_KERNEL, key=lambda n: call_ms[n])
     achieved = bytes_[dom] / (call_ms[dom] * 1e-3) / 1e9
     traffic = None
     tf = os.path.join(ROOT, "profiles", "traffic.json")
@@ -325,7 +404,7 @@ def run_gpu(args, rank, world, local):
                    "rows_per_step": c.R, "U": int(P["U"]), "deterministic": bool(args.det),
                    "l2": "flushed between timed steps (256 MB write outside the event pair)",
                    "parallelism": f"replicas x{world}"},
-        "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peaks["hbm_gbs"],
+        "roofline": {"bound": "hbm", "kernel": SINGLE_KERNEL[dom], "call": dom, "achieved": achieved, "peak": peaks["hbm_gbs"],
                      "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"], "traffic": traffic,
                      "algorithmic_bytes": bytes_[dom], "peak_source": peaks["source"]},
         "step_roofline": {"algorithmic_bytes": total_bytes, "algorithmic_flops": total_flops,
@@ -360,6 +439,7 @@ def oracle_sample(cfg_name, seed, expertwise, frac, rng_seed=0):
     sel_p = np.sort(rng.choice(c.R, n_p, replace=False)).astype(np.int32)
     sel_t = np.sort(rng.choice(c.T, n_t, replace=False)).astype(np.int32)
     sel_r = np.sort(rng.choice(int(L.rank_off[-1]), n_r, replace=False)).astype(np.int32)
+    _ = (L.topk_idx, L.e2g, L.G)
     ins = {"X": L.X(), "h": L.h(), "dY": {p: L.dY(p) for p in ("gate", "up", "down")},
            "A": {p: L.A(p) for p in ("gate", "up", "down")}, "Bt": {p: L.Bt(p) for p in ("gate", "up", "down")}}
     t0 = time.perf_counter()
@@ -386,16 +466,32 @@ def cpu_cores():
         return os.cpu_count() or 1
 
 
+def calibrate_fraction(cfg_name, seed, expertwise, target_s):
+    """Sample fraction whose oracle time is about target_s: the time of a
+    sample is a fixed part (permutations, per-call setup) plus a part linear
+    in the fraction, so two short probes fix both."""
+    f1, f2 = 1.0 / 1024, 1.0 / 256
+    t1, _ = oracle_sample(cfg_name, seed, expertwise, f1)
+    t2, _ = oracle_sample(cfg_name, seed, expertwise, f2)
+    slope = max((t2 - t1) / (f2 - f1), 1e-6)
+    fixed = max(t1 - slope * f1, 0.0)
+    return float(min(1.0, max(f1, (target_s - fixed) / slope)))
+
+
 def cpu_baseline(cfg_name, seed, expertwise, target_s):
     """Calibrate a sample fraction to ~target_s seconds of oracle work, then time it."""
     os.environ.setdefault("OMP_NUM_THREADS", str(cpu_cores()))
-    frac = 1.0 / 512
-    dt, _ = oracle_sample(cfg_name, seed, expertwise, frac)
-    frac = min(1.0, frac * target_s / max(dt, 1e-3))
+    frac = calibrate_fraction(cfg_name, seed, expertwise, target_s)
     dt, rows = oracle_sample(cfg_name, seed, expertwise, frac)
+    reps = 1
+    while frac >= 1.0 and dt < 0.75 * target_s and reps < 16:  # whole steps are short: time several
+        t, r = oracle_sample(cfg_name, seed, expertwise, frac, rng_seed=reps)
+        dt, rows, reps = dt + t, rows + r, reps + 1
+    what = (f"{reps} whole step(s) (permutation, forward, dX/dh, dA, dB^T of all 3 projections)" if frac >= 1.0 else
+            f"one step's permutation plus {frac:.4f} of its pairs (forward, dX/dh) and of its rank rows "
+            f"(dA, dB^T), all 3 projections")
     return {"value": rows / dt, "unit": UNIT, "cores": int(os.environ["OMP_NUM_THREADS"]), "kind": "oracle",
-            "sample": f"one step's permutation plus {frac:.4f} of its pairs (forward, dX/dh) and of its rank "
-                      f"rows (dA, dB^T), all 3 projections; {dt:.1f} s", "seconds": dt}
+            "sample": f"{what}; {dt:.1f} s", "seconds": dt}
 
 
 def run_reference(args, rank, world):
@@ -406,9 +502,7 @@ def run_reference(args, rank, world):
     c = W.get_config(args.config)
     # per step: a bounded sample sized so that warmup + steps end within minutes
     per_step_s = max(2.0, min(20.0, 120.0 / max(1, args.steps + args.warmup)))
-    frac = 1.0 / 512
-    dt, _ = oracle_sample(args.config, args.seed, args.expertwise, frac)
-    frac = min(1.0, frac * per_step_s / max(dt, 1e-3))
+    frac = calibrate_fraction(args.config, args.seed, args.expertwise, per_step_s)
     for _ in range(args.warmup):
         oracle_sample(args.config, args.seed, args.expertwise, frac)
     times, rows = [], 0.0
@@ -434,7 +528,7 @@ def run_reference(args, rank, world):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ace", choices=["ace", "reference"])
     ap.add_argument("--config", default="olmoe")

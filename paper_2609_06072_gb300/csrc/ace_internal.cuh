@@ -117,13 +117,14 @@ cudaError_t launch_fwd_h(const PlanTables& pt, const FwdHLaunch& a, cudaStream_t
 // MODE down: H_row = A_g h_row computed here (K loop over h);  gate/up:
 // H_row = H_u gathered from the unique-pair H of launch_fwd_h.
 struct FwdRowsLaunch {
-  CUtensorMap tm_x;      // down: Hin [R, d_in], box 64 x 128
-  CUtensorMap tm_a;      // down: A [n_rank, d_in], box 64 x rank_pad
-  CUtensorMap tm_bt[2];  // Bt [n_rank, d_out], box 64 x rank_pad
-  CUtensorMap tm_y[2];   // Y [R, d_out], box 64 x 128
-  const Tile* tiles;     // row tiles
-  const int32_t* counts;
-  int32_t max_tiles;
+  CUtensorMap tm_x;       // down: Hin [R, d_in], box 64 x 128
+  CUtensorMap tm_x16;     // down: Hin, box 64 x 16 (short tiles)
+  CUtensorMap tm_a;       // down: A [n_rank, d_in], box 64 x rank_pad
+  CUtensorMap tm_bt[2];   // Bt [n_rank, d_out], box 64 x rank_pad
+  CUtensorMap tm_y[2];    // Y [R, d_out], box 64 x 128
+  CUtensorMap tm_y16[2];  // Y, box 64 x 16 (short tiles)
+  const int32_t* group_off;  // [G + 1] row offsets of the groups
+  int32_t grid;              // persistent CTAs (the SM count)
   const int32_t* row_uniq;
   const float* Hu[2];    // gate/up: H per unique pair
   uint16_t* Y[2];

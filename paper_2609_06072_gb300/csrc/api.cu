@@ -48,6 +48,7 @@ struct ace_plan {
   int32_t T_max;
   uint32_t flags;
   int device;
+  int num_sms;  // persistent kernels launch one CTA per SM
 };
 
 namespace {
@@ -156,6 +157,9 @@ ace_status ace_plan_create(ace_plan** out, const ace_layer_desc* desc) {
   cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
   if (!(major == 10 && minor == 3))
     return fail(ACE_ERR_UNSUPPORTED, "device %d is sm_%d%d; this library is built for sm_103a only", dev, major, minor);
+  int num_sms = 0;
+  ce = cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, dev);
+  if (ce != cudaSuccess || num_sms <= 0) return cuda_status(ce, "multiprocessor count");
   ace_plan* p = new (std::nothrow) ace_plan();
   if (!p) return fail(ACE_ERR_ARG, "out of host memory");
   std::memset(&p->pt, 0, sizeof(p->pt));
@@ -172,6 +176,7 @@ ace_status ace_plan_create(ace_plan** out, const ace_layer_desc* desc) {
   p->T_max = D.T_max;
   p->flags = D.flags;
   p->device = dev;
+  p->num_sms = num_sms;
   *out = p;
   return ACE_OK;
 }
@@ -272,16 +277,17 @@ static ace_status fwd_common(const ace_plan* plan, const ace_perm* perm, const u
   bool ok = true;
   if (!shared) {
     ok = ok && make_tmap_bf16(&r.tm_x, X, (uint64_t)R, (uint64_t)d_in, kTileM);
+    ok = ok && make_tmap_bf16(&r.tm_x16, X, (uint64_t)R, (uint64_t)d_in, 16);
     ok = ok && make_tmap_bf16(&r.tm_a, A[0], (uint64_t)n_rank, (uint64_t)d_in, pt.rank_pad);
   }
   for (int j = 0; j < nproj; ++j) {
     ok = ok && make_tmap_bf16(&r.tm_bt[j], Bt[j], (uint64_t)n_rank, (uint64_t)d_out, pt.rank_pad);
     ok = ok && make_tmap_bf16(&r.tm_y[j], Y[j], (uint64_t)R, (uint64_t)d_out, kTileM);
+    ok = ok && make_tmap_bf16(&r.tm_y16[j], Y[j], (uint64_t)R, (uint64_t)d_out, 16);
   }
   if (!ok) return fail(ACE_ERR_UNSUPPORTED, "tensor-map encoding failed for this layout");
-  r.tiles = at<Tile>(perm->ws, L.tiles_row);
-  r.counts = perm->counts;
-  r.max_tiles = L.max_tiles;
+  r.group_off = perm->group_off;
+  r.grid = R > 0 ? plan->num_sms : 0;
   r.row_uniq = at<int32_t>(perm->ws, L.row_uniq);
   for (int j = 0; j < 2; ++j) {
     const int jj = j < nproj ? j : 0;

@@ -78,7 +78,7 @@ typedef int32_t ace_status;
 
 /* Layer description (host memory; copied into the plan). */
 typedef struct ace_layer_desc {
-  int32_t T_max;           /* largest T a call will use */
+  int32_t T_max;           /* largest T a call will use; T_max * k <= 2^30 */
   int32_t k;               /* top-k, 1 <= k <= E, k <= 32 */
   int32_t E;               /* experts, 1 <= E <= ACE_MAX_EXPERTS */
   int32_t G;               /* groups, 1 <= G <= E */

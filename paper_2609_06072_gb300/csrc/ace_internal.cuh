@@ -27,25 +27,28 @@ struct PlanTables {
   int32_t rank_off[ACE_MAX_EXPERTS + 1];
 };
 
-// A unit of work: rows [start, start + cnt) of group g (row tiles) or unique
-// pairs [start, start + cnt) of group g (shared tiles).  `id` is the split
-// index for backward splits.
+// A unit of work: unique pairs [start, start + cnt) of group g (shared tiles)
+// or rows [start, start + cnt) of group g (row tiles, backward splits).  `id`
+// is the tile's or split's index.
 struct Tile {
   int32_t g, start, cnt, id;
 };
 
 // Byte layout of the permutation workspace for T tokens.
 struct PermLayout {
-  size_t err, counts, group_off, expert_off, expert_cnt, uniq_off, row_pair, pair_row, pair_g, row_uniq, uniq_tok,
+  size_t err, counts, sched, group_off, expert_off, expert_cnt, uniq_off, row_pair, pair_row, pair_g, row_uniq, uniq_tok,
       tok_uniq;
   size_t chunk_cntE, chunk_cntU, chunk_baseE, chunk_baseU, chunk_err;
-  size_t tiles_sh, tiles_row, splits_sh, splits_row;
+  size_t tiles_sh, tiles_row, splits_row;
   size_t total;
   int32_t n_chunks, max_tiles, max_splits;
 };
 
 // counts[] slots
-constexpr int kCntU = 0, kCntRows = 1, kCntTilesSh = 2, kCntTilesRow = 3, kCntSplitsSh = 4, kCntSplitsRow = 5;
+constexpr int kCntU = 0, kCntRows = 1, kCntTilesSh = 2, kCntTilesRow = 3, kCntSplitsRow = 4;
+// sched[] slots: work counters of the dynamically scheduled kernels (zeroed
+// by the host before each launch)
+constexpr int kSchedFwdRows = 0;
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
@@ -64,6 +67,7 @@ inline PermLayout perm_layout(const PlanTables& pt, int32_t T) {
   };
   L.err = take(4 * 8);
   L.counts = take(4 * 8);
+  L.sched = take(4 * 8);
   L.group_off = take(4 * (size_t)(pt.G + 1));
   L.expert_off = take(4 * (size_t)pt.E);
   L.expert_cnt = take(4 * (size_t)pt.E);
@@ -81,7 +85,6 @@ inline PermLayout perm_layout(const PlanTables& pt, int32_t T) {
   L.chunk_err = take(4 * (size_t)(L.n_chunks + 1));
   L.tiles_sh = take(sizeof(Tile) * (size_t)L.max_tiles);
   L.tiles_row = take(sizeof(Tile) * (size_t)L.max_tiles);
-  L.splits_sh = take(sizeof(Tile) * (size_t)L.max_splits);
   L.splits_row = take(sizeof(Tile) * (size_t)L.max_splits);
   L.total = off;
   return L;
@@ -123,7 +126,9 @@ struct FwdRowsLaunch {
   CUtensorMap tm_bt[2];   // Bt [n_rank, d_out], box 64 x rank_pad
   CUtensorMap tm_y[2];    // Y [R, d_out], box 64 x 128
   CUtensorMap tm_y16[2];  // Y, box 64 x 16 (short tiles)
-  const int32_t* group_off;  // [G + 1] row offsets of the groups
+  const Tile* tiles;         // row tiles (<= 128 rows of one group), in row order
+  const int32_t* counts;     // counts[kCntTilesRow] = number of row tiles
+  int32_t* sched;            // work counter, zero at launch
   int32_t grid;              // persistent CTAs (the SM count)
   const int32_t* row_uniq;
   const float* Hu[2];    // gate/up: H per unique pair

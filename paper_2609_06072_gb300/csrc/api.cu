@@ -71,7 +71,6 @@ ace_status cuda_status(cudaError_t e, const char* what) {
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 // Row tiles per backward split: (tiles + 2) * rank_pad TMEM columns <= 256.
-int nt_split_for(int rank_pad) { return rank_pad <= 32 ? 4 : rank_pad == 64 ? 2 : 1; }
 
 ace_status check_perm(const ace_plan* plan, const ace_perm* perm) {
   if (!plan || !perm || !perm->ws) return fail(ACE_ERR_ARG, "null plan or perm");
@@ -79,6 +78,8 @@ ace_status check_perm(const ace_plan* plan, const ace_perm* perm) {
   if (perm->R != perm->T * plan->pt.k) return fail(ACE_ERR_ARG, "perm R does not match T*k");
   return ACE_OK;
 }
+
+int pt_nt_split(int rank_pad) { return rank_pad <= 32 ? 4 : rank_pad == 64 ? 2 : 1; }
 
 struct BwdWs {
   float* dHrow[2];
@@ -93,7 +94,8 @@ int n_rank_pad_of(const PlanTables& pt) { return (pt.rank_off[pt.G] + 63) / 64 *
 // Backward scratch: dH per row (fp32, per projection), the deterministic
 // split-K partials of dB^T (per projection) and dA (down), and the
 // token-major dense dH of gate/up (bf16).
-BwdWs bwd_layout(const PlanTables& pt, int32_t T, void* base) {
+BwdWs bwd_layout(const ace_plan* plan, int32_t T, void* base) {
+  const PlanTables& pt = plan->pt;
   const PermLayout L = perm_layout(pt, T);
   const int64_t R = (int64_t)T * pt.k;
   const size_t dhrow = align_up(4 * (size_t)R * pt.rank_pad, 256);
@@ -170,7 +172,7 @@ ace_status ace_plan_create(ace_plan** out, const ace_layer_desc* desc) {
   p->pt.f = D.f;
   p->pt.rank_max = rank_max;
   p->pt.rank_pad = rank_max <= 16 ? 16 : rank_max <= 32 ? 32 : rank_max <= 64 ? 64 : 128;
-  p->pt.nt_split = nt_split_for(p->pt.rank_pad);
+  p->pt.nt_split = pt_nt_split(p->pt.rank_pad);
   for (int e = 0; e < D.E; ++e) p->pt.e2g[e] = (int16_t)D.e2g[e];
   for (int g = 0; g <= D.G; ++g) p->pt.rank_off[g] = D.rank_off[g];
   p->T_max = D.T_max;
@@ -191,7 +193,7 @@ ace_status ace_workspace_size(const ace_plan* plan, int32_t T, size_t* perm_byte
   if (T < 0 || T > plan->T_max) return fail(ACE_ERR_SHAPE, "T=%d outside [0, %d]", T, plan->T_max);
   if (perm_bytes) *perm_bytes = perm_layout(plan->pt, T).total;
   if (fwd_bytes) *fwd_bytes = 2 * align_up(4 * (size_t)T * plan->pt.k * plan->pt.rank_max, 256);
-  if (bwd_bytes) *bwd_bytes = bwd_layout(plan->pt, T, nullptr).total;
+  if (bwd_bytes) *bwd_bytes = bwd_layout(plan, T, nullptr).total;
   return ACE_OK;
 }
 
@@ -286,8 +288,14 @@ static ace_status fwd_common(const ace_plan* plan, const ace_perm* perm, const u
     ok = ok && make_tmap_bf16(&r.tm_y16[j], Y[j], (uint64_t)R, (uint64_t)d_out, 16);
   }
   if (!ok) return fail(ACE_ERR_UNSUPPORTED, "tensor-map encoding failed for this layout");
-  r.group_off = perm->group_off;
+  r.tiles = at<Tile>(perm->ws, L.tiles_row);
+  r.counts = perm->counts;
+  r.sched = at<int32_t>(perm->ws, L.sched) + kSchedFwdRows;
   r.grid = R > 0 ? plan->num_sms : 0;
+  if (R > 0) {
+    st = cuda_status(cudaMemsetAsync(r.sched, 0, sizeof(int32_t), cs), "work counter reset");
+    if (st != ACE_OK) return st;
+  }
   r.row_uniq = at<int32_t>(perm->ws, L.row_uniq);
   for (int j = 0; j < 2; ++j) {
     const int jj = j < nproj ? j : 0;
@@ -334,11 +342,11 @@ ace_status ace_bwd_shared(const ace_plan* plan, const ace_perm* perm, int32_t np
         !aligned16(dBt[j]))
       return fail(ACE_ERR_ARG, "tensor of projection %d not 16-byte aligned", j);
   }
-  const BwdWs need = bwd_layout(plan->pt, perm->T, nullptr);
+  const BwdWs need = bwd_layout(plan, perm->T, nullptr);
   if (!ws || ws_bytes < need.total) return fail(ACE_ERR_WORKSPACE, "backward workspace %zu < %zu bytes", ws_bytes, need.total);
   if (!aligned16(ws)) return fail(ACE_ERR_WORKSPACE, "backward workspace misaligned");
   const PermLayout L = perm_layout(plan->pt, perm->T);
-  const BwdWs w = bwd_layout(plan->pt, perm->T, ws);
+  const BwdWs w = bwd_layout(plan, perm->T, ws);
   cudaStream_t cs = static_cast<cudaStream_t>(stream);
   BwdLaunch a{};
   bool ok = true;
@@ -412,11 +420,11 @@ ace_status ace_bwd_row(const ace_plan* plan, const ace_perm* perm, const uint16_
   if (!aligned16(dY) || !aligned16(Hin) || !aligned16(H) || !aligned16(A) || !aligned16(Bt) || !aligned16(dHin) ||
       !aligned16(dA) || !aligned16(dBt))
     return fail(ACE_ERR_ARG, "tensor not 16-byte aligned");
-  const BwdWs need = bwd_layout(plan->pt, perm->T, nullptr);
+  const BwdWs need = bwd_layout(plan, perm->T, nullptr);
   if (!ws || ws_bytes < need.total) return fail(ACE_ERR_WORKSPACE, "backward workspace %zu < %zu bytes", ws_bytes, need.total);
   if (!aligned16(ws)) return fail(ACE_ERR_WORKSPACE, "backward workspace misaligned");
   const PermLayout L = perm_layout(plan->pt, perm->T);
-  const BwdWs w = bwd_layout(plan->pt, perm->T, ws);
+  const BwdWs w = bwd_layout(plan, perm->T, ws);
   BwdLaunch a{};
   bool ok = true;
   const uint64_t R = (uint64_t)perm->R, nr = (uint64_t)plan->pt.rank_off[plan->pt.G];

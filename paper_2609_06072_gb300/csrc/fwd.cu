@@ -6,19 +6,18 @@
 //   X rows gathered by token with cp.async into 128-byte-swizzled smem,
 //   tcgen05 MMA with N = nproj * rank_pad (gate and up share the gather),
 //   fp32 H written per unique pair.
-// k_fwd_rows: persistent, one CTA per SM; each CTA takes an equal share of
-//   the rows (16-row quanta) and walks it in tiles of <= 128 consecutive rows
-//   of one group (expert segments are contiguous inside group segments).
-//   Warp-specialised:
+// k_fwd_rows: persistent, one CTA per SM; tiles of <= 128 consecutive rows
+//   of one group (expert segments are contiguous inside group segments) are
+//   taken dynamically from a counter.  Warp-specialised:
 //     warp 0     TMA producer: row tiles of Y (and of h for down) and chunks of
 //                B_g^T / A_g into a ring of shared-memory slots
 //     warp 1     MMA issuer: (down) H = h . A_g^T over the K loop, then per
-//                64-column chunk D = H . B_g^T into double-buffered TMEM
-//     warps 2-9  epilogue, two groups of four (one warp per TMEM lane
+//                64-column chunk D = H . B_g^T into one of four TMEM buffers
+//     warps 2-17 epilogue, four groups of four (one warp per TMEM lane
 //                quarter): H -> bf16 operand (down: from TMEM; gate/up:
 //                gathered from the unique pair of each row), then group p
-//                takes the chunks of parity p: Y += s * D on its own 32 rows
-//                in swizzled smem (TMEM lane = row) and stores those rows.
+//                takes the chunks cc with cc % 4 == p: Y += s * D on its own
+//                32 rows in swizzled smem (TMEM lane = row) and stores them.
 //   For gate/up the K = r_g product B_g H_u is evaluated per routed row; the
 //   K = d product A_g x -- the one that dominates -- stays deduplicated.
 #include <cstdint>
@@ -151,144 +150,200 @@ __global__ void __launch_bounds__(kHThreads) k_fwd_h(const __grid_constant__ Pla
 }
 
 // --------------------------------------------------------------- k_fwd_rows
-constexpr int kRowsThreads = 320;  // 10 warps: producer, MMA, 2 x 4 epilogue warps
+constexpr int kNGrp = 4;                        // epilogue groups (4 warps each, one per TMEM lane quarter)
+constexpr int kRowsThreads = 64 + 128 * kNGrp;  // producer warp, MMA warp, epilogue warps
+constexpr int kRowsTmem = 512;
 constexpr int kChunk = 64;         // output columns per D chunk
-constexpr int kQuant = 16;         // rows per work quantum and per small TMA box
+constexpr int kQuant = 16;         // rows per small TMA box (short tiles)
+constexpr int kQ = 4;              // depth of the tile queue
 
-template <int RP, int NPROJ>
+template <int RP, int NPROJ, bool SHARED>
 struct RowsFwdCfg {
   static constexpr int kWBlk = RP * 128;                    // [RP x 64] weight block
   static constexpr int kSlot = NPROJ * (kBlk + kWBlk);      // Y tiles + B^T blocks (down K-step: h + A)
-  static constexpr int kHs = ((NPROJ * RP + 63) / 64) * kBlk;
-  static constexpr int kBudget = 200 * 1024;
-  static constexpr int kS0 = (kBudget - kHs) / kSlot;
+  static constexpr int kHs = ((NPROJ * RP + 63) / 64) * kBlk;  // bf16 H operand of one tile
+  static constexpr int kBudget = 210 * 1024;
+  static constexpr int NBH = 2 * kHs + 4 * kSlot <= kBudget ? 2 : 1;  // H operand buffers
+  static constexpr int kS0 = (kBudget - NBH * kHs) / kSlot;
   static constexpr int S = kS0 > 8 ? 8 : (kS0 < 2 ? 2 : kS0);
-  static constexpr int kSmem = kHs + S * kSlot + 1024;
-};
-
-// Rows of one CTA of a persistent row kernel: equal shares of 16-row quanta
-// over the CTAs that have work (at least 128 rows each).
-struct RowRange {
-  int begin, end;
-};
-__device__ __forceinline__ RowRange cta_rows(int R) {
-  const int ncta = min((int)gridDim.x, max(1, (R + kTileM - 1) / kTileM));
-  if ((int)blockIdx.x >= ncta) return {0, 0};
-  const int nq = (R + kQuant - 1) / kQuant;
-  const int q0 = (int)((int64_t)blockIdx.x * nq / ncta), q1 = (int)((int64_t)(blockIdx.x + 1) * nq / ncta);
-  return {min(R, q0 * kQuant), min(R, q1 * kQuant)};
-}
-
-// Walks a row range in tiles of at most 128 rows that never cross a group
-// boundary (every row of a tile uses the same A_g, B_g).  goff: group_off in
-// shared memory.  Every role of a CTA walks the same sequence.
-struct TileWalk {
-  int cur, end, g;
-  __device__ __forceinline__ bool next(const int32_t* goff, Tile& t) {
-    if (cur >= end) return false;
-    while (goff[g + 1] <= cur) ++g;
-    t.g = g;
-    t.start = cur;
-    t.cnt = min(kTileM, min(end, goff[g + 1]) - cur);
-    t.id = 0;
-    cur += t.cnt;
-    return true;
-  }
+  static constexpr int kSmem = NBH * kHs + S * kSlot + 1024;
+  static constexpr int kHcol = RP <= 64 ? 64 : 128;         // down: TMEM columns of one H accumulator
+  static constexpr uint32_t kDBase = SHARED ? 0u : 2u * kHcol;
+  static_assert(kDBase + kNGrp * NPROJ * kChunk <= kRowsTmem, "TMEM budget");
 };
 
 // Rows [y, y + cnt) of a 64-column box at column x: one 128-row box for a
 // whole tile, else ceil(cnt / 16) boxes of 16 rows (so a short tile reads at
-// most 15 rows it does not use).  Returns the bytes the copies deliver.
-__device__ __forceinline__ uint32_t load_rows(uint32_t dst, const CUtensorMap* m128, const CUtensorMap* m16, int x,
-                                              int y, int cnt, uint64_t* bar) {
+// most 15 rows it does not use).
+__device__ __forceinline__ void load_rows(uint32_t dst, const CUtensorMap* m128, const CUtensorMap* m16, int x, int y,
+                                          int cnt, uint64_t* bar) {
   if (cnt == kTileM) {
     tma_load_2d(dst, m128, x, y, bar);
-    return kBlk;
+    return;
   }
   const int nb = (cnt + kQuant - 1) / kQuant;
   for (int b = 0; b < nb; ++b) tma_load_2d(dst + b * kQuant * 128, m16, x, y + b * kQuant, bar);
-  return nb * kQuant * 128;
 }
 __device__ __forceinline__ uint32_t rows_bytes(int cnt) {
   return cnt == kTileM ? (uint32_t)kBlk : (uint32_t)((cnt + kQuant - 1) / kQuant) * kQuant * 128;
 }
 
-// Persistent: one CTA per SM walks its share of the rows tile by tile; the
-// producer, the MMA issuer and the epilogue run ahead of one another across
-// tile boundaries.  The eight epilogue warps form two groups of four (one warp
-// per TMEM lane quarter); group p owns the D chunks of parity p, and each warp
-// updates and stores only its own 32 rows, so a chunk needs no barrier wider
-// than its group.
+// Tile queue: the producer takes row tiles from a global counter (so faster
+// SMs take more tiles) and hands each tile index to the MMA warp and the
+// epilogue warps through a small ring in shared memory; -1 ends.
+struct TileQueue {
+  int32_t item[kQ];
+  uint64_t full[kQ], empty[kQ];
+};
+// Consumer side: the next non-empty tile (false at the end or if a wait gave
+// up; *ok tells which).  Every lane of a warp calls it; lane 0 releases the
+// entries it reads.
+__device__ __forceinline__ bool queue_next(TileQueue& tq, int& q, const Tile* tiles, Tile& t, bool single_lane,
+                                           bool* ok) {
+  while (true) {
+    const int e = q % kQ;
+    bool w = mbar_wait(&tq.full[e], (q / kQ) & 1);
+    if (!single_lane) w = __all_sync(0xffffffffu, w);
+    if (!w) {
+      *ok = false;
+      return false;
+    }
+    const int item = *reinterpret_cast<volatile int32_t*>(&tq.item[e]);
+    if (!single_lane) __syncwarp();
+    if (single_lane || (threadIdx.x & 31) == 0) mbar_arrive(&tq.empty[e]);
+    ++q;
+    if (item < 0) return false;
+    t = tiles[item];
+    if (t.cnt > 0) return true;  // (an empty tile is skipped)
+  }
+}
+// Persistent: one CTA per SM; tiles of <= 128 consecutive rows of one group
+// are taken dynamically.  The producer, the MMA issuer and the epilogue run
+// ahead of one another across tile boundaries: for down, the K loop of the
+// next tile (H = h . A_g^T into the other of two TMEM accumulators) follows
+// the D chunks of the current tile in the ring; for gate/up the next tile's
+// H is gathered while the current one streams (the H operand is
+// double-buffered in shared memory where it fits).  (Interleaving the next
+// K loop into the chunk stream measured slower.)  The epilogue warps form kNGrp groups of four (one warp
+// per TMEM lane quarter); group p owns the D chunks cc with cc % kNGrp == p,
+// and each warp updates and stores only its own 32 rows, so no barrier spans
+// more than one warp: every hand-off is an mbarrier (a ring slot is released
+// by the MMA commit after a K step, or by the four warps of the group after a
+// chunk, each on its own barrier).
 template <int RP, int NPROJ, bool SHARED>
 __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_constant__ PlanTables pt,
                                                               const __grid_constant__ FwdRowsLaunch a) {
-  using C = RowsFwdCfg<RP, NPROJ>;
-  constexpr int S = C::S;
+  using C = RowsFwdCfg<RP, NPROJ, SHARED>;
+  constexpr int S = C::S, NBH = C::NBH;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  __shared__ __align__(8) uint64_t full[S], empty[S], dfull[2], dempty[2], hacc, hs_ready;
+  __shared__ __align__(8) uint64_t full[S], emptyK[S], emptyC[S], dfull[kNGrp], dempty[kNGrp];
+  __shared__ __align__(8) uint64_t hacc[2], hs_ready[2], hs_free[2];
+  __shared__ __align__(8) TileQueue tq;
   __shared__ uint32_t tslot;
-  __shared__ int32_t goff[ACE_MAX_EXPERTS + 1];
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  for (int i = tid; i <= pt.G; i += kRowsThreads) goff[i] = a.group_off[i];
   if (tid == 0) {
     for (int i = 0; i < S; ++i) {
       mbar_init(&full[i], 1);
-      mbar_init(&empty[i], 1);
+      mbar_init(&emptyK[i], 1);  // MMA commit after a K step
+      mbar_init(&emptyC[i], 4);  // the four warps of the group that owns the chunk
+    }
+    for (int i = 0; i < kNGrp; ++i) {
+      mbar_init(&dfull[i], 1);
+      mbar_init(&dempty[i], 4);
+    }
+    for (int i = 0; i < kQ; ++i) {
+      mbar_init(&tq.full[i], 1);
+      mbar_init(&tq.empty[i], 1 + 4 * kNGrp);  // MMA thread + every epilogue warp
     }
     for (int i = 0; i < 2; ++i) {
-      mbar_init(&dfull[i], 1);
-      mbar_init(&dempty[i], 4);  // the four warps of the group that owns the buffer
+      mbar_init(&hacc[i], 1);              // down: H of the tiles of this parity accumulated
+      mbar_init(&hs_ready[i], 4 * kNGrp);  // H operand of the tiles of this parity staged (every epilogue warp)
+      mbar_init(&hs_free[i], 1);           // D chunks reading H buffer i done (MMA commit)
     }
-    mbar_init(&hacc, 1);
-    mbar_init(&hs_ready, 8);  // every epilogue warp
     fence_mbar_init();
   }
-  if (warp == 0) tmem_alloc(&tslot, 256);
+  if (warp == 0) tmem_alloc(&tslot, kRowsTmem);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = tslot;
-  const RowRange rr = cta_rows(goff[pt.G]);
+  const int n_items = a.counts[kCntTilesRow];
   const int d_in = a.d_in, d_out = a.d_out;
   const int NK = SHARED ? 0 : (d_in + 63) / 64;  // K steps of the down H GEMM
   const int nch = (d_out + kChunk - 1) / kChunk;
-  const uint32_t sHs = smem_u32(smem);
-  const uint32_t slot0 = sHs + C::kHs;
-  const uint32_t dbase = SHARED ? 0u : 128u;  // down: H accumulator in columns [0, RP)
+  const uint32_t sHs0 = smem_u32(smem);
+  const uint32_t slot0 = sHs0 + NBH * C::kHs;
   bool bad = false;
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
-      TileWalk w{rr.begin, rr.end, 0};
-      Tile tl;
-      int i = 0;
-      while (!bad && w.next(goff, tl)) {
-        const int r0 = pt.rank_off[tl.g];
-        const uint32_t rb = rows_bytes(tl.cnt);
-        for (int it = 0; it < NK + nch; ++it, ++i) {
-          const int s = i % S, u = i / S;
-          if (u >= 1 && !mbar_wait(&empty[s], (u - 1) & 1)) {
-            bad = true;
-            break;
-          }
-          const uint32_t base = slot0 + s * C::kSlot;
-          if (it < NK) {
-            mbar_arrive_expect_tx(&full[s], rb + C::kWBlk);
-            load_rows(base, &a.tm_x, &a.tm_x16, it * 64, tl.start, tl.cnt, &full[s]);
-            tma_load_2d(base + NPROJ * kBlk, &a.tm_a, it * 64, r0, &full[s]);
-          } else {
-            const int n0 = (it - NK) * kChunk;
-            mbar_arrive_expect_tx(&full[s], NPROJ * (rb + C::kWBlk));
+      int last[S], nK[S], nC[S];  // per slot: kind of the last use (0 none, 1 K step, 2 chunk), use counts
 #pragma unroll
-            for (int j = 0; j < NPROJ; ++j) {
-              load_rows(base + j * kBlk, &a.tm_y[j], &a.tm_y16[j], n0, tl.start, tl.cnt, &full[s]);
-              tma_load_2d(base + NPROJ * kBlk + j * C::kWBlk, &a.tm_bt[j], n0, r0, &full[s]);
-            }
+      for (int k = 0; k < S; ++k) last[k] = nK[k] = nC[k] = 0;
+      int i = 0, q = 0;
+      // grab tiles until a non-empty one or the end, handing each index on
+      auto grab = [&](Tile& t) -> bool {
+        while (true) {
+          const int e = q % kQ;
+          if (q >= kQ && !mbar_wait(&tq.empty[e], ((q - kQ) / kQ) & 1)) {
+            bad = true;
+            return false;
           }
+          int item = atomicAdd(a.sched, 1);
+          if (item >= n_items) item = -1;
+          tq.item[e] = item;
+          mbar_arrive(&tq.full[e]);
+          ++q;
+          if (item < 0) return false;
+          t = a.tiles[item];
+          if (t.cnt > 0) return true;
         }
+      };
+      auto acquire = [&](bool kstep) -> uint32_t {  // next ring slot, once its last user released it
+        const int s = i % S;
+        if ((last[s] == 1 && !mbar_wait(&emptyK[s], (nK[s] - 1) & 1)) ||
+            (last[s] == 2 && !mbar_wait(&emptyC[s], (nC[s] - 1) & 1)))
+          bad = true;
+        last[s] = kstep ? 1 : 2;
+        if (kstep) ++nK[s]; else ++nC[s];
+        return (uint32_t)s;
+      };
+      auto load_k = [&](const Tile& t, int k) {
+        const uint32_t s = acquire(true);
+        if (bad) return;
+        const uint32_t base = slot0 + s * C::kSlot;
+        mbar_arrive_expect_tx(&full[s], rows_bytes(t.cnt) + C::kWBlk);
+        load_rows(base, &a.tm_x, &a.tm_x16, k * 64, t.start, t.cnt, &full[s]);
+        tma_load_2d(base + NPROJ * kBlk, &a.tm_a, k * 64, pt.rank_off[t.g], &full[s]);
+        ++i;
+      };
+      auto load_c = [&](const Tile& t, int c) {
+        const uint32_t s = acquire(false);
+        if (bad) return;
+        const uint32_t base = slot0 + s * C::kSlot;
+        const int n0 = c * kChunk;
+        mbar_arrive_expect_tx(&full[s], NPROJ * (rows_bytes(t.cnt) + C::kWBlk));
+#pragma unroll
+        for (int j = 0; j < NPROJ; ++j) {
+          load_rows(base + j * kBlk, &a.tm_y[j], &a.tm_y16[j], n0, t.start, t.cnt, &full[s]);
+          tma_load_2d(base + NPROJ * kBlk + j * C::kWBlk, &a.tm_bt[j], n0, pt.rank_off[t.g], &full[s]);
+        }
+        ++i;
+      };
+      Tile cur, nxt;
+      bool has_cur = grab(cur);
+      if (has_cur && !SHARED)
+        for (int k = 0; k < NK && !bad; ++k) load_k(cur, k);
+      while (has_cur && !bad) {
+        const bool has_nxt = grab(nxt);
+        for (int c = 0; c < nch && !bad; ++c) load_c(cur, c);
+        if (!SHARED && has_nxt)
+          for (int k = 0; k < NK && !bad; ++k) load_k(nxt, k);
+        cur = nxt;
+        has_cur = has_nxt;
       }
       // every copy issued has landed before the CTA can exit
       for (int k = max(0, i - S); k < i; ++k)
@@ -299,89 +354,95 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
     if (lane == 0) {
       constexpr uint32_t idesc_h = idesc_bf16_f32(128, RP, 0, 0);
       constexpr uint32_t idesc_d = idesc_bf16_f32(128, kChunk, 0, 1);
-      TileWalk w{rr.begin, rr.end, 0};
-      Tile tl;
-      int i = 0, cc = 0, ti = 0;
-      while (!bad && w.next(goff, tl)) {
-        for (int it = 0; it < NK + nch; ++it, ++i) {
-          const int s = i % S, u = i / S;
-          if (!mbar_wait(&full[s], u & 1)) {
-            bad = true;
-            break;
-          }
-          tc_fence_after();
-          const uint32_t base = slot0 + s * C::kSlot;
-          if (it < NK) {
-#pragma unroll
-            for (int kk = 0; kk < 4; ++kk)
-              tc_mma_bf16(tmem, sdesc_sw128(base + kk * 32, 16, 1024),
-                          sdesc_sw128(base + NPROJ * kBlk + kk * 32, 16, 1024), idesc_h,
-                          (it > 0 || kk > 0) ? 1u : 0u);
-            tc_commit(&empty[s]);
-            if (it == NK - 1) tc_commit(&hacc);
-          } else {
-            const int b = cc & 1;
-            if (it == NK && !mbar_wait(&hs_ready, ti & 1)) {
-              bad = true;
-              break;
-            }
-            if (cc >= 2 && !mbar_wait(&dempty[b], ((cc - 2) >> 1) & 1)) {
-              bad = true;
-              break;
-            }
-            tc_fence_after();
-#pragma unroll
-            for (int j = 0; j < NPROJ; ++j)
-#pragma unroll
-              for (int kk = 0; kk < RP / 16; ++kk) {
-                const int kg = (j * RP) / 16 + kk;
-                tc_mma_bf16(tmem + dbase + (b * NPROJ + j) * kChunk,
-                            sdesc_sw128(sHs + (kg >> 2) * kBlk + (kg & 3) * 32, 16, 1024),
-                            sdesc_sw128(base + NPROJ * kBlk + j * C::kWBlk + kk * 2048, C::kWBlk, 1024), idesc_d,
-                            kk > 0 ? 1u : 0u);
-              }
-            tc_commit(&dfull[b]);
-            ++cc;
-          }
+      int i = 0, cc = 0, ti = 0, q = 0;
+      auto mma_k = [&](int hb, int k) {  // K step k of the tile whose H accumulator is hb
+        const int s = i % S;
+        if (!mbar_wait(&full[s], (i / S) & 1)) {
+          bad = true;
+          return;
         }
+        tc_fence_after();
+        const uint32_t base = slot0 + s * C::kSlot;
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk)
+          tc_mma_bf16(tmem + hb * C::kHcol, sdesc_sw128(base + kk * 32, 16, 1024),
+                      sdesc_sw128(base + NPROJ * kBlk + kk * 32, 16, 1024), idesc_h, (k > 0 || kk > 0) ? 1u : 0u);
+        tc_commit(&emptyK[s]);
+        if (k == NK - 1) tc_commit(&hacc[hb]);
+        ++i;
+      };
+      auto mma_c = [&](int c) {  // D chunk c of tile ti
+        const int s = i % S, b = cc % kNGrp;
+        if ((c == 0 && !mbar_wait(&hs_ready[ti & 1], (ti >> 1) & 1)) ||
+            (cc >= kNGrp && !mbar_wait(&dempty[b], ((cc - kNGrp) / kNGrp) & 1)) ||
+            !mbar_wait(&full[s], (i / S) & 1)) {
+          bad = true;
+          return;
+        }
+        tc_fence_after();
+        const uint32_t base = slot0 + s * C::kSlot;
+        const uint32_t sHs = sHs0 + (ti % NBH) * C::kHs;
+#pragma unroll
+        for (int j = 0; j < NPROJ; ++j)
+#pragma unroll
+          for (int kk = 0; kk < RP / 16; ++kk) {
+            const int kg = (j * RP) / 16 + kk;
+            tc_mma_bf16(tmem + C::kDBase + (b * NPROJ + j) * kChunk,
+                        sdesc_sw128(sHs + (kg >> 2) * kBlk + (kg & 3) * 32, 16, 1024),
+                        sdesc_sw128(base + NPROJ * kBlk + j * C::kWBlk + kk * 2048, C::kWBlk, 1024), idesc_d,
+                        kk > 0 ? 1u : 0u);
+          }
+        tc_commit(&dfull[b]);
+        if (c == nch - 1) tc_commit(&hs_free[ti % NBH]);
+        ++cc;
+        ++i;
+      };
+      Tile cur, nxt;
+      bool qok = true;
+      bool has_cur = queue_next(tq, q, a.tiles, cur, true, &qok);
+      if (has_cur && !SHARED)
+        for (int k = 0; k < NK && !bad; ++k) mma_k(0, k);
+      while (has_cur && !bad) {
+        const bool has_nxt = queue_next(tq, q, a.tiles, nxt, true, &qok);
+        for (int c = 0; c < nch && !bad; ++c) mma_c(c);
+        if (!SHARED && has_nxt)
+          for (int k = 0; k < NK && !bad; ++k) mma_k((ti + 1) & 1, k);
         ++ti;
+        cur = nxt;
+        has_cur = has_nxt;
       }
+      if (!qok) bad = true;
+      // the last commit must land before the CTA exits
+      if (!bad && ti > 0 && !mbar_wait(&hs_free[(ti - 1) % NBH], ((ti - 1) / NBH) & 1)) bad = true;
     }
   } else {
     // ------------------------------------------------------------ epilogue
-    const int grp = (warp - 2) >> 2;        // chunk parity of this warp's group
+    const int grp = (warp - 2) >> 2;        // this warp's group: chunks cc with cc % kNGrp == grp
     const int quarter = warp & 3;           // TMEM lane quarter of this warp
     const int m = quarter * 32 + lane;      // tile row owned by this thread
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
     const float s = a.s;
-    TileWalk w{rr.begin, rr.end, 0};
-    Tile tl;
-    int i0 = 0, cc0 = 0, ti = 0;
-    bool ok = true;
-    // Every decision to stop is made jointly by the four warps of a group
-    // (bar.red.and), so no warp is ever left waiting at its group's barrier.
-    while (ok && w.next(goff, tl)) {
-      const int r0 = pt.rank_off[tl.g], rg = pt.rank_off[tl.g + 1] - r0;
-      const bool live = m < tl.cnt;
-      // sHs is free once the previous tile's last D chunk has completed
-      bool w_ok = ti == 0 || mbar_wait(&dfull[(cc0 - 1) & 1], ((cc0 - 1) >> 1) & 1);
-      // H -> bf16 operand (row m), columns split between the two groups
+    // H operand of tile t (tile number tn) into buffer tn % NBH: this warp's
+    // rows, its group's share of the columns
+    auto stage_h = [&](const Tile& t, int tn) {
+      const uint32_t sHs = sHs0 + (tn % NBH) * C::kHs;
+      if (quarter * 32 >= t.cnt) return;  // no live row: these H rows feed only D rows nobody reads
+      const bool live = m < t.cnt;
+      const int rg = pt.rank_off[t.g + 1] - pt.rank_off[t.g];
       if (!SHARED) {
-        w_ok = w_ok && mbar_wait(&hacc, ti & 1);
-        w_ok = __all_sync(0xffffffffu, w_ok);
         tc_fence_after();
-        for (int c0 = grp * 16; c0 < RP && w_ok; c0 += 32) {
+        for (int c0 = grp * 16; c0 < RP; c0 += 16 * kNGrp) {
           uint32_t r[16];
-          tmem_ld16(tmem + lane_base + c0, r);
+          tmem_ld16(tmem + lane_base + (tn & 1) * C::kHcol + c0, r);
           tmem_ld_wait();
           float v[16];
 #pragma unroll
-          for (int q = 0; q < 16; ++q) v[q] = (live && c0 + q < rg) ? __uint_as_float(r[q]) : 0.f;
+          for (int qq = 0; qq < 16; ++qq) v[qq] = (live && c0 + qq < rg) ? __uint_as_float(r[qq]) : 0.f;
           if (live && a.Hsave != nullptr) {
-            float* hrow = a.Hsave + (int64_t)(tl.start + m) * pt.rank_max;
+            float* hrow = a.Hsave + (int64_t)(t.start + m) * pt.rank_max;
 #pragma unroll
-            for (int q = 0; q < 16; ++q)
-              if (c0 + q < pt.rank_max) hrow[c0 + q] = v[q];
+            for (int qq = 0; qq < 16; ++qq)
+              if (c0 + qq < pt.rank_max) hrow[c0 + qq] = v[qq];
           }
 #pragma unroll
           for (int h = 0; h < 2; ++h) {
@@ -394,15 +455,15 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
             sts128(sHs + (col >> 6) * kBlk + sw128_off(m, (col & 63) >> 3), o);
           }
         }
-      } else if (w_ok) {
-        const int u = live ? a.row_uniq[tl.start + m] : -1;
+      } else {
+        const int u = live ? a.row_uniq[t.start + m] : -1;
 #pragma unroll
         for (int j = 0; j < NPROJ; ++j) {
           const float* hp = a.Hu[j] + (int64_t)(u < 0 ? 0 : u) * pt.rank_max;
-          for (int c8 = grp * 8; c8 < RP; c8 += 16) {
+          for (int c8 = grp * 8; c8 < RP; c8 += 8 * kNGrp) {
             float v[8];
 #pragma unroll
-            for (int q = 0; q < 8; ++q) v[q] = (u >= 0 && c8 + q < rg) ? hp[c8 + q] : 0.f;
+            for (int qq = 0; qq < 8; ++qq) v[qq] = (u >= 0 && c8 + qq < rg) ? hp[c8 + qq] : 0.f;
             uint4 o;
             o.x = pack_bf16x2(v[0], v[1]);
             o.y = pack_bf16x2(v[2], v[3]);
@@ -413,22 +474,45 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
           }
         }
       }
+    };
+    // H of tile tn (tile t): wait until the buffer's previous tile is done
+    // with it and (down) tn's K loop has completed, stage, publish
+    auto prepare_h = [&](const Tile& t, int tn) -> bool {
+      bool w = true;
+      if (tn >= NBH) w = mbar_wait(&hs_free[tn % NBH], ((tn - NBH) / NBH) & 1);
+      if (!SHARED) w = w && mbar_wait(&hacc[tn & 1], (tn >> 1) & 1);
+      if (!__all_sync(0xffffffffu, w)) return false;
+      stage_h(t, tn);
       fence_proxy_async_smem();
       tc_fence_before();
-      ok = named_bar_and(1 + grp, 128, w_ok);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&hs_ready[tn & 1]);
+      return true;
+    };
+    int q = 0, ib = SHARED ? 0 : NK, cc0 = 0, ti = 0;
+    bool ok = true;
+    Tile cur, nxt;
+    bool has_cur = queue_next(tq, q, a.tiles, cur, false, &ok);
+    if (has_cur) ok = prepare_h(cur, 0);
+    while (has_cur && ok) {
+      const bool has_nxt = queue_next(tq, q, a.tiles, nxt, false, &ok);
       if (!ok) break;
-      if (lane == 0) mbar_arrive(&hs_ready);
-      // the chunks of this group's parity: Y += s * D on this warp's 32 rows, then row stores
-      for (int c = (grp ^ cc0) & 1; c < nch; c += 2) {
-        const int cc = cc0 + c, i = i0 + NK + c, sl = i % S, b = cc & 1, n0 = c * kChunk;
-        bool c_ok = mbar_wait(&full[sl], (i / S) & 1) && mbar_wait(&dfull[b], (cc >> 1) & 1);
-        c_ok = __all_sync(0xffffffffu, c_ok);
+      const bool inter = !SHARED && has_nxt;
+      // gate/up with two H buffers: gather the next tile's H now, while this tile streams
+      const bool early = SHARED && NBH == 2 && has_nxt;
+      if (early && !(ok = prepare_h(nxt, ti + 1))) break;
+      const bool qlive = quarter * 32 < cur.cnt;  // this warp has live rows (warp-uniform)
+      for (int c = ((grp - cc0) % kNGrp + kNGrp) % kNGrp; c < nch; c += kNGrp) {
+        const int cc = cc0 + c, i = ib + c;
+        const int sl = i % S, b = cc % kNGrp, n0 = c * kChunk;
+        ok = __all_sync(0xffffffffu, mbar_wait(&full[sl], (i / S) & 1) && mbar_wait(&dfull[b], (cc / kNGrp) & 1));
+        if (!ok) break;
+        tc_fence_after();
         const uint32_t base = slot0 + sl * C::kSlot;
-        if (c_ok) {
-          tc_fence_after();
+        if (qlive) {
 #pragma unroll
           for (int j = 0; j < NPROJ; ++j) {
-            const uint32_t ta = tmem + lane_base + dbase + (b * NPROJ + j) * kChunk;
+            const uint32_t ta = tmem + lane_base + C::kDBase + (b * NPROJ + j) * kChunk;
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
               uint32_t r[32];
@@ -436,10 +520,10 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
               tmem_ld16(ta + h * 32 + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
               tmem_ld_wait();
 #pragma unroll
-              for (int q = 0; q < 4; ++q) {
-                const uint32_t addr = base + j * kBlk + sw128_off(m, h * 4 + q);
+              for (int qq = 0; qq < 4; ++qq) {
+                const uint32_t addr = base + j * kBlk + sw128_off(m, h * 4 + qq);
                 const uint4 y = lds128(addr);
-                const uint32_t* dq = &r[q * 8];
+                const uint32_t* dq = &r[qq * 8];
                 const float2 f0 = unpack_bf16x2(y.x), f1 = unpack_bf16x2(y.y), f2 = unpack_bf16x2(y.z),
                              f3 = unpack_bf16x2(y.w);
                 uint4 o;
@@ -451,36 +535,41 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
               }
             }
           }
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&dempty[b]);
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&dempty[b]);
+        if (qlive) {
           // this warp's 32 rows, 128 contiguous bytes each: 4 rows per instruction
 #pragma unroll
           for (int j = 0; j < NPROJ; ++j)
 #pragma unroll
             for (int it = 0; it < 8; ++it) {
               const int row = quarter * 32 + it * 4 + (lane >> 3), ch = lane & 7, col = n0 + ch * 8;
-              if (row < tl.cnt && col < d_out) {
+              if (row < cur.cnt && col < d_out) {
                 const uint4 v = lds128(base + j * kBlk + sw128_off(row, ch));
-                *reinterpret_cast<uint4*>(a.Y[j] + (int64_t)(tl.start + row) * d_out + col) = v;
+                *reinterpret_cast<uint4*>(a.Y[j] + (int64_t)(cur.start + row) * d_out + col) = v;
               }
             }
-          fence_proxy_async_smem();
         }
-        ok = named_bar_and(1 + grp, 128, c_ok);
-        if (!ok) break;
-        if (warp == 2 + 4 * grp && lane == 0) mbar_arrive(&empty[sl]);
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&emptyC[sl]);
       }
-      i0 += NK + nch;
+      if (!ok) break;
+      if (has_nxt && !early && !(ok = prepare_h(nxt, ti + 1))) break;
+      ib += nch + (inter ? NK : 0);
       cc0 += nch;
       ++ti;
+      cur = nxt;
+      has_cur = has_nxt;
     }
     if (!ok) bad = true;
   }
   __syncwarp();  // reconverge the single-lane roles before the CTA barrier
   tc_fence_before();
   if (__syncthreads_or(bad) && tid == 0) atomicOr(a.err, kErrTimeout);
-  if (warp == 0) tmem_dealloc(tmem, 256);
+  if (warp == 0) tmem_dealloc(tmem, kRowsTmem);
 }
 
 template <typename K>
@@ -500,7 +589,7 @@ cudaError_t launch_h_t(const PlanTables& pt, const FwdHLaunch& a, cudaStream_t s
 
 template <int RP, int NPROJ, bool SHARED>
 cudaError_t launch_rows_t(const PlanTables& pt, const FwdRowsLaunch& a, cudaStream_t st) {
-  using C = RowsFwdCfg<RP, NPROJ>;
+  using C = RowsFwdCfg<RP, NPROJ, SHARED>;
   auto kern = k_fwd_rows<RP, NPROJ, SHARED>;
   cudaError_t e = set_smem(kern, C::kSmem);
   if (e != cudaSuccess || a.grid <= 0) return e;

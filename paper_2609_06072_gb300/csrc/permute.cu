@@ -4,8 +4,9 @@
 // A(x) of Sec. 3.5 are deduplicated into a (g, t)-sorted unique list.
 //
 // Three launches, no inter-CTA waiting:
-//   k_perm_count   per 256-token chunk: pairs per expert, unique pairs per group
-//   k_perm_scan    one CTA: totals, segment offsets, per-chunk bases, tile tables
+//   k_perm_count   per 64-token chunk: pairs per expert, unique pairs per group
+//   k_perm_scan    one CTA: totals, segment offsets, per-chunk bases, the
+//                  unique-pair tile, row tile and row split tables
 //   k_perm_scatter per chunk: rank of each pair inside its expert (bitmask
 //                  popcounts over the chunk's earlier tokens) -> row
 // Integer-only and order-independent, so bit-exact and deterministic.
@@ -152,8 +153,7 @@ __global__ void __launch_bounds__(1024) k_perm_scan(const __grid_constant__ Plan
                                                     int32_t* __restrict__ expert_off,
                                                     int32_t* __restrict__ expert_cnt,
                                                     int32_t* __restrict__ uniq_off, Tile* __restrict__ tiles_sh,
-                                                    Tile* __restrict__ tiles_row, Tile* __restrict__ splits_sh,
-                                                    Tile* __restrict__ splits_row) {
+                                                    Tile* __restrict__ tiles_row, Tile* __restrict__ splits_row) {
   __shared__ int32_t totE[ACE_MAX_EXPERTS];
   __shared__ int32_t rowsG[ACE_MAX_EXPERTS];
   __shared__ int32_t totU[ACE_MAX_EXPERTS];
@@ -203,15 +203,11 @@ __global__ void __launch_bounds__(1024) k_perm_scan(const __grid_constant__ Plan
   __syncthreads();
   column_bases(chunk_cntE, n_chunks, E, partE, eoff, chunk_baseE);
   column_bases(chunk_cntU, n_chunks, G, partU, uofs, chunk_baseU);
-  const int per_split = kTileM * pt.nt_split;
-  int n;
-  n = build_tiles(totU, uofs, G, kTileM, tiles_sh, scratch);
+  int n = build_tiles(totU, uofs, G, kTileM, tiles_sh, scratch);
   if (tid == 0) counts[kCntTilesSh] = n;
   n = build_tiles(rowsG, gofs, G, kTileM, tiles_row, scratch);
   if (tid == 0) counts[kCntTilesRow] = n;
-  n = build_tiles(totU, uofs, G, per_split, splits_sh, scratch);
-  if (tid == 0) counts[kCntSplitsSh] = n;
-  n = build_tiles(rowsG, gofs, G, per_split, splits_row, scratch);
+  n = build_tiles(rowsG, gofs, G, kTileM * pt.nt_split, splits_row, scratch);
   if (tid == 0) counts[kCntSplitsRow] = n;
 }
 
@@ -322,7 +318,7 @@ cudaError_t launch_permute(const PlanTables& pt, const int32_t* topk_idx, int32_
                                   at<int32_t>(ws, L.counts), at<int32_t>(ws, L.group_off),
                                   at<int32_t>(ws, L.expert_off), at<int32_t>(ws, L.expert_cnt),
                                   at<int32_t>(ws, L.uniq_off), at<Tile>(ws, L.tiles_sh), at<Tile>(ws, L.tiles_row),
-                                  at<Tile>(ws, L.splits_sh), at<Tile>(ws, L.splits_row));
+                                  at<Tile>(ws, L.splits_row));
   if (C > 0) {
     size_t sm3 = sizeof(uint32_t) * (size_t)(pt.E + pt.G) * (kPermTB / 32);
     k_perm_scatter<<<C, kPermTB, sm3, st>>>(pt, topk_idx, T, at<int32_t>(ws, L.chunk_baseE),

@@ -24,6 +24,8 @@ struct PlanTables {
   int32_t rank_pad;  // MMA N of one projection's rank block (16/32/64/128)
   int32_t nt_split;  // tiles per backward split
   int16_t e2g[ACE_MAX_EXPERTS];
+  int16_t eorder[ACE_MAX_EXPERTS];  // experts in (g, e) order
+  int16_t gfirst[ACE_MAX_EXPERTS];  // position in eorder of group g's first expert
   int32_t rank_off[ACE_MAX_EXPERTS + 1];
 };
 
@@ -36,8 +38,8 @@ struct Tile {
 
 // Byte layout of the permutation workspace for T tokens.
 struct PermLayout {
-  size_t err, counts, sched, group_off, expert_off, expert_cnt, uniq_off, row_pair, pair_row, pair_g, row_uniq, uniq_tok,
-      tok_uniq;
+  size_t err, counts, sched, group_off, expert_off, expert_cnt, uniq_off, tot_u, row_pair, pair_row, pair_g, row_uniq,
+      uniq_tok, tok_uniq;
   size_t chunk_cntE, chunk_cntU, chunk_baseE, chunk_baseU, chunk_err;
   size_t tiles_sh, tiles_row, splits_row;
   size_t total;
@@ -72,6 +74,7 @@ inline PermLayout perm_layout(const PlanTables& pt, int32_t T) {
   L.expert_off = take(4 * (size_t)pt.E);
   L.expert_cnt = take(4 * (size_t)pt.E);
   L.uniq_off = take(4 * (size_t)(pt.G + 1));
+  L.tot_u = take(4 * (size_t)pt.G);
   L.row_pair = take(4 * (size_t)R);
   L.pair_row = take(4 * (size_t)R);
   L.pair_g = take(4 * (size_t)R);

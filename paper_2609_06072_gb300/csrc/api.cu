@@ -174,6 +174,14 @@ ace_status ace_plan_create(ace_plan** out, const ace_layer_desc* desc) {
   p->pt.rank_pad = rank_max <= 16 ? 16 : rank_max <= 32 ? 32 : rank_max <= 64 ? 64 : 128;
   p->pt.nt_split = pt_nt_split(p->pt.rank_pad);
   for (int e = 0; e < D.E; ++e) p->pt.e2g[e] = (int16_t)D.e2g[e];
+  {
+    int pos = 0;
+    for (int g = 0; g < D.G; ++g) {
+      p->pt.gfirst[g] = (int16_t)pos;
+      for (int e = 0; e < D.E; ++e)
+        if (D.e2g[e] == g) p->pt.eorder[pos++] = (int16_t)e;
+    }
+  }
   for (int g = 0; g <= D.G; ++g) p->pt.rank_off[g] = D.rank_off[g];
   p->T_max = D.T_max;
   p->flags = D.flags;

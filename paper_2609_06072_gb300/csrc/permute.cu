@@ -5,10 +5,13 @@
 //
 // Three launches, no inter-CTA waiting:
 //   k_perm_count   per 64-token chunk: pairs per expert, unique pairs per group
-//   k_perm_scan    one CTA: totals, segment offsets, per-chunk bases, the
-//                  unique-pair tile, row tile and row split tables
-//   k_perm_scatter per chunk: rank of each pair inside its expert (bitmask
-//                  popcounts over the chunk's earlier tokens) -> row
+//   k_perm_colscan one CTA per expert and per group: prefix over the chunks
+//                  of that column and its total; CTA 0 also gathers the
+//                  routing-error flags
+//   k_perm_scatter per chunk: segment offsets from the totals (a warp scan in
+//                  (g, e) order), rank of each pair inside its expert
+//                  (bitmask popcounts over the chunk's earlier tokens) -> row;
+//                  CTA 0 writes the offsets and the tile tables
 // Integer-only and order-independent, so bit-exact and deterministic.
 #include <algorithm>
 #include <cstdint>
@@ -99,116 +102,58 @@ __device__ int build_tiles(const int32_t* n_g, const int32_t* off_g, int G, int 
   return total;
 }
 
-// Per-column prefix over chunks of a [C x ncol] count matrix, parallel over
-// (column, part) with P parts per column.  Pass 1 writes each column's total;
-// pass 2 writes base[c][col] = col_base[col] + sum_{c' < c} cnt[c'][col].
-__device__ void column_totals(const int32_t* __restrict__ cnt, int C, int ncol, int32_t* part_sum /*smem 1024*/,
-                              int32_t* total /*smem [ncol]*/) {
-  const int tid = threadIdx.x;
-  int P = 1;
-  while (P * 2 * ncol <= (int)blockDim.x && P < 32) P *= 2;
-  const int len = (C + P - 1) / P;
-  if (tid < ncol * P) {
-    const int col = tid / P, part = tid % P;
-    int s = 0;
-    for (int c = part * len; c < min(C, (part + 1) * len); ++c) s += cnt[(int64_t)c * ncol + col];
-    part_sum[tid] = s;
+__device__ __forceinline__ int warp_incl_scan(int v) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int x = __shfl_up_sync(0xffffffffu, v, o);
+    if (lane >= o) v += x;
   }
-  __syncthreads();
-  for (int col = tid; col < ncol; col += blockDim.x) {
-    int run = 0;
-    for (int part = 0; part < P; ++part) {
-      const int v = part_sum[col * P + part];
-      part_sum[col * P + part] = run;
-      run += v;
-    }
-    total[col] = run;
-  }
-  __syncthreads();
-}
-__device__ void column_bases(const int32_t* __restrict__ cnt, int C, int ncol, const int32_t* part_sum,
-                             const int32_t* col_base, int32_t* __restrict__ base) {
-  const int tid = threadIdx.x;
-  int P = 1;
-  while (P * 2 * ncol <= (int)blockDim.x && P < 32) P *= 2;
-  const int len = (C + P - 1) / P;
-  if (tid < ncol * P) {
-    const int col = tid / P, part = tid % P;
-    int run = col_base[col] + part_sum[tid];
-    for (int c = part * len; c < min(C, (part + 1) * len); ++c) {
-      base[(int64_t)c * ncol + col] = run;
-      run += cnt[(int64_t)c * ncol + col];
-    }
-  }
-  __syncthreads();
+  return v;
 }
 
-__global__ void __launch_bounds__(1024) k_perm_scan(const __grid_constant__ PlanTables pt, int n_chunks,
-                                                    const int32_t* __restrict__ chunk_cntE,
-                                                    const int32_t* __restrict__ chunk_cntU,
-                                                    const int32_t* __restrict__ chunk_err,
-                                                    int32_t* __restrict__ chunk_baseE,
-                                                    int32_t* __restrict__ chunk_baseU, int32_t* __restrict__ err,
-                                                    int32_t* __restrict__ counts, int32_t* __restrict__ group_off,
-                                                    int32_t* __restrict__ expert_off,
-                                                    int32_t* __restrict__ expert_cnt,
-                                                    int32_t* __restrict__ uniq_off, Tile* __restrict__ tiles_sh,
-                                                    Tile* __restrict__ tiles_row, Tile* __restrict__ splits_row) {
-  __shared__ int32_t totE[ACE_MAX_EXPERTS];
-  __shared__ int32_t rowsG[ACE_MAX_EXPERTS];
-  __shared__ int32_t totU[ACE_MAX_EXPERTS];
-  __shared__ int32_t gofs[ACE_MAX_EXPERTS + 1];
-  __shared__ int32_t uofs[ACE_MAX_EXPERTS + 1];
-  __shared__ int32_t scratch[ACE_MAX_EXPERTS + 1];
-  __shared__ int32_t eoff[ACE_MAX_EXPERTS];
-  __shared__ int32_t partE[1024];
-  __shared__ int32_t partU[1024];
+// Column col of the [C x ncol] chunk-count matrix (experts, then groups):
+// base[c][col] = sum of cnt[c'][col] over c' < c, and the column total.
+__global__ void __launch_bounds__(256) k_perm_colscan(const __grid_constant__ PlanTables pt, int n_chunks,
+                                                      const int32_t* __restrict__ chunk_cntE,
+                                                      const int32_t* __restrict__ chunk_cntU,
+                                                      const int32_t* __restrict__ chunk_err,
+                                                      int32_t* __restrict__ chunk_baseE,
+                                                      int32_t* __restrict__ chunk_baseU, int32_t* __restrict__ totE,
+                                                      int32_t* __restrict__ totU, int32_t* __restrict__ err) {
+  __shared__ int32_t wsum[8];
   __shared__ int32_t err_s;
-  const int tid = threadIdx.x;
-  const int E = pt.E, G = pt.G;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const bool isE = (int)blockIdx.x < pt.E;
+  const int ncol = isE ? pt.E : pt.G, col = isE ? blockIdx.x : blockIdx.x - pt.E;
+  const int32_t* cnt = isE ? chunk_cntE : chunk_cntU;
+  int32_t* base = isE ? chunk_baseE : chunk_baseU;
   if (tid == 0) err_s = 0;
-  for (int g = tid; g < G; g += blockDim.x) rowsG[g] = 0;
-  __syncthreads();
-  for (int c = tid; c < n_chunks; c += blockDim.x)
-    if (chunk_err[c]) atomicOr(&err_s, chunk_err[c]);
-  column_totals(chunk_cntE, n_chunks, E, partE, totE);
-  column_totals(chunk_cntU, n_chunks, G, partU, totU);
-  for (int e = tid; e < E; e += blockDim.x) atomicAdd(&rowsG[pt.e2g[e]], totE[e]);
-  __syncthreads();
-  if (tid == 0) {
-    gofs[0] = 0;
-    uofs[0] = 0;
-    for (int g = 0; g < G; ++g) {
-      gofs[g + 1] = gofs[g] + rowsG[g];
-      uofs[g + 1] = uofs[g] + totU[g];
+  int carry = 0;
+  for (int c0 = 0; c0 < n_chunks; c0 += 256) {
+    const int c = c0 + tid;
+    const int v = c < n_chunks ? cnt[(int64_t)c * ncol + col] : 0;
+    const int x = warp_incl_scan(v);
+    if (lane == 31) wsum[warp] = x;
+    __syncthreads();
+    if (warp == 0) {
+      int w = lane < 8 ? wsum[lane] : 0;
+      w = warp_incl_scan(w);
+      if (lane < 8) wsum[lane] = w;
     }
-    *err = err_s ? kErrIndex : 0;
-    counts[kCntU] = uofs[G];
-    counts[kCntRows] = gofs[G];
+    __syncthreads();
+    if (c < n_chunks) base[(int64_t)c * ncol + col] = carry + (warp > 0 ? wsum[warp - 1] : 0) + x - v;
+    carry += wsum[7];
+    __syncthreads();
   }
-  __syncthreads();
-  for (int g = tid; g <= G; g += blockDim.x) {
-    group_off[g] = gofs[g];
-    uniq_off[g] = uofs[g];
+  if (tid == 0) (isE ? totE : totU)[col] = carry;
+  if (blockIdx.x == 0) {
+    int e = 0;
+    for (int c = tid; c < n_chunks; c += 256) e |= chunk_err[c];
+    if (e) atomicOr(&err_s, e);
+    __syncthreads();
+    if (tid == 0) *err = err_s ? kErrIndex : 0;
   }
-  for (int e = tid; e < E; e += blockDim.x) {
-    const int g = pt.e2g[e];
-    int start = gofs[g];
-    for (int e2 = 0; e2 < e; ++e2)
-      if (pt.e2g[e2] == g) start += totE[e2];
-    eoff[e] = start;
-    expert_off[e] = start;
-    expert_cnt[e] = totE[e];
-  }
-  __syncthreads();
-  column_bases(chunk_cntE, n_chunks, E, partE, eoff, chunk_baseE);
-  column_bases(chunk_cntU, n_chunks, G, partU, uofs, chunk_baseU);
-  int n = build_tiles(totU, uofs, G, kTileM, tiles_sh, scratch);
-  if (tid == 0) counts[kCntTilesSh] = n;
-  n = build_tiles(rowsG, gofs, G, kTileM, tiles_row, scratch);
-  if (tid == 0) counts[kCntTilesRow] = n;
-  n = build_tiles(rowsG, gofs, G, kTileM * pt.nt_split, splits_row, scratch);
-  if (tid == 0) counts[kCntSplitsRow] = n;
 }
 
 __device__ __forceinline__ int prefix_bits(const uint32_t* mask, int tid) {
@@ -218,30 +163,90 @@ __device__ __forceinline__ int prefix_bits(const uint32_t* mask, int tid) {
   return r + __popc(mask[w] & ((1u << (tid & 31)) - 1u));
 }
 
+struct ScatterOut {
+  int32_t* row_pair;
+  int32_t* pair_row;
+  int32_t* pair_g;
+  int32_t* row_uniq;
+  int32_t* uniq_tok;
+  int32_t* tok_uniq;
+  int32_t* counts;
+  int32_t* group_off;
+  int32_t* uniq_off;
+  int32_t* expert_off;
+  Tile* tiles_sh;
+  Tile* tiles_row;
+  Tile* splits_row;
+};
+
 __global__ void __launch_bounds__(kPermTB) k_perm_scatter(const __grid_constant__ PlanTables pt,
                                                           const int32_t* __restrict__ idx, int T,
                                                           const int32_t* __restrict__ chunk_baseE,
                                                           const int32_t* __restrict__ chunk_baseU,
-                                                          int32_t* __restrict__ row_pair,
-                                                          int32_t* __restrict__ pair_row,
-                                                          int32_t* __restrict__ pair_g,
-                                                          int32_t* __restrict__ row_uniq,
-                                                          int32_t* __restrict__ uniq_tok,
-                                                          int32_t* __restrict__ tok_uniq) {
+                                                          const int32_t* __restrict__ totE,
+                                                          const int32_t* __restrict__ totU, const ScatterOut o) {
   constexpr int W = kPermTB / 32;
   extern __shared__ uint32_t msk[];
   uint32_t* mE = msk;                    // [E][W]
   uint32_t* mU = msk + (size_t)pt.E * W; // [G][W]
-  const int tid = threadIdx.x;
-  for (int i = tid; i < (pt.E + pt.G) * W; i += blockDim.x) msk[i] = 0;
+  __shared__ int32_t eoff[ACE_MAX_EXPERTS];      // first row of each expert segment
+  __shared__ int32_t uoff[ACE_MAX_EXPERTS + 1];  // first unique pair of each group
+  __shared__ int32_t goff[ACE_MAX_EXPERTS + 1];  // first row of each group
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int E = pt.E, G = pt.G;
+  for (int i = tid; i < (E + G) * W; i += blockDim.x) msk[i] = 0;
+  // segment offsets: rows in (g, e) order (warp 0), unique pairs in g order (warp 1)
+  if (warp == 0) {
+    int carry = 0;
+    for (int i0 = 0; i0 < E; i0 += 32) {
+      const int i = i0 + lane, e = i < E ? pt.eorder[i] : 0;
+      const int v = i < E ? totE[e] : 0, x = warp_incl_scan(v);
+      if (i < E) eoff[e] = carry + x - v;
+      carry += __shfl_sync(0xffffffffu, x, 31);
+    }
+    if (lane == 0) goff[G] = carry;
+  } else if (warp == 1) {
+    int carry = 0;
+    for (int g0 = 0; g0 < G; g0 += 32) {
+      const int g = g0 + lane;
+      const int v = g < G ? totU[g] : 0, x = warp_incl_scan(v);
+      if (g < G) uoff[g] = carry + x - v;
+      carry += __shfl_sync(0xffffffffu, x, 31);
+    }
+    if (lane == 0) uoff[G] = carry;
+  }
   __syncthreads();
+  for (int g = tid; g < G; g += blockDim.x) goff[g] = eoff[pt.eorder[pt.gfirst[g]]];
+  __syncthreads();
+  if (blockIdx.x == 0) {
+    // the offsets and the tile tables the other calls read
+    __shared__ int32_t rows_g[ACE_MAX_EXPERTS];
+    __shared__ int32_t scratch[ACE_MAX_EXPERTS + 1];
+    for (int g = tid; g <= G; g += blockDim.x) {
+      o.group_off[g] = goff[g];
+      o.uniq_off[g] = uoff[g];
+      if (g < G) rows_g[g] = goff[g + 1] - goff[g];
+    }
+    for (int e = tid; e < E; e += blockDim.x) o.expert_off[e] = eoff[e];
+    if (tid == 0) {
+      o.counts[kCntU] = uoff[G];
+      o.counts[kCntRows] = goff[G];
+    }
+    __syncthreads();
+    int n = build_tiles(totU, uoff, G, kTileM, o.tiles_sh, scratch);
+    if (tid == 0) o.counts[kCntTilesSh] = n;
+    n = build_tiles(rows_g, goff, G, kTileM, o.tiles_row, scratch);
+    if (tid == 0) o.counts[kCntTilesRow] = n;
+    n = build_tiles(rows_g, goff, G, kTileM * pt.nt_split, o.splits_row, scratch);
+    if (tid == 0) o.counts[kCntSplitsRow] = n;
+  }
   const int c = blockIdx.x;
   const int t = c * kPermTB + tid;
   const int k = pt.k;
   int e[kMaxK];
   bool ok = false;
   if (t < T) {
-    ok = read_token(idx, t, k, pt.E, e);
+    ok = read_token(idx, t, k, E, e);
     if (ok) {
       const uint32_t bit = 1u << (tid & 31);
       for (int j = 0; j < k; ++j) {
@@ -254,19 +259,19 @@ __global__ void __launch_bounds__(kPermTB) k_perm_scatter(const __grid_constant_
   if (t >= T) return;
   if (!ok) {
     for (int j = 0; j < k; ++j) {
-      tok_uniq[(int64_t)t * k + j] = -1;
-      pair_g[(int64_t)t * k + j] = -1;
+      o.tok_uniq[(int64_t)t * k + j] = -1;
+      o.pair_g[(int64_t)t * k + j] = -1;
     }
     return;
   }
   int rows_j[kMaxK];
   for (int j = 0; j < k; ++j) {
-    const int row = chunk_baseE[(int64_t)c * pt.E + e[j]] + prefix_bits(&mE[e[j] * W], tid);
+    const int row = eoff[e[j]] + chunk_baseE[(int64_t)c * E + e[j]] + prefix_bits(&mE[e[j] * W], tid);
     const int p = t * k + j;
     rows_j[j] = row;
-    pair_row[p] = row;
-    pair_g[p] = pt.e2g[e[j]];
-    row_pair[row] = p;
+    o.pair_row[p] = row;
+    o.pair_g[p] = pt.e2g[e[j]];
+    o.row_pair[row] = p;
   }
   // distinct groups of the token, ascending
   int n_u = 0;
@@ -278,15 +283,15 @@ __global__ void __launch_bounds__(kPermTB) k_perm_scatter(const __grid_constant_
       if (g > last && g < nxt) nxt = g;
     }
     if (nxt == 0x7fffffff) break;
-    const int u = chunk_baseU[(int64_t)c * pt.G + nxt] + prefix_bits(&mU[nxt * W], tid);
-    uniq_tok[u] = t;
-    tok_uniq[(int64_t)t * k + n_u] = u;
+    const int u = uoff[nxt] + chunk_baseU[(int64_t)c * G + nxt] + prefix_bits(&mU[nxt * W], tid);
+    o.uniq_tok[u] = t;
+    o.tok_uniq[(int64_t)t * k + n_u] = u;
     for (int j = 0; j < k; ++j)
-      if (pt.e2g[e[j]] == nxt) row_uniq[rows_j[j]] = u;
+      if (pt.e2g[e[j]] == nxt) o.row_uniq[rows_j[j]] = u;
     ++n_u;
     last = nxt;
   }
-  for (int j = n_u; j < k; ++j) tok_uniq[(int64_t)t * k + j] = -1;
+  for (int j = n_u; j < k; ++j) o.tok_uniq[(int64_t)t * k + j] = -1;
 }
 
 __global__ void k_rows_copy(const int32_t* __restrict__ row_pair, const uint4* __restrict__ src,
@@ -312,21 +317,29 @@ cudaError_t launch_permute(const PlanTables& pt, const int32_t* topk_idx, int32_
     k_perm_count<<<C, kPermTB, sm1, st>>>(pt, topk_idx, T, at<int32_t>(ws, L.chunk_cntE),
                                           at<int32_t>(ws, L.chunk_cntU), at<int32_t>(ws, L.chunk_err));
   }
-  k_perm_scan<<<1, 1024, 0, st>>>(pt, C, at<int32_t>(ws, L.chunk_cntE), at<int32_t>(ws, L.chunk_cntU),
-                                  at<int32_t>(ws, L.chunk_err), at<int32_t>(ws, L.chunk_baseE),
-                                  at<int32_t>(ws, L.chunk_baseU), at<int32_t>(ws, L.err),
-                                  at<int32_t>(ws, L.counts), at<int32_t>(ws, L.group_off),
-                                  at<int32_t>(ws, L.expert_off), at<int32_t>(ws, L.expert_cnt),
-                                  at<int32_t>(ws, L.uniq_off), at<Tile>(ws, L.tiles_sh), at<Tile>(ws, L.tiles_row),
-                                  at<Tile>(ws, L.splits_row));
-  if (C > 0) {
-    size_t sm3 = sizeof(uint32_t) * (size_t)(pt.E + pt.G) * (kPermTB / 32);
-    k_perm_scatter<<<C, kPermTB, sm3, st>>>(pt, topk_idx, T, at<int32_t>(ws, L.chunk_baseE),
-                                            at<int32_t>(ws, L.chunk_baseU), at<int32_t>(ws, L.row_pair),
-                                            at<int32_t>(ws, L.pair_row), at<int32_t>(ws, L.pair_g),
-                                            at<int32_t>(ws, L.row_uniq), at<int32_t>(ws, L.uniq_tok),
-                                            at<int32_t>(ws, L.tok_uniq));
-  }
+  k_perm_colscan<<<pt.E + pt.G, 256, 0, st>>>(pt, C, at<int32_t>(ws, L.chunk_cntE), at<int32_t>(ws, L.chunk_cntU),
+                                                at<int32_t>(ws, L.chunk_err), at<int32_t>(ws, L.chunk_baseE),
+                                                at<int32_t>(ws, L.chunk_baseU), at<int32_t>(ws, L.expert_cnt),
+                                                at<int32_t>(ws, L.tot_u), at<int32_t>(ws, L.err));
+  ScatterOut o;
+  o.row_pair = at<int32_t>(ws, L.row_pair);
+  o.pair_row = at<int32_t>(ws, L.pair_row);
+  o.pair_g = at<int32_t>(ws, L.pair_g);
+  o.row_uniq = at<int32_t>(ws, L.row_uniq);
+  o.uniq_tok = at<int32_t>(ws, L.uniq_tok);
+  o.tok_uniq = at<int32_t>(ws, L.tok_uniq);
+  o.counts = at<int32_t>(ws, L.counts);
+  o.group_off = at<int32_t>(ws, L.group_off);
+  o.uniq_off = at<int32_t>(ws, L.uniq_off);
+  o.expert_off = at<int32_t>(ws, L.expert_off);
+  o.tiles_sh = at<Tile>(ws, L.tiles_sh);
+  o.tiles_row = at<Tile>(ws, L.tiles_row);
+  o.splits_row = at<Tile>(ws, L.splits_row);
+  size_t sm3 = sizeof(uint32_t) * (size_t)(pt.E + pt.G) * (kPermTB / 32);
+  // one CTA at least: CTA 0 writes the offsets and tables even when T = 0
+  k_perm_scatter<<<C > 0 ? C : 1, kPermTB, sm3, st>>>(pt, topk_idx, T, at<int32_t>(ws, L.chunk_baseE),
+                                                     at<int32_t>(ws, L.chunk_baseU), at<int32_t>(ws, L.expert_cnt),
+                                                     at<int32_t>(ws, L.tot_u), o);
   return cudaGetLastError();
 }
 

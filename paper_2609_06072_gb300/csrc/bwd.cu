@@ -140,7 +140,7 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   __shared__ __align__(8) uint64_t fullA[SA], emptyA[SA], fullB[SB], emptyB[SB];
   __shared__ __align__(8) uint64_t dbt_full[2], dbt_empty[2], d_full[2], d_empty[2], da_full[2], da_empty[2];
-  __shared__ __align__(8) uint64_t dh_full, hs_ready;
+  __shared__ __align__(8) uint64_t dh_full, hs_ready, ops_ready;
   __shared__ uint32_t tslot;
   static_assert(NT * RP <= 128, "dH accumulators must fit below the dB^T columns");
 
@@ -178,25 +178,10 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
     }
     mbar_init(&dh_full, 1);
     mbar_init(&hs_ready, 1);
+    mbar_init(&ops_ready, 8);  // the epilogue warps, once the H operand is staged
     fence_mbar_init();
   }
   if (warp == 0) tmem_alloc(&tslot, C::kTmem);
-  // H operand slots (all threads): bf16 of the saved H of each row
-  for (int idx = tid; idx < ntiles * kTileM; idx += kThreadsWS) {
-    const int i = idx / kTileM, m = idx % kTileM;
-    const int row = sp.start + i * kTileM + m;
-    const bool live = i * kTileM + m < sp.cnt;
-    const int hrow = !live ? -1 : (MODE == MODE_SHARED ? a.row_uniq[row] : row);
-    const float* hp = a.H[proj] + (int64_t)(hrow < 0 ? 0 : hrow) * pt.rank_max;
-#pragma unroll
-    for (int c8 = 0; c8 < RP; c8 += 8) {
-      float v[8];
-#pragma unroll
-      for (int q = 0; q < 8; ++q) v[q] = (hrow >= 0 && c8 + q < rg) ? hp[c8 + q] : 0.f;
-      sts128(sOps + SL::elem(i, m, c8), pack8(v));
-    }
-  }
-  fence_proxy_async_smem();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -244,6 +229,7 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
     if (lane == 0) {
       constexpr uint32_t id_dh = idesc_bf16_f32(128, RP, 0, 0);
       constexpr uint32_t id_w = idesc_bf16_f32(128, RP, 1, 1);
+      if (!mbar_wait(&ops_ready, 0)) bad = true;
       for (int q = 0; q < NI1 && !bad; ++q) {
         const int c = q / ntiles, i = q % ntiles, s = q % SA, u = q / SA;
         if (!mbar_wait(&fullA[s], u & 1)) {
@@ -311,6 +297,45 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
     const int m = quarter * 32 + lane;
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
     const int fmode = a.deterministic ? kPartial : kAtomic;
+    // H operand slots: bf16 of the saved H of each row, staged while the
+    // producer already streams the first dY tiles
+    {
+      const bool vec = (pt.rank_max & 3) == 0;
+      for (int idx = et; idx < ntiles * kTileM; idx += kEpiThreads) {
+        const int i = idx / kTileM, mm = idx % kTileM;
+        const int row = sp.start + idx;
+        const int hrow = idx >= sp.cnt ? -1 : (MODE == MODE_SHARED ? a.row_uniq[row] : row);
+        const float* hp = a.H[proj] + (int64_t)(hrow < 0 ? 0 : hrow) * pt.rank_max;
+#pragma unroll
+        for (int c0 = 0; c0 < RP; c0 += 32) {
+          float v[32];
+          if (vec) {
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+              const int c = c0 + 4 * q;
+              const float4 x = (hrow >= 0 && c < pt.rank_max) ? *reinterpret_cast<const float4*>(hp + c)
+                                                             : make_float4(0.f, 0.f, 0.f, 0.f);
+              v[4 * q] = x.x;
+              v[4 * q + 1] = x.y;
+              v[4 * q + 2] = x.z;
+              v[4 * q + 3] = x.w;
+            }
+          } else {
+#pragma unroll
+            for (int q = 0; q < 32; ++q) v[q] = (hrow >= 0 && c0 + q < pt.rank_max) ? hp[c0 + q] : 0.f;
+          }
+#pragma unroll
+          for (int q = 0; q < 32; ++q)
+            if (c0 + q >= rg) v[q] = 0.f;
+#pragma unroll
+          for (int c8 = 0; c8 < 4; ++c8)
+            if (c0 + 8 * c8 < RP) sts128(sOps + SL::elem(i, mm, c0 + 8 * c8), pack8(v + 8 * c8));
+        }
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ops_ready);
+    }
     bool ok = true;
     for (int c = 0; c < nch1 && ok; ++c) {
       ok = named_bar_and(kEpiBar, kEpiThreads, mbar_wait(&dbt_full[c & 1], (c >> 1) & 1));

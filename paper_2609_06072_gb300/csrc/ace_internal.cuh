@@ -191,6 +191,7 @@ struct DenseBwdLaunch {
   uint16_t* dX;
   float* dA[2];
   int32_t T, d, n_rank, n_rank_pad, nproj;
+  int32_t grid;  // persistent CTAs of the dX GEMM (the SM count)
   int32_t* err;
 };
 cudaError_t launch_dense_bwd(const DenseBwdLaunch& a, cudaStream_t st);

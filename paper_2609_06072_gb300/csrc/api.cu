@@ -415,6 +415,7 @@ ace_status ace_bwd_shared(const ace_plan* plan, const ace_perm* perm, int32_t np
   x.n_rank = n_rank;
   x.n_rank_pad = nrp;
   x.nproj = nproj;
+  x.grid = plan->num_sms;
   x.err = a.err;
   return cuda_status(launch_dense_bwd(x, cs), "dense dX / dA launch");
 }

@@ -7,9 +7,10 @@
 // products over contiguous rows:
 //   k_gemm_dx:  dX[t] += sum_j dHx_j[t] . A_j            (M = T, N = d, K = rank)
 //   k_gemm_da:  dA_j   = dHx_j^T . X                      (M = rank, N = d, K = T)
-// Each CTA owns one output tile and its whole K loop, so both are
+// Each output tile is computed with its whole K loop by one CTA, so both are
 // deterministic.  Warp-specialised: TMA producer warp, MMA warp, 8 epilogue
 // warps.  Operands arrive by TMA in 128-byte-swizzled boxes.
+#include <algorithm>
 #include <cstdint>
 
 #include "ace_internal.cuh"
@@ -25,33 +26,43 @@ constexpr int kBlk = 128 * 128;       // [128 rows x 64 bf16]
 constexpr int kHalfBlk = 64 * 128;    // [64 rows x 64 bf16]
 
 // ------------------------------------------------------------------ dX
-constexpr int kDxN = 256;                               // d columns per CTA
+// Persistent: one CTA per SM walks the [128-token x 256-column] output tiles
+// (column-fastest, so concurrent CTAs share dHx rows in L2).  Two TMEM
+// accumulators let the epilogue of one tile overlap the K loop of the next.
+// Each epilogue warp owns 32 rows x 128 columns: it reads the old dX of its
+// block with coalesced loads into its own swizzled shared-memory block (while
+// the K loop still runs), adds its accumulator rows there (thread = row) and
+// writes the block back with coalesced stores.
+constexpr int kDxN = 256;                               // d columns per tile
 constexpr int kDxStage = kBlk + (kDxN / 64) * kHalfBlk; // dHx [128 t x 64 k] + A [64 k x 256 d]
 constexpr int kDxS = 3;
-constexpr int kDxStaging = (kDxN / 64) * kBlk;          // dX tile [128 x 256]
-constexpr int kDxSmem = kDxS * kDxStage + kDxStaging + 1024;
+constexpr int kDxWarpBlk = 32 * 256;                    // [32 rows x 128 bf16] per epilogue warp
+constexpr int kDxSmem = kDxS * kDxStage + 8 * kDxWarpBlk + 1024;
+// byte offset of 16-byte chunk c (0..15) of row r (0..31) in a warp block
+__device__ __forceinline__ uint32_t dx_off(int r, int c) { return (uint32_t)(r * 256 + ((c ^ (r & 15)) << 4)); }
 
 __global__ void __launch_bounds__(kThreads, 1) k_gemm_dx(const __grid_constant__ DenseBwdLaunch a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  __shared__ __align__(8) uint64_t full[kDxS], empty[kDxS], acc_full, dx_full;
+  __shared__ __align__(8) uint64_t full[kDxS], empty[kDxS], acc_full[2], acc_empty[2];
   __shared__ uint32_t tslot;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int t0 = blockIdx.x * 128, c0 = blockIdx.y * kDxN;
+  const int ncol = (a.d + kDxN - 1) / kDxN, ntile = ((a.T + 127) / 128) * ncol;
   const int ksteps = a.n_rank_pad / 64;
   const int NK = a.nproj * ksteps;
   const uint32_t s0 = smem_u32(smem);
-  const uint32_t stg = s0 + kDxS * kDxStage;
   if (tid == 0) {
     for (int i = 0; i < kDxS; ++i) {
       mbar_init(&full[i], 1);
       mbar_init(&empty[i], 1);
     }
-    mbar_init(&acc_full, 1);
-    mbar_init(&dx_full, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&acc_full[i], 1);
+      mbar_init(&acc_empty[i], 8);  // every epilogue warp
+    }
     fence_mbar_init();
   }
-  if (warp == 0) tmem_alloc(&tslot, 256);
+  if (warp == 0) tmem_alloc(&tslot, 2 * kDxN);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -59,92 +70,114 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemm_dx(const __grid_constant__
   bool bad = false;
   if (warp == 0) {
     if (lane == 0) {
-      // the dX tile to update, then the K loop operands
-      mbar_arrive_expect_tx(&dx_full, kDxStaging);
-      for (int q = 0; q < kDxN / 64; ++q) tma_load_2d(stg + q * kBlk, &a.tm_dx, c0 + q * 64, t0, &dx_full);
-      for (int i = 0; i < NK; ++i) {
-        const int s = i % kDxS, u = i / kDxS;
-        if (u >= 1 && !mbar_wait(&empty[s], (u - 1) & 1)) {
-          bad = true;
-          break;
+      int i = 0;
+      for (int tile = blockIdx.x; tile < ntile && !bad; tile += gridDim.x) {
+        const int t0 = (tile / ncol) * 128, c0 = (tile % ncol) * kDxN;
+        for (int kb = 0; kb < NK; ++kb, ++i) {
+          const int s = i % kDxS, u = i / kDxS;
+          if (u >= 1 && !mbar_wait(&empty[s], (u - 1) & 1)) {
+            bad = true;
+            break;
+          }
+          const int j = kb / ksteps, ks = kb % ksteps;
+          const uint32_t base = s0 + s * kDxStage;
+          mbar_arrive_expect_tx(&full[s], kDxStage);
+          tma_load_2d(base, &a.tm_dhx, j * a.n_rank_pad + ks * 64, t0, &full[s]);
+          for (int q = 0; q < kDxN / 64; ++q)
+            tma_load_2d(base + kBlk + q * kHalfBlk, &a.tm_acat[j], c0 + q * 64, ks * 64, &full[s]);
         }
-        const int j = i / ksteps, ks = i % ksteps;
-        const uint32_t base = s0 + s * kDxStage;
-        mbar_arrive_expect_tx(&full[s], kDxStage);
-        tma_load_2d(base, &a.tm_dhx, j * a.n_rank_pad + ks * 64, t0, &full[s]);
-        for (int q = 0; q < kDxN / 64; ++q)
-          tma_load_2d(base + kBlk + q * kHalfBlk, &a.tm_acat[j], c0 + q * 64, ks * 64, &full[s]);
       }
+      // every copy issued has landed before the CTA can exit
+      for (int k = max(0, i - kDxS); k < i; ++k)
+        if (!mbar_wait(&full[k % kDxS], (k / kDxS) & 1)) bad = true;
     }
   } else if (warp == 1) {
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(128, kDxN, 0, 1);
-      for (int i = 0; i < NK; ++i) {
-        const int s = i % kDxS;
-        if (!mbar_wait(&full[s], (i / kDxS) & 1)) {
+      int i = 0, it = 0;
+      for (int tile = blockIdx.x; tile < ntile && !bad; tile += gridDim.x, ++it) {
+        const int b = it & 1;
+        if (it >= 2 && !mbar_wait(&acc_empty[b], ((it - 2) >> 1) & 1)) {
           bad = true;
           break;
         }
         tc_fence_after();
-        const uint32_t base = s0 + s * kDxStage;
+        for (int kb = 0; kb < NK; ++kb, ++i) {
+          const int s = i % kDxS;
+          if (!mbar_wait(&full[s], (i / kDxS) & 1)) {
+            bad = true;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t base = s0 + s * kDxStage;
 #pragma unroll
-        for (int kk = 0; kk < 4; ++kk)
-          tc_mma_bf16(tmem, sdesc_sw128(base + kk * 32, 16, 1024), sdesc_sw128(base + kBlk + kk * 2048, kHalfBlk, 1024),
-                      idesc, (i > 0 || kk > 0) ? 1u : 0u);
-        tc_commit(&empty[s]);
+          for (int kk = 0; kk < 4; ++kk)
+            tc_mma_bf16(tmem + b * kDxN, sdesc_sw128(base + kk * 32, 16, 1024),
+                        sdesc_sw128(base + kBlk + kk * 2048, kHalfBlk, 1024), idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+          tc_commit(&empty[s]);
+        }
+        if (!bad) tc_commit(&acc_full[b]);
       }
-      if (!bad) tc_commit(&acc_full);
     }
   } else {
-    const int et = tid - 64, quarter = warp & 3, ehalf = (warp - 2) >> 2;
-    const int m = quarter * 32 + lane;
+    const int quarter = warp & 3, ehalf = (warp - 2) >> 2;  // this warp: 32 rows x 128 columns
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
-    bool ok = mbar_wait(&dx_full, 0);
-    ok = ok && (NK == 0 || mbar_wait(&acc_full, 0));
-    ok = named_bar_and(kEpiBar, kEpiThreads, ok);
-    if (ok) {
+    const uint32_t wb = s0 + kDxS * kDxStage + (warp - 2) * kDxWarpBlk;
+    int it = 0;
+    for (int tile = blockIdx.x; tile < ntile; tile += gridDim.x, ++it) {
+      const int b = it & 1;
+      const int tq = (tile / ncol) * 128 + quarter * 32;  // first token of this warp's rows
+      const int cb = (tile % ncol) * kDxN + ehalf * 128;  // first column of this warp's block
+      // old dX of the block: two 256-byte rows per instruction
+#pragma unroll
+      for (int k2 = 0; k2 < 16; ++k2) {
+        const int r = k2 * 2 + (lane >> 4), c = lane & 15, t = tq + r, col = cb + c * 8;
+        const uint4 v = (t < a.T && col < a.d) ? *reinterpret_cast<const uint4*>(a.dX + (int64_t)t * a.d + col)
+                                               : make_uint4(0, 0, 0, 0);
+        sts128(wb + dx_off(r, c), v);
+      }
+      if (!__all_sync(0xffffffffu, mbar_wait(&acc_full[b], (it >> 1) & 1))) {
+        bad = true;
+        break;
+      }
       tc_fence_after();
-      if (NK > 0) {
 #pragma unroll
-        for (int hq = 0; hq < 4; ++hq) {  // 4 x 32 columns of this warp half's 128
-          const int h = ehalf * 4 + hq;    // 32-column group 0..7
-          uint32_t r[32];
-          tmem_ld16(tmem + lane_base + h * 32, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
-          tmem_ld16(tmem + lane_base + h * 32 + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
-          tmem_ld_wait();
+      for (int h = 0; h < 4; ++h) {  // 32-column groups of this warp's 128
+        uint32_t r[32];
+        const uint32_t ta = tmem + lane_base + b * kDxN + ehalf * 128 + h * 32;
+        tmem_ld16(ta, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
+        tmem_ld16(ta + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
+        tmem_ld_wait();
 #pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            const int chunk = h * 4 + q;  // 16-byte chunk 0..31 of the 256-column row
-            const uint32_t addr = stg + (chunk >> 3) * kBlk + sw128_off(m, chunk & 7);
-            const uint4 y = lds128(addr);
-            const uint32_t* dq = &r[q * 8];
-            const float2 f0 = unpack_bf16x2(y.x), f1 = unpack_bf16x2(y.y), f2 = unpack_bf16x2(y.z),
-                         f3 = unpack_bf16x2(y.w);
-            uint4 o;
-            o.x = pack_bf16x2(f0.x + __uint_as_float(dq[0]), f0.y + __uint_as_float(dq[1]));
-            o.y = pack_bf16x2(f1.x + __uint_as_float(dq[2]), f1.y + __uint_as_float(dq[3]));
-            o.z = pack_bf16x2(f2.x + __uint_as_float(dq[4]), f2.y + __uint_as_float(dq[5]));
-            o.w = pack_bf16x2(f3.x + __uint_as_float(dq[6]), f3.y + __uint_as_float(dq[7]));
-            sts128(addr, o);
-          }
+        for (int q = 0; q < 4; ++q) {
+          const uint32_t addr = wb + dx_off(lane, h * 4 + q);
+          const uint4 y = lds128(addr);
+          const uint32_t* dq = &r[q * 8];
+          const float2 f0 = unpack_bf16x2(y.x), f1 = unpack_bf16x2(y.y), f2 = unpack_bf16x2(y.z),
+                       f3 = unpack_bf16x2(y.w);
+          uint4 o;
+          o.x = pack_bf16x2(f0.x + __uint_as_float(dq[0]), f0.y + __uint_as_float(dq[1]));
+          o.y = pack_bf16x2(f1.x + __uint_as_float(dq[2]), f1.y + __uint_as_float(dq[3]));
+          o.z = pack_bf16x2(f2.x + __uint_as_float(dq[4]), f2.y + __uint_as_float(dq[5]));
+          o.w = pack_bf16x2(f3.x + __uint_as_float(dq[6]), f3.y + __uint_as_float(dq[7]));
+          sts128(addr, o);
         }
       }
-      named_bar(kEpiBar, kEpiThreads);
-#pragma unroll 4
-      for (int it = et; it < 128 * (kDxN / 8); it += kEpiThreads) {
-        const int row = it / (kDxN / 8), ch = it % (kDxN / 8), col = c0 + ch * 8;
-        if (t0 + row < a.T && col < a.d) {
-          const uint4 v = lds128(stg + (ch >> 3) * kBlk + sw128_off(row, ch & 7));
-          *reinterpret_cast<uint4*>(a.dX + (int64_t)(t0 + row) * a.d + col) = v;
-        }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&acc_empty[b]);
+#pragma unroll
+      for (int k2 = 0; k2 < 16; ++k2) {
+        const int r = k2 * 2 + (lane >> 4), c = lane & 15, t = tq + r, col = cb + c * 8;
+        if (t < a.T && col < a.d) *reinterpret_cast<uint4*>(a.dX + (int64_t)t * a.d + col) = lds128(wb + dx_off(r, c));
       }
+      __syncwarp();
     }
-    if (!ok) bad = true;
   }
   __syncwarp();
   tc_fence_before();
   if (__syncthreads_or(bad) && tid == 0) atomicOr(a.err, kErrTimeout);
-  if (warp == 0) tmem_dealloc(tmem, 256);
+  if (warp == 0) tmem_dealloc(tmem, 2 * kDxN);
 }
 
 // ------------------------------------------------------------------ dA
@@ -259,7 +292,8 @@ cudaError_t launch_dense_bwd(const DenseBwdLaunch& a, cudaStream_t st) {
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(k_gemm_da, cudaFuncAttributeMaxDynamicSharedMemorySize, kDaSmem);
   if (e != cudaSuccess) return e;
-  k_gemm_dx<<<dim3((a.T + 127) / 128, (a.d + kDxN - 1) / kDxN), kThreads, kDxSmem, st>>>(a);
+  const int dx_tiles = ((a.T + 127) / 128) * ((a.d + kDxN - 1) / kDxN);
+  k_gemm_dx<<<std::min(dx_tiles, a.grid), kThreads, kDxSmem, st>>>(a);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   k_gemm_da<<<dim3(a.nproj * a.n_rank_pad / 128 + (a.nproj * a.n_rank_pad % 128 ? 1 : 0), (a.d + kDaN - 1) / kDaN),
               kThreads, kDaSmem, st>>>(a);

@@ -147,6 +147,8 @@ cudaError_t launch_fwd_rows(const PlanTables& pt, const FwdRowsLaunch& a, bool s
 // and 128-byte swizzle.  Returns false when the encoder is unavailable or
 // rejects the layout.
 bool make_tmap_bf16(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows);
+// 2-D fp32 tensor map with a 32-column x box_rows box and 128-byte swizzle.
+bool make_tmap_f32(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows);
 
 struct BwdLaunch {
   CUtensorMap tm_dy[2];    // dY [R, d_out], box 64 x 128
@@ -188,6 +190,7 @@ struct DenseBwdLaunch {
   CUtensorMap tm_acat[2];  // A_j [n_rank, d], box 64 x 64
   CUtensorMap tm_x;        // X [T, d], box 64 x 64
   CUtensorMap tm_dx;       // dX [T, d], box 64 x 128
+  CUtensorMap tm_da[2];    // dA_j [n_rank, d] fp32, box 32 x 32 (bulk reduce-add)
   uint16_t* dX;
   float* dA[2];
   int32_t T, d, n_rank, n_rank_pad, nproj;

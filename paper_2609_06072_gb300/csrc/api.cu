@@ -43,6 +43,18 @@ bool ace::make_tmap_bf16(CUtensorMap* m, const void* base, uint64_t rows, uint64
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+bool ace::make_tmap_f32(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows) {
+  EncodeTiledFn fn = tensor_map_encoder();
+  if (!fn || rows == 0 || cols == 0) return false;
+  cuuint64_t gdim[2] = {cols, rows};
+  cuuint64_t gstr[1] = {cols * 4};
+  cuuint32_t box[2] = {32, box_rows};
+  cuuint32_t es[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<void*>(base), gdim, gstr, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 struct ace_plan {
   PlanTables pt;
   int32_t T_max;
@@ -405,9 +417,12 @@ ace_status ace_bwd_shared(const ace_plan* plan, const ace_perm* perm, int32_t np
   const uint64_t T = (uint64_t)perm->T, kw = (uint64_t)nproj * nrp;
   bool okm = make_tmap_bf16(&x.tm_dhx, w.dHx, T, kw, kTileM) && make_tmap_bf16(&x.tm_dhx_t, w.dHx, T, kw, 64) &&
              make_tmap_bf16(&x.tm_x, X, T, (uint64_t)pt.d, 64) && make_tmap_bf16(&x.tm_dx, dX, T, (uint64_t)pt.d, kTileM);
-  for (int j = 0; j < nproj; ++j) okm = okm && make_tmap_bf16(&x.tm_acat[j], A[j], (uint64_t)n_rank, (uint64_t)pt.d, 64);
+  for (int j = 0; j < nproj; ++j) {
+    okm = okm && make_tmap_bf16(&x.tm_acat[j], A[j], (uint64_t)n_rank, (uint64_t)pt.d, 64);
+    okm = okm && make_tmap_f32(&x.tm_da[j], dA[j], (uint64_t)n_rank, (uint64_t)pt.d, 32);
+  }
   if (!okm) return fail(ACE_ERR_UNSUPPORTED, "tensor-map encoding failed for this layout");
-  if (nproj == 1) x.tm_acat[1] = x.tm_acat[0];
+  if (nproj == 1) x.tm_acat[1] = x.tm_acat[0], x.tm_da[1] = x.tm_da[0];
   x.dX = dX;
   for (int j = 0; j < 2; ++j) x.dA[j] = dA[j < nproj ? j : 0];
   x.T = perm->T;

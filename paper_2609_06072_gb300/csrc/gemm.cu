@@ -181,10 +181,18 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemm_dx(const __grid_constant__
 }
 
 // ------------------------------------------------------------------ dA
-constexpr int kDaN = 128;                              // d columns per CTA
-constexpr int kDaStage = 2 * kHalfBlk + (kDaN / 64) * kHalfBlk;  // dHx^T [64 t x 128 k] + X [64 t x 128 d]
-constexpr int kDaS = 6;
-constexpr int kDaSmem = kDaS * kDaStage + 1024;
+// Output tiles of [128 stacked rank rows x 256 columns]; when the tiles alone
+// leave SMs idle the token (K) loop is split in two halves, and each CTA adds
+// its fp32 tile into the zeroed dA with bulk tensor reduce-adds.  Each element
+// then receives at most two addends on top of 0, and a + b == b + a in
+// floating point, so the result does not depend on their order.
+constexpr int kDaN = 256;                                        // d columns per tile
+constexpr int kDaStage = 2 * kHalfBlk + (kDaN / 64) * kHalfBlk;  // dHx^T [64 t x 128 k] + X [64 t x 256 d]
+constexpr int kDaS = 4;
+constexpr int kDaWarpStg = 32 * 128;                             // [32 rows x 32 fp32] per epilogue warp
+constexpr int kDaSmem = kDaS * kDaStage + 8 * kDaWarpStg + 1024;
+
+__host__ __device__ inline int da_ksplit(int tiles, int grid) { return tiles * 2 <= grid ? 2 : 1; }
 
 __global__ void __launch_bounds__(kThreads, 1) k_gemm_da(const __grid_constant__ DenseBwdLaunch a) {
   extern __shared__ uint8_t smem_raw[];
@@ -192,9 +200,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemm_da(const __grid_constant__
   __shared__ __align__(8) uint64_t full[kDaS], empty[kDaS], acc_full;
   __shared__ uint32_t tslot;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int m0 = blockIdx.x * 128;  // row of the stacked [nproj * n_rank_pad] rank dimension
-  const int c0 = blockIdx.y * kDaN;
-  const int NK = (a.T + 63) / 64;
+  const int mt = (a.nproj * a.n_rank_pad + 127) / 128, nt = (a.d + kDaN - 1) / kDaN;
+  const int ks = da_ksplit(mt * nt, a.grid);
+  const int tile = blockIdx.x / ks, half = blockIdx.x % ks;
+  const int m0 = (tile / nt) * 128;  // row of the stacked [nproj * n_rank_pad] rank dimension
+  const int c0 = (tile % nt) * kDaN;
+  const int nkb = (a.T + 63) / 64;
+  const int kb0 = half * nkb / ks, kb1 = (half + 1) * nkb / ks, NK = kb1 - kb0;
   const uint32_t s0 = smem_u32(smem);
   if (tid == 0) {
     for (int i = 0; i < kDaS; ++i) {
@@ -204,7 +216,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemm_da(const __grid_constant__
     mbar_init(&acc_full, 1);
     fence_mbar_init();
   }
-  if (warp == 0) tmem_alloc(&tslot, 128);
+  if (warp == 0) tmem_alloc(&tslot, kDaN);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -212,19 +224,23 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemm_da(const __grid_constant__
   bool bad = false;
   if (warp == 0) {
     if (lane == 0) {
-      for (int i = 0; i < NK; ++i) {
+      int i = 0;
+      for (; i < NK; ++i) {
         const int s = i % kDaS, u = i / kDaS;
         if (u >= 1 && !mbar_wait(&empty[s], (u - 1) & 1)) {
           bad = true;
           break;
         }
+        const int t0 = (kb0 + i) * 64;
         const uint32_t base = s0 + s * kDaStage;
         mbar_arrive_expect_tx(&full[s], kDaStage);
-        tma_load_2d(base, &a.tm_dhx_t, m0, i * 64, &full[s]);
-        tma_load_2d(base + kHalfBlk, &a.tm_dhx_t, m0 + 64, i * 64, &full[s]);
+        tma_load_2d(base, &a.tm_dhx_t, m0, t0, &full[s]);
+        tma_load_2d(base + kHalfBlk, &a.tm_dhx_t, m0 + 64, t0, &full[s]);
         for (int q = 0; q < kDaN / 64; ++q)
-          tma_load_2d(base + 2 * kHalfBlk + q * kHalfBlk, &a.tm_x, c0 + q * 64, i * 64, &full[s]);
+          tma_load_2d(base + 2 * kHalfBlk + q * kHalfBlk, &a.tm_x, c0 + q * 64, t0, &full[s]);
       }
+      for (int k = max(0, i - kDaS); k < i; ++k)
+        if (!mbar_wait(&full[k % kDaS], (k / kDaS) & 1)) bad = true;
     }
   } else if (warp == 1) {
     if (lane == 0) {
@@ -246,42 +262,42 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemm_da(const __grid_constant__
       if (!bad) tc_commit(&acc_full);
     }
   } else {
-    const int quarter = warp & 3, ehalf = (warp - 2) >> 2;
-    const int m = quarter * 32 + lane;
+    const int quarter = warp & 3, ehalf = (warp - 2) >> 2;  // this warp: 32 rank rows x 128 columns
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
+    const uint32_t stg = s0 + kDaS * kDaStage + (warp - 2) * kDaWarpStg;
+    const int r0 = m0 + quarter * 32, j = r0 / a.n_rank_pad, rr0 = r0 % a.n_rank_pad;
     bool ok = NK == 0 || mbar_wait(&acc_full, 0);
-    ok = named_bar_and(kEpiBar, kEpiThreads, ok);
-    if (ok) {
+    ok = __all_sync(0xffffffffu, ok);
+    if (ok && NK > 0 && j < a.nproj && rr0 < a.n_rank) {
       tc_fence_after();
-      const int r = m0 + m, j = r / a.n_rank_pad, rr = r % a.n_rank_pad;
-      const bool live = j < a.nproj && rr < a.n_rank;
-      float* out = live ? a.dA[j] + (int64_t)rr * a.d : nullptr;
-#pragma unroll
-      for (int hq = 0; hq < 2; ++hq) {
-        const int h = ehalf * 2 + hq;  // 32-column group 0..3
+#pragma unroll 1
+      for (int h = 0; h < 4; ++h) {  // 32-column groups of this warp's 128
+        const int col = c0 + ehalf * 128 + h * 32;
         uint32_t v[32];
-        tmem_ld16(tmem + lane_base + h * 32, *reinterpret_cast<uint32_t(*)[16]>(&v[0]));
-        tmem_ld16(tmem + lane_base + h * 32 + 16, *reinterpret_cast<uint32_t(*)[16]>(&v[16]));
+        tmem_ld16(tmem + lane_base + ehalf * 128 + h * 32, *reinterpret_cast<uint32_t(*)[16]>(&v[0]));
+        tmem_ld16(tmem + lane_base + ehalf * 128 + h * 32 + 16, *reinterpret_cast<uint32_t(*)[16]>(&v[16]));
         tmem_ld_wait();
-        if (live) {
+        if (lane == 0) bulk_wait_read0();  // the previous group's box has been read
+        __syncwarp();
+        // row = lane, 128-byte swizzle of the tensor map
 #pragma unroll
-          for (int q = 0; q < 8; ++q) {
-            const int col = c0 + h * 32 + q * 4;
-            if (col < a.d)
-              *reinterpret_cast<float4*>(out + col) =
-                  NK == 0 ? make_float4(0.f, 0.f, 0.f, 0.f)
-                          : make_float4(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]),
-                                        __uint_as_float(v[4 * q + 2]), __uint_as_float(v[4 * q + 3]));
-          }
+        for (int q = 0; q < 8; ++q)
+          sts128(stg + lane * 128 + ((q ^ (lane & 7)) << 4), make_uint4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]));
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0 && col < a.d) {
+          tma_reduce_add_2d(&a.tm_da[j], stg, col, rr0);
+          bulk_commit();
         }
       }
+      if (lane == 0) bulk_wait0();
     }
     if (!ok) bad = true;
   }
   __syncwarp();
   tc_fence_before();
   if (__syncthreads_or(bad) && tid == 0) atomicOr(a.err, kErrTimeout);
-  if (warp == 0) tmem_dealloc(tmem, 128);
+  if (warp == 0) tmem_dealloc(tmem, kDaN);
 }
 
 }  // namespace
@@ -295,8 +311,11 @@ cudaError_t launch_dense_bwd(const DenseBwdLaunch& a, cudaStream_t st) {
   const int dx_tiles = ((a.T + 127) / 128) * ((a.d + kDxN - 1) / kDxN);
   k_gemm_dx<<<std::min(dx_tiles, a.grid), kThreads, kDxSmem, st>>>(a);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  k_gemm_da<<<dim3(a.nproj * a.n_rank_pad / 128 + (a.nproj * a.n_rank_pad % 128 ? 1 : 0), (a.d + kDaN - 1) / kDaN),
-              kThreads, kDaSmem, st>>>(a);
+  // dA accumulates bulk reduce-adds: zero it first
+  for (int j = 0; j < a.nproj; ++j)
+    if ((e = cudaMemsetAsync(a.dA[j], 0, sizeof(float) * (size_t)a.n_rank * a.d, st)) != cudaSuccess) return e;
+  const int da_tiles = ((a.nproj * a.n_rank_pad + 127) / 128) * ((a.d + kDaN - 1) / kDaN);
+  k_gemm_da<<<da_tiles * da_ksplit(da_tiles, a.grid), kThreads, kDaSmem, st>>>(a);
   return cudaGetLastError();
 }
 

@@ -48,9 +48,10 @@ struct PermLayout {
 
 // counts[] slots
 constexpr int kCntU = 0, kCntRows = 1, kCntTilesSh = 2, kCntTilesRow = 3, kCntSplitsRow = 4;
-// sched[] slots: work counters of the dynamically scheduled kernels (zeroed
-// by the host before each launch)
-constexpr int kSchedFwdRows = 0;
+// sched[] slots: work counter and finished-CTA counter of the dynamically
+// scheduled forward row kernel; the permutation zeroes them and the last CTA
+// of every launch resets them, so each launch starts from zero
+constexpr int kSchedFwdRows = 0, kSchedFwdDone = 1;
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
@@ -102,6 +103,9 @@ inline T* at(void* base, size_t off) {
 // cudaError_t of its launches.
 cudaError_t launch_permute(const PlanTables& pt, const int32_t* topk_idx, int32_t T, void* ws, const PermLayout& L,
                            cudaStream_t st);
+// Zeroes n (<= kZeroMax) device buffers in one launch (null / empty ones skipped).
+constexpr int kZeroMax = 6;
+cudaError_t launch_zero(void* const* ptrs, const size_t* bytes, int n, cudaStream_t st);
 cudaError_t launch_rows_copy(const int32_t* row_pair, const uint16_t* src, uint16_t* dst, int64_t R, int32_t cols,
                              bool gather, cudaStream_t st);
 
@@ -131,7 +135,7 @@ struct FwdRowsLaunch {
   CUtensorMap tm_y16[2];  // Y, box 64 x 16 (short tiles)
   const Tile* tiles;         // row tiles (<= 128 rows of one group), in row order
   const int32_t* counts;     // counts[kCntTilesRow] = number of row tiles
-  int32_t* sched;            // work counter, zero at launch
+  int32_t* sched;            // [kSchedFwdRows] work counter, [kSchedFwdDone] finished CTAs; zero at launch
   int32_t grid;              // persistent CTAs (the SM count)
   const int32_t* row_uniq;
   const float* Hu[2];    // gate/up: H per unique pair
@@ -197,6 +201,7 @@ struct DenseBwdLaunch {
   int32_t grid;  // persistent CTAs of the dX GEMM (the SM count)
   int32_t* err;
 };
+// dA must be zero on entry (the GEMM adds its tiles into it).
 cudaError_t launch_dense_bwd(const DenseBwdLaunch& a, cudaStream_t st);
 
 }  // namespace ace

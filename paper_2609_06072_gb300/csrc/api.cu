@@ -310,12 +310,8 @@ static ace_status fwd_common(const ace_plan* plan, const ace_perm* perm, const u
   if (!ok) return fail(ACE_ERR_UNSUPPORTED, "tensor-map encoding failed for this layout");
   r.tiles = at<Tile>(perm->ws, L.tiles_row);
   r.counts = perm->counts;
-  r.sched = at<int32_t>(perm->ws, L.sched) + kSchedFwdRows;
+  r.sched = at<int32_t>(perm->ws, L.sched);
   r.grid = R > 0 ? plan->num_sms : 0;
-  if (R > 0) {
-    st = cuda_status(cudaMemsetAsync(r.sched, 0, sizeof(int32_t), cs), "work counter reset");
-    if (st != ACE_OK) return st;
-  }
   r.row_uniq = at<int32_t>(perm->ws, L.row_uniq);
   for (int j = 0; j < 2; ++j) {
     const int jj = j < nproj ? j : 0;

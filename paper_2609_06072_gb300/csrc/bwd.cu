@@ -538,19 +538,24 @@ cudaError_t launch_bwd_t(const PlanTables& pt, const BwdLaunch& a, bool shared, 
   cudaError_t e;
   const int n_rank = pt.rank_off[pt.G];
   const int nproj = shared ? a.nproj : 1;
-  if (!a.deterministic) {
-    for (int j = 0; j < nproj; ++j)
-      if ((e = cudaMemsetAsync(a.dBt[j], 0, sizeof(float) * (size_t)n_rank * a.d_out, st)) != cudaSuccess) return e;
+  // one launch zeroes every accumulation target of the call: the fast-mode
+  // atomic dB^T (and down dA), and for gate/up the dense dH and the dA that
+  // the dense GEMM adds its tiles into
+  void* zp[kZeroMax] = {};
+  size_t zb[kZeroMax] = {};
+  int nz = 0;
+  if (!a.deterministic)
+    for (int j = 0; j < nproj; ++j) zp[nz] = a.dBt[j], zb[nz++] = sizeof(float) * (size_t)n_rank * a.d_out;
+  if (!shared && !a.deterministic) zp[nz] = a.dA[0], zb[nz++] = sizeof(float) * (size_t)n_rank * a.d_in;
+  if (shared) {
+    zp[nz] = a.dHx, zb[nz++] = sizeof(uint16_t) * (size_t)a.T * nproj * a.n_rank_pad;
+    for (int j = 0; j < nproj; ++j) zp[nz] = a.dA[j], zb[nz++] = sizeof(float) * (size_t)n_rank * a.d_in;
   }
+  if ((e = launch_zero(zp, zb, nz, st)) != cudaSuccess) return e;
   if (!shared) {
-    if (!a.deterministic &&
-        (e = cudaMemsetAsync(a.dA[0], 0, sizeof(float) * (size_t)n_rank * a.d_in, st)) != cudaSuccess)
-      return e;
     if ((e = launch_rows<RP, MODE_DOWN>(pt, a, 1, st)) != cudaSuccess) return e;
   } else {
     if ((e = launch_rows<RP, MODE_SHARED>(pt, a, nproj, st)) != cudaSuccess) return e;
-    const size_t dhx = sizeof(uint16_t) * (size_t)a.T * nproj * a.n_rank_pad;
-    if ((e = cudaMemsetAsync(a.dHx, 0, dhx, st)) != cudaSuccess) return e;
     k_dh_reduce<RP><<<dim3(a.max_tiles_sh, nproj), 128, 0, st>>>(pt, a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }

@@ -292,7 +292,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
             bad = true;
             return false;
           }
-          int item = atomicAdd(a.sched, 1);
+          int item = atomicAdd(a.sched + kSchedFwdRows, 1);
           if (item >= n_items) item = -1;
           tq.item[e] = item;
           mbar_arrive(&tq.full[e]);
@@ -569,6 +569,15 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
   __syncwarp();  // reconverge the single-lane roles before the CTA barrier
   tc_fence_before();
   if (__syncthreads_or(bad) && tid == 0) atomicOr(a.err, kErrTimeout);
+  if (tid == 0) {
+    // the last CTA to finish (every producer has taken its final index) resets
+    // the counters for the next launch
+    __threadfence();
+    if (atomicAdd(a.sched + kSchedFwdDone, 1) == (int)gridDim.x - 1) {
+      atomicExch(a.sched + kSchedFwdRows, 0);
+      atomicExch(a.sched + kSchedFwdDone, 0);
+    }
+  }
   if (warp == 0) tmem_dealloc(tmem, kRowsTmem);
 }
 

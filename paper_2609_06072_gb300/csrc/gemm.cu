@@ -311,9 +311,8 @@ cudaError_t launch_dense_bwd(const DenseBwdLaunch& a, cudaStream_t st) {
   const int dx_tiles = ((a.T + 127) / 128) * ((a.d + kDxN - 1) / kDxN);
   k_gemm_dx<<<std::min(dx_tiles, a.grid), kThreads, kDxSmem, st>>>(a);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  // dA accumulates bulk reduce-adds: zero it first
-  for (int j = 0; j < a.nproj; ++j)
-    if ((e = cudaMemsetAsync(a.dA[j], 0, sizeof(float) * (size_t)a.n_rank * a.d, st)) != cudaSuccess) return e;
+  // dA accumulates bulk reduce-adds: the caller has zeroed it (with the
+  // backward's other accumulation targets, in one launch)
   const int da_tiles = ((a.nproj * a.n_rank_pad + 127) / 128) * ((a.d + kDaN - 1) / kDaN);
   k_gemm_da<<<da_tiles * da_ksplit(da_tiles, a.grid), kThreads, kDaSmem, st>>>(a);
   return cudaGetLastError();

@@ -120,7 +120,8 @@ __global__ void __launch_bounds__(256) k_perm_colscan(const __grid_constant__ Pl
                                                       const int32_t* __restrict__ chunk_err,
                                                       int32_t* __restrict__ chunk_baseE,
                                                       int32_t* __restrict__ chunk_baseU, int32_t* __restrict__ totE,
-                                                      int32_t* __restrict__ totU, int32_t* __restrict__ err) {
+                                                      int32_t* __restrict__ totU, int32_t* __restrict__ err,
+                                                      int32_t* __restrict__ sched) {
   __shared__ int32_t wsum[8];
   __shared__ int32_t err_s;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -148,6 +149,7 @@ __global__ void __launch_bounds__(256) k_perm_colscan(const __grid_constant__ Pl
   }
   if (tid == 0) (isE ? totE : totU)[col] = carry;
   if (blockIdx.x == 0) {
+    if (tid < 8) sched[tid] = 0;  // work counters of the row kernels start at zero
     int e = 0;
     for (int c = tid; c < n_chunks; c += 256) e |= chunk_err[c];
     if (e) atomicOr(&err_s, e);
@@ -294,6 +296,20 @@ __global__ void __launch_bounds__(kPermTB) k_perm_scatter(const __grid_constant_
   for (int j = n_u; j < k; ++j) o.tok_uniq[(int64_t)t * k + j] = -1;
 }
 
+// Zeroes up to kZeroMax buffers (16-byte aligned, sizes multiples of 16) in
+// one launch.
+struct ZeroList {
+  uint4* p[kZeroMax];
+  int64_t n16[kZeroMax];  // 16-byte words of each
+  int n;
+};
+__global__ void __launch_bounds__(256) k_zero(const __grid_constant__ ZeroList z) {
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int b = 0; b < z.n; ++b)
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < z.n16[b]; i += stride)
+      z.p[b][i] = make_uint4(0, 0, 0, 0);
+}
+
 __global__ void k_rows_copy(const int32_t* __restrict__ row_pair, const uint4* __restrict__ src,
                             uint4* __restrict__ dst, int64_t R, int vec_per_row, bool gather) {
   const int64_t n = R * vec_per_row;
@@ -320,7 +336,8 @@ cudaError_t launch_permute(const PlanTables& pt, const int32_t* topk_idx, int32_
   k_perm_colscan<<<pt.E + pt.G, 256, 0, st>>>(pt, C, at<int32_t>(ws, L.chunk_cntE), at<int32_t>(ws, L.chunk_cntU),
                                                 at<int32_t>(ws, L.chunk_err), at<int32_t>(ws, L.chunk_baseE),
                                                 at<int32_t>(ws, L.chunk_baseU), at<int32_t>(ws, L.expert_cnt),
-                                                at<int32_t>(ws, L.tot_u), at<int32_t>(ws, L.err));
+                                                at<int32_t>(ws, L.tot_u), at<int32_t>(ws, L.err),
+                                                at<int32_t>(ws, L.sched));
   ScatterOut o;
   o.row_pair = at<int32_t>(ws, L.row_pair);
   o.pair_row = at<int32_t>(ws, L.pair_row);
@@ -340,6 +357,22 @@ cudaError_t launch_permute(const PlanTables& pt, const int32_t* topk_idx, int32_
   k_perm_scatter<<<C > 0 ? C : 1, kPermTB, sm3, st>>>(pt, topk_idx, T, at<int32_t>(ws, L.chunk_baseE),
                                                      at<int32_t>(ws, L.chunk_baseU), at<int32_t>(ws, L.expert_cnt),
                                                      at<int32_t>(ws, L.tot_u), o);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_zero(void* const* ptrs, const size_t* bytes, int n, cudaStream_t st) {
+  ZeroList z{};
+  int64_t total = 0;
+  for (int i = 0; i < n && i < kZeroMax; ++i) {
+    if (!ptrs[i] || bytes[i] == 0) continue;
+    z.p[z.n] = static_cast<uint4*>(ptrs[i]);
+    z.n16[z.n] = (int64_t)(bytes[i] / 16);
+    total += z.n16[z.n];
+    ++z.n;
+  }
+  if (z.n == 0) return cudaSuccess;
+  const int blocks = (int)std::min<int64_t>((total + 255) / 256, 152 * 4);
+  k_zero<<<blocks, 256, 0, st>>>(z);
   return cudaGetLastError();
 }
 

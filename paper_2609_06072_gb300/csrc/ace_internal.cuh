@@ -23,6 +23,7 @@ struct PlanTables {
   int32_t rank_max;  // max_g r_g
   int32_t rank_pad;  // MMA N of one projection's rank block (16/32/64/128)
   int32_t nt_split;  // tiles per backward split
+  int32_t nsm;       // SMs of the plan's device (the last nsm forward row tiles are split in column halves)
   int16_t e2g[ACE_MAX_EXPERTS];
   int16_t eorder[ACE_MAX_EXPERTS];  // experts in (g, e) order
   int16_t gfirst[ACE_MAX_EXPERTS];  // position in eorder of group g's first expert
@@ -31,7 +32,8 @@ struct PlanTables {
 
 // A unit of work: unique pairs [start, start + cnt) of group g (shared tiles)
 // or rows [start, start + cnt) of group g (row tiles, backward splits).  `id`
-// is the tile's or split's index.
+// is the tile's or split's index, except for forward row tiles, where it
+// names the output columns: 0 all, 1 the first half, 2 the second half.
 struct Tile {
   int32_t g, start, cnt, id;
 };
@@ -88,7 +90,7 @@ inline PermLayout perm_layout(const PlanTables& pt, int32_t T) {
   L.chunk_baseU = take(4 * (size_t)L.n_chunks * pt.G);
   L.chunk_err = take(4 * (size_t)(L.n_chunks + 1));
   L.tiles_sh = take(sizeof(Tile) * (size_t)L.max_tiles);
-  L.tiles_row = take(sizeof(Tile) * (size_t)L.max_tiles);
+  L.tiles_row = take(sizeof(Tile) * (size_t)(L.max_tiles + pt.nsm));
   L.splits_row = take(sizeof(Tile) * (size_t)L.max_splits);
   L.total = off;
   return L;

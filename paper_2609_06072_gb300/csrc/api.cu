@@ -185,6 +185,7 @@ ace_status ace_plan_create(ace_plan** out, const ace_layer_desc* desc) {
   p->pt.rank_max = rank_max;
   p->pt.rank_pad = rank_max <= 16 ? 16 : rank_max <= 32 ? 32 : rank_max <= 64 ? 64 : 128;
   p->pt.nt_split = pt_nt_split(p->pt.rank_pad);
+  p->pt.nsm = num_sms;
   for (int e = 0; e < D.E; ++e) p->pt.e2g[e] = (int16_t)D.e2g[e];
   {
     int pos = 0;

@@ -8,7 +8,8 @@
 //   fp32 H written per unique pair.
 // k_fwd_rows: persistent, one CTA per SM; tiles of <= 128 consecutive rows
 //   of one group (expert segments are contiguous inside group segments) are
-//   taken dynamically from a counter.  Warp-specialised:
+//   taken dynamically from a counter (the last ones in column halves, so the
+//   SMs finish together).  Warp-specialised:
 //     warp 0     TMA producer: row tiles of Y (and of h for down) and chunks of
 //                B_g^T / A_g into a ring of shared-memory slots
 //     warp 1     MMA issuer: (down) H = h . A_g^T over the K loop, then per
@@ -184,6 +185,17 @@ __device__ __forceinline__ void load_rows(uint32_t dst, const CUtensorMap* m128,
   const int nb = (cnt + kQuant - 1) / kQuant;
   for (int b = 0; b < nb; ++b) tma_load_2d(dst + b * kQuant * 128, m16, x, y + b * kQuant, bar);
 }
+// Output chunks [lo, hi) of a row tile (its id names all, or one half of, the
+// columns).  `whole` (down): a split tile is done whole under its first half's
+// entry and its second half's entry is skipped -- cutting it would make both
+// halves repeat the tile's K loop, which measured slower.
+__device__ __forceinline__ bool tile_live(const Tile& t, bool whole) { return t.cnt > 0 && !(whole && t.id == 2); }
+__device__ __forceinline__ int chunk_lo(const Tile& t, int nch, bool whole) {
+  return !whole && t.id == 2 ? (nch + 1) / 2 : 0;
+}
+__device__ __forceinline__ int chunk_hi(const Tile& t, int nch, bool whole) {
+  return !whole && t.id == 1 ? (nch + 1) / 2 : nch;
+}
 __device__ __forceinline__ uint32_t rows_bytes(int cnt) {
   return cnt == kTileM ? (uint32_t)kBlk : (uint32_t)((cnt + kQuant - 1) / kQuant) * kQuant * 128;
 }
@@ -199,7 +211,7 @@ struct TileQueue {
 // up; *ok tells which).  Every lane of a warp calls it; lane 0 releases the
 // entries it reads.
 __device__ __forceinline__ bool queue_next(TileQueue& tq, int& q, const Tile* tiles, Tile& t, bool single_lane,
-                                           bool* ok) {
+                                           bool* ok, bool whole) {
   while (true) {
     const int e = q % kQ;
     bool w = mbar_wait(&tq.full[e], (q / kQ) & 1);
@@ -214,7 +226,7 @@ __device__ __forceinline__ bool queue_next(TileQueue& tq, int& q, const Tile* ti
     ++q;
     if (item < 0) return false;
     t = tiles[item];
-    if (t.cnt > 0) return true;  // (an empty tile is skipped)
+    if (tile_live(t, whole)) return true;
   }
 }
 // Persistent: one CTA per SM; tiles of <= 128 consecutive rows of one group
@@ -299,7 +311,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
           ++q;
           if (item < 0) return false;
           t = a.tiles[item];
-          if (t.cnt > 0) return true;
+          if (tile_live(t, !SHARED)) return true;
         }
       };
       auto acquire = [&](bool kstep) -> uint32_t {  // next ring slot, once its last user released it
@@ -339,7 +351,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
         for (int k = 0; k < NK && !bad; ++k) load_k(cur, k);
       while (has_cur && !bad) {
         const bool has_nxt = grab(nxt);
-        for (int c = 0; c < nch && !bad; ++c) load_c(cur, c);
+        for (int c = chunk_lo(cur, nch, !SHARED); c < chunk_hi(cur, nch, !SHARED) && !bad; ++c) load_c(cur, c);
         if (!SHARED && has_nxt)
           for (int k = 0; k < NK && !bad; ++k) load_k(nxt, k);
         cur = nxt;
@@ -371,9 +383,9 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
         if (k == NK - 1) tc_commit(&hacc[hb]);
         ++i;
       };
-      auto mma_c = [&](int c) {  // D chunk c of tile ti
+      auto mma_c = [&](bool first, bool last) {  // a D chunk of tile ti
         const int s = i % S, b = cc % kNGrp;
-        if ((c == 0 && !mbar_wait(&hs_ready[ti & 1], (ti >> 1) & 1)) ||
+        if ((first && !mbar_wait(&hs_ready[ti & 1], (ti >> 1) & 1)) ||
             (cc >= kNGrp && !mbar_wait(&dempty[b], ((cc - kNGrp) / kNGrp) & 1)) ||
             !mbar_wait(&full[s], (i / S) & 1)) {
           bad = true;
@@ -393,18 +405,19 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
                         kk > 0 ? 1u : 0u);
           }
         tc_commit(&dfull[b]);
-        if (c == nch - 1) tc_commit(&hs_free[ti % NBH]);
+        if (last) tc_commit(&hs_free[ti % NBH]);
         ++cc;
         ++i;
       };
       Tile cur, nxt;
       bool qok = true;
-      bool has_cur = queue_next(tq, q, a.tiles, cur, true, &qok);
+      bool has_cur = queue_next(tq, q, a.tiles, cur, true, &qok, !SHARED);
       if (has_cur && !SHARED)
         for (int k = 0; k < NK && !bad; ++k) mma_k(0, k);
       while (has_cur && !bad) {
-        const bool has_nxt = queue_next(tq, q, a.tiles, nxt, true, &qok);
-        for (int c = 0; c < nch && !bad; ++c) mma_c(c);
+        const bool has_nxt = queue_next(tq, q, a.tiles, nxt, true, &qok, !SHARED);
+        const int lo = chunk_lo(cur, nch, !SHARED), hi = chunk_hi(cur, nch, !SHARED);
+        for (int c = lo; c < hi && !bad; ++c) mma_c(c == lo, c == hi - 1);
         if (!SHARED && has_nxt)
           for (int k = 0; k < NK && !bad; ++k) mma_k((ti + 1) & 1, k);
         ++ti;
@@ -492,18 +505,19 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
     int q = 0, ib = SHARED ? 0 : NK, cc0 = 0, ti = 0;
     bool ok = true;
     Tile cur, nxt;
-    bool has_cur = queue_next(tq, q, a.tiles, cur, false, &ok);
+    bool has_cur = queue_next(tq, q, a.tiles, cur, false, &ok, !SHARED);
     if (has_cur) ok = prepare_h(cur, 0);
     while (has_cur && ok) {
-      const bool has_nxt = queue_next(tq, q, a.tiles, nxt, false, &ok);
+      const bool has_nxt = queue_next(tq, q, a.tiles, nxt, false, &ok, !SHARED);
       if (!ok) break;
       const bool inter = !SHARED && has_nxt;
       // gate/up with two H buffers: gather the next tile's H now, while this tile streams
       const bool early = SHARED && NBH == 2 && has_nxt;
       if (early && !(ok = prepare_h(nxt, ti + 1))) break;
       const bool qlive = quarter * 32 < cur.cnt;  // this warp has live rows (warp-uniform)
-      for (int c = ((grp - cc0) % kNGrp + kNGrp) % kNGrp; c < nch; c += kNGrp) {
-        const int cc = cc0 + c, i = ib + c;
+      const int lo = chunk_lo(cur, nch, !SHARED), hi = chunk_hi(cur, nch, !SHARED);
+      for (int c = lo + ((grp - cc0) % kNGrp + kNGrp) % kNGrp; c < hi; c += kNGrp) {
+        const int cc = cc0 + (c - lo), i = ib + (c - lo);
         const int sl = i % S, b = cc % kNGrp, n0 = c * kChunk;
         ok = __all_sync(0xffffffffu, mbar_wait(&full[sl], (i / S) & 1) && mbar_wait(&dfull[b], (cc / kNGrp) & 1));
         if (!ok) break;
@@ -558,8 +572,8 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
       }
       if (!ok) break;
       if (has_nxt && !early && !(ok = prepare_h(nxt, ti + 1))) break;
-      ib += nch + (inter ? NK : 0);
-      cc0 += nch;
+      ib += (hi - lo) + (inter ? NK : 0);
+      cc0 += hi - lo;
       ++ti;
       cur = nxt;
       has_cur = has_nxt;

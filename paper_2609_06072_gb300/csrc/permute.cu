@@ -102,6 +102,33 @@ __device__ int build_tiles(const int32_t* n_g, const int32_t* off_g, int G, int 
   return total;
 }
 
+// Forward row tiles in dispatch order: every group's rows in tiles of 128
+// (id 0: all output columns), except that each of the last `tail` tiles of the
+// list becomes two entries covering one half of the columns each (ids 1, 2),
+// so the work left when SMs run dry comes in halves.
+__device__ int build_row_tiles(const int32_t* n_g, const int32_t* off_g, int G, int tail, Tile* __restrict__ out,
+                               int32_t* scratch /* smem [G+1] */) {
+  const int n = build_tiles(n_g, off_g, G, kTileM, out, scratch);
+  const int ns = min(n, tail), first = n - ns;
+  for (int j = threadIdx.x; j < first; j += blockDim.x) out[j].id = 0;
+  // read the tiles to split before any of them is overwritten
+  Tile mine[8];
+  int cnt = 0;
+  for (int j = first + (int)threadIdx.x; j < n && cnt < 8; j += blockDim.x) mine[cnt++] = out[j];
+  __syncthreads();
+  cnt = 0;
+  for (int j = first + (int)threadIdx.x; j < n && cnt < 8; j += blockDim.x) {
+    Tile t = mine[cnt++];
+    const int k = first + 2 * (j - first);
+    t.id = 1;
+    out[k] = t;
+    t.id = 2;
+    out[k + 1] = t;
+  }
+  __syncthreads();
+  return n + ns;
+}
+
 __device__ __forceinline__ int warp_incl_scan(int v) {
   const int lane = threadIdx.x & 31;
 #pragma unroll
@@ -237,7 +264,7 @@ __global__ void __launch_bounds__(kPermTB) k_perm_scatter(const __grid_constant_
     __syncthreads();
     int n = build_tiles(totU, uoff, G, kTileM, o.tiles_sh, scratch);
     if (tid == 0) o.counts[kCntTilesSh] = n;
-    n = build_tiles(rows_g, goff, G, kTileM, o.tiles_row, scratch);
+    n = build_row_tiles(rows_g, goff, G, min(pt.nsm, 8 * (int)blockDim.x), o.tiles_row, scratch);
     if (tid == 0) o.counts[kCntTilesRow] = n;
     n = build_tiles(rows_g, goff, G, kTileM * pt.nt_split, o.splits_row, scratch);
     if (tid == 0) o.counts[kCntSplitsRow] = n;

@@ -11,7 +11,7 @@
 //   k_perm_scatter per chunk: segment offsets from the totals (a warp scan in
 //                  (g, e) order), rank of each pair inside its expert
 //                  (bitmask popcounts over the chunk's earlier tokens) -> row;
-//                  CTA 0 writes the offsets and the tile tables
+//                  one extra CTA writes the offsets and the tile tables
 // Integer-only and order-independent, so bit-exact and deterministic.
 #include <algorithm>
 #include <cstdint>
@@ -247,8 +247,9 @@ __global__ void __launch_bounds__(kPermTB) k_perm_scatter(const __grid_constant_
   __syncthreads();
   for (int g = tid; g < G; g += blockDim.x) goff[g] = eoff[pt.eorder[pt.gfirst[g]]];
   __syncthreads();
-  if (blockIdx.x == 0) {
-    // the offsets and the tile tables the other calls read
+  if (blockIdx.x == gridDim.x - 1) {
+    // the last CTA, which owns no chunk: the offsets and the tile tables the
+    // other calls read (in parallel with the chunks' scatter)
     __shared__ int32_t rows_g[ACE_MAX_EXPERTS];
     __shared__ int32_t scratch[ACE_MAX_EXPERTS + 1];
     for (int g = tid; g <= G; g += blockDim.x) {
@@ -268,6 +269,7 @@ __global__ void __launch_bounds__(kPermTB) k_perm_scatter(const __grid_constant_
     if (tid == 0) o.counts[kCntTilesRow] = n;
     n = build_tiles(rows_g, goff, G, kTileM * pt.nt_split, o.splits_row, scratch);
     if (tid == 0) o.counts[kCntSplitsRow] = n;
+    return;
   }
   const int c = blockIdx.x;
   const int t = c * kPermTB + tid;
@@ -380,8 +382,8 @@ cudaError_t launch_permute(const PlanTables& pt, const int32_t* topk_idx, int32_
   o.tiles_row = at<Tile>(ws, L.tiles_row);
   o.splits_row = at<Tile>(ws, L.splits_row);
   size_t sm3 = sizeof(uint32_t) * (size_t)(pt.E + pt.G) * (kPermTB / 32);
-  // one CTA at least: CTA 0 writes the offsets and tables even when T = 0
-  k_perm_scatter<<<C > 0 ? C : 1, kPermTB, sm3, st>>>(pt, topk_idx, T, at<int32_t>(ws, L.chunk_baseE),
+  // one CTA per chunk, plus the one that writes the offsets and tables
+  k_perm_scatter<<<C + 1, kPermTB, sm3, st>>>(pt, topk_idx, T, at<int32_t>(ws, L.chunk_baseE),
                                                      at<int32_t>(ws, L.chunk_baseU), at<int32_t>(ws, L.expert_cnt),
                                                      at<int32_t>(ws, L.tot_u), o);
   return cudaGetLastError();

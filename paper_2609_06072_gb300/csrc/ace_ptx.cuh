@@ -53,6 +53,16 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
   return false;
 }
 
+// Programmatic dependent launch: wait until the kernels this grid depends on
+// (launched before it on the stream) have completed and their writes are
+// visible.  Every kernel calls it before its first global-memory access; when
+// the grid was launched without the attribute it returns at once.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+// Lets the next kernel on the stream start launching once every CTA of this
+// grid has started (its own pdl_wait() still orders its memory accesses after
+// this grid's completion).
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 // ---------------------------------------------------------------- fences
 __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");

@@ -144,6 +144,8 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
   __shared__ uint32_t tslot;
   static_assert(NT * RP <= 128, "dH accumulators must fit below the dB^T columns");
 
+  pdl_wait();
+  pdl_trigger();
   const int n_splits = a.counts[kCntSplitsRow];
   if ((int)blockIdx.x >= n_splits) return;
   const int proj = blockIdx.y;
@@ -453,6 +455,8 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
 template <int RP>
 __global__ void __launch_bounds__(128) k_dh_reduce(const __grid_constant__ PlanTables pt,
                                                    const __grid_constant__ BwdLaunch a) {
+  pdl_wait();
+  pdl_trigger();
   const int n_tiles = a.counts[kCntTilesSh];
   if ((int)blockIdx.x >= n_tiles) return;
   const int proj = blockIdx.y;
@@ -498,6 +502,8 @@ __global__ void __launch_bounds__(256) k_splitk_reduce(const __grid_constant__ P
                                                        const int32_t* __restrict__ counts, int slot,
                                                        const float* __restrict__ part, int RP, int width,
                                                        float* __restrict__ out) {
+  pdl_wait();
+  pdl_trigger();
   const int i = blockIdx.x;  // global rank row
   int g = 0;
   while (pt.rank_off[g + 1] <= i) ++g;
@@ -529,8 +535,7 @@ cudaError_t launch_rows(const PlanTables& pt, const BwdLaunch& a, int nproj, cud
   auto kern = k_bwd_rows<RP, MODE>;
   cudaError_t e = set_smem(kern, C::kSmem);
   if (e != cudaSuccess) return e;
-  kern<<<dim3(a.max_splits_row, nproj), kThreadsWS, C::kSmem, st>>>(pt, a);
-  return cudaGetLastError();
+  return launch_k(kern, dim3(a.max_splits_row, nproj), kThreadsWS, C::kSmem, st, pt, a);
 }
 
 template <int RP>
@@ -556,21 +561,20 @@ cudaError_t launch_bwd_t(const PlanTables& pt, const BwdLaunch& a, bool shared, 
     if ((e = launch_rows<RP, MODE_DOWN>(pt, a, 1, st)) != cudaSuccess) return e;
   } else {
     if ((e = launch_rows<RP, MODE_SHARED>(pt, a, nproj, st)) != cudaSuccess) return e;
-    k_dh_reduce<RP><<<dim3(a.max_tiles_sh, nproj), 128, 0, st>>>(pt, a);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if ((e = launch_k(k_dh_reduce<RP>, dim3(a.max_tiles_sh, nproj), 128, 0, st, pt, a)) != cudaSuccess) return e;
   }
   if (a.deterministic) {
     for (int j = 0; j < nproj; ++j) {
       dim3 grid(n_rank, (a.d_out / 4 + 255) / 256);
-      k_splitk_reduce<<<grid, 256, 0, st>>>(pt, a.splits_row, a.counts, kCntSplitsRow, a.part_dBt[j], RP, a.d_out,
-                                            a.dBt[j]);
-      if ((e = cudaGetLastError()) != cudaSuccess) return e;
+      if ((e = launch_k(k_splitk_reduce, grid, 256, 0, st, pt, a.splits_row, a.counts, kCntSplitsRow, a.part_dBt[j],
+                        (int)RP, a.d_out, a.dBt[j])) != cudaSuccess)
+        return e;
     }
     if (!shared) {
       dim3 grid(n_rank, (a.d_in / 4 + 255) / 256);
-      k_splitk_reduce<<<grid, 256, 0, st>>>(pt, a.splits_row, a.counts, kCntSplitsRow, a.part_dA[0], RP, a.d_in,
-                                            a.dA[0]);
-      if ((e = cudaGetLastError()) != cudaSuccess) return e;
+      if ((e = launch_k(k_splitk_reduce, grid, 256, 0, st, pt, a.splits_row, a.counts, kCntSplitsRow, a.part_dA[0],
+                        (int)RP, a.d_in, a.dA[0])) != cudaSuccess)
+        return e;
     }
   }
   return cudaSuccess;

@@ -53,6 +53,8 @@ __global__ void __launch_bounds__(kHThreads) k_fwd_h(const __grid_constant__ Pla
   __shared__ uint32_t tslot;
   __shared__ int32_t src_row[kTileM];
 
+  pdl_wait();
+  pdl_trigger();
   const int n_tiles = a.counts[kCntTilesSh];
   if ((int)blockIdx.x >= n_tiles) return;
   const Tile tl = a.tiles[blockIdx.x];
@@ -281,6 +283,8 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = tslot;
+  pdl_wait();
+  pdl_trigger();
   const int n_items = a.counts[kCntTilesRow];
   const int d_in = a.d_in, d_out = a.d_out;
   const int NK = SHARED ? 0 : (d_in + 63) / 64;  // K steps of the down H GEMM
@@ -606,8 +610,7 @@ cudaError_t launch_h_t(const PlanTables& pt, const FwdHLaunch& a, cudaStream_t s
   auto kern = k_fwd_h<RP, NPROJ>;
   cudaError_t e = set_smem(kern, C::kSmem);
   if (e != cudaSuccess || a.max_tiles <= 0) return e;
-  kern<<<a.max_tiles, kHThreads, C::kSmem, st>>>(pt, a);
-  return cudaGetLastError();
+  return launch_k(kern, a.max_tiles, kHThreads, C::kSmem, st, pt, a);
 }
 
 template <int RP, int NPROJ, bool SHARED>
@@ -616,6 +619,8 @@ cudaError_t launch_rows_t(const PlanTables& pt, const FwdRowsLaunch& a, cudaStre
   auto kern = k_fwd_rows<RP, NPROJ, SHARED>;
   cudaError_t e = set_smem(kern, C::kSmem);
   if (e != cudaSuccess || a.grid <= 0) return e;
+  // a plain launch: with programmatic serialization after k_fwd_h the gate/up
+  // call measured slower
   kern<<<a.grid, kRowsThreads, C::kSmem, st>>>(pt, a);
   return cudaGetLastError();
 }

@@ -66,6 +66,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemm_dx(const __grid_constant__
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  pdl_wait();
+  pdl_trigger();
   const uint32_t tmem = tslot;
   bool bad = false;
   if (warp == 0) {
@@ -220,6 +222,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemm_da(const __grid_constant__
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  pdl_wait();
+  pdl_trigger();
   const uint32_t tmem = tslot;
   bool bad = false;
   if (warp == 0) {
@@ -309,13 +313,11 @@ cudaError_t launch_dense_bwd(const DenseBwdLaunch& a, cudaStream_t st) {
   e = cudaFuncSetAttribute(k_gemm_da, cudaFuncAttributeMaxDynamicSharedMemorySize, kDaSmem);
   if (e != cudaSuccess) return e;
   const int dx_tiles = ((a.T + 127) / 128) * ((a.d + kDxN - 1) / kDxN);
-  k_gemm_dx<<<std::min(dx_tiles, a.grid), kThreads, kDxSmem, st>>>(a);
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  if ((e = launch_k(k_gemm_dx, std::min(dx_tiles, a.grid), kThreads, kDxSmem, st, a)) != cudaSuccess) return e;
   // dA accumulates bulk reduce-adds: the caller has zeroed it (with the
   // backward's other accumulation targets, in one launch)
   const int da_tiles = ((a.nproj * a.n_rank_pad + 127) / 128) * ((a.d + kDaN - 1) / kDaN);
-  k_gemm_da<<<da_tiles * da_ksplit(da_tiles, a.grid), kThreads, kDaSmem, st>>>(a);
-  return cudaGetLastError();
+  return launch_k(k_gemm_da, da_tiles * da_ksplit(da_tiles, a.grid), kThreads, kDaSmem, st, a);
 }
 
 }  // namespace ace

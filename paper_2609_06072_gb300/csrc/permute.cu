@@ -17,6 +17,7 @@
 #include <cstdint>
 
 #include "ace_internal.cuh"
+#include "ace_ptx.cuh"
 
 namespace ace {
 namespace {
@@ -47,6 +48,8 @@ __global__ void __launch_bounds__(kPermTB) k_perm_count(const __grid_constant__ 
   int32_t* cntU = sm + pt.E;         // [G]
   __shared__ int32_t err_s;
   const int tid = threadIdx.x;
+  pdl_wait();
+  pdl_trigger();
   for (int i = tid; i < pt.E + pt.G; i += blockDim.x) sm[i] = 0;
   if (tid == 0) err_s = 0;
   __syncthreads();
@@ -152,6 +155,8 @@ __global__ void __launch_bounds__(256) k_perm_colscan(const __grid_constant__ Pl
   __shared__ int32_t wsum[8];
   __shared__ int32_t err_s;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  pdl_wait();
+  pdl_trigger();
   const bool isE = (int)blockIdx.x < pt.E;
   const int ncol = isE ? pt.E : pt.G, col = isE ? blockIdx.x : blockIdx.x - pt.E;
   const int32_t* cnt = isE ? chunk_cntE : chunk_cntU;
@@ -223,6 +228,8 @@ __global__ void __launch_bounds__(kPermTB) k_perm_scatter(const __grid_constant_
   __shared__ int32_t goff[ACE_MAX_EXPERTS + 1];  // first row of each group
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int E = pt.E, G = pt.G;
+  pdl_wait();
+  pdl_trigger();
   for (int i = tid; i < (E + G) * W; i += blockDim.x) msk[i] = 0;
   // segment offsets: rows in (g, e) order (warp 0), unique pairs in g order (warp 1)
   if (warp == 0) {
@@ -333,6 +340,8 @@ struct ZeroList {
   int n;
 };
 __global__ void __launch_bounds__(256) k_zero(const __grid_constant__ ZeroList z) {
+  pdl_wait();
+  pdl_trigger();
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int b = 0; b < z.n; ++b)
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < z.n16[b]; i += stride)
@@ -341,6 +350,8 @@ __global__ void __launch_bounds__(256) k_zero(const __grid_constant__ ZeroList z
 
 __global__ void k_rows_copy(const int32_t* __restrict__ row_pair, const uint4* __restrict__ src,
                             uint4* __restrict__ dst, int64_t R, int vec_per_row, bool gather) {
+  pdl_wait();
+  pdl_trigger();
   const int64_t n = R * vec_per_row;
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
     const int64_t row = i / vec_per_row, v = i % vec_per_row;
@@ -359,14 +370,15 @@ cudaError_t launch_permute(const PlanTables& pt, const int32_t* topk_idx, int32_
   const int C = L.n_chunks;
   if (C > 0) {
     size_t sm1 = sizeof(int32_t) * (pt.E + pt.G);
-    k_perm_count<<<C, kPermTB, sm1, st>>>(pt, topk_idx, T, at<int32_t>(ws, L.chunk_cntE),
-                                          at<int32_t>(ws, L.chunk_cntU), at<int32_t>(ws, L.chunk_err));
+    cudaError_t e = launch_k(k_perm_count, C, kPermTB, sm1, st, pt, topk_idx, T, at<int32_t>(ws, L.chunk_cntE),
+                             at<int32_t>(ws, L.chunk_cntU), at<int32_t>(ws, L.chunk_err));
+    if (e != cudaSuccess) return e;
   }
-  k_perm_colscan<<<pt.E + pt.G, 256, 0, st>>>(pt, C, at<int32_t>(ws, L.chunk_cntE), at<int32_t>(ws, L.chunk_cntU),
-                                                at<int32_t>(ws, L.chunk_err), at<int32_t>(ws, L.chunk_baseE),
-                                                at<int32_t>(ws, L.chunk_baseU), at<int32_t>(ws, L.expert_cnt),
-                                                at<int32_t>(ws, L.tot_u), at<int32_t>(ws, L.err),
-                                                at<int32_t>(ws, L.sched));
+  cudaError_t e = launch_k(k_perm_colscan, pt.E + pt.G, 256, 0, st, pt, C, at<int32_t>(ws, L.chunk_cntE),
+                           at<int32_t>(ws, L.chunk_cntU), at<int32_t>(ws, L.chunk_err), at<int32_t>(ws, L.chunk_baseE),
+                           at<int32_t>(ws, L.chunk_baseU), at<int32_t>(ws, L.expert_cnt), at<int32_t>(ws, L.tot_u),
+                           at<int32_t>(ws, L.err), at<int32_t>(ws, L.sched));
+  if (e != cudaSuccess) return e;
   ScatterOut o;
   o.row_pair = at<int32_t>(ws, L.row_pair);
   o.pair_row = at<int32_t>(ws, L.pair_row);
@@ -383,10 +395,8 @@ cudaError_t launch_permute(const PlanTables& pt, const int32_t* topk_idx, int32_
   o.splits_row = at<Tile>(ws, L.splits_row);
   size_t sm3 = sizeof(uint32_t) * (size_t)(pt.E + pt.G) * (kPermTB / 32);
   // one CTA per chunk, plus the one that writes the offsets and tables
-  k_perm_scatter<<<C + 1, kPermTB, sm3, st>>>(pt, topk_idx, T, at<int32_t>(ws, L.chunk_baseE),
-                                                     at<int32_t>(ws, L.chunk_baseU), at<int32_t>(ws, L.expert_cnt),
-                                                     at<int32_t>(ws, L.tot_u), o);
-  return cudaGetLastError();
+  return launch_k(k_perm_scatter, C + 1, kPermTB, sm3, st, pt, topk_idx, T, at<int32_t>(ws, L.chunk_baseE),
+                  at<int32_t>(ws, L.chunk_baseU), at<int32_t>(ws, L.expert_cnt), at<int32_t>(ws, L.tot_u), o);
 }
 
 cudaError_t launch_zero(void* const* ptrs, const size_t* bytes, int n, cudaStream_t st) {
@@ -401,8 +411,7 @@ cudaError_t launch_zero(void* const* ptrs, const size_t* bytes, int n, cudaStrea
   }
   if (z.n == 0) return cudaSuccess;
   const int blocks = (int)std::min<int64_t>((total + 255) / 256, 152 * 4);
-  k_zero<<<blocks, 256, 0, st>>>(z);
-  return cudaGetLastError();
+  return launch_k(k_zero, blocks, 256, 0, st, z);
 }
 
 cudaError_t launch_rows_copy(const int32_t* row_pair, const uint16_t* src, uint16_t* dst, int64_t R, int32_t cols,
@@ -411,9 +420,8 @@ cudaError_t launch_rows_copy(const int32_t* row_pair, const uint16_t* src, uint1
   const int vpr = cols / 8;
   const int64_t n = R * vpr;
   int blocks = (int)std::min<int64_t>((n + 255) / 256, 152 * 16);
-  k_rows_copy<<<blocks, 256, 0, st>>>(row_pair, reinterpret_cast<const uint4*>(src), reinterpret_cast<uint4*>(dst),
-                                      R, vpr, gather);
-  return cudaGetLastError();
+  return launch_k(k_rows_copy, blocks, 256, 0, st, row_pair, reinterpret_cast<const uint4*>(src),
+                  reinterpret_cast<uint4*>(dst), R, vpr, gather);
 }
 
 }  // namespace ace

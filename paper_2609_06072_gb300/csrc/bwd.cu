@@ -451,47 +451,54 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
 
 // ---------------------------------------------------------------- dH_u
 // dH_u = sum of the dH rows of unique pair u (fixed slot order), written into
-// the token-major dense matrix dHx[t][j * n_rank_pad + rank_off[g] + k].
+// the token-major dense matrix dHx[t][j * n_rank_pad + rank_off[g] + k].  One
+// thread per (unique pair, 8 columns): the RP / 8 threads of a pair read its
+// rows' 32-byte pieces side by side, and many pairs' loads are in flight.
 template <int RP>
 __global__ void __launch_bounds__(128) k_dh_reduce(const __grid_constant__ PlanTables pt,
                                                    const __grid_constant__ BwdLaunch a) {
+  constexpr int CH = RP / 8;  // threads per unique pair
   pdl_wait();
   pdl_trigger();
   const int n_tiles = a.counts[kCntTilesSh];
-  if ((int)blockIdx.x >= n_tiles) return;
+  const int tile = blockIdx.x / CH;
+  if (tile >= n_tiles) return;
   const int proj = blockIdx.y;
-  const Tile tl = a.tiles_sh[blockIdx.x];
-  const int m = threadIdx.x;
+  const Tile tl = a.tiles_sh[tile];
+  const int m = (blockIdx.x % CH) * (128 / CH) + threadIdx.x / CH, q = threadIdx.x % CH;
   if (m >= tl.cnt) return;
   const int u = tl.start + m, t = a.uniq_tok[u], k = pt.k, g = tl.g;
   const int r0 = pt.rank_off[g], rg = pt.rank_off[g + 1] - r0;
-  float acc[RP];
+  int rows[kMaxK];
+  int n = 0;
+  for (int j = 0; j < k; ++j)
+    if (a.pair_g[(int64_t)t * k + j] == g) rows[n++] = a.pair_row[(int64_t)t * k + j];
+  float acc[8];
 #pragma unroll
-  for (int q = 0; q < RP; ++q) acc[q] = 0.f;
-  for (int j = 0; j < k; ++j) {
-    if (a.pair_g[(int64_t)t * k + j] != g) continue;
-    const float4* src = reinterpret_cast<const float4*>(a.dHrow[proj] + (int64_t)a.pair_row[(int64_t)t * k + j] * RP);
-#pragma unroll
-    for (int q = 0; q < RP / 4; ++q) {
-      const float4 v = src[q];
-      acc[4 * q] += v.x;
-      acc[4 * q + 1] += v.y;
-      acc[4 * q + 2] += v.z;
-      acc[4 * q + 3] += v.w;
-    }
+  for (int c = 0; c < 8; ++c) acc[c] = 0.f;
+  for (int i = 0; i < n; ++i) {
+    const float4* src = reinterpret_cast<const float4*>(a.dHrow[proj] + (int64_t)rows[i] * RP + q * 8);
+    const float4 v0 = src[0], v1 = src[1];
+    acc[0] += v0.x;
+    acc[1] += v0.y;
+    acc[2] += v0.z;
+    acc[3] += v0.w;
+    acc[4] += v1.x;
+    acc[5] += v1.y;
+    acc[6] += v1.z;
+    acc[7] += v1.w;
   }
+  if (q * 8 >= rg) return;
   const int kw = a.nproj * a.n_rank_pad;
-  uint16_t* dst = a.dHx + (int64_t)t * kw + proj * a.n_rank_pad + r0;
-  if ((r0 & 7) == 0 && (rg & 7) == 0) {
-#pragma unroll
-    for (int q = 0; q < RP / 8; ++q)
-      if (q * 8 < rg) reinterpret_cast<uint4*>(dst)[q] = pack8(&acc[8 * q]);
+  uint16_t* dst = a.dHx + (int64_t)t * kw + proj * a.n_rank_pad + r0 + q * 8;
+  if ((r0 & 7) == 0 && q * 8 + 8 <= rg) {
+    *reinterpret_cast<uint4*>(dst) = pack8(acc);
   } else {
 #pragma unroll
-    for (int q = 0; q < RP; ++q)
-      if (q < rg) {
-        const __nv_bfloat16 h = __float2bfloat16_rn(acc[q]);
-        dst[q] = *reinterpret_cast<const uint16_t*>(&h);
+    for (int c = 0; c < 8; ++c)
+      if (q * 8 + c < rg) {
+        const __nv_bfloat16 h = __float2bfloat16_rn(acc[c]);
+        dst[c] = *reinterpret_cast<const uint16_t*>(&h);
       }
   }
 }
@@ -561,7 +568,8 @@ cudaError_t launch_bwd_t(const PlanTables& pt, const BwdLaunch& a, bool shared, 
     if ((e = launch_rows<RP, MODE_DOWN>(pt, a, 1, st)) != cudaSuccess) return e;
   } else {
     if ((e = launch_rows<RP, MODE_SHARED>(pt, a, nproj, st)) != cudaSuccess) return e;
-    if ((e = launch_k(k_dh_reduce<RP>, dim3(a.max_tiles_sh, nproj), 128, 0, st, pt, a)) != cudaSuccess) return e;
+    if ((e = launch_k(k_dh_reduce<RP>, dim3(a.max_tiles_sh * (RP / 8), nproj), 128, 0, st, pt, a)) != cudaSuccess)
+      return e;
   }
   if (a.deterministic) {
     for (int j = 0; j < nproj; ++j) {

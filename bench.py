@@ -42,6 +42,18 @@ def dist_env():
     return rank, world, local
 
 
+def reduce_max(x, device):
+    """Max of x over the ranks of the default process group (x itself when
+    there is none): timed regions are reported as the slowest rank's."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -308,6 +320,40 @@ CALLS = ["permute", "fwd_shared", "fwd_row", "bwd_row", "bwd_shared"]
 SINGLE_KERNEL = {"fwd_row": "k_fwd_rows<down>"}
 
 
+def time_steps(lay, steps, warmup, flush):
+    """Mean step time (ms) of `steps` steps, events at step boundaries only;
+    flush: a buffer larger than L2 written before each step, or None."""
+    import torch
+    for _ in range(warmup):
+        lay.step()
+    torch.cuda.synchronize()
+    evs = [[torch.cuda.Event(enable_timing=True), None, None, None, None, torch.cuda.Event(enable_timing=True)]
+           for _ in range(steps)]
+    for e in evs:
+        if flush is not None:
+            flush.zero_()
+        lay.step(e)
+    torch.cuda.synchronize()
+    assert lay.plan.get_error(lay.perm) == 0
+    return float(np.mean([e[0].elapsed_time(e[5]) for e in evs]))
+
+
+def run_variants(args, flush, main_layer):
+    """The other timings of the same workload: the expert-wise layout at the
+    matched adapter budget, the deterministic split-K mode, and no L2 flush."""
+    out = {}
+    c_rows = main_layer.c.R
+    for name, ew, det in (("expertwise_matched_budget", not args.expertwise, args.det),
+                          ("deterministic" if not args.det else "fast_atomics", args.expertwise, not args.det)):
+        lay = Layer(args.config, args.seed, ew, det)
+        ms = time_steps(lay, args.steps, args.warmup, flush)
+        out[name] = {"value": c_rows / (ms * 1e-3), "ms_per_step": ms, "expertwise": ew, "deterministic": det}
+        del lay
+    ms = time_steps(main_layer, args.steps, args.warmup, None)
+    out["unflushed"] = {"value": c_rows / (ms * 1e-3), "ms_per_step": ms}
+    return out
+
+
 def run_gpu(args, rank, world, local):
     import torch
     torch.cuda.set_device(local)
@@ -348,6 +394,8 @@ def run_gpu(args, rank, world, local):
     step_ms = [e[0].elapsed_time(e[5]) for e in evs]
     fwd_row_ms = float(np.mean([e[2].elapsed_time(e[3]) for e in evs]))
     ms = float(np.sum(step_ms))
+    step_stats = {"median_ms": float(np.median(step_ms)), "mean_ms": float(np.mean(step_ms)),
+                  "std_ms": float(np.std(step_ms)), "min_ms": float(np.min(step_ms))}
     # per-call breakdown (diagnostic, not part of `value`): a second pass with
     # events at every call boundary
     evs_b = [[new_ev() for _ in range(6)] for _ in range(args.steps)]
@@ -357,9 +405,7 @@ def run_gpu(args, rank, world, local):
     torch.cuda.synchronize()
     per_call = {n: [e[j].elapsed_time(e[j + 1]) for e in evs_b] for j, n in enumerate(CALLS)}
     if world > 1:
-        t = torch.tensor([ms], device="cuda")
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms = float(t.item())
+        ms = reduce_max(ms, "cuda")
         torch.distributed.barrier()
     ms_per_step = ms / args.steps
     value = world * c.R / (ms_per_step * 1e-3)
@@ -382,9 +428,7 @@ def run_gpu(args, rank, world, local):
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1)
     if world > 1:
-        t = torch.tensor([e2e_ms], device="cuda")
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        e2e_ms = float(t.item())
+        e2e_ms = reduce_max(e2e_ms, "cuda")
     e2e_value = world * c.R * args.steps / (e2e_ms * 1e-3)
 
     peaks = load_peaks()
@@ -422,6 +466,7 @@ def run_gpu(args, rank, world, local):
                           "achieved_GBps": total_bytes / (ms_per_step * 1e-3) / 1e9,
                           "frac_hbm": total_bytes / (ms_per_step * 1e-3) / 1e9 / peaks["hbm_gbs"],
                           "tensor_TFLOPs": total_flops / (ms_per_step * 1e-3) / 1e12},
+        "step_ms_stats": step_stats,
         "per_call_ms": call_ms,
         "per_call_frac_hbm": {n: bytes_[n] / (call_ms[n] * 1e-3) / 1e9 / peaks["hbm_gbs"] for n in CALLS},
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": lay.h2d_bytes(),
@@ -430,6 +475,8 @@ def run_gpu(args, rank, world, local):
         "clocks": clocks,
         "wall_s_timed": t_wall,
     }
+    if not args.no_variants:
+        out["variants"] = run_variants(args, flush, lay)
     return out, lay
 
 
@@ -548,6 +595,8 @@ def main():
     ap.add_argument("--det", action="store_true", help="deterministic two-stage split-K for dA / dB^T")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU-oracle baseline leg")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--no-variants", action="store_true",
+                    help="skip the expert-wise, deterministic-mode and unflushed timings")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

@@ -22,22 +22,45 @@
 namespace ace {
 namespace {
 
-// Reads token t's k expert ids; returns false (and leaves `e` partially
-// filled) when an id is out of range or repeated within the token.
-__device__ __forceinline__ bool read_token(const int32_t* __restrict__ idx, int t, int k, int E, int* e) {
+// Reads token t's k expert ids into e[0..k) (KB >= k; the loops unroll so e
+// stays in registers); false when an id is out of range or repeated within
+// the token.
+template <int KB>
+__device__ __forceinline__ bool read_token(const int32_t* __restrict__ idx, int t, int k, int E, int (&e)[KB]) {
   bool ok = true;
-  for (int j = 0; j < k; ++j) {
-    int v = idx[(int64_t)t * k + j];
-    e[j] = v;
-    if (v < 0 || v >= E) ok = false;
+#pragma unroll
+  for (int j = 0; j < KB; ++j) {
+    e[j] = -1;
+    if (j < k) {
+      const int v = idx[(int64_t)t * k + j];
+      e[j] = v;
+      if (v < 0 || v >= E) ok = false;
+    }
   }
-  if (!ok) return false;
-  for (int j = 1; j < k; ++j)
+#pragma unroll
+  for (int j = 1; j < KB; ++j)
+#pragma unroll
     for (int jj = 0; jj < j; ++jj)
-      if (e[j] == e[jj]) return false;
-  return true;
+      if (j < k && e[j] == e[jj]) ok = false;
+  return ok;
 }
 
+// Bit j set when slot j is the first of the token's slots routed into its group.
+template <int KB>
+__device__ __forceinline__ uint32_t first_of_group(const int (&g)[KB], int k) {
+  uint32_t m = 0;
+#pragma unroll
+  for (int j = 0; j < KB; ++j) {
+    bool first = j < k;
+#pragma unroll
+    for (int jj = 0; jj < j; ++jj)
+      if (g[jj] == g[j]) first = false;
+    if (first) m |= 1u << j;
+  }
+  return m;
+}
+
+template <int KB>
 __global__ void __launch_bounds__(kPermTB) k_perm_count(const __grid_constant__ PlanTables pt,
                                                         const int32_t* __restrict__ idx, int T,
                                                         int32_t* __restrict__ chunk_cntE,
@@ -46,26 +69,29 @@ __global__ void __launch_bounds__(kPermTB) k_perm_count(const __grid_constant__ 
   extern __shared__ int32_t sm[];
   int32_t* cntE = sm;                // [E]
   int32_t* cntU = sm + pt.E;         // [G]
+  int32_t* e2g = sm + pt.E + pt.G;   // [E] expert -> group, staged from the plan
   __shared__ int32_t err_s;
   const int tid = threadIdx.x;
   pdl_wait();
   pdl_trigger();
   for (int i = tid; i < pt.E + pt.G; i += blockDim.x) sm[i] = 0;
+  for (int i = tid; i < pt.E; i += blockDim.x) e2g[i] = pt.e2g[i];
   if (tid == 0) err_s = 0;
   __syncthreads();
   const int t = blockIdx.x * kPermTB + tid;
   if (t < T) {
-    int e[kMaxK];
-    if (!read_token(idx, t, pt.k, pt.E, e)) {
+    int e[KB];
+    if (!read_token<KB>(idx, t, pt.k, pt.E, e)) {
       atomicOr(&err_s, kErrIndex);
     } else {
-      for (int j = 0; j < pt.k; ++j) {
-        atomicAdd(&cntE[e[j]], 1);
-        int g = pt.e2g[e[j]];
-        bool first = true;
-        for (int jj = 0; jj < j; ++jj)
-          if (pt.e2g[e[jj]] == g) first = false;
-        if (first) atomicAdd(&cntU[g], 1);
+      int g[KB];
+#pragma unroll
+      for (int j = 0; j < KB; ++j) g[j] = j < pt.k ? e2g[e[j]] : -1 - j;
+      const uint32_t first = first_of_group<KB>(g, pt.k);
+#pragma unroll
+      for (int j = 0; j < KB; ++j) {
+        if (j < pt.k) atomicAdd(&cntE[e[j]], 1);
+        if ((first >> j) & 1u) atomicAdd(&cntU[g[j]], 1);
       }
     }
   }
@@ -213,6 +239,7 @@ struct ScatterOut {
   Tile* splits_row;
 };
 
+template <int KB>
 __global__ void __launch_bounds__(kPermTB) k_perm_scatter(const __grid_constant__ PlanTables pt,
                                                           const int32_t* __restrict__ idx, int T,
                                                           const int32_t* __restrict__ chunk_baseE,
@@ -226,11 +253,22 @@ __global__ void __launch_bounds__(kPermTB) k_perm_scatter(const __grid_constant_
   __shared__ int32_t eoff[ACE_MAX_EXPERTS];      // first row of each expert segment
   __shared__ int32_t uoff[ACE_MAX_EXPERTS + 1];  // first unique pair of each group
   __shared__ int32_t goff[ACE_MAX_EXPERTS + 1];  // first row of each group
+  __shared__ int32_t baseE[ACE_MAX_EXPERTS];     // this chunk's rows before it, per expert
+  __shared__ int32_t baseU[ACE_MAX_EXPERTS];     // this chunk's unique pairs before it, per group
+  __shared__ int32_t e2g[ACE_MAX_EXPERTS];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int E = pt.E, G = pt.G;
   pdl_wait();
   pdl_trigger();
   for (int i = tid; i < (E + G) * W; i += blockDim.x) msk[i] = 0;
+  const int c = blockIdx.x;
+  if (c < (int)gridDim.x - 1) {
+    for (int i = tid; i < E; i += blockDim.x) {
+      baseE[i] = chunk_baseE[(int64_t)c * E + i];
+      e2g[i] = pt.e2g[i];
+    }
+    for (int i = tid; i < G; i += blockDim.x) baseU[i] = chunk_baseU[(int64_t)c * G + i];
+  }
   // segment offsets: rows in (g, e) order (warp 0), unique pairs in g order (warp 1)
   if (warp == 0) {
     int carry = 0;
@@ -278,19 +316,20 @@ __global__ void __launch_bounds__(kPermTB) k_perm_scatter(const __grid_constant_
     if (tid == 0) o.counts[kCntSplitsRow] = n;
     return;
   }
-  const int c = blockIdx.x;
   const int t = c * kPermTB + tid;
   const int k = pt.k;
-  int e[kMaxK];
+  int e[KB];
   bool ok = false;
   if (t < T) {
-    ok = read_token(idx, t, k, E, e);
+    ok = read_token<KB>(idx, t, k, E, e);
     if (ok) {
       const uint32_t bit = 1u << (tid & 31);
-      for (int j = 0; j < k; ++j) {
-        atomicOr(&mE[e[j] * W + (tid >> 5)], bit);
-        atomicOr(&mU[pt.e2g[e[j]] * W + (tid >> 5)], bit);
-      }
+#pragma unroll
+      for (int j = 0; j < KB; ++j)
+        if (j < k) {
+          atomicOr(&mE[e[j] * W + (tid >> 5)], bit);
+          atomicOr(&mU[e2g[e[j]] * W + (tid >> 5)], bit);
+        }
     }
   }
   __syncthreads();
@@ -302,34 +341,31 @@ __global__ void __launch_bounds__(kPermTB) k_perm_scatter(const __grid_constant_
     }
     return;
   }
-  int rows_j[kMaxK];
-  for (int j = 0; j < k; ++j) {
-    const int row = eoff[e[j]] + chunk_baseE[(int64_t)c * E + e[j]] + prefix_bits(&mE[e[j] * W], tid);
+  int g[KB];
+#pragma unroll
+  for (int j = 0; j < KB; ++j) g[j] = j < k ? e2g[e[j]] : -1 - j;
+  const uint32_t first = first_of_group<KB>(g, k);
+#pragma unroll
+  for (int j = 0; j < KB; ++j) {
+    if (j >= k) break;
+    const int row = eoff[e[j]] + baseE[e[j]] + prefix_bits(&mE[e[j] * W], tid);
+    const int u = uoff[g[j]] + baseU[g[j]] + prefix_bits(&mU[g[j] * W], tid);
     const int p = t * k + j;
-    rows_j[j] = row;
     o.pair_row[p] = row;
-    o.pair_g[p] = pt.e2g[e[j]];
+    o.pair_g[p] = g[j];
     o.row_pair[row] = p;
-  }
-  // distinct groups of the token, ascending
-  int n_u = 0;
-  int last = -1;
-  while (true) {
-    int nxt = 0x7fffffff;
-    for (int j = 0; j < k; ++j) {
-      int g = pt.e2g[e[j]];
-      if (g > last && g < nxt) nxt = g;
+    o.row_uniq[row] = u;
+    if ((first >> j) & 1u) {
+      // position among the token's distinct groups in ascending order
+      int n_below = 0;
+#pragma unroll
+      for (int jj = 0; jj < KB; ++jj)
+        if (((first >> jj) & 1u) && g[jj] < g[j]) ++n_below;
+      o.uniq_tok[u] = t;
+      o.tok_uniq[(int64_t)t * k + n_below] = u;
     }
-    if (nxt == 0x7fffffff) break;
-    const int u = uoff[nxt] + chunk_baseU[(int64_t)c * G + nxt] + prefix_bits(&mU[nxt * W], tid);
-    o.uniq_tok[u] = t;
-    o.tok_uniq[(int64_t)t * k + n_u] = u;
-    for (int j = 0; j < k; ++j)
-      if (pt.e2g[e[j]] == nxt) o.row_uniq[rows_j[j]] = u;
-    ++n_u;
-    last = nxt;
   }
-  for (int j = n_u; j < k; ++j) o.tok_uniq[(int64_t)t * k + j] = -1;
+  for (int j = __popc(first); j < k; ++j) o.tok_uniq[(int64_t)t * k + j] = -1;
 }
 
 // Zeroes up to kZeroMax buffers (16-byte aligned, sizes multiples of 16) in
@@ -369,8 +405,8 @@ cudaError_t launch_permute(const PlanTables& pt, const int32_t* topk_idx, int32_
                            cudaStream_t st) {
   const int C = L.n_chunks;
   if (C > 0) {
-    size_t sm1 = sizeof(int32_t) * (pt.E + pt.G);
-    cudaError_t e = launch_k(k_perm_count, C, kPermTB, sm1, st, pt, topk_idx, T, at<int32_t>(ws, L.chunk_cntE),
+    size_t sm1 = sizeof(int32_t) * (2 * pt.E + pt.G);
+    cudaError_t e = launch_k(pt.k <= 8 ? k_perm_count<8> : k_perm_count<kMaxK>, C, kPermTB, sm1, st, pt, topk_idx, T, at<int32_t>(ws, L.chunk_cntE),
                              at<int32_t>(ws, L.chunk_cntU), at<int32_t>(ws, L.chunk_err));
     if (e != cudaSuccess) return e;
   }
@@ -395,7 +431,7 @@ cudaError_t launch_permute(const PlanTables& pt, const int32_t* topk_idx, int32_
   o.splits_row = at<Tile>(ws, L.splits_row);
   size_t sm3 = sizeof(uint32_t) * (size_t)(pt.E + pt.G) * (kPermTB / 32);
   // one CTA per chunk, plus the one that writes the offsets and tables
-  return launch_k(k_perm_scatter, C + 1, kPermTB, sm3, st, pt, topk_idx, T, at<int32_t>(ws, L.chunk_baseE),
+  return launch_k(pt.k <= 8 ? k_perm_scatter<8> : k_perm_scatter<kMaxK>, C + 1, kPermTB, sm3, st, pt, topk_idx, T, at<int32_t>(ws, L.chunk_baseE),
                   at<int32_t>(ws, L.chunk_baseU), at<int32_t>(ws, L.expert_cnt), at<int32_t>(ws, L.tot_u), o);
 }
 

@@ -36,6 +36,7 @@ constexpr int MODE_DOWN = 0, MODE_SHARED = 1;
 constexpr int kThreadsWS = 320;     // producer, MMA, 8 epilogue warps (two per TMEM lane quarter)
 constexpr int kEpiThreads = 256;
 constexpr int kEpiBar = 1;
+constexpr int kIssueBar = 2;        // epilogue -> producer: the H prefetches are out
 
 // Operand slots of [128 x RP] bf16 (H or dH tiles).  For RP <= 64 several
 // slots share one 128-byte-swizzled block side by side (column offset
@@ -192,6 +193,9 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
+    // the dY stream starts once the epilogue has sent out its H prefetches,
+    // so they are not queued behind it
+    named_bar(kIssueBar, kEpiThreads + 32);
     if (lane == 0) {
       for (int q = 0; q < NI1 + NI2 && !bad; ++q) {
         const int s = q % SA, u = q / SA;
@@ -300,8 +304,15 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
     const int fmode = a.deterministic ? kPartial : kAtomic;
     // H operand slots: bf16 of the saved H of each row, staged while the
-    // producer already streams the first dY tiles
+    // producer already streams the first dY tiles.  The rows' lines are
+    // prefetched into L2 first, ahead of the stream.
     {
+      for (int idx = et; idx < sp.cnt; idx += kEpiThreads) {
+        const int hrow = MODE == MODE_SHARED ? a.row_uniq[sp.start + idx] : sp.start + idx;
+        const float* hp = a.H[proj] + (int64_t)hrow * pt.rank_max;
+        for (int c = 0; c < RP && c < pt.rank_max; c += 32) prefetch_l2(hp + c);
+      }
+      named_bar_arrive(kIssueBar, kEpiThreads + 32);
       const bool vec = (pt.rank_max & 3) == 0;
       for (int idx = et; idx < ntiles * kTileM; idx += kEpiThreads) {
         const int i = idx / kTileM, mm = idx % kTileM;

@@ -196,10 +196,10 @@ class Layer:
 
     def kernels_per_step(self):
         # permute 3, fwd_shared 2 (H per unique pair, row stream), fwd_row 1,
-        # bwd_row 2 (zeroing, row stream), bwd_shared 5 (zeroing, row stream, dH_u sum, dX, dA);
+        # bwd_row 2 (zeroing, row stream), bwd_shared 4 (zeroing, row stream, dX, dA);
         # deterministic mode: bwd_row has nothing to zero and adds a dB^T and a dA reduce,
-        # bwd_shared adds one dB^T reduce per projection
-        return 13 + (3 if self.det else 0)
+        # bwd_shared adds the fixed-order dH_u sum and one dB^T reduce per projection
+        return 12 + (4 if self.det else 0)
 
     def step(self, ev=None):
         """One pass of the hot path.  ev: 6 CUDA events or None at the call

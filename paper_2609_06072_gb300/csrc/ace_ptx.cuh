@@ -132,6 +132,17 @@ __device__ __forceinline__ void named_bar_arrive(int id, int nthreads) {
   asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
+// Relaxed, gpu-scope reductions into bf16 global memory: 8 values at a
+// 16-byte aligned address, or one value.
+__device__ __forceinline__ void red_add_bf16x8(void* p, uint4 v) {
+  asm volatile("red.global.add.noftz.v4.bf16x2 [%0], {%1, %2, %3, %4};" ::"l"(p), "r"(v.x), "r"(v.y), "r"(v.z),
+               "r"(v.w)
+               : "memory");
+}
+__device__ __forceinline__ void red_add_bf16(void* p, uint16_t h) {
+  asm volatile("red.global.add.noftz.bf16 [%0], %1;" ::"l"(p), "h"(h) : "memory");
+}
+
 // Hint: bring the 128-byte line holding p into L2.
 __device__ __forceinline__ void prefetch_l2(const void* p) {
   asm volatile("prefetch.global.L2 [%0];" ::"l"(p));

@@ -16,10 +16,11 @@
 //     dA_c   = sum_i h_i^T . dH_i         (flushed like dB^T)
 //   For gate/up (MODE_SHARED) the rows of one unique pair (g, t) share H_u and
 //   dC_u . B_g = sum_rows dY_row . B_g, so streaming contiguous rows moves the
-//   bytes of the deduplicated form; dH per row goes to fp32 scratch.
-// k_dh_reduce: dH_u = sum of the dH rows of unique pair u (fixed slot order),
-//   written into the token-major dense dHx consumed by the dense dX / dA
-//   GEMMs of gemm.cu.
+//   bytes of the deduplicated form.  dH_u, the sum of its rows' dH, lands in
+//   the token-major dense dHx consumed by the dense dX / dA GEMMs of gemm.cu:
+//   in the fast mode each row adds its dH there with bf16 vector reductions;
+//   in the deterministic mode the rows go to fp32 scratch and
+// k_dh_reduce sums them per unique pair in a fixed slot order.
 // k_splitk_reduce: deterministic stage 2 of dB^T / dA (split order); empty groups
 //   -> exact zeros.
 #include <cstdint>
@@ -143,6 +144,7 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
   __shared__ __align__(8) uint64_t dbt_full[2], dbt_empty[2], d_full[2], d_empty[2], da_full[2], da_empty[2];
   __shared__ __align__(8) uint64_t dh_full, hs_ready, ops_ready;
   __shared__ uint32_t tslot;
+  __shared__ int32_t tok_s[MODE == MODE_SHARED ? NT * kTileM : 1];  // token of each row (gate/up)
   static_assert(NT * RP <= 128, "dH accumulators must fit below the dB^T columns");
 
   pdl_wait();
@@ -319,6 +321,7 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
         const int row = sp.start + idx;
         const int hrow = idx >= sp.cnt ? -1 : (MODE == MODE_SHARED ? a.row_uniq[row] : row);
         const float* hp = a.H[proj] + (int64_t)(hrow < 0 ? 0 : hrow) * pt.rank_max;
+        if (MODE == MODE_SHARED) tok_s[idx] = hrow < 0 ? -1 : a.uniq_tok[hrow];
 #pragma unroll
         for (int c0 = 0; c0 < RP; c0 += 32) {
           float v[32];
@@ -377,10 +380,28 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
           // columns >= r_g come from the next group's rank rows of the B^T box: zero them
           for (int q = 0; q < 16; ++q) v[q] = (live && c0 + q < rg) ? a.s * __uint_as_float(r[q]) : 0.f;
           if (MODE == MODE_SHARED) {
-            if (live) {
+            if (live && a.deterministic) {
               float4* dst = reinterpret_cast<float4*>(a.dHrow[proj] + row * RP + c0);
 #pragma unroll
               for (int q = 0; q < 4; ++q) dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+            } else if (live) {
+              // dHx[t][proj * n_rank_pad + r0 + k] += dH_row[k], k < r_g
+              uint16_t* dst = a.dHx + (int64_t)tok_s[i * kTileM + m] * (a.nproj * a.n_rank_pad) +
+                              proj * a.n_rank_pad + r0 + c0;
+#pragma unroll
+              for (int h8 = 0; h8 < 2; ++h8) {
+                const int k0 = c0 + h8 * 8;
+                if (((r0 & 7) == 0) && k0 + 8 <= rg) {
+                  red_add_bf16x8(dst + h8 * 8, pack8(v + h8 * 8));
+                } else {
+#pragma unroll
+                  for (int q = 0; q < 8; ++q)
+                    if (k0 + q < rg) {
+                      const __nv_bfloat16 b = __float2bfloat16_rn(v[h8 * 8 + q]);
+                      red_add_bf16(dst + h8 * 8 + q, *reinterpret_cast<const uint16_t*>(&b));
+                    }
+                }
+              }
             }
           } else {
             sts128(sOps + SL::elem(i, m, c0), pack8(v));
@@ -579,7 +600,8 @@ cudaError_t launch_bwd_t(const PlanTables& pt, const BwdLaunch& a, bool shared, 
     if ((e = launch_rows<RP, MODE_DOWN>(pt, a, 1, st)) != cudaSuccess) return e;
   } else {
     if ((e = launch_rows<RP, MODE_SHARED>(pt, a, nproj, st)) != cudaSuccess) return e;
-    if ((e = launch_k(k_dh_reduce<RP>, dim3(a.max_tiles_sh * (RP / 8), nproj), 128, 0, st, pt, a)) != cudaSuccess)
+    if (a.deterministic &&
+        (e = launch_k(k_dh_reduce<RP>, dim3(a.max_tiles_sh * (RP / 8), nproj), 128, 0, st, pt, a)) != cudaSuccess)
       return e;
   }
   if (a.deterministic) {

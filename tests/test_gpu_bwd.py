@@ -84,7 +84,9 @@ def _row_case(L, deterministic, with_base=False):
 
 
 CASES = [("tiny", 0, {}), ("tiny", 1, {"T": 300}), ("olmoe", 0, {"T": 1024}), ("qwen", 0, {"T": 1024}),
-         ("deepseek_g16", 0, {"T": 1024})]
+         ("deepseek_g16", 0, {"T": 1024}),
+         # r_g = 12: rank offsets that are not multiples of 8 (unaligned dH_u columns)
+         ("tiny", 4, {"r": 3})]
 
 
 @pytest.mark.parametrize("det", [True, False])

@@ -117,7 +117,7 @@ def _fwd_shared_case(L, s, with_base, nproj=2):
 
 @pytest.mark.parametrize("name,seed,over", [("tiny", 0, {}), ("tiny", 1, {"T": 300}), ("olmoe", 0, {"T": 1024}),
                                             ("olmoe", 2, {"T": 4096}), ("qwen", 0, {"T": 1024}),
-                                            ("deepseek_g16", 0, {"T": 1024})])
+                                            ("deepseek_g16", 0, {"T": 1024}), ("tiny", 4, {"r": 3})])
 def test_fwd_shared_parity(name, seed, over):
     L = W.Layer(W.get_config(name, **over), seed=seed)
     _fwd_shared_case(L, L.cfg.s, with_base=False)
@@ -160,7 +160,7 @@ def _fwd_row_case(L, s, with_base):
 @pytest.mark.parametrize("name,seed,over,base", [("tiny", 0, {}, False), ("tiny", 5, {"T": 77}, True),
                                                  ("olmoe", 0, {"T": 512}, False), ("olmoe", 2, {"T": 4096}, True),
                                                  ("qwen", 1, {"T": 512}, False),
-                                                 ("deepseek_g16", 0, {"T": 512}, True)])
+                                                 ("deepseek_g16", 0, {"T": 512}, True), ("tiny", 4, {"r": 3}, False)])
 def test_fwd_row_parity(name, seed, over, base):
     L = W.Layer(W.get_config(name, **over), seed=seed)
     _fwd_row_case(L, L.cfg.s, with_base=base)

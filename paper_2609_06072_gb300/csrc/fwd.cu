@@ -203,33 +203,31 @@ __device__ __forceinline__ uint32_t rows_bytes(int cnt) {
 }
 
 // Tile queue: the producer takes row tiles from a global counter (so faster
-// SMs take more tiles) and hands each tile index to the MMA warp and the
-// epilogue warps through a small ring in shared memory; -1 ends.
+// SMs take more tiles), skips the ones this kernel does not run, and hands
+// each live tile index to the MMA warp and the epilogue warps through a small
+// ring in shared memory; -1 ends.
 struct TileQueue {
   int32_t item[kQ];
   uint64_t full[kQ], empty[kQ];
 };
-// Consumer side: the next non-empty tile (false at the end or if a wait gave
-// up; *ok tells which).  Every lane of a warp calls it; lane 0 releases the
-// entries it reads.
+// Consumer side: the next tile (false at the end or if a wait gave up; *ok
+// tells which).  Every lane of a warp calls it; lane 0 releases the entry.
 __device__ __forceinline__ bool queue_next(TileQueue& tq, int& q, const Tile* tiles, Tile& t, bool single_lane,
-                                           bool* ok, bool whole) {
-  while (true) {
-    const int e = q % kQ;
-    bool w = mbar_wait(&tq.full[e], (q / kQ) & 1);
-    if (!single_lane) w = __all_sync(0xffffffffu, w);
-    if (!w) {
-      *ok = false;
-      return false;
-    }
-    const int item = *reinterpret_cast<volatile int32_t*>(&tq.item[e]);
-    if (!single_lane) __syncwarp();
-    if (single_lane || (threadIdx.x & 31) == 0) mbar_arrive(&tq.empty[e]);
-    ++q;
-    if (item < 0) return false;
-    t = tiles[item];
-    if (tile_live(t, whole)) return true;
+                                           bool* ok) {
+  const int e = q % kQ;
+  bool w = mbar_wait(&tq.full[e], (q / kQ) & 1);
+  if (!single_lane) w = __all_sync(0xffffffffu, w);
+  if (!w) {
+    *ok = false;
+    return false;
   }
+  const int item = *reinterpret_cast<volatile int32_t*>(&tq.item[e]);
+  if (!single_lane) __syncwarp();
+  if (single_lane || (threadIdx.x & 31) == 0) mbar_arrive(&tq.empty[e]);
+  ++q;
+  if (item < 0) return false;
+  t = tiles[item];
+  return true;
 }
 // Persistent: one CTA per SM; tiles of <= 128 consecutive rows of one group
 // are taken dynamically.  The producer, the MMA issuer and the epilogue run
@@ -300,23 +298,27 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
 #pragma unroll
       for (int k = 0; k < S; ++k) last[k] = nK[k] = nC[k] = 0;
       int i = 0, q = 0;
-      // grab tiles until a non-empty one or the end, handing each index on
+      // take tiles until one this kernel runs, or the end; hand it on
       auto grab = [&](Tile& t) -> bool {
+        int item;
         while (true) {
-          const int e = q % kQ;
-          if (q >= kQ && !mbar_wait(&tq.empty[e], ((q - kQ) / kQ) & 1)) {
-            bad = true;
-            return false;
+          item = atomicAdd(a.sched + kSchedFwdRows, 1);
+          if (item >= n_items) {
+            item = -1;
+            break;
           }
-          int item = atomicAdd(a.sched + kSchedFwdRows, 1);
-          if (item >= n_items) item = -1;
-          tq.item[e] = item;
-          mbar_arrive(&tq.full[e]);
-          ++q;
-          if (item < 0) return false;
           t = a.tiles[item];
-          if (tile_live(t, !SHARED)) return true;
+          if (tile_live(t, !SHARED)) break;
         }
+        const int e = q % kQ;
+        if (q >= kQ && !mbar_wait(&tq.empty[e], ((q - kQ) / kQ) & 1)) {
+          bad = true;
+          return false;
+        }
+        tq.item[e] = item;
+        mbar_arrive(&tq.full[e]);
+        ++q;
+        return item >= 0;
       };
       auto acquire = [&](bool kstep) -> uint32_t {  // next ring slot, once its last user released it
         const int s = i % S;
@@ -415,11 +417,11 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
       };
       Tile cur, nxt;
       bool qok = true;
-      bool has_cur = queue_next(tq, q, a.tiles, cur, true, &qok, !SHARED);
+      bool has_cur = queue_next(tq, q, a.tiles, cur, true, &qok);
       if (has_cur && !SHARED)
         for (int k = 0; k < NK && !bad; ++k) mma_k(0, k);
       while (has_cur && !bad) {
-        const bool has_nxt = queue_next(tq, q, a.tiles, nxt, true, &qok, !SHARED);
+        const bool has_nxt = queue_next(tq, q, a.tiles, nxt, true, &qok);
         const int lo = chunk_lo(cur, nch, !SHARED), hi = chunk_hi(cur, nch, !SHARED);
         for (int c = lo; c < hi && !bad; ++c) mma_c(c == lo, c == hi - 1);
         if (!SHARED && has_nxt)
@@ -509,10 +511,10 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
     int q = 0, ib = SHARED ? 0 : NK, cc0 = 0, ti = 0;
     bool ok = true;
     Tile cur, nxt;
-    bool has_cur = queue_next(tq, q, a.tiles, cur, false, &ok, !SHARED);
+    bool has_cur = queue_next(tq, q, a.tiles, cur, false, &ok);
     if (has_cur) ok = prepare_h(cur, 0);
     while (has_cur && ok) {
-      const bool has_nxt = queue_next(tq, q, a.tiles, nxt, false, &ok, !SHARED);
+      const bool has_nxt = queue_next(tq, q, a.tiles, nxt, false, &ok);
       if (!ok) break;
       const bool inter = !SHARED && has_nxt;
       // gate/up with two H buffers: gather the next tile's H now, while this tile streams

@@ -27,7 +27,9 @@ constexpr int kHalfBlk = 64 * 128;    // [64 rows x 64 bf16]
 
 // ------------------------------------------------------------------ dX
 // Persistent: one CTA per SM walks the [128-token x 256-column] output tiles
-// (column-fastest, so concurrent CTAs share dHx rows in L2).  Two TMEM
+// (column-fastest, so concurrent CTAs share dHx rows in L2); the tiles left
+// over after the last whole round go out as column halves, so that round
+// takes half as long and reaches twice as many SMs.  Two TMEM
 // accumulators let the epilogue of one tile overlap the K loop of the next.
 // Each epilogue warp owns 32 rows x 128 columns: it reads the old dX of its
 // block with coalesced loads into its own swizzled shared-memory block (while
@@ -40,6 +42,23 @@ constexpr int kDxWarpBlk = 32 * 256;                    // [32 rows x 128 bf16] 
 constexpr int kDxSmem = kDxS * kDxStage + 8 * kDxWarpBlk + 1024;
 // byte offset of 16-byte chunk c (0..15) of row r (0..31) in a warp block
 __device__ __forceinline__ uint32_t dx_off(int r, int c) { return (uint32_t)(r * 256 + ((c ^ (r & 15)) << 4)); }
+
+// Work item `it` of this CTA: a whole tile (half = -1) for the first
+// ntile / grid rounds, then one column half of a left-over tile.  False past
+// the end.
+__device__ __forceinline__ bool dx_item(int it, int ntile, int& tile, int& half) {
+  const int grid = gridDim.x, full = ntile / grid, rem = ntile % grid;
+  if (it < full) {
+    tile = it * grid + blockIdx.x;
+    half = -1;
+    return true;
+  }
+  const int h = (it - full) * grid + blockIdx.x;
+  if (h >= 2 * rem) return false;
+  tile = full * grid + h / 2;
+  half = h & 1;
+  return true;
+}
 
 __global__ void __launch_bounds__(kThreads, 1) k_gemm_dx(const __grid_constant__ DenseBwdLaunch a) {
   extern __shared__ uint8_t smem_raw[];
@@ -72,9 +91,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemm_dx(const __grid_constant__
   bool bad = false;
   if (warp == 0) {
     if (lane == 0) {
-      int i = 0;
-      for (int tile = blockIdx.x; tile < ntile && !bad; tile += gridDim.x) {
-        const int t0 = (tile / ncol) * 128, c0 = (tile % ncol) * kDxN;
+      int i = 0, tile, half;
+      for (int it = 0; dx_item(it, ntile, tile, half) && !bad; ++it) {
+        const int t0 = (tile / ncol) * 128, c0 = (tile % ncol) * kDxN + (half > 0 ? kDxN / 2 : 0);
+        const int nq = half < 0 ? kDxN / 64 : kDxN / 128;  // 64-column boxes of A
         for (int kb = 0; kb < NK; ++kb, ++i) {
           const int s = i % kDxS, u = i / kDxS;
           if (u >= 1 && !mbar_wait(&empty[s], (u - 1) & 1)) {
@@ -83,9 +103,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemm_dx(const __grid_constant__
           }
           const int j = kb / ksteps, ks = kb % ksteps;
           const uint32_t base = s0 + s * kDxStage;
-          mbar_arrive_expect_tx(&full[s], kDxStage);
+          mbar_arrive_expect_tx(&full[s], kBlk + nq * kHalfBlk);
           tma_load_2d(base, &a.tm_dhx, j * a.n_rank_pad + ks * 64, t0, &full[s]);
-          for (int q = 0; q < kDxN / 64; ++q)
+          for (int q = 0; q < nq; ++q)
             tma_load_2d(base + kBlk + q * kHalfBlk, &a.tm_acat[j], c0 + q * 64, ks * 64, &full[s]);
         }
       }
@@ -96,9 +116,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemm_dx(const __grid_constant__
   } else if (warp == 1) {
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(128, kDxN, 0, 1);
-      int i = 0, it = 0;
-      for (int tile = blockIdx.x; tile < ntile && !bad; tile += gridDim.x, ++it) {
+      constexpr uint32_t idesc_half = idesc_bf16_f32(128, kDxN / 2, 0, 1);
+      int i = 0, tile, half;
+      for (int it = 0; dx_item(it, ntile, tile, half) && !bad; ++it) {
         const int b = it & 1;
+        const uint32_t id = half < 0 ? idesc : idesc_half;
         if (it >= 2 && !mbar_wait(&acc_empty[b], ((it - 2) >> 1) & 1)) {
           bad = true;
           break;
@@ -115,7 +137,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemm_dx(const __grid_constant__
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk)
             tc_mma_bf16(tmem + b * kDxN, sdesc_sw128(base + kk * 32, 16, 1024),
-                        sdesc_sw128(base + kBlk + kk * 2048, kHalfBlk, 1024), idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+                        sdesc_sw128(base + kBlk + kk * 2048, kHalfBlk, 1024), id, (kb > 0 || kk > 0) ? 1u : 0u);
           tc_commit(&empty[s]);
         }
         if (!bad) tc_commit(&acc_full[b]);
@@ -125,11 +147,24 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemm_dx(const __grid_constant__
     const int quarter = warp & 3, ehalf = (warp - 2) >> 2;  // this warp: 32 rows x 128 columns
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
     const uint32_t wb = s0 + kDxS * kDxStage + (warp - 2) * kDxWarpBlk;
-    int it = 0;
-    for (int tile = blockIdx.x; tile < ntile; tile += gridDim.x, ++it) {
+    int tile, half;
+    for (int it = 0; dx_item(it, ntile, tile, half); ++it) {
       const int b = it & 1;
       const int tq = (tile / ncol) * 128 + quarter * 32;  // first token of this warp's rows
-      const int cb = (tile % ncol) * kDxN + ehalf * 128;  // first column of this warp's block
+      // first column of this warp's block; of a half tile only the ehalf 0
+      // warps have one (the accumulator's first 128 columns)
+      const int cb = (tile % ncol) * kDxN + (half < 0 ? ehalf : half) * 128;
+      const bool idle = half >= 0 && ehalf == 1;
+      if (idle) {
+        if (!__all_sync(0xffffffffu, mbar_wait(&acc_full[b], (it >> 1) & 1))) {
+          bad = true;
+          break;
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&acc_empty[b]);
+        continue;
+      }
       // old dX of the block: two 256-byte rows per instruction
 #pragma unroll
       for (int k2 = 0; k2 < 16; ++k2) {

@@ -31,17 +31,19 @@ constexpr int kHalfBlk = 64 * 128;    // [64 rows x 64 bf16]
 // over after the last whole round go out as column halves, so that round
 // takes half as long and reaches twice as many SMs.  Two TMEM
 // accumulators let the epilogue of one tile overlap the K loop of the next.
-// Each epilogue warp owns 32 rows x 128 columns: it reads the old dX of its
-// block with coalesced loads into its own swizzled shared-memory block (while
-// the K loop still runs), adds its accumulator rows there (thread = row) and
-// writes the block back with coalesced stores.
+// Each epilogue warp owns 32 rows x 128 columns, done in two passes of 64
+// columns through its own swizzled shared-memory block: the old dX is read
+// with coalesced loads (pass 0 into the block, pass 1 into registers, both
+// while the K loop still runs), the accumulator rows are added there (thread =
+// row) and the block is written back with coalesced stores.  (The small block
+// leaves room for four pipeline stages.)
 constexpr int kDxN = 256;                               // d columns per tile
 constexpr int kDxStage = kBlk + (kDxN / 64) * kHalfBlk; // dHx [128 t x 64 k] + A [64 k x 256 d]
-constexpr int kDxS = 3;
-constexpr int kDxWarpBlk = 32 * 256;                    // [32 rows x 128 bf16] per epilogue warp
+constexpr int kDxS = 4;
+constexpr int kDxWarpBlk = 32 * 128;                    // [32 rows x 64 bf16] per epilogue warp
 constexpr int kDxSmem = kDxS * kDxStage + 8 * kDxWarpBlk + 1024;
-// byte offset of 16-byte chunk c (0..15) of row r (0..31) in a warp block
-__device__ __forceinline__ uint32_t dx_off(int r, int c) { return (uint32_t)(r * 256 + ((c ^ (r & 15)) << 4)); }
+// byte offset of 16-byte chunk c (0..7) of row r (0..31) in a warp block
+__device__ __forceinline__ uint32_t dx_off(int r, int c) { return (uint32_t)(r * 128 + ((c ^ (r & 7)) << 4)); }
 
 // Work item `it` of this CTA: a whole tile (half = -1) for the first
 // ntile / grid rounds, then one column half of a left-over tile.  False past
@@ -165,12 +167,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemm_dx(const __grid_constant__
         if (lane == 0) mbar_arrive(&acc_empty[b]);
         continue;
       }
-      // old dX of the block: two 256-byte rows per instruction
+      // old dX of the block, four 128-byte rows per instruction: columns
+      // [0, 64) into the block, [64, 128) into registers
+      uint4 later[8];
 #pragma unroll
-      for (int k2 = 0; k2 < 16; ++k2) {
-        const int r = k2 * 2 + (lane >> 4), c = lane & 15, t = tq + r, col = cb + c * 8;
+      for (int k2 = 0; k2 < 8; ++k2) {
+        const int r = k2 * 4 + (lane >> 3), c = lane & 7, t = tq + r, col = cb + c * 8;
         const uint4 v = (t < a.T && col < a.d) ? *reinterpret_cast<const uint4*>(a.dX + (int64_t)t * a.d + col)
                                                : make_uint4(0, 0, 0, 0);
+        later[k2] = (t < a.T && col + 64 < a.d) ? *reinterpret_cast<const uint4*>(a.dX + (int64_t)t * a.d + col + 64)
+                                                : make_uint4(0, 0, 0, 0);
         sts128(wb + dx_off(r, c), v);
       }
       if (!__all_sync(0xffffffffu, mbar_wait(&acc_full[b], (it >> 1) & 1))) {
@@ -179,34 +185,47 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemm_dx(const __grid_constant__
       }
       tc_fence_after();
 #pragma unroll
-      for (int h = 0; h < 4; ++h) {  // 32-column groups of this warp's 128
-        uint32_t r[32];
-        const uint32_t ta = tmem + lane_base + b * kDxN + ehalf * 128 + h * 32;
-        tmem_ld16(ta, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
-        tmem_ld16(ta + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
-        tmem_ld_wait();
+      for (int pass = 0; pass < 2; ++pass) {
+        if (pass == 1) {
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const uint32_t addr = wb + dx_off(lane, h * 4 + q);
-          const uint4 y = lds128(addr);
-          const uint32_t* dq = &r[q * 8];
-          const float2 f0 = unpack_bf16x2(y.x), f1 = unpack_bf16x2(y.y), f2 = unpack_bf16x2(y.z),
-                       f3 = unpack_bf16x2(y.w);
-          uint4 o;
-          o.x = pack_bf16x2(f0.x + __uint_as_float(dq[0]), f0.y + __uint_as_float(dq[1]));
-          o.y = pack_bf16x2(f1.x + __uint_as_float(dq[2]), f1.y + __uint_as_float(dq[3]));
-          o.z = pack_bf16x2(f2.x + __uint_as_float(dq[4]), f2.y + __uint_as_float(dq[5]));
-          o.w = pack_bf16x2(f3.x + __uint_as_float(dq[6]), f3.y + __uint_as_float(dq[7]));
-          sts128(addr, o);
+          for (int k2 = 0; k2 < 8; ++k2) sts128(wb + dx_off(k2 * 4 + (lane >> 3), lane & 7), later[k2]);
+          __syncwarp();
         }
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&acc_empty[b]);
 #pragma unroll
-      for (int k2 = 0; k2 < 16; ++k2) {
-        const int r = k2 * 2 + (lane >> 4), c = lane & 15, t = tq + r, col = cb + c * 8;
-        if (t < a.T && col < a.d) *reinterpret_cast<uint4*>(a.dX + (int64_t)t * a.d + col) = lds128(wb + dx_off(r, c));
+        for (int h = 0; h < 2; ++h) {  // 32-column groups of the pass's 64
+          uint32_t r[32];
+          const uint32_t ta = tmem + lane_base + b * kDxN + ehalf * 128 + pass * 64 + h * 32;
+          tmem_ld16(ta, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
+          tmem_ld16(ta + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
+          tmem_ld_wait();
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const uint32_t addr = wb + dx_off(lane, h * 4 + q);
+            const uint4 y = lds128(addr);
+            const uint32_t* dq = &r[q * 8];
+            const float2 f0 = unpack_bf16x2(y.x), f1 = unpack_bf16x2(y.y), f2 = unpack_bf16x2(y.z),
+                         f3 = unpack_bf16x2(y.w);
+            uint4 o;
+            o.x = pack_bf16x2(f0.x + __uint_as_float(dq[0]), f0.y + __uint_as_float(dq[1]));
+            o.y = pack_bf16x2(f1.x + __uint_as_float(dq[2]), f1.y + __uint_as_float(dq[3]));
+            o.z = pack_bf16x2(f2.x + __uint_as_float(dq[4]), f2.y + __uint_as_float(dq[5]));
+            o.w = pack_bf16x2(f3.x + __uint_as_float(dq[6]), f3.y + __uint_as_float(dq[7]));
+            sts128(addr, o);
+          }
+        }
+        if (pass == 1) {  // the accumulator is read out
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&acc_empty[b]);
+        }
+        __syncwarp();
+#pragma unroll
+        for (int k2 = 0; k2 < 8; ++k2) {
+          const int r = k2 * 4 + (lane >> 3), c = lane & 7, t = tq + r, col = cb + pass * 64 + c * 8;
+          if (t < a.T && col < a.d)
+            *reinterpret_cast<uint4*>(a.dX + (int64_t)t * a.d + col) = lds128(wb + dx_off(r, c));
+        }
+        __syncwarp();
       }
       __syncwarp();
     }

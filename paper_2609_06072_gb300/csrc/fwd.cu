@@ -168,7 +168,9 @@ struct RowsFwdCfg {
   static constexpr int kBudget = 210 * 1024;
   static constexpr int NBH = 2 * kHs + 4 * kSlot <= kBudget ? 2 : 1;  // H operand buffers
   static constexpr int kS0 = (kBudget - NBH * kHs) / kSlot;
-  static constexpr int S = kS0 > 8 ? 8 : (kS0 < 2 ? 2 : kS0);
+  // ring slots: down keeps at most 6 (7 or 8 measured slower, 6 the fastest)
+  static constexpr int kSmax = SHARED ? 8 : 6;
+  static constexpr int S = kS0 > kSmax ? kSmax : (kS0 < 2 ? 2 : kS0);
   static constexpr int kSmem = NBH * kHs + S * kSlot + 1024;
   static constexpr int kHcol = RP <= 64 ? 64 : 128;         // down: TMEM columns of one H accumulator
   static constexpr uint32_t kDBase = SHARED ? 0u : 2u * kHcol;

@@ -54,7 +54,6 @@ __global__ void __launch_bounds__(kHThreads) k_fwd_h(const __grid_constant__ Pla
   __shared__ int32_t src_row[kTileM];
 
   pdl_wait();
-  pdl_trigger();
   const int n_tiles = a.counts[kCntTilesSh];
   if ((int)blockIdx.x >= n_tiles) return;
   const Tile tl = a.tiles[blockIdx.x];
@@ -149,6 +148,9 @@ __global__ void __launch_bounds__(kHThreads) k_fwd_h(const __grid_constant__ Pla
   if (aborted && tid == 0) atomicOr(a.err, kErrTimeout);
   tc_fence_before();
   __syncthreads();
+  // the row kernel that follows takes a whole SM per CTA: let it launch only
+  // as this grid's CTAs finish (an early launch measured slower)
+  pdl_trigger();
   if (warp == 0) tmem_dealloc(tmem, C::kTmem);
 }
 
@@ -623,10 +625,7 @@ cudaError_t launch_rows_t(const PlanTables& pt, const FwdRowsLaunch& a, cudaStre
   auto kern = k_fwd_rows<RP, NPROJ, SHARED>;
   cudaError_t e = set_smem(kern, C::kSmem);
   if (e != cudaSuccess || a.grid <= 0) return e;
-  // a plain launch: with programmatic serialization after k_fwd_h the gate/up
-  // call measured slower
-  kern<<<a.grid, kRowsThreads, C::kSmem, st>>>(pt, a);
-  return cudaGetLastError();
+  return launch_k(kern, a.grid, kRowsThreads, C::kSmem, st, pt, a);
 }
 
 }  // namespace

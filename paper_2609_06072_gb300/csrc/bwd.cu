@@ -148,7 +148,6 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
   static_assert(NT * RP <= 128, "dH accumulators must fit below the dB^T columns");
 
   pdl_wait();
-  pdl_trigger();
   const int n_splits = a.counts[kCntSplitsRow];
   if ((int)blockIdx.x >= n_splits) return;
   const int proj = blockIdx.y;
@@ -478,6 +477,9 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
   __syncwarp();
   tc_fence_before();
   if (__syncthreads_or(bad) && tid == 0) atomicOr(a.err, kErrTimeout);
+  // signal dependents only as this CTA finishes: an earlier launch of the
+  // next kernel (a whole SM per CTA) measured slower
+  pdl_trigger();
   if (warp == 0) tmem_dealloc(tmem, C::kTmem);
 }
 

@@ -286,7 +286,6 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
   tc_fence_after();
   const uint32_t tmem = tslot;
   pdl_wait();
-  pdl_trigger();
   const int n_items = a.counts[kCntTilesRow];
   const int d_in = a.d_in, d_out = a.d_out;
   const int NK = SHARED ? 0 : (d_in + 63) / 64;  // K steps of the down H GEMM
@@ -602,6 +601,9 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
       atomicExch(a.sched + kSchedFwdDone, 0);
     }
   }
+  // signal dependents only as this CTA finishes: an earlier launch of the
+  // next kernel (a whole SM per CTA) measured slower
+  pdl_trigger();
   if (warp == 0) tmem_dealloc(tmem, kRowsTmem);
 }
 

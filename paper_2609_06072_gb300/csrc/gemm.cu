@@ -88,7 +88,6 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemm_dx(const __grid_constant__
   __syncthreads();
   tc_fence_after();
   pdl_wait();
-  pdl_trigger();
   const uint32_t tmem = tslot;
   bool bad = false;
   if (warp == 0) {
@@ -233,6 +232,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemm_dx(const __grid_constant__
   __syncwarp();
   tc_fence_before();
   if (__syncthreads_or(bad) && tid == 0) atomicOr(a.err, kErrTimeout);
+  // signal dependents only as this CTA finishes: an earlier launch of the
+  // next kernel (a whole SM per CTA) measured slower
+  pdl_trigger();
   if (warp == 0) tmem_dealloc(tmem, 2 * kDxN);
 }
 
@@ -277,7 +279,6 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemm_da(const __grid_constant__
   __syncthreads();
   tc_fence_after();
   pdl_wait();
-  pdl_trigger();
   const uint32_t tmem = tslot;
   bool bad = false;
   if (warp == 0) {
@@ -355,6 +356,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemm_da(const __grid_constant__
   __syncwarp();
   tc_fence_before();
   if (__syncthreads_or(bad) && tid == 0) atomicOr(a.err, kErrTimeout);
+  // signal dependents only as this CTA finishes: an earlier launch of the
+  // next kernel (a whole SM per CTA) measured slower
+  pdl_trigger();
   if (warp == 0) tmem_dealloc(tmem, kDaN);
 }
 

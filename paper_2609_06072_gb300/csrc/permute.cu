@@ -260,8 +260,14 @@ __global__ void __launch_bounds__(kPermTB) k_perm_scatter(const __grid_constant_
   const int E = pt.E, G = pt.G;
   pdl_wait();
   pdl_trigger();
-  for (int i = tid; i < (E + G) * W; i += blockDim.x) msk[i] = 0;
   const int c = blockIdx.x;
+  const int t = c * kPermTB + tid;
+  const int k = pt.k;
+  // the token's expert ids, in flight while the offsets are computed
+  int e[KB];
+  bool ok = false;
+  if (c < (int)gridDim.x - 1 && t < T) ok = read_token<KB>(idx, t, k, E, e);
+  for (int i = tid; i < (E + G) * W; i += blockDim.x) msk[i] = 0;
   if (c < (int)gridDim.x - 1) {
     for (int i = tid; i < E; i += blockDim.x) {
       baseE[i] = chunk_baseE[(int64_t)c * E + i];
@@ -316,21 +322,14 @@ __global__ void __launch_bounds__(kPermTB) k_perm_scatter(const __grid_constant_
     if (tid == 0) o.counts[kCntSplitsRow] = n;
     return;
   }
-  const int t = c * kPermTB + tid;
-  const int k = pt.k;
-  int e[KB];
-  bool ok = false;
-  if (t < T) {
-    ok = read_token<KB>(idx, t, k, E, e);
-    if (ok) {
-      const uint32_t bit = 1u << (tid & 31);
+  if (ok) {
+    const uint32_t bit = 1u << (tid & 31);
 #pragma unroll
-      for (int j = 0; j < KB; ++j)
-        if (j < k) {
-          atomicOr(&mE[e[j] * W + (tid >> 5)], bit);
-          atomicOr(&mU[e2g[e[j]] * W + (tid >> 5)], bit);
-        }
-    }
+    for (int j = 0; j < KB; ++j)
+      if (j < k) {
+        atomicOr(&mE[e[j] * W + (tid >> 5)], bit);
+        atomicOr(&mU[e2g[e[j]] * W + (tid >> 5)], bit);
+      }
   }
   __syncthreads();
   if (t >= T) return;

@@ -320,9 +320,28 @@ CALLS = ["permute", "fwd_shared", "fwd_row", "bwd_row", "bwd_shared"]
 SINGLE_KERNEL = {"fwd_row": "k_fwd_rows<down>"}
 
 
+class L2Flush:
+    """Leaves L2 cold and clean between timed steps: a 256 MB write (evicts
+    the step's lines) followed by a 256 MB read (evicts the write's dirty
+    lines, so their write-back is not charged to the next timed step).  Both
+    run on the stream outside the event pair."""
+
+    def __init__(self):
+        import torch
+        n = 256 * 1024 * 1024  # each > L2 (~126 MB)
+        self.w = torch.empty(n, dtype=torch.uint8, device="cuda")
+        self.r = torch.ones(n // 4, dtype=torch.float32, device="cuda")
+        self.out = torch.empty((), dtype=torch.float32, device="cuda")
+
+    def __call__(self):
+        import torch
+        self.w.zero_()
+        torch.sum(self.r, dim=0, out=self.out)
+
+
 def time_steps(lay, steps, warmup, flush):
     """Mean step time (ms) of `steps` steps, events at step boundaries only;
-    flush: a buffer larger than L2 written before each step, or None."""
+    flush: an L2Flush run before each step, or None."""
     import torch
     for _ in range(warmup):
         lay.step()
@@ -331,7 +350,7 @@ def time_steps(lay, steps, warmup, flush):
            for _ in range(steps)]
     for e in evs:
         if flush is not None:
-            flush.zero_()
+            flush()
         lay.step(e)
     torch.cuda.synchronize()
     assert lay.plan.get_error(lay.perm) == 0
@@ -361,7 +380,7 @@ def run_gpu(args, rank, world, local):
     ace.load()
     lay = Layer(args.config, args.seed, args.expertwise, args.det)
     c = lay.c
-    flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device="cuda")  # > L2 (~126 MB)
+    flush = L2Flush()
     for _ in range(args.warmup):
         lay.step()
     torch.cuda.synchronize()
@@ -386,7 +405,7 @@ def run_gpu(args, rank, world, local):
     nv.start()
     t_wall0 = time.perf_counter()
     for i in range(args.steps):
-        flush.zero_()  # L2 flush between timed steps (outside the event pair)
+        flush()  # L2 flush between timed steps (outside the event pair)
         lay.step(evs[i])
     torch.cuda.synchronize()
     t_wall = time.perf_counter() - t_wall0
@@ -400,7 +419,7 @@ def run_gpu(args, rank, world, local):
     # events at every call boundary
     evs_b = [[new_ev() for _ in range(6)] for _ in range(args.steps)]
     for i in range(args.steps):
-        flush.zero_()
+        flush()
         lay.step(evs_b[i])
     torch.cuda.synchronize()
     per_call = {n: [e[j].elapsed_time(e[j + 1]) for e in evs_b] for j, n in enumerate(CALLS)}
@@ -456,7 +475,8 @@ def run_gpu(args, rank, world, local):
                    "T": c.T, "d": c.d, "f": c.f, "E": c.E, "k": c.k, "G": lay.L.G, "r": c.r,
                    "rank_g": int(np.max(np.diff(lay.L.rank_off))), "s": c.s, "routing": f"{c.routing}({c.alpha})",
                    "rows_per_step": c.R, "U": int(P["U"]), "deterministic": bool(args.det),
-                   "l2": "flushed between timed steps (256 MB write outside the event pair)",
+                   "l2": "flushed between timed steps (256 MB write, then 256 MB read so no dirty line "
+                         "is left; outside the event pair)",
                    "parallelism": f"replicas x{world}"},
         "roofline": {"bound": "hbm", "kernel": SINGLE_KERNEL[dom], "call": dom, "achieved": achieved,
                      "launch_ms": fwd_row_ms, "peak": peaks["hbm_gbs"],

@@ -339,6 +339,18 @@ class L2Flush:
         torch.sum(self.r, dim=0, out=self.out)
 
 
+def load_stats(expert_cnt, R, U):
+    """Realised routing of the step: rows per unique (token, group) pair and
+    the expert load spread (max / min rows, entropy of the load in bits and
+    its ratio to the uniform log2 E)."""
+    cnt = np.asarray(expert_cnt, dtype=np.float64)
+    p = cnt / max(1.0, cnt.sum())
+    nz = p[p > 0]
+    h = float(-(nz * np.log2(nz)).sum())
+    return {"R_over_U": R / max(1, U), "expert_rows_max": int(cnt.max()), "expert_rows_min": int(cnt.min()),
+            "load_entropy_bits": h, "load_entropy_ratio": float(h / np.log2(len(cnt))) if len(cnt) > 1 else 1.0}
+
+
 def time_steps(lay, steps, warmup, flush):
     """Mean step time (ms) of `steps` steps, events at step boundaries only;
     flush: an L2Flush run before each step, or None."""
@@ -474,7 +486,8 @@ def run_gpu(args, rank, world, local):
                                f"{' (expert-wise, matched budget)' if args.expertwise else ' (grouped)'}",
                    "T": c.T, "d": c.d, "f": c.f, "E": c.E, "k": c.k, "G": lay.L.G, "r": c.r,
                    "rank_g": int(np.max(np.diff(lay.L.rank_off))), "s": c.s, "routing": f"{c.routing}({c.alpha})",
-                   "rows_per_step": c.R, "U": int(P["U"]), "deterministic": bool(args.det),
+                   "rows_per_step": c.R, "U": int(P["U"]), **load_stats(P["expert_cnt"], c.R, int(P["U"])),
+                   "deterministic": bool(args.det),
                    "l2": "flushed between timed steps (256 MB write, then 256 MB read so no dirty line "
                          "is left; outside the event pair)",
                    "parallelism": f"replicas x{world}"},
@@ -572,6 +585,27 @@ def cpu_baseline(cfg_name, seed, expertwise, target_s):
             "sample": f"{what}; {dt:.1f} s", "seconds": dt}
 
 
+def oracle_single_thread(seed, expertwise):
+    """The oracle on one host core (a child process with OMP_NUM_THREADS=1):
+    whole steps of the tiny layer, and a ~3 s sample of the OLMoE-shaped one."""
+    code = ("import json, sys; sys.path.insert(0, %r); import bench\n"
+            "out = {}\n"
+            "t = r = 0.0; n = 0\n"
+            "while t < 1.0 and n < 100:\n"
+            "    dt, dr = bench.oracle_sample('tiny', %d, %r, 1.0, rng_seed=n); t += dt; r += dr; n += 1\n"
+            "out['tiny'] = {'value': r / t, 'sample': '%%d whole steps' %% n, 'seconds': t}\n"
+            "f = bench.calibrate_fraction('olmoe', %d, %r, 3.0)\n"
+            "t, r = bench.oracle_sample('olmoe', %d, %r, f)\n"
+            "out['olmoe'] = {'value': r / t, 'sample': 'permutation plus %%.5f of one step' %% f, 'seconds': t}\n"
+            "print(json.dumps(out))\n") % (ROOT, seed, expertwise, seed, expertwise, seed, expertwise)
+    env = dict(os.environ, OMP_NUM_THREADS="1")
+    r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True, timeout=300)
+    if r.returncode != 0:
+        return {"error": r.stderr.strip().splitlines()[-1] if r.stderr.strip() else "failed"}
+    res = json.loads(r.stdout.strip().splitlines()[-1])
+    return {"cores": 1, "unit": UNIT, **res}
+
+
 def run_reference(args, rank, world):
     if rank != 0:
         return None
@@ -635,6 +669,7 @@ def main():
     if rank == 0:
         if world == 1 and not args.no_cpu:
             out["cpu_baseline"] = cpu_baseline(args.config, args.seed, args.expertwise, args.cpu_seconds)
+            out["cpu_baseline"]["single_thread"] = oracle_single_thread(args.seed, args.expertwise)
         print(json.dumps(out))
     if world > 1:
         import torch.distributed as dist

@@ -6,8 +6,12 @@ both the CUDA path and the CPU oracle can consume exactly the same bytes.
 
 Shapes follow the paper's backbones (Tab. "model_configs": OLMoE-1B-7B
 d=2048/ff=1024/E=64/top-8, Qwen1.5-MoE d=2048/ff=1408/E=60/top-4, the
-Moonlight-style DeepSeek layer d=2048/ff=1408/E=64/top-6) plus a
-Mixtral-shaped layer and a tiny oracle-scale layer.  Nothing here comes from
+Moonlight-style DeepSeek layer d=2048/ff=1408/E=64/top-6, Kimi-Linear
+d=2304/ff=1024/E=256/top-8) plus a Mixtral-shaped layer and a tiny
+oracle-scale layer.  The "paperlike" grouping mimics the group statistics
+of the Louvain-resolution study (one large group of 43 experts, mid-size
+groups and unmerged singletons per 64 experts), at the paper's OLMoE rank
+r = 2, so r_g runs from 2 to 86.  Nothing here comes from
 any dataset; routing is synthetic:
 
 * router logits l_{t,e} = log w_e + Gumbel(0,1) (tiny layer: l ~ N(0,1)),
@@ -80,6 +84,9 @@ CONFIGS: Dict[str, LayerConfig] = {
     "deepseek_g32": LayerConfig("deepseek_g32", 16384, 2048, 1408, 64, 6, 8, "zipf", 1.2, "pairs"),
     "deepseek_g16": LayerConfig("deepseek_g16", 16384, 2048, 1408, 64, 6, 8, "zipf", 1.2, "uneven16"),
     "deepseek_g8": LayerConfig("deepseek_g8", 16384, 2048, 1408, 64, 6, 8, "zipf", 1.2, "all8"),
+    # paper-like uneven groups at r = 2: OLMoE-shaped, and a Kimi-Linear-shaped layer (many small segments)
+    "olmoe_uneven": LayerConfig("olmoe_uneven", 8192, 2048, 1024, 64, 8, 2, "zipf", 1.0, "paperlike"),
+    "kimi": LayerConfig("kimi", 8192, 2304, 1024, 256, 8, 2, "zipf", 1.0, "paperlike"),
 }
 
 
@@ -92,6 +99,8 @@ def get_config(name: str, **overrides) -> LayerConfig:
 # admissible size mixes (a, b, c) of groups of sizes 2, 4, 8 with 16 groups
 # covering 64 experts, the all-4 mix excluded
 _UNEVEN16_MIXES = [(2, 13, 1), (4, 10, 2), (6, 7, 3), (8, 4, 4), (10, 1, 5)]
+# group sizes per block of 64 experts for the "paperlike" grouping
+_PAPERLIKE64 = [43, 9, 5, 3, 1, 1, 1, 1]
 
 
 class Layer:
@@ -133,10 +142,14 @@ class Layer:
             return (np.arange(c.E) // 2).astype(np.int32), np.full(c.E // 2, 2, dtype=np.int64)
         if c.groups == "all8":
             return (np.arange(c.E) // 8).astype(np.int32), np.full(c.E // 8, 8, dtype=np.int64)
-        if c.groups == "uneven16":
+        if c.groups in ("uneven16", "paperlike"):
             rng = self._rng("groups")
-            a, b, cc = _UNEVEN16_MIXES[int(rng.integers(len(_UNEVEN16_MIXES)))]
-            sizes = np.array([2] * a + [4] * b + [8] * cc, dtype=np.int64)
+            if c.groups == "uneven16":
+                a, b, cc = _UNEVEN16_MIXES[int(rng.integers(len(_UNEVEN16_MIXES)))]
+                sizes = np.array([2] * a + [4] * b + [8] * cc, dtype=np.int64)
+            else:
+                assert c.E % 64 == 0
+                sizes = np.array(_PAPERLIKE64 * (c.E // 64), dtype=np.int64)
             rng.shuffle(sizes)
             perm = rng.permutation(c.E)
             e2g = np.empty(c.E, dtype=np.int32)

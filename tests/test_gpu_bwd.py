@@ -86,7 +86,9 @@ def _row_case(L, deterministic, with_base=False):
 CASES = [("tiny", 0, {}), ("tiny", 1, {"T": 300}), ("olmoe", 0, {"T": 1024}), ("qwen", 0, {"T": 1024}),
          ("deepseek_g16", 0, {"T": 1024}),
          # r_g = 12: rank offsets that are not multiples of 8 (unaligned dH_u columns)
-         ("tiny", 4, {"r": 3})]
+         ("tiny", 4, {"r": 3}),
+         # paper-like uneven groups, r_g from 2 to 86 (128-wide rank tiles), and E = 256
+         ("olmoe_uneven", 0, {"T": 512}), ("kimi", 0, {"T": 256})]
 
 
 @pytest.mark.parametrize("det", [True, False])

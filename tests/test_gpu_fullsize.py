@@ -81,6 +81,6 @@ def _full_case(name, seed):
         check_close(host_f64(dBt[p][ri]), rdBt, f"dBt_{p}[sampled]")
 
 
-@pytest.mark.parametrize("name", ["olmoe", "qwen", "deepseek_g16"])
+@pytest.mark.parametrize("name", ["olmoe", "qwen", "deepseek_g16", "olmoe_uneven", "kimi"])
 def test_full_size_sampled_parity(name):
     _full_case(name, 0)

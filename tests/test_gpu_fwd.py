@@ -41,7 +41,7 @@ def compare_perm(G_arr, O):
 
 PERM_CASES = [("tiny", 0, {}), ("tiny", 1, {}), ("olmoe", 0, {}), ("qwen", 0, {"T": 4096}),
               ("deepseek_g16", 0, {"T": 4096}), ("mixtral", 0, {"T": 2048}), ("tiny", 2, {"T": 1}),
-              ("tiny", 3, {"T": 300})]
+              ("tiny", 3, {"T": 300}), ("olmoe_uneven", 0, {"T": 2048}), ("kimi", 0, {"T": 1024})]
 
 
 @pytest.mark.parametrize("name,seed,over", PERM_CASES)
@@ -117,7 +117,8 @@ def _fwd_shared_case(L, s, with_base, nproj=2):
 
 @pytest.mark.parametrize("name,seed,over", [("tiny", 0, {}), ("tiny", 1, {"T": 300}), ("olmoe", 0, {"T": 1024}),
                                             ("olmoe", 2, {"T": 4096}), ("qwen", 0, {"T": 1024}),
-                                            ("deepseek_g16", 0, {"T": 1024}), ("tiny", 4, {"r": 3})])
+                                            ("deepseek_g16", 0, {"T": 1024}), ("tiny", 4, {"r": 3}),
+                                            ("olmoe_uneven", 0, {"T": 512}), ("kimi", 0, {"T": 256})])
 def test_fwd_shared_parity(name, seed, over):
     L = W.Layer(W.get_config(name, **over), seed=seed)
     _fwd_shared_case(L, L.cfg.s, with_base=False)
@@ -160,7 +161,8 @@ def _fwd_row_case(L, s, with_base):
 @pytest.mark.parametrize("name,seed,over,base", [("tiny", 0, {}, False), ("tiny", 5, {"T": 77}, True),
                                                  ("olmoe", 0, {"T": 512}, False), ("olmoe", 2, {"T": 4096}, True),
                                                  ("qwen", 1, {"T": 512}, False),
-                                                 ("deepseek_g16", 0, {"T": 512}, True), ("tiny", 4, {"r": 3}, False)])
+                                                 ("deepseek_g16", 0, {"T": 512}, True), ("tiny", 4, {"r": 3}, False),
+                                                 ("olmoe_uneven", 0, {"T": 512}, True), ("kimi", 0, {"T": 256}, False)])
 def test_fwd_row_parity(name, seed, over, base):
     L = W.Layer(W.get_config(name, **over), seed=seed)
     _fwd_row_case(L, L.cfg.s, with_base=base)

@@ -195,10 +195,15 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
   if (warp == 0) {
     // ------------------------------------------------------------ producer
     // the dY stream starts once the epilogue has sent out its H prefetches,
-    // so they are not queued behind it
+    // and runs two slots ahead until the H operand is staged, so the H loads
+    // are not queued behind a full ring of dY
     named_bar(kIssueBar, kEpiThreads + 32);
     if (lane == 0) {
       for (int q = 0; q < NI1 + NI2 && !bad; ++q) {
+        if (q == 2 && !mbar_wait(&ops_ready, 0)) {
+          bad = true;
+          break;
+        }
         const int s = q % SA, u = q / SA;
         if (u >= 1 && !mbar_wait(&emptyA[s], (u - 1) & 1)) {
           bad = true;

@@ -11,7 +11,7 @@
 //   k_perm_scatter per chunk: segment offsets from the totals (a warp scan in
 //                  (g, e) order), rank of each pair inside its expert
 //                  (bitmask popcounts over the chunk's earlier tokens) -> row;
-//                  one extra CTA writes the offsets and the tile tables
+//                  three extra CTAs write the offsets and the tile tables
 // Integer-only and order-independent, so bit-exact and deterministic.
 #include <algorithm>
 #include <cstdint>
@@ -223,6 +223,8 @@ __device__ __forceinline__ int prefix_bits(const uint32_t* mask, int tid) {
   return r + __popc(mask[w] & ((1u << (tid & 31)) - 1u));
 }
 
+constexpr int kTableCtas = 3;  // scatter CTAs that build the offsets and tile tables
+
 struct ScatterOut {
   int32_t* row_pair;
   int32_t* pair_row;
@@ -266,9 +268,10 @@ __global__ void __launch_bounds__(kPermTB) k_perm_scatter(const __grid_constant_
   // the token's expert ids, in flight while the offsets are computed
   int e[KB];
   bool ok = false;
-  if (c < (int)gridDim.x - 1 && t < T) ok = read_token<KB>(idx, t, k, E, e);
+  const int n_chunk_ctas = (int)gridDim.x - kTableCtas;
+  if (c < n_chunk_ctas && t < T) ok = read_token<KB>(idx, t, k, E, e);
   for (int i = tid; i < (E + G) * W; i += blockDim.x) msk[i] = 0;
-  if (c < (int)gridDim.x - 1) {
+  if (c < n_chunk_ctas) {
     for (int i = tid; i < E; i += blockDim.x) {
       baseE[i] = chunk_baseE[(int64_t)c * E + i];
       e2g[i] = pt.e2g[i];
@@ -298,28 +301,35 @@ __global__ void __launch_bounds__(kPermTB) k_perm_scatter(const __grid_constant_
   __syncthreads();
   for (int g = tid; g < G; g += blockDim.x) goff[g] = eoff[pt.eorder[pt.gfirst[g]]];
   __syncthreads();
-  if (blockIdx.x == gridDim.x - 1) {
-    // the last CTA, which owns no chunk: the offsets and the tile tables the
-    // other calls read (in parallel with the chunks' scatter)
+  if (c >= n_chunk_ctas) {
+    // the CTAs that own no chunk write, in parallel with the chunks' scatter,
+    // the offsets and the tile tables the other calls read: one table each
     __shared__ int32_t rows_g[ACE_MAX_EXPERTS];
     __shared__ int32_t scratch[ACE_MAX_EXPERTS + 1];
-    for (int g = tid; g <= G; g += blockDim.x) {
-      o.group_off[g] = goff[g];
-      o.uniq_off[g] = uoff[g];
-      if (g < G) rows_g[g] = goff[g + 1] - goff[g];
-    }
-    for (int e = tid; e < E; e += blockDim.x) o.expert_off[e] = eoff[e];
-    if (tid == 0) {
-      o.counts[kCntU] = uoff[G];
-      o.counts[kCntRows] = goff[G];
+    const int job = c - n_chunk_ctas;
+    for (int g = tid; g < G; g += blockDim.x) rows_g[g] = goff[g + 1] - goff[g];
+    if (job == 0) {
+      for (int g = tid; g <= G; g += blockDim.x) {
+        o.group_off[g] = goff[g];
+        o.uniq_off[g] = uoff[g];
+      }
+      for (int e = tid; e < E; e += blockDim.x) o.expert_off[e] = eoff[e];
+      if (tid == 0) {
+        o.counts[kCntU] = uoff[G];
+        o.counts[kCntRows] = goff[G];
+      }
     }
     __syncthreads();
-    int n = build_tiles(totU, uoff, G, kTileM, o.tiles_sh, scratch);
-    if (tid == 0) o.counts[kCntTilesSh] = n;
-    n = build_row_tiles(rows_g, goff, G, min(pt.nsm, 8 * (int)blockDim.x), o.tiles_row, scratch);
-    if (tid == 0) o.counts[kCntTilesRow] = n;
-    n = build_tiles(rows_g, goff, G, kTileM * pt.nt_split, o.splits_row, scratch);
-    if (tid == 0) o.counts[kCntSplitsRow] = n;
+    if (job == 0) {
+      const int n = build_tiles(totU, uoff, G, kTileM, o.tiles_sh, scratch);
+      if (tid == 0) o.counts[kCntTilesSh] = n;
+    } else if (job == 1) {
+      const int n = build_row_tiles(rows_g, goff, G, min(pt.nsm, 8 * (int)blockDim.x), o.tiles_row, scratch);
+      if (tid == 0) o.counts[kCntTilesRow] = n;
+    } else {
+      const int n = build_tiles(rows_g, goff, G, kTileM * pt.nt_split, o.splits_row, scratch);
+      if (tid == 0) o.counts[kCntSplitsRow] = n;
+    }
     return;
   }
   if (ok) {
@@ -429,8 +439,8 @@ cudaError_t launch_permute(const PlanTables& pt, const int32_t* topk_idx, int32_
   o.tiles_row = at<Tile>(ws, L.tiles_row);
   o.splits_row = at<Tile>(ws, L.splits_row);
   size_t sm3 = sizeof(uint32_t) * (size_t)(pt.E + pt.G) * (kPermTB / 32);
-  // one CTA per chunk, plus the one that writes the offsets and tables
-  return launch_k(pt.k <= 8 ? k_perm_scatter<8> : k_perm_scatter<kMaxK>, C + 1, kPermTB, sm3, st, pt, topk_idx, T, at<int32_t>(ws, L.chunk_baseE),
+  // one CTA per chunk, plus the ones that write the offsets and tables
+  return launch_k(pt.k <= 8 ? k_perm_scatter<8> : k_perm_scatter<kMaxK>, C + kTableCtas, kPermTB, sm3, st, pt, topk_idx, T, at<int32_t>(ws, L.chunk_baseE),
                   at<int32_t>(ws, L.chunk_baseU), at<int32_t>(ws, L.expert_cnt), at<int32_t>(ws, L.tot_u), o);
 }
 

@@ -63,7 +63,9 @@ inline PermLayout perm_layout(const PlanTables& pt, int32_t T) {
   L.n_chunks = (T + kPermTB - 1) / kPermTB;
   L.max_tiles = (int32_t)((R + kTileM - 1) / kTileM + pt.G);
   const int64_t split_rows = (int64_t)kTileM * pt.nt_split;
-  L.max_splits = (int32_t)((R + split_rows - 1) / split_rows + pt.G);
+  // pieces of split_rows rows, rounded up to whole waves of nsm CTAs
+  const int64_t min_splits = (R + split_rows - 1) / split_rows + pt.G;
+  L.max_splits = (int32_t)((min_splits + pt.nsm - 1) / pt.nsm * pt.nsm);
   size_t off = 0;
   auto take = [&](size_t bytes) {
     size_t o = off;

@@ -91,7 +91,7 @@ ace_status check_perm(const ace_plan* plan, const ace_perm* perm) {
   return ACE_OK;
 }
 
-int pt_nt_split(int rank_pad) { return rank_pad <= 32 ? 4 : rank_pad == 64 ? 2 : 1; }
+int pt_nt_split(int rank_pad) { return rank_pad <= 64 ? 4 : 1; }
 
 struct BwdWs {
   float* dHrow[2];

@@ -116,7 +116,7 @@ __device__ __forceinline__ void flush_wgrad(uint32_t taddr, int n0, int ld, int 
 // ----------------------------------------------------------------- k_bwd_rows
 template <int RP, int MODE>
 struct RowsCfg {
-  static constexpr int NT = RP <= 32 ? 4 : (RP == 64 ? 2 : 1);
+  static constexpr int NT = RP <= 64 ? 4 : 1;
   static constexpr int kOps = Slots<RP>::bytes(NT);
   static constexpr int kWBlk = RP * 128;
   static constexpr int kSlotA = 2 * kBlk + 2 * kWBlk;  // dY tile + B^T chunk (down phase 2: A chunk + h tile)
@@ -126,10 +126,12 @@ struct RowsCfg {
   static constexpr int kSA0 = (kBudget - kOps - SB * kSlotB) / kSlotA;
   static constexpr int SA = kSA0 > 6 ? 6 : (kSA0 < 2 ? 2 : kSA0);
   static constexpr int kSmem = kOps + SA * kSlotA + SB * kSlotB + 1024;
-  static constexpr int kTB = 128;  // dB^T (phase 1) / dA (phase 2) accumulators, 2 x RP columns
-  static constexpr int ND = RP > 64 ? 1 : 2;            // down: dh D buffers of 128 columns
-  static constexpr int kDB = RP > 64 ? 384 : 256;
-  static constexpr int kTmem = (MODE == MODE_DOWN || RP > 64) ? 512 : 256;
+  // dH accumulators of the split's tiles below kTB; dB^T (phase 1) / dA
+  // (phase 2) accumulators, 2 x RP columns, from kTB
+  static constexpr int kTB = NT * RP > 128 ? 256 : 128;
+  static constexpr int ND = (RP > 64 || kTB > 128) ? 1 : 2;  // down: dh D buffers of 128 columns
+  static constexpr int kDB = (RP > 64 || kTB > 128) ? 384 : 256;
+  static constexpr int kTmem = (MODE == MODE_DOWN || RP > 64 || kTB > 128) ? 512 : 256;
 };
 
 template <int RP, int MODE>
@@ -145,7 +147,7 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
   __shared__ __align__(8) uint64_t dh_full, hs_ready, ops_ready;
   __shared__ uint32_t tslot;
   __shared__ int32_t tok_s[MODE == MODE_SHARED ? NT * kTileM : 1];  // token of each row (gate/up)
-  static_assert(NT * RP <= 128, "dH accumulators must fit below the dB^T columns");
+  static_assert(NT * RP <= C::kTB, "dH accumulators must fit below the dB^T columns");
 
   pdl_wait();
   const int n_splits = a.counts[kCntSplitsRow];

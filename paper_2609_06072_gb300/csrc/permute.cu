@@ -158,6 +158,61 @@ __device__ int build_row_tiles(const int32_t* n_g, const int32_t* off_g, int G, 
   return n + ns;
 }
 
+// Sum of ceil(n_g / per) over the groups (every thread gets the total).
+__device__ int count_pieces(const int32_t* n_g, int G, int per, int32_t* red /* smem [32] */) {
+  int v = 0;
+  for (int g = threadIdx.x; g < G; g += blockDim.x) v += (n_g[g] + per - 1) / per;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+  __syncthreads();
+  int tot = 0;
+  for (int w = 0; w < (int)(blockDim.x + 31) / 32; ++w) tot += red[w];
+  return tot;
+}
+
+// Backward splits: every group's rows in near-equal pieces of at most `cap`
+// rows.  When pieces of `cap` rows leave the last wave of `nsm` CTAs less than
+// 90% full, the piece size shrinks so that the pieces fill whole waves:
+// per = ceil(R / (waves * nsm - G)) gives at most R / per + G <= waves * nsm
+// pieces.  Returns the number of splits.
+__device__ int build_splits(const int32_t* n_g, const int32_t* off_g, int G, int cap, int nsm,
+                            Tile* __restrict__ out, int32_t* scratch /* smem [G+1] */, int32_t* red) {
+  const int min_total = count_pieces(n_g, G, cap, red);
+  const int target = (min_total + nsm - 1) / nsm * nsm;
+  int per = cap;
+  if (min_total > 0 && 10 * (min_total - (target - nsm)) < 9 * nsm && target > G) {
+    int rows = 0;
+    for (int g = 0; g < G; ++g) rows += n_g[g];  // (every thread; G <= 512)
+    per = min(cap, max(1, (rows + target - G - 1) / (target - G)));
+  }
+  const int tid = threadIdx.x;
+  for (int g = tid; g < G; g += blockDim.x) scratch[g + 1] = (n_g[g] + per - 1) / per;
+  __syncthreads();
+  if (tid == 0) {
+    scratch[0] = 0;
+    for (int g = 0; g < G; ++g) scratch[g + 1] += scratch[g];
+  }
+  __syncthreads();
+  for (int g = tid; g < G; g += blockDim.x) {
+    const int n = n_g[g], base = scratch[g], np = scratch[g + 1] - base;
+    for (int i = 0; i < np; ++i) {
+      const int b0 = (int)((int64_t)i * n / np), b1 = (int)((int64_t)(i + 1) * n / np);
+      Tile tl;
+      tl.g = g;
+      tl.start = off_g[g] + b0;
+      tl.cnt = b1 - b0;
+      tl.id = base + i;
+      out[base + i] = tl;
+    }
+  }
+  __syncthreads();
+  const int total = scratch[G];
+  __syncthreads();
+  return total;
+}
+
 __device__ __forceinline__ int warp_incl_scan(int v) {
   const int lane = threadIdx.x & 31;
 #pragma unroll
@@ -327,7 +382,8 @@ __global__ void __launch_bounds__(kPermTB) k_perm_scatter(const __grid_constant_
       const int n = build_row_tiles(rows_g, goff, G, min(pt.nsm, 8 * (int)blockDim.x), o.tiles_row, scratch);
       if (tid == 0) o.counts[kCntTilesRow] = n;
     } else {
-      const int n = build_tiles(rows_g, goff, G, kTileM * pt.nt_split, o.splits_row, scratch);
+      __shared__ int32_t red[32];
+      const int n = build_splits(rows_g, goff, G, kTileM * pt.nt_split, pt.nsm, o.splits_row, scratch, red);
       if (tid == 0) o.counts[kCntSplitsRow] = n;
     }
     return;

@@ -146,6 +146,20 @@ struct FwdHLaunch {
 };
 cudaError_t launch_fwd_h(const PlanTables& pt, const FwdHLaunch& a, cudaStream_t st);
 
+// Token-major H of the gate/up forward (gemm.cu): the same H_u as
+// launch_fwd_h, from 128-token blocks of X read once by TMA.
+constexpr int kDenseHMaxRank = 512;  // stacked ranks of a projection up to which H is token-major
+struct DenseHLaunch {
+  CUtensorMap tm_x;         // X [T, d], box 64 x 128
+  CUtensorMap tm_a[2];      // A_j [n_rank, d], box 64 x 256
+  const int32_t* tok_uniq;  // [T, k]: the token's unique pairs, ascending g, -1 padded
+  const int32_t* uniq_off;  // [G + 1]
+  float* H[2];              // [U, rank_max] fp32, row u (columns past r_g written as 0)
+  int32_t T, d, n_rank, nproj, rank_max, grid;
+  int32_t* err;
+};
+cudaError_t launch_dense_h(const PlanTables& pt, const DenseHLaunch& a, cudaStream_t st);
+
 // Row-tile forward: Y[row] += s * B_g H_row over contiguous rows of a group.
 // MODE down: H_row = A_g h_row computed here (K loop over h);  gate/up:
 // H_row = H_u gathered from the unique-pair H of launch_fwd_h.

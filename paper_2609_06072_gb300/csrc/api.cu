@@ -278,7 +278,29 @@ static ace_status fwd_common(const ace_plan* plan, const ace_perm* perm, const u
     for (int j = 0; j < nproj; ++j)
       if (!Hbuf[j]) Hbuf[j] = reinterpret_cast<float*>(static_cast<char*>(ws) + j * align_up(4 * (size_t)R * pt.rank_max, 256));
   }
-  if (shared) {
+  // H_u of gate/up: token-major dense tiles when the stacked ranks of a
+  // projection are few (the MMA then also forms the products of the groups a
+  // token skips, cheaper than gathering X once per active group), else
+  // gathered per unique pair
+  const bool dense_h = shared && n_rank <= kDenseHMaxRank;
+  if (dense_h) {
+    DenseHLaunch h{};
+    bool okh = make_tmap_bf16(&h.tm_x, X, (uint64_t)perm->T, (uint64_t)d_in, kTileM);
+    for (int j = 0; j < nproj; ++j) okh = okh && make_tmap_bf16(&h.tm_a[j], A[j], (uint64_t)n_rank, (uint64_t)d_in, 256);
+    if (!okh) return fail(ACE_ERR_UNSUPPORTED, "tensor-map encoding failed for this layout");
+    h.tok_uniq = perm->tok_uniq;
+    h.uniq_off = perm->uniq_off;
+    for (int j = 0; j < 2; ++j) h.H[j] = Hbuf[j < nproj ? j : 0];
+    h.T = perm->T;
+    h.d = d_in;
+    h.n_rank = n_rank;
+    h.nproj = nproj;
+    h.rank_max = pt.rank_max;
+    h.grid = plan->num_sms;
+    h.err = err;
+    st = cuda_status(launch_dense_h(pt, h, cs), "forward H launch");
+    if (st != ACE_OK) return st;
+  } else if (shared) {
     FwdHLaunch h{};
     h.tiles = at<Tile>(perm->ws, L.tiles_sh);
     h.counts = perm->counts;

@@ -362,7 +362,185 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemm_da(const __grid_constant__
   if (warp == 0) tmem_dealloc(tmem, kDaN);
 }
 
+// ------------------------------------------------------------------ H
+// Token-major H of the gate/up forward: H_u = A_g x_t for every active pair
+// u = (g, t) (Sec. 3.5), for a block of 128 consecutive tokens against 256
+// stacked rank rows of A_j at a time.  X is read once per token block by TMA
+// instead of once per active group of each token, and the MMA also forms the
+// products of the groups a token does not route to, which the epilogue drops:
+// each H_u is still computed once and written once, into the same
+// per-unique-pair layout as the gathering kernel of fwd.cu.  Persistent over
+// [128-token x 256-rank] tiles (rank blocks fastest, so concurrent CTAs share
+// the X block in L2), two TMEM accumulators, four 48 KB stages.
+constexpr int kHN = 256;                                // rank rows per tile
+constexpr int kHStageB = kBlk + (kHN / 64) * kHalfBlk;  // X [128 t x 64 d] + A [256 r x 64 d]
+constexpr int kHS = 4;
+constexpr int kHSmem = kHS * kHStageB + 1024;
+
+// Largest i with off[i] <= v over off[0..n] (off ascending, off[0] <= v).
+__device__ __forceinline__ int upper_idx(const int32_t* off, int n, int v) {
+  int lo = 0, hi = n;
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (off[mid] <= v)
+      lo = mid;
+    else
+      hi = mid;
+  }
+  return lo;
+}
+
+template <int KB>
+__global__ void __launch_bounds__(kThreads, 1) k_gemm_h(const __grid_constant__ PlanTables pt,
+                                                        const __grid_constant__ DenseHLaunch a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  __shared__ __align__(8) uint64_t full[kHS], empty[kHS], acc_full[2], acc_empty[2];
+  __shared__ uint32_t tslot;
+  __shared__ int32_t uoff_s[ACE_MAX_EXPERTS + 1], roff_s[ACE_MAX_EXPERTS + 1];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int G = pt.G, k = pt.k;
+  const int ncb = (a.n_rank + kHN - 1) / kHN, nper = a.nproj * ncb;
+  const int ntile = ((a.T + 127) / 128) * nper;
+  const int NK = (a.d + 63) / 64;
+  const uint32_t s0 = smem_u32(smem);
+  if (tid == 0) {
+    for (int i = 0; i < kHS; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&acc_full[i], 1);
+      mbar_init(&acc_empty[i], 8);  // every epilogue warp
+    }
+    fence_mbar_init();
+  }
+  if (warp == 0) tmem_alloc(&tslot, 2 * kHN);
+  for (int i = tid; i <= G; i += blockDim.x) roff_s[i] = pt.rank_off[i];
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  pdl_wait();
+  for (int i = tid; i <= G; i += blockDim.x) uoff_s[i] = a.uniq_off[i];
+  __syncthreads();
+  const uint32_t tmem = tslot;
+  bool bad = false;
+  if (warp == 0) {
+    if (lane == 0) {
+      int i = 0;
+      for (int tile = blockIdx.x; tile < ntile && !bad; tile += gridDim.x) {
+        const int t0 = (tile / nper) * 128, j = (tile % nper) / ncb, r0 = (tile % ncb) * kHN;
+        for (int kb = 0; kb < NK; ++kb, ++i) {
+          const int s = i % kHS, u = i / kHS;
+          if (u >= 1 && !mbar_wait(&empty[s], (u - 1) & 1)) {
+            bad = true;
+            break;
+          }
+          const uint32_t base = s0 + s * kHStageB;
+          mbar_arrive_expect_tx(&full[s], kHStageB);
+          tma_load_2d(base, &a.tm_x, kb * 64, t0, &full[s]);
+          tma_load_2d(base + kBlk, &a.tm_a[j], kb * 64, r0, &full[s]);
+        }
+      }
+      // every copy issued has landed before the CTA can exit
+      for (int k2 = max(0, i - kHS); k2 < i; ++k2)
+        if (!mbar_wait(&full[k2 % kHS], (k2 / kHS) & 1)) bad = true;
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(128, kHN, 0, 0);
+      int i = 0, it = 0;
+      for (int tile = blockIdx.x; tile < ntile && !bad; tile += gridDim.x, ++it) {
+        const int b = it & 1;
+        if (it >= 2 && !mbar_wait(&acc_empty[b], ((it - 2) >> 1) & 1)) {
+          bad = true;
+          break;
+        }
+        tc_fence_after();
+        for (int kb = 0; kb < NK; ++kb, ++i) {
+          const int s = i % kHS;
+          if (!mbar_wait(&full[s], (i / kHS) & 1)) {
+            bad = true;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t base = s0 + s * kHStageB;
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            tc_mma_bf16(tmem + b * kHN, sdesc_sw128(base + kk * 32, 16, 1024),
+                        sdesc_sw128(base + kBlk + kk * 32, 16, 1024), idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+          tc_commit(&empty[s]);
+        }
+        if (!bad) tc_commit(&acc_full[b]);
+      }
+    }
+  } else {
+    // this warp: TMEM lane quarter `quarter` (32 tokens) x 128 of the tile's 256 rank columns
+    const int quarter = warp & 3, ehalf = (warp - 2) >> 2;
+    const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
+    int it = 0;
+    for (int tile = blockIdx.x; tile < ntile; tile += gridDim.x, ++it) {
+      const int b = it & 1;
+      const int t = (tile / nper) * 128 + quarter * 32 + lane, j = (tile % nper) / ncb;
+      const int c_lo = (tile % ncb) * kHN + ehalf * 128;  // first rank column of this warp
+      // this token's active pairs and their groups (ascending g)
+      int uu[KB], gu[KB];
+#pragma unroll
+      for (int n = 0; n < KB; ++n) {
+        uu[n] = (t < a.T && n < k) ? a.tok_uniq[(int64_t)t * k + n] : -1;
+        gu[n] = uu[n] >= 0 ? upper_idx(uoff_s, G, uu[n]) : -1;
+      }
+      if (!__all_sync(0xffffffffu, mbar_wait(&acc_full[b], (it >> 1) & 1))) {
+        bad = true;
+        break;
+      }
+      tc_fence_after();
+      float* __restrict__ Hj = a.H[j];
+      for (int c16 = 0; c16 < 8; ++c16) {
+        const int c = c_lo + c16 * 16;
+        if (c >= a.n_rank) break;  // warp-uniform
+        uint32_t r[16];
+        tmem_ld16(tmem + lane_base + b * kHN + ehalf * 128 + c16 * 16, r);
+        tmem_ld_wait();
+        // the groups whose rank rows meet columns [c, c + 16)
+        const int g_lo = upper_idx(roff_s, G, c), g_hi = upper_idx(roff_s, G, min(c + 15, a.n_rank - 1));
+        for (int gg = g_lo; gg <= g_hi; ++gg) {
+          int u = -1;
+#pragma unroll
+          for (int n = 0; n < KB; ++n)
+            if (gu[n] == gg) u = uu[n];
+          if (u < 0) continue;
+          const int off = roff_s[gg], end = roff_s[gg + 1];
+          float* hrow = Hj + (int64_t)u * a.rank_max - off;
+#pragma unroll
+          for (int q = 0; q < 16; ++q)
+            if (c + q >= off && c + q < end) hrow[c + q] = __uint_as_float(r[q]);
+          if (end <= c + 16)  // the group ends here: zero its row's columns past r_g
+            for (int q = end - off; q < a.rank_max; ++q) hrow[off + q] = 0.f;
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&acc_empty[b]);
+    }
+  }
+  __syncwarp();
+  tc_fence_before();
+  if (__syncthreads_or(bad) && tid == 0) atomicOr(a.err, kErrTimeout);
+  pdl_trigger();
+  if (warp == 0) tmem_dealloc(tmem, 2 * kHN);
+}
+
 }  // namespace
+
+cudaError_t launch_dense_h(const PlanTables& pt, const DenseHLaunch& a, cudaStream_t st) {
+  if (a.T == 0) return cudaSuccess;
+  auto kern = pt.k <= 8 ? k_gemm_h<8> : k_gemm_h<kMaxK>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kHSmem);
+  if (e != cudaSuccess) return e;
+  const int tiles = ((a.T + 127) / 128) * a.nproj * ((a.n_rank + kHN - 1) / kHN);
+  return launch_k(kern, std::min(tiles, a.grid), kThreads, kHSmem, st, pt, a);
+}
 
 cudaError_t launch_dense_bwd(const DenseBwdLaunch& a, cudaStream_t st) {
   if (a.T == 0) return cudaSuccess;

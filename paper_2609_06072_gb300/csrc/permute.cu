@@ -102,8 +102,23 @@ __global__ void __launch_bounds__(kPermTB) k_perm_count(const __grid_constant__ 
   if (tid == 0) chunk_err[c] = err_s;
 }
 
+// Group whose pieces [pre[g], pre[g + 1]) contain piece i (pre ascending, G + 1 entries).
+__device__ __forceinline__ int piece_group(const int32_t* pre, int G, int i) {
+  int lo = 0, hi = G;
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (pre[mid] <= i)
+      lo = mid;
+    else
+      hi = mid;
+  }
+  return lo;
+}
+
 // Writes the tiles of every group: group g has ceil(n_g / per) tiles of at
-// most `per` items; returns the total (thread 0's view after the call).
+// most `per` items; returns the total (thread 0's view after the call).  The
+// threads share the tiles (not the groups), so a large group costs no more
+// than many small ones.
 __device__ int build_tiles(const int32_t* n_g, const int32_t* off_g, int G, int per, Tile* __restrict__ out,
                            int32_t* scratch /* smem [G+1] */) {
   const int tid = threadIdx.x;
@@ -114,16 +129,14 @@ __device__ int build_tiles(const int32_t* n_g, const int32_t* off_g, int G, int 
     for (int g = 0; g < G; ++g) scratch[g + 1] += scratch[g];
   }
   __syncthreads();
-  for (int g = tid; g < G; g += blockDim.x) {
-    int n = n_g[g], base = scratch[g];
-    for (int i = 0; i * per < n; ++i) {
-      Tile tl;
-      tl.g = g;
-      tl.start = off_g[g] + i * per;
-      tl.cnt = min(per, n - i * per);
-      tl.id = base + i;
-      out[base + i] = tl;
-    }
+  for (int p = tid; p < scratch[G]; p += blockDim.x) {
+    const int g = piece_group(scratch, G, p), i = p - scratch[g], n = n_g[g];
+    Tile tl;
+    tl.g = g;
+    tl.start = off_g[g] + i * per;
+    tl.cnt = min(per, n - i * per);
+    tl.id = p;
+    out[p] = tl;
   }
   __syncthreads();
   int total = scratch[G];
@@ -195,17 +208,15 @@ __device__ int build_splits(const int32_t* n_g, const int32_t* off_g, int G, int
     for (int g = 0; g < G; ++g) scratch[g + 1] += scratch[g];
   }
   __syncthreads();
-  for (int g = tid; g < G; g += blockDim.x) {
-    const int n = n_g[g], base = scratch[g], np = scratch[g + 1] - base;
-    for (int i = 0; i < np; ++i) {
-      const int b0 = (int)((int64_t)i * n / np), b1 = (int)((int64_t)(i + 1) * n / np);
-      Tile tl;
-      tl.g = g;
-      tl.start = off_g[g] + b0;
-      tl.cnt = b1 - b0;
-      tl.id = base + i;
-      out[base + i] = tl;
-    }
+  for (int p = tid; p < scratch[G]; p += blockDim.x) {
+    const int g = piece_group(scratch, G, p), i = p - scratch[g], n = n_g[g], np = scratch[g + 1] - scratch[g];
+    const int b0 = (int)((int64_t)i * n / np), b1 = (int)((int64_t)(i + 1) * n / np);
+    Tile tl;
+    tl.g = g;
+    tl.start = off_g[g] + b0;
+    tl.cnt = b1 - b0;
+    tl.id = p;
+    out[p] = tl;
   }
   __syncthreads();
   const int total = scratch[G];

@@ -50,6 +50,7 @@ struct PermLayout {
 
 // counts[] slots
 constexpr int kCntU = 0, kCntRows = 1, kCntTilesSh = 2, kCntTilesRow = 3, kCntSplitsRow = 4;
+constexpr int kCntRowSplit = 5;  // index of the first split (column-half) entry of the row tiles
 // sched[] slots: work counter and finished-CTA counter of the dynamically
 // scheduled forward row kernel; the permutation zeroes them and the last CTA
 // of every launch resets them, so each launch starts from zero
@@ -74,7 +75,7 @@ inline PermLayout perm_layout(const PlanTables& pt, int32_t T) {
   };
   L.err = take(4 * 8);
   L.counts = take(4 * 8);
-  L.sched = take(4 * 8);
+  L.sched = take(4 * (8 + (size_t)pt.nsm));  // 8 counters, then one H-ready flag per split row tile
   L.group_off = take(4 * (size_t)(pt.G + 1));
   L.expert_off = take(4 * (size_t)pt.E);
   L.expert_cnt = take(4 * (size_t)pt.E);
@@ -178,6 +179,8 @@ struct FwdRowsLaunch {
   const float* Hu[2];    // gate/up: H per unique pair
   uint16_t* Y[2];
   float* Hsave;          // down: H per row out (may be null)
+  float* Hpre;           // down: where the split row tiles' H is computed first (Hsave or scratch), or null
+  int32_t pre;           // down: split row tiles take their H from Hpre (computed up front), not a K loop
   float s;
   int32_t d_in, d_out, nproj;
   int32_t* err;

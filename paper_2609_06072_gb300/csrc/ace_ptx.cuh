@@ -143,6 +143,14 @@ __device__ __forceinline__ void red_add_bf16(void* p, uint16_t h) {
   asm volatile("red.global.add.noftz.bf16 [%0], %1;" ::"l"(p), "h"(h) : "memory");
 }
 
+// Load with acquire semantics at gpu scope (pairs with a writer's fence +
+// atomic).
+__device__ __forceinline__ int ld_acquire(const int32_t* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
 // Hint: bring the 128-byte line holding p into L2.
 __device__ __forceinline__ void prefetch_l2(const void* p) {
   asm volatile("prefetch.global.L2 [%0];" ::"l"(p));

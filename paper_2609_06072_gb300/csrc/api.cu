@@ -342,6 +342,13 @@ static ace_status fwd_common(const ace_plan* plan, const ace_perm* perm, const u
     r.Y[j] = Y[jj];
   }
   r.Hsave = shared ? nullptr : (H ? H[0] : nullptr);
+  if (!shared) {
+    // the split row tiles' H is computed up front into the saved H, or into
+    // the forward workspace when H is not saved (else they run whole)
+    r.Hpre = r.Hsave;
+    if (!r.Hpre && ws && aligned16(ws) && ws_bytes >= 4 * (size_t)R * pt.rank_max) r.Hpre = static_cast<float*>(ws);
+    r.pre = r.Hpre != nullptr;
+  }
   r.s = s;
   r.d_in = d_in;
   r.d_out = d_out;

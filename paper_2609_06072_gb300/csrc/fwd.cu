@@ -191,17 +191,25 @@ __device__ __forceinline__ void load_rows(uint32_t dst, const CUtensorMap* m128,
   const int nb = (cnt + kQuant - 1) / kQuant;
   for (int b = 0; b < nb; ++b) tma_load_2d(dst + b * kQuant * 128, m16, x, y + b * kQuant, bar);
 }
-// Output chunks [lo, hi) of a row tile (its id names all, or one half of, the
-// columns).  `whole` (down): a split tile is done whole under its first half's
-// entry and its second half's entry is skipped -- cutting it would make both
-// halves repeat the tile's K loop, which measured slower.
-__device__ __forceinline__ bool tile_live(const Tile& t, bool whole) { return t.cnt > 0 && !(whole && t.id == 2); }
+// Output chunks [lo, hi) of a row tile: id 0 names all columns; split b has
+// ids 1 + 2b (first half) and 2 + 2b (second half).  `whole` (down without an
+// up-front H): a split tile is done whole under its first half's entry and its
+// second half's entry is skipped -- cutting it would make both halves repeat
+// the tile's K loop.
+__device__ __forceinline__ int split_half(const Tile& t) { return (t.id - 1) & 1; }
+__device__ __forceinline__ int split_index(const Tile& t) { return (t.id - 1) >> 1; }
+__device__ __forceinline__ bool tile_live(const Tile& t, bool whole) {
+  return t.cnt > 0 && !(whole && t.id > 0 && split_half(t) == 1);
+}
 __device__ __forceinline__ int chunk_lo(const Tile& t, int nch, bool whole) {
-  return !whole && t.id == 2 ? (nch + 1) / 2 : 0;
+  return !whole && t.id > 0 && split_half(t) == 1 ? (nch + 1) / 2 : 0;
 }
 __device__ __forceinline__ int chunk_hi(const Tile& t, int nch, bool whole) {
-  return !whole && t.id == 1 ? (nch + 1) / 2 : nch;
+  return !whole && t.id > 0 && split_half(t) == 0 ? (nch + 1) / 2 : nch;
 }
+// Up-front H of the split row tiles (down): ready once every epilogue warp of
+// the CTA that computed it has added 1.
+constexpr int kPreWriters = 4 * 4;
 __device__ __forceinline__ uint32_t rows_bytes(int cnt) {
   return cnt == kTileM ? (uint32_t)kBlk : (uint32_t)((cnt + kQuant - 1) / kQuant) * kQuant * 128;
 }
@@ -287,6 +295,17 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
   const uint32_t tmem = tslot;
   pdl_wait();
   const int n_items = a.counts[kCntTilesRow];
+  // down with an up-front H: CTA b first computes the H of split row tile b
+  // (K loop only) into Hpre; the split tiles' column halves then read it
+  // instead of repeating the K loop, so the last work comes in halves
+  const bool pre = !SHARED && a.pre != 0;
+  const bool whole = !SHARED && !pre;
+  const int split0 = a.counts[kCntRowSplit], n_split = (n_items - split0) / 2;
+  const bool has_pre = pre && (int)blockIdx.x < n_split;
+  Tile pre_t{};
+  if (has_pre) pre_t = a.tiles[split0 + 2 * (int)blockIdx.x];
+  int32_t* const hflag = a.sched + 8;
+  auto needs_k = [&](const Tile& t) { return !SHARED && !(pre && t.id > 0); };
   const int d_in = a.d_in, d_out = a.d_out;
   const int NK = SHARED ? 0 : (d_in + 63) / 64;  // K steps of the down H GEMM
   const int nch = (d_out + kChunk - 1) / kChunk;
@@ -311,7 +330,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
             break;
           }
           t = a.tiles[item];
-          if (tile_live(t, !SHARED)) break;
+          if (tile_live(t, whole)) break;
         }
         const int e = q % kQ;
         if (q >= kQ && !mbar_wait(&tq.empty[e], ((q - kQ) / kQ) & 1)) {
@@ -355,13 +374,15 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
         ++i;
       };
       Tile cur, nxt;
+      if (has_pre)
+        for (int k = 0; k < NK && !bad; ++k) load_k(pre_t, k);
       bool has_cur = grab(cur);
-      if (has_cur && !SHARED)
+      if (has_cur && needs_k(cur))
         for (int k = 0; k < NK && !bad; ++k) load_k(cur, k);
       while (has_cur && !bad) {
         const bool has_nxt = grab(nxt);
-        for (int c = chunk_lo(cur, nch, !SHARED); c < chunk_hi(cur, nch, !SHARED) && !bad; ++c) load_c(cur, c);
-        if (!SHARED && has_nxt)
+        for (int c = chunk_lo(cur, nch, whole); c < chunk_hi(cur, nch, whole) && !bad; ++c) load_c(cur, c);
+        if (has_nxt && needs_k(nxt))
           for (int k = 0; k < NK && !bad; ++k) load_k(nxt, k);
         cur = nxt;
         has_cur = has_nxt;
@@ -375,7 +396,9 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
     if (lane == 0) {
       constexpr uint32_t idesc_h = idesc_bf16_f32(128, RP, 0, 0);
       constexpr uint32_t idesc_d = idesc_bf16_f32(128, kChunk, 0, 1);
-      int i = 0, cc = 0, ti = 0, q = 0;
+      // ci counts the tiles with D chunks (H operand buffers, hs_ready / hs_free),
+      // kc the tiles with a K loop (H accumulators, hacc)
+      int i = 0, cc = 0, ci = 0, kc = 0, q = 0;
       auto mma_k = [&](int hb, int k) {  // K step k of the tile whose H accumulator is hb
         const int s = i % S;
         if (!mbar_wait(&full[s], (i / S) & 1)) {
@@ -392,9 +415,9 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
         if (k == NK - 1) tc_commit(&hacc[hb]);
         ++i;
       };
-      auto mma_c = [&](bool first, bool last) {  // a D chunk of tile ti
+      auto mma_c = [&](bool first, bool last) {  // a D chunk of chunk-tile ci
         const int s = i % S, b = cc % kNGrp;
-        if ((first && !mbar_wait(&hs_ready[ti & 1], (ti >> 1) & 1)) ||
+        if ((first && !mbar_wait(&hs_ready[ci & 1], (ci >> 1) & 1)) ||
             (cc >= kNGrp && !mbar_wait(&dempty[b], ((cc - kNGrp) / kNGrp) & 1)) ||
             !mbar_wait(&full[s], (i / S) & 1)) {
           bad = true;
@@ -402,7 +425,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
         }
         tc_fence_after();
         const uint32_t base = slot0 + s * C::kSlot;
-        const uint32_t sHs = sHs0 + (ti % NBH) * C::kHs;
+        const uint32_t sHs = sHs0 + (ci % NBH) * C::kHs;
 #pragma unroll
         for (int j = 0; j < NPROJ; ++j)
 #pragma unroll
@@ -414,28 +437,37 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
                         kk > 0 ? 1u : 0u);
           }
         tc_commit(&dfull[b]);
-        if (last) tc_commit(&hs_free[ti % NBH]);
+        if (last) tc_commit(&hs_free[ci % NBH]);
         ++cc;
         ++i;
       };
       Tile cur, nxt;
       bool qok = true;
+      if (has_pre) {
+        for (int k = 0; k < NK && !bad; ++k) mma_k(kc & 1, k);
+        ++kc;
+      }
       bool has_cur = queue_next(tq, q, a.tiles, cur, true, &qok);
-      if (has_cur && !SHARED)
-        for (int k = 0; k < NK && !bad; ++k) mma_k(0, k);
+      if (has_cur && needs_k(cur)) {
+        for (int k = 0; k < NK && !bad; ++k) mma_k(kc & 1, k);
+        ++kc;
+      }
       while (has_cur && !bad) {
         const bool has_nxt = queue_next(tq, q, a.tiles, nxt, true, &qok);
-        const int lo = chunk_lo(cur, nch, !SHARED), hi = chunk_hi(cur, nch, !SHARED);
+        const int lo = chunk_lo(cur, nch, whole), hi = chunk_hi(cur, nch, whole);
         for (int c = lo; c < hi && !bad; ++c) mma_c(c == lo, c == hi - 1);
-        if (!SHARED && has_nxt)
-          for (int k = 0; k < NK && !bad; ++k) mma_k((ti + 1) & 1, k);
-        ++ti;
+        ++ci;
+        if (has_nxt && needs_k(nxt)) {
+          for (int k = 0; k < NK && !bad; ++k) mma_k(kc & 1, k);
+          ++kc;
+        }
         cur = nxt;
         has_cur = has_nxt;
       }
       if (!qok) bad = true;
-      // the last commit must land before the CTA exits
-      if (!bad && ti > 0 && !mbar_wait(&hs_free[(ti - 1) % NBH], ((ti - 1) / NBH) & 1)) bad = true;
+      // the last commits must land before the CTA exits
+      if (!bad && ci > 0 && !mbar_wait(&hs_free[(ci - 1) % NBH], ((ci - 1) / NBH) & 1)) bad = true;
+      if (!bad && kc > 0 && ci == 0 && !mbar_wait(&hacc[(kc - 1) & 1], ((kc - 1) >> 1) & 1)) bad = true;
     }
   } else {
     // ------------------------------------------------------------ epilogue
@@ -444,18 +476,18 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
     const int m = quarter * 32 + lane;      // tile row owned by this thread
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
     const float s = a.s;
-    // H operand of tile t (tile number tn) into buffer tn % NBH: this warp's
-    // rows, its group's share of the columns
-    auto stage_h = [&](const Tile& t, int tn) {
-      const uint32_t sHs = sHs0 + (tn % NBH) * C::kHs;
+    // H operand of chunk-tile ci (tile t, K-tile kt or -1) into buffer
+    // ci % NBH: this warp's rows, its group's share of the columns
+    auto stage_h = [&](const Tile& t, int ci, int kt) {
+      const uint32_t sHs = sHs0 + (ci % NBH) * C::kHs;
       if (quarter * 32 >= t.cnt) return;  // no live row: these H rows feed only D rows nobody reads
       const bool live = m < t.cnt;
       const int rg = pt.rank_off[t.g + 1] - pt.rank_off[t.g];
-      if (!SHARED) {
+      if (!SHARED && kt >= 0) {
         tc_fence_after();
         for (int c0 = grp * 16; c0 < RP; c0 += 16 * kNGrp) {
           uint32_t r[16];
-          tmem_ld16(tmem + lane_base + (tn & 1) * C::kHcol + c0, r);
+          tmem_ld16(tmem + lane_base + (kt & 1) * C::kHcol + c0, r);
           tmem_ld_wait();
           float v[16];
 #pragma unroll
@@ -478,10 +510,11 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
           }
         }
       } else {
-        const int u = live ? a.row_uniq[t.start + m] : -1;
+        // gate/up: H of the row's unique pair; down split tile: its up-front H row
+        const int u = live ? (SHARED ? a.row_uniq[t.start + m] : t.start + m) : -1;
 #pragma unroll
         for (int j = 0; j < NPROJ; ++j) {
-          const float* hp = a.Hu[j] + (int64_t)(u < 0 ? 0 : u) * pt.rank_max;
+          const float* hp = (SHARED ? a.Hu[j] : a.Hpre) + (int64_t)(u < 0 ? 0 : u) * pt.rank_max;
           for (int c8 = grp * 8; c8 < RP; c8 += 8 * kNGrp) {
             float v[8];
 #pragma unroll
@@ -497,34 +530,85 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
         }
       }
     };
-    // H of tile tn (tile t): wait until the buffer's previous tile is done
-    // with it and (down) tn's K loop has completed, stage, publish
-    auto prepare_h = [&](const Tile& t, int tn) -> bool {
+    // H of chunk-tile ci (tile t; kt: its K-tile number, -1 without a K
+    // loop): wait until the buffer's previous tile is done with it and the H
+    // exists (down: the K loop, or the up-front H of a split tile), stage,
+    // publish
+    auto prepare_h = [&](const Tile& t, int ci, int kt) -> bool {
       bool w = true;
-      if (tn >= NBH) w = mbar_wait(&hs_free[tn % NBH], ((tn - NBH) / NBH) & 1);
-      if (!SHARED) w = w && mbar_wait(&hacc[tn & 1], (tn >> 1) & 1);
+      if (ci >= NBH) w = mbar_wait(&hs_free[ci % NBH], ((ci - NBH) / NBH) & 1);
+      if (kt >= 0) w = w && mbar_wait(&hacc[kt & 1], (kt >> 1) & 1);
+      if (!SHARED && kt < 0) {  // split tile: wait for its up-front H
+        bool w2 = true;
+        if (lane == 0) {
+          const uint64_t t0 = globaltimer_ns();
+          while (ld_acquire(hflag + split_index(t)) < kPreWriters)
+            if (globaltimer_ns() - t0 > kWaitLimitNs) {
+              w2 = false;
+              break;
+            }
+        }
+        w = w && __shfl_sync(0xffffffffu, w2, 0);
+        if (w) (void)ld_acquire(hflag + split_index(t));  // every lane's H loads follow an acquire
+      }
       if (!__all_sync(0xffffffffu, w)) return false;
-      stage_h(t, tn);
+      stage_h(t, ci, kt);
       fence_proxy_async_smem();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&hs_ready[tn & 1]);
+      if (lane == 0) mbar_arrive(&hs_ready[ci & 1]);
       return true;
     };
-    int q = 0, ib = SHARED ? 0 : NK, cc0 = 0, ti = 0;
+    // the up-front H of split tile blockIdx.x: this warp's rows and columns
+    // into Hpre, then count this warp in the tile's flag
+    auto drain_pre = [&](const Tile& t, int kt) -> bool {
+      if (!__all_sync(0xffffffffu, mbar_wait(&hacc[kt & 1], (kt >> 1) & 1))) return false;
+      tc_fence_after();
+      const bool live = m < t.cnt;
+      const int rg = pt.rank_off[t.g + 1] - pt.rank_off[t.g];
+      for (int c0 = grp * 16; c0 < RP; c0 += 16 * kNGrp) {
+        uint32_t r[16];
+        tmem_ld16(tmem + lane_base + (kt & 1) * C::kHcol + c0, r);
+        tmem_ld_wait();
+        if (live) {
+          float* hrow = a.Hpre + (int64_t)(t.start + m) * pt.rank_max;
+#pragma unroll
+          for (int qq = 0; qq < 16; ++qq)
+            if (c0 + qq < pt.rank_max) hrow[c0 + qq] = c0 + qq < rg ? __uint_as_float(r[qq]) : 0.f;
+        }
+      }
+      tc_fence_before();
+      __threadfence();
+      __syncwarp();
+      if (lane == 0) atomicAdd(hflag + blockIdx.x, 1);
+      return true;
+    };
+    int q = 0, ib = 0, cc0 = 0, ci = 0, kc = 0;
     bool ok = true;
     Tile cur, nxt;
-    bool has_cur = queue_next(tq, q, a.tiles, cur, false, &ok);
-    if (has_cur) ok = prepare_h(cur, 0);
+    if (has_pre) {
+      ok = drain_pre(pre_t, kc);
+      ++kc;
+      ib += NK;
+    }
+    bool has_cur = ok && queue_next(tq, q, a.tiles, cur, false, &ok);
+    if (has_cur) {
+      int kt = -1;
+      if (needs_k(cur)) {
+        kt = kc++;
+        ib += NK;
+      }
+      ok = prepare_h(cur, ci, kt);
+    }
     while (has_cur && ok) {
       const bool has_nxt = queue_next(tq, q, a.tiles, nxt, false, &ok);
       if (!ok) break;
-      const bool inter = !SHARED && has_nxt;
+      const bool inter = has_nxt && needs_k(nxt);
       // gate/up with two H buffers: gather the next tile's H now, while this tile streams
       const bool early = SHARED && NBH == 2 && has_nxt;
-      if (early && !(ok = prepare_h(nxt, ti + 1))) break;
+      if (early && !(ok = prepare_h(nxt, ci + 1, -1))) break;
       const bool qlive = quarter * 32 < cur.cnt;  // this warp has live rows (warp-uniform)
-      const int lo = chunk_lo(cur, nch, !SHARED), hi = chunk_hi(cur, nch, !SHARED);
+      const int lo = chunk_lo(cur, nch, whole), hi = chunk_hi(cur, nch, whole);
       for (int c = lo + ((grp - cc0) % kNGrp + kNGrp) % kNGrp; c < hi; c += kNGrp) {
         const int cc = cc0 + (c - lo), i = ib + (c - lo);
         const int sl = i % S, b = cc % kNGrp, n0 = c * kChunk;
@@ -580,10 +664,10 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
         if (lane == 0) mbar_arrive(&emptyC[sl]);
       }
       if (!ok) break;
-      if (has_nxt && !early && !(ok = prepare_h(nxt, ti + 1))) break;
+      if (has_nxt && !early && !(ok = prepare_h(nxt, ci + 1, inter ? kc++ : -1))) break;
       ib += (hi - lo) + (inter ? NK : 0);
       cc0 += hi - lo;
-      ++ti;
+      ++ci;
       cur = nxt;
       has_cur = has_nxt;
     }
@@ -592,14 +676,21 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
   __syncwarp();  // reconverge the single-lane roles before the CTA barrier
   tc_fence_before();
   if (__syncthreads_or(bad) && tid == 0) atomicOr(a.err, kErrTimeout);
+  __shared__ int last_cta;
   if (tid == 0) {
     // the last CTA to finish (every producer has taken its final index) resets
-    // the counters for the next launch
+    // the counters (and the H-ready flags) for the next launch
     __threadfence();
-    if (atomicAdd(a.sched + kSchedFwdDone, 1) == (int)gridDim.x - 1) {
+    last_cta = atomicAdd(a.sched + kSchedFwdDone, 1) == (int)gridDim.x - 1;
+    if (last_cta) {
       atomicExch(a.sched + kSchedFwdRows, 0);
       atomicExch(a.sched + kSchedFwdDone, 0);
     }
+  }
+  if (pre) {
+    __syncthreads();
+    if (last_cta)
+      for (int b = tid; b < n_split; b += blockDim.x) hflag[b] = 0;
   }
   // signal dependents only as this CTA finishes: an earlier launch of the
   // next kernel (a whole SM per CTA) measured slower

@@ -146,12 +146,14 @@ __device__ int build_tiles(const int32_t* n_g, const int32_t* off_g, int G, int 
 
 // Forward row tiles in dispatch order: every group's rows in tiles of 128
 // (id 0: all output columns), except that each of the last `tail` tiles of the
-// list becomes two entries covering one half of the columns each (ids 1, 2),
-// so the work left when SMs run dry comes in halves.
+// list (split b) becomes two entries covering one half of the columns each
+// (ids 1 + 2b and 2 + 2b), so the work left when SMs run dry comes in halves.
+// *split_first receives the index of the first split entry.
 __device__ int build_row_tiles(const int32_t* n_g, const int32_t* off_g, int G, int tail, Tile* __restrict__ out,
-                               int32_t* scratch /* smem [G+1] */) {
+                               int32_t* scratch /* smem [G+1] */, int32_t* split_first) {
   const int n = build_tiles(n_g, off_g, G, kTileM, out, scratch);
   const int ns = min(n, tail), first = n - ns;
+  if (threadIdx.x == 0) split_first[0] = first;
   for (int j = threadIdx.x; j < first; j += blockDim.x) out[j].id = 0;
   // read the tiles to split before any of them is overwritten
   Tile mine[8];
@@ -162,9 +164,9 @@ __device__ int build_row_tiles(const int32_t* n_g, const int32_t* off_g, int G, 
   for (int j = first + (int)threadIdx.x; j < n && cnt < 8; j += blockDim.x) {
     Tile t = mine[cnt++];
     const int k = first + 2 * (j - first);
-    t.id = 1;
+    t.id = 1 + 2 * (j - first);  // split b = j - first: ids 1 + 2b (first half), 2 + 2b (second half)
     out[k] = t;
-    t.id = 2;
+    t.id = 2 + 2 * (j - first);
     out[k + 1] = t;
   }
   __syncthreads();
@@ -273,7 +275,7 @@ __global__ void __launch_bounds__(256) k_perm_colscan(const __grid_constant__ Pl
   }
   if (tid == 0) (isE ? totE : totU)[col] = carry;
   if (blockIdx.x == 0) {
-    if (tid < 8) sched[tid] = 0;  // work counters of the row kernels start at zero
+    for (int i = tid; i < 8 + pt.nsm; i += blockDim.x) sched[i] = 0;  // row-kernel counters and flags start at zero
     int e = 0;
     for (int c = tid; c < n_chunks; c += 256) e |= chunk_err[c];
     if (e) atomicOr(&err_s, e);
@@ -390,7 +392,8 @@ __global__ void __launch_bounds__(kPermTB) k_perm_scatter(const __grid_constant_
       const int n = build_tiles(totU, uoff, G, kTileM, o.tiles_sh, scratch);
       if (tid == 0) o.counts[kCntTilesSh] = n;
     } else if (job == 1) {
-      const int n = build_row_tiles(rows_g, goff, G, min(pt.nsm, 8 * (int)blockDim.x), o.tiles_row, scratch);
+      const int n = build_row_tiles(rows_g, goff, G, min(pt.nsm, 8 * (int)blockDim.x), o.tiles_row, scratch,
+                                    o.counts + kCntRowSplit);
       if (tid == 0) o.counts[kCntTilesRow] = n;
     } else {
       __shared__ int32_t red[32];

@@ -50,7 +50,8 @@ struct PermLayout {
 
 // counts[] slots
 constexpr int kCntU = 0, kCntRows = 1, kCntTilesSh = 2, kCntTilesRow = 3, kCntSplitsRow = 4;
-constexpr int kCntRowSplit = 5;  // index of the first split (column-half) entry of the row tiles
+constexpr int kCntRowSplit = 5;  // index of the first split entry of the row tiles
+constexpr int kSplitParts = 4;   // column parts of each split row tile (the last wave's tiles)
 // sched[] slots: work counter and finished-CTA counter of the dynamically
 // scheduled forward row kernel; the permutation zeroes them and the last CTA
 // of every launch resets them, so each launch starts from zero
@@ -93,7 +94,7 @@ inline PermLayout perm_layout(const PlanTables& pt, int32_t T) {
   L.chunk_baseU = take(4 * (size_t)L.n_chunks * pt.G);
   L.chunk_err = take(4 * (size_t)(L.n_chunks + 1));
   L.tiles_sh = take(sizeof(Tile) * (size_t)L.max_tiles);
-  L.tiles_row = take(sizeof(Tile) * (size_t)(L.max_tiles + pt.nsm));
+  L.tiles_row = take(sizeof(Tile) * (size_t)(L.max_tiles + (kSplitParts - 1) * pt.nsm));
   L.splits_row = take(sizeof(Tile) * (size_t)L.max_splits);
   L.total = off;
   return L;

@@ -192,20 +192,22 @@ __device__ __forceinline__ void load_rows(uint32_t dst, const CUtensorMap* m128,
   for (int b = 0; b < nb; ++b) tma_load_2d(dst + b * kQuant * 128, m16, x, y + b * kQuant, bar);
 }
 // Output chunks [lo, hi) of a row tile: id 0 names all columns; split b has
-// ids 1 + 2b (first half) and 2 + 2b (second half).  `whole` (down without an
-// up-front H): a split tile is done whole under its first half's entry and its
-// second half's entry is skipped -- cutting it would make both halves repeat
-// the tile's K loop.
-__device__ __forceinline__ int split_half(const Tile& t) { return (t.id - 1) & 1; }
-__device__ __forceinline__ int split_index(const Tile& t) { return (t.id - 1) >> 1; }
-__device__ __forceinline__ bool tile_live(const Tile& t, bool whole) {
-  return t.cnt > 0 && !(whole && t.id > 0 && split_half(t) == 1);
+// ids 1 + P b + p for its column parts p < P = kSplitParts.  A kernel takes
+// the parts of a split tile `merge` at a time (the entries of the other parts
+// are skipped): gate/up merges 2 (a part then costs a gather of H per row; 4
+// parts measured slower), down with an up-front H takes single parts, down
+// without one takes the tile whole (cutting it would make every part repeat
+// the tile's K loop).
+__device__ __forceinline__ int split_part(const Tile& t) { return (t.id - 1) % kSplitParts; }
+__device__ __forceinline__ int split_index(const Tile& t) { return (t.id - 1) / kSplitParts; }
+__device__ __forceinline__ bool tile_live(const Tile& t, int merge) {
+  return t.cnt > 0 && !(t.id > 0 && split_part(t) % merge != 0);
 }
-__device__ __forceinline__ int chunk_lo(const Tile& t, int nch, bool whole) {
-  return !whole && t.id > 0 && split_half(t) == 1 ? (nch + 1) / 2 : 0;
+__device__ __forceinline__ int chunk_lo(const Tile& t, int nch, int merge) {
+  return t.id > 0 && merge < kSplitParts ? split_part(t) * nch / kSplitParts : 0;
 }
-__device__ __forceinline__ int chunk_hi(const Tile& t, int nch, bool whole) {
-  return !whole && t.id > 0 && split_half(t) == 0 ? (nch + 1) / 2 : nch;
+__device__ __forceinline__ int chunk_hi(const Tile& t, int nch, int merge) {
+  return t.id > 0 && merge < kSplitParts ? (split_part(t) + merge) * nch / kSplitParts : nch;
 }
 // Up-front H of the split row tiles (down): ready once every epilogue warp of
 // the CTA that computed it has added 1.
@@ -299,11 +301,11 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
   // (K loop only) into Hpre; the split tiles' column halves then read it
   // instead of repeating the K loop, so the last work comes in halves
   const bool pre = !SHARED && a.pre != 0;
-  const bool whole = !SHARED && !pre;
-  const int split0 = a.counts[kCntRowSplit], n_split = (n_items - split0) / 2;
+  const int merge = SHARED ? 2 : (pre ? 1 : kSplitParts);  // parts of a split tile taken together
+  const int split0 = a.counts[kCntRowSplit], n_split = (n_items - split0) / kSplitParts;
   const bool has_pre = pre && (int)blockIdx.x < n_split;
   Tile pre_t{};
-  if (has_pre) pre_t = a.tiles[split0 + 2 * (int)blockIdx.x];
+  if (has_pre) pre_t = a.tiles[split0 + kSplitParts * (int)blockIdx.x];
   int32_t* const hflag = a.sched + 8;
   auto needs_k = [&](const Tile& t) { return !SHARED && !(pre && t.id > 0); };
   const int d_in = a.d_in, d_out = a.d_out;
@@ -320,17 +322,21 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
 #pragma unroll
       for (int k = 0; k < S; ++k) last[k] = nK[k] = nC[k] = 0;
       int i = 0, q = 0;
-      // take tiles until one this kernel runs, or the end; hand it on
+      // take the next tile (the counter runs over the entries this kernel
+      // takes: every unsplit tile, then every merge-th part entry), or the
+      // end; hand it on
+      const int n_take = split0 + (n_items - split0) / merge;
       auto grab = [&](Tile& t) -> bool {
         int item;
         while (true) {
-          item = atomicAdd(a.sched + kSchedFwdRows, 1);
-          if (item >= n_items) {
+          const int v = atomicAdd(a.sched + kSchedFwdRows, 1);
+          if (v >= n_take) {
             item = -1;
             break;
           }
+          item = v < split0 ? v : split0 + (v - split0) * merge;
           t = a.tiles[item];
-          if (tile_live(t, whole)) break;
+          if (tile_live(t, merge)) break;
         }
         const int e = q % kQ;
         if (q >= kQ && !mbar_wait(&tq.empty[e], ((q - kQ) / kQ) & 1)) {
@@ -381,7 +387,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
         for (int k = 0; k < NK && !bad; ++k) load_k(cur, k);
       while (has_cur && !bad) {
         const bool has_nxt = grab(nxt);
-        for (int c = chunk_lo(cur, nch, whole); c < chunk_hi(cur, nch, whole) && !bad; ++c) load_c(cur, c);
+        for (int c = chunk_lo(cur, nch, merge); c < chunk_hi(cur, nch, merge) && !bad; ++c) load_c(cur, c);
         if (has_nxt && needs_k(nxt))
           for (int k = 0; k < NK && !bad; ++k) load_k(nxt, k);
         cur = nxt;
@@ -454,7 +460,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
       }
       while (has_cur && !bad) {
         const bool has_nxt = queue_next(tq, q, a.tiles, nxt, true, &qok);
-        const int lo = chunk_lo(cur, nch, whole), hi = chunk_hi(cur, nch, whole);
+        const int lo = chunk_lo(cur, nch, merge), hi = chunk_hi(cur, nch, merge);
         for (int c = lo; c < hi && !bad; ++c) mma_c(c == lo, c == hi - 1);
         ++ci;
         if (has_nxt && needs_k(nxt)) {
@@ -608,7 +614,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
       const bool early = SHARED && NBH == 2 && has_nxt;
       if (early && !(ok = prepare_h(nxt, ci + 1, -1))) break;
       const bool qlive = quarter * 32 < cur.cnt;  // this warp has live rows (warp-uniform)
-      const int lo = chunk_lo(cur, nch, whole), hi = chunk_hi(cur, nch, whole);
+      const int lo = chunk_lo(cur, nch, merge), hi = chunk_hi(cur, nch, merge);
       for (int c = lo + ((grp - cc0) % kNGrp + kNGrp) % kNGrp; c < hi; c += kNGrp) {
         const int cc = cc0 + (c - lo), i = ib + (c - lo);
         const int sl = i % S, b = cc % kNGrp, n0 = c * kChunk;

@@ -146,8 +146,8 @@ __device__ int build_tiles(const int32_t* n_g, const int32_t* off_g, int G, int 
 
 // Forward row tiles in dispatch order: every group's rows in tiles of 128
 // (id 0: all output columns), except that each of the last `tail` tiles of the
-// list (split b) becomes two entries covering one half of the columns each
-// (ids 1 + 2b and 2 + 2b), so the work left when SMs run dry comes in halves.
+// list (split b) becomes kSplitParts entries covering one part of the columns
+// each (ids 1 + P b + p), so the work left when SMs run dry comes in parts.
 // *split_first receives the index of the first split entry.
 __device__ int build_row_tiles(const int32_t* n_g, const int32_t* off_g, int G, int tail, Tile* __restrict__ out,
                                int32_t* scratch /* smem [G+1] */, int32_t* split_first) {
@@ -163,14 +163,14 @@ __device__ int build_row_tiles(const int32_t* n_g, const int32_t* off_g, int G, 
   cnt = 0;
   for (int j = first + (int)threadIdx.x; j < n && cnt < 8; j += blockDim.x) {
     Tile t = mine[cnt++];
-    const int k = first + 2 * (j - first);
-    t.id = 1 + 2 * (j - first);  // split b = j - first: ids 1 + 2b (first half), 2 + 2b (second half)
-    out[k] = t;
-    t.id = 2 + 2 * (j - first);
-    out[k + 1] = t;
+    // split b = j - first: ids 1 + P b + p for its column parts p < P
+    for (int p = 0; p < kSplitParts; ++p) {
+      t.id = 1 + kSplitParts * (j - first) + p;
+      out[first + kSplitParts * (j - first) + p] = t;
+    }
   }
   __syncthreads();
-  return n + ns;
+  return n + (kSplitParts - 1) * ns;
 }
 
 // Sum of ceil(n_g / per) over the groups (every thread gets the total).

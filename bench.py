@@ -100,11 +100,15 @@ def model(T, k, d, f, rank_off, U_g, R_g, nproj_shared=2):
 
 # ------------------------------------------------------------------ clocks
 class ClockSampler:
-    def __init__(self, index: int):
+    """nvidia-smi clock samples during the timed region, into `path` (a temp
+    file unless --clocks-csv names one; {rank} in it becomes the rank)."""
+
+    def __init__(self, index: int, path: str = ""):
         self.index = index
         self.proc = None
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{index}.csv") if os.path.isdir(
-            os.path.join(ROOT, "gpurun_out")) else f"/tmp/ace_clocks_{os.getpid()}.csv"
+        import tempfile
+        self.path = (path.format(rank=index) if path else
+                     os.path.join(tempfile.gettempdir(), f"ace_clocks_{os.getpid()}_{index}.csv"))
 
     def start(self):
         q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
@@ -411,7 +415,7 @@ def run_gpu(args, rank, world, local):
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
-    clk = ClockSampler(local)
+    clk = ClockSampler(local, args.clocks_csv)
     nv = NvmlSampler(torch.cuda.get_device_properties(local))
     clk.start()
     nv.start()
@@ -642,6 +646,8 @@ def main():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--clocks-csv", default="",
+                    help="keep the nvidia-smi clock samples of the timed region in this file ({rank} = rank)")
     ap.add_argument("--impl", default="ace", choices=["ace", "reference"])
     ap.add_argument("--config", default="olmoe")
     ap.add_argument("--seed", type=int, default=0)

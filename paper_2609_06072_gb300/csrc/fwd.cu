@@ -1,15 +1,17 @@
 // Fused LoRA forward (Sec. 3.3-3.5; App. "Implementation and Profiling of
 // Grouped Adapter Execution").
 //
-// k_fwd_h (gate/up): per tile of up to 128 unique (g, t) pairs of one group,
+// k_fwd_h (gate/up, when the token-major k_gemm_h of gemm.cu does not
+//   apply): per tile of up to 128 unique (g, t) pairs of one group,
 //   H_u = A_g x_t is computed ONCE per active group of a token (Sec. 3.5):
 //   X rows gathered by token with cp.async into 128-byte-swizzled smem,
 //   tcgen05 MMA with N = nproj * rank_pad (gate and up share the gather),
 //   fp32 H written per unique pair.
 // k_fwd_rows: persistent, one CTA per SM; tiles of <= 128 consecutive rows
 //   of one group (expert segments are contiguous inside group segments) are
-//   taken dynamically from a counter (the last ones in column halves, so the
-//   SMs finish together).  Warp-specialised:
+//   taken dynamically from a counter; the last wave's tiles come in column
+//   parts (down: their H computed up front, one tile per CTA), so the SMs
+//   finish together.  Warp-specialised:
 //     warp 0     TMA producer: row tiles of Y (and of h for down) and chunks of
 //                B_g^T / A_g into a ring of shared-memory slots
 //     warp 1     MMA issuer: (down) H = h . A_g^T over the K loop, then per

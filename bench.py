@@ -65,9 +65,15 @@ def load_peaks():
 
 
 def csrc_sha():
+    """Hash of the kernel sources with comments and blank space taken out, so
+    that a comment edit does not orphan counters taken from the same code."""
+    import re
     h = hashlib.sha256()
     for p in sorted(glob.glob(os.path.join(ROOT, "paper_2609_06072_gb300", "csrc", "*"))):
-        h.update(open(p, "rb").read())
+        src = open(p, encoding="utf-8").read()
+        src = re.sub(r"/\*.*?\*/", " ", src, flags=re.S)
+        src = re.sub(r"//[^\n]*", " ", src)
+        h.update(" ".join(src.split()).encode())
     return h.hexdigest()[:16]
 
 

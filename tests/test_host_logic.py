@@ -1,0 +1,65 @@
+"""Host-side logic that needs no GPU: the seeded groupings of the workloads,
+the benchmark's routing statistics and byte model, and the kernel-source hash
+that ties stored ncu counters to the code they were taken from."""
+import os
+import sys
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+
+import bench  # noqa: E402
+from paper_2609_06072_gb300 import workloads as W  # noqa: E402
+
+
+def test_paperlike_grouping_sizes_and_budget():
+    for name in ("olmoe_uneven", "kimi"):
+        L = W.Layer(W.get_config(name), seed=0)
+        c = L.cfg
+        sizes = np.bincount(L.e2g, minlength=L.G)
+        # per block of 64 experts: one group of 43, mid-size groups, four singletons
+        assert sizes.sum() == c.E and sizes.min() >= 1
+        assert sorted(sizes.tolist(), reverse=True)[: c.E // 64] == [43] * (c.E // 64)
+        assert (sizes == 1).sum() == 4 * (c.E // 64)
+        # matched budget: sum_g r_g = E * r
+        assert int(L.rank_off[-1]) == c.E * c.r
+        assert np.array_equal(np.diff(L.rank_off), sizes * c.r)
+        # seeded: the same grouping on every draw, another seed another shuffle
+        assert np.array_equal(L.e2g, W.Layer(W.get_config(name), seed=0).e2g)
+        assert not np.array_equal(L.e2g, W.Layer(W.get_config(name), seed=1).e2g)
+
+
+def test_load_stats():
+    st = bench.load_stats([5, 0, 10, 20], 35, 30)
+    assert st["expert_rows_max"] == 20 and st["expert_rows_min"] == 0
+    assert abs(st["R_over_U"] - 35 / 30) < 1e-12
+    p = np.array([5, 10, 20]) / 35
+    assert abs(st["load_entropy_bits"] - float(-(p * np.log2(p)).sum())) < 1e-12
+    uni = bench.load_stats([7] * 8, 56, 56)
+    assert abs(uni["load_entropy_ratio"] - 1.0) < 1e-12
+
+
+def test_byte_model_counts_each_tensor_once():
+    # two groups, equal ranks: bytes of the forward per row call follow the
+    # stated formula term by term
+    T, k, d, f = 64, 2, 32, 16
+    rank_off = [0, 8, 16]
+    U_g, R_g = np.array([40, 30]), np.array([64, 64])
+    b, fl = bench.model(T, k, d, f, rank_off, U_g, R_g)
+    R, Pw = T * k, 16 * (d + f)
+    assert b["fwd_row"] == 2 * R * f + 4 * R * d + 4 * int((R_g * 8).sum()) + 2 * Pw
+    assert fl["fwd_row"] == 2 * int((R_g * 8).sum()) * (d + f)
+    assert b["bwd_row"] == 2 * R * d + 2 * R * f + 4 * int((R_g * 8).sum()) + 4 * R * f + 6 * Pw
+
+
+def test_source_hash_ignores_comments(tmp_path, monkeypatch):
+    src = tmp_path / "paper_2609_06072_gb300" / "csrc"
+    src.mkdir(parents=True)
+    (src / "a.cu").write_text("int f() {  // one\n  return 1; /* two */ }\n")
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    h0 = bench.csrc_sha()
+    (src / "a.cu").write_text("// header\nint f() {\n  return 1;\n}\n")
+    assert bench.csrc_sha() == h0
+    (src / "a.cu").write_text("int f() { return 2; }\n")
+    assert bench.csrc_sha() != h0

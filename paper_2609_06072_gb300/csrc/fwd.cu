@@ -221,7 +221,10 @@ __device__ __forceinline__ uint32_t rows_bytes(int cnt) {
 // Tile queue: the producer takes row tiles from a global counter (so faster
 // SMs take more tiles), skips the ones this kernel does not run, and hands
 // each live tile index to the MMA warp and the epilogue warps through a small
-// ring in shared memory; -1 ends.
+// ring in shared memory; -1 ends.  The consumers take an entry at the start
+// of the tile before it, so a claim that finds the ring full waits only for
+// them to reach the start of a tile whose loads are already issued: the wait
+// always ends.
 struct TileQueue {
   int32_t item[kQ];
   uint64_t full[kQ], empty[kQ];

@@ -122,7 +122,11 @@ int32_t ace_plan_rank_max(const ace_plan* plan);
 
 /* Workspace bytes for T tokens:
  *   perm_bytes  -- ace_permute (lives as long as the ace_perm views are used)
- *   fwd_bytes   -- ace_fwd_shared scratch, used only when its H argument is NULL
+ *   fwd_bytes   -- forward scratch, used only when the call's H argument is NULL:
+ *                  ace_fwd_shared keeps H per unique pair there, ace_fwd_row the H
+ *                  of the rows of its last wave of tiles (computed first, so that
+ *                  wave can run in column parts; with neither H nor scratch that
+ *                  wave runs whole tiles)
  *   bwd_bytes   -- ace_bwd_shared / ace_bwd_row scratch
  * A NULL output pointer is skipped. */
 ace_status ace_workspace_size(const ace_plan* plan, int32_t T, size_t* perm_bytes, size_t* fwd_bytes,
@@ -175,7 +179,8 @@ ace_status ace_fwd_shared_noalloc(const ace_plan* plan, const ace_perm* perm, co
  *   Hin  [R, f] bf16 expert-specific inputs h_e in row order
  *   A    [rank_off[G], f] bf16 (A_g);  Bt [rank_off[G], d] bf16 (B_g^T)
  *   Y    [R, d] bf16 IN/OUT: Y[row] += s * B_g (A_g Hin[row])
- *   H    [R, rank_max] fp32 OUT or NULL: A_g Hin[row] */
+ *   H    [R, rank_max] fp32 OUT or NULL: A_g Hin[row]
+ *   ws   forward scratch (ace_workspace_size fwd_bytes) or NULL; read only when H is NULL */
 ace_status ace_fwd_row(const ace_plan* plan, const ace_perm* perm, const uint16_t* Hin, const uint16_t* A,
                        const uint16_t* Bt, float s, uint16_t* Y, float* H, void* ws, size_t ws_bytes,
                        void* stream);

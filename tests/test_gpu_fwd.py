@@ -158,6 +158,31 @@ def _fwd_row_case(L, s, with_base):
     check_close(host_f64(H), Href[O["row_pair"]][:, : plan.rank_max], "H_down", max_rel=H_MAX_REL, fro_rel=H_FRO_REL)
 
 
+@pytest.mark.parametrize("with_ws", [False, True])
+def test_fwd_row_without_saved_h(with_ws):
+    """No H to save: with forward scratch the last wave's tiles get their H up
+    front in the scratch and run in column parts; without it they run whole.
+    Y is the same either way."""
+    import torch
+    L = W.Layer(W.get_config("olmoe", T=4096), seed=3)
+    c = L.cfg
+    plan = make_plan(L)
+    perm, P = run_perm(L, plan)
+    O = oracle.permute(L.topk_idx, L.e2g, L.G)
+    Y = dev_bf16(np.zeros((c.R, c.d), np.uint16))
+    ws = None
+    if with_ws:
+        _, fwd_bytes, _ = plan.workspace_size(c.T)
+        ws = torch.empty(fwd_bytes, dtype=torch.uint8, device="cuda")
+    plan.fwd_row(perm, dev_bf16(L.h()[O["row_pair"]]), dev_bf16(L.A("down")), dev_bf16(L.Bt("down")), c.s, Y,
+                 None, ws)
+    assert plan.get_error(perm) == 0
+    ref, _ = oracle.fwd(L.topk_idx, L.e2g, L.rank_off, L.h(), L.A("down"), L.Bt("down"), c.s, x_per_pair=True)
+    got = np.empty((c.R, c.d))
+    got[O["row_pair"]] = host_f64(Y)
+    check_close(got, ref, "Y_down")
+
+
 @pytest.mark.parametrize("name,seed,over,base", [("tiny", 0, {}, False), ("tiny", 5, {"T": 77}, True),
                                                  ("olmoe", 0, {"T": 512}, False), ("olmoe", 2, {"T": 4096}, True),
                                                  ("qwen", 1, {"T": 512}, False),

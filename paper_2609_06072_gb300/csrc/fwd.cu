@@ -255,12 +255,16 @@ __device__ __forceinline__ bool queue_next(TileQueue& tq, int& q, const Tile* ti
 // the D chunks of the current tile in the ring; for gate/up the next tile's
 // H is gathered while the current one streams (the H operand is
 // double-buffered in shared memory where it fits).  (Interleaving the next
-// K loop into the chunk stream measured slower.)  The epilogue warps form kNGrp groups of four (one warp
-// per TMEM lane quarter); group p owns the D chunks cc with cc % kNGrp == p,
-// and each warp updates and stores only its own 32 rows, so no barrier spans
-// more than one warp: every hand-off is an mbarrier (a ring slot is released
-// by the MMA commit after a K step, or by the four warps of the group after a
-// chunk, each on its own barrier).
+// K loop into the chunk stream measured slower.)  Down with an up-front H
+// starts with the K loop of its split tile (H to global memory, no chunks);
+// the split tiles' parts later stage that H like gate/up stages H_u, so the
+// H accumulators count only the tiles with a K loop (kc) and the H operand
+// buffers only the tiles with chunks (ci).  The epilogue warps form kNGrp
+// groups of four (one warp per TMEM lane quarter); group p owns the D chunks
+// cc with cc % kNGrp == p, and each warp updates and stores only its own 32
+// rows, so no barrier spans more than one warp: every hand-off is an mbarrier
+// (a ring slot is released by the MMA commit after a K step, or by the four
+// warps of the group after a chunk, each on its own barrier).
 template <int RP, int NPROJ, bool SHARED>
 __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_constant__ PlanTables pt,
                                                               const __grid_constant__ FwdRowsLaunch a) {

@@ -18,6 +18,11 @@ Functions and the passages they follow (arxiv 2609.06072):
 * ``bwd_w``    -- dA_g, dB_g^T: shared adapter updates (Sec. 3.4) from the
                   gradient form of Sec. 3.1.2.
 * ``budget``   -- parameter budget of Sec. 3.1.1 / Sec. 3.3 (pure Python).
+* ``combine_fwd``, ``combine_bwd_dh``, ``combine_bwd_w``
+               -- the down projection's delta weighted by the gate p_e(x) and
+                  summed over a token's routed experts (the combine of
+                  Sec. 3.1's y(x)), and its adjoint: dh, the gate-weight
+                  gradient, dA_g and dB_g^T.
 """
 from __future__ import annotations
 
@@ -67,6 +72,15 @@ def _load():
         lib.oracle_bwd_w.restype = ctypes.c_int
         lib.oracle_bwd_w.argtypes = [i32, i32, i32, i32, vp, vp, vp, i32, i32, vp, i32, vp, vp, vp, dbl, vp, vp,
                                      vp, i64]
+        lib.oracle_combine_fwd.restype = ctypes.c_int
+        lib.oracle_combine_fwd.argtypes = [i32, i32, i32, i32, vp, vp, vp, i32, i32, vp, vp, vp, vp, dbl, vp, vp,
+                                           vp, i64]
+        lib.oracle_combine_bwd_dh.restype = ctypes.c_int
+        lib.oracle_combine_bwd_dh.argtypes = [i32, i32, i32, i32, vp, vp, vp, i32, i32, vp, vp, vp, vp, vp, dbl,
+                                              vp, vp, vp, vp, i64]
+        lib.oracle_combine_bwd_w.restype = ctypes.c_int
+        lib.oracle_combine_bwd_w.argtypes = [i32, i32, i32, i32, vp, vp, vp, i32, i32, vp, vp, vp, vp, vp, dbl,
+                                             vp, vp, vp, i64]
         _lib = lib
     return _lib
 
@@ -195,6 +209,82 @@ def bwd_w(topk_idx, e2g, rank_off, X, dy, A_all, Bt_all, s, x_per_pair=False, se
                           _p(sel_a), 0 if sel_a is None else sel_a.shape[0])
     if st != OR_OK:
         raise OracleError(st, "bwd_w")
+    return dA, dBt
+
+
+def _combine_args(topk_idx, e2g, rank_off, w, A_all, Bt_all):
+    idx = _c(topk_idx, np.int32)
+    e2g = _c(e2g, np.int32)
+    rank_off = _c(rank_off, np.int32)
+    A_all = _c(A_all, np.uint16)
+    Bt_all = _c(Bt_all, np.uint16)
+    w = _c(np.asarray(w).reshape(-1), np.float32)
+    if w.shape[0] != idx.size:
+        raise ValueError("gate weights must hold one value per (token, slot) pair")
+    return idx, e2g, rank_off, w, A_all, Bt_all
+
+
+def combine_fwd(topk_idx, e2g, rank_off, h, w, A_all, Bt_all, s, z_in=None, sel=None):
+    """z_out[t] = z_in[t] + sum_j w[t,j] s B_g (A_g h_{t*k+j}): token rows
+    [T, d_out] float64 (or [len(sel), d_out], row i holding token sel[i])."""
+    lib = _load()
+    idx, e2g, rank_off, w, A_all, Bt_all = _combine_args(topk_idx, e2g, rank_off, w, A_all, Bt_all)
+    T, k = idx.shape
+    G = rank_off.shape[0] - 1
+    h = _c(h, np.uint16)
+    d_in, d_out = A_all.shape[1], Bt_all.shape[1]
+    sel_a = _c(sel, np.int32)
+    z = np.empty((T if sel_a is None else sel_a.shape[0], d_out))
+    st = lib.oracle_combine_fwd(T, k, e2g.shape[0], G, _p(idx), _p(e2g), _p(rank_off), d_in, d_out, _p(h), _p(w),
+                                _p(A_all), _p(Bt_all), float(s), _p(_c(z_in, np.uint16)), _p(z), _p(sel_a),
+                                0 if sel_a is None else sel_a.shape[0])
+    if st != OR_OK:
+        raise OracleError(st, "combine_fwd")
+    return z
+
+
+def combine_bwd_dh(topk_idx, e2g, rank_off, dz, h, w, A_all, Bt_all, s, dh_in=None, sel=None):
+    """(dh [T*k, d_in], dw [T*k]) in float64 for the token-space gradient dz
+    [T, d_out]; with ``sel``, row i holds pair sel[i]."""
+    lib = _load()
+    idx, e2g, rank_off, w, A_all, Bt_all = _combine_args(topk_idx, e2g, rank_off, w, A_all, Bt_all)
+    T, k = idx.shape
+    G = rank_off.shape[0] - 1
+    dz = _c(dz, np.uint16)
+    h = _c(h, np.uint16)
+    d_in, d_out = A_all.shape[1], Bt_all.shape[1]
+    sel_a = _c(sel, np.int32)
+    n = T * k if sel_a is None else sel_a.shape[0]
+    dh = np.empty((n, d_in))
+    dw = np.empty(n)
+    st = lib.oracle_combine_bwd_dh(T, k, e2g.shape[0], G, _p(idx), _p(e2g), _p(rank_off), d_in, d_out, _p(dz),
+                                   _p(h), _p(w), _p(A_all), _p(Bt_all), float(s), _p(_c(dh_in, np.uint16)), _p(dh),
+                                   _p(dw), _p(sel_a), 0 if sel_a is None else sel_a.shape[0])
+    if st != OR_OK:
+        raise OracleError(st, "combine_bwd_dh")
+    return dh, dw
+
+
+def combine_bwd_w(topk_idx, e2g, rank_off, h, dz, w, A_all, Bt_all, s, sel=None):
+    """(dA [sum r_g, d_in], dBt [sum r_g, d_out]) in float64 for the combine;
+    with ``sel``, row i holds rank row sel[i]."""
+    lib = _load()
+    idx, e2g, rank_off, w, A_all, Bt_all = _combine_args(topk_idx, e2g, rank_off, w, A_all, Bt_all)
+    T, k = idx.shape
+    G = rank_off.shape[0] - 1
+    h = _c(h, np.uint16)
+    dz = _c(dz, np.uint16)
+    d_in, d_out = A_all.shape[1], Bt_all.shape[1]
+    n_rank = int(rank_off[-1])
+    sel_a = _c(sel, np.int32)
+    n = n_rank if sel_a is None else sel_a.shape[0]
+    dA = np.empty((n, d_in))
+    dBt = np.empty((n, d_out))
+    st = lib.oracle_combine_bwd_w(T, k, e2g.shape[0], G, _p(idx), _p(e2g), _p(rank_off), d_in, d_out, _p(h),
+                                  _p(dz), _p(w), _p(A_all), _p(Bt_all), float(s), _p(dA), _p(dBt), _p(sel_a),
+                                  0 if sel_a is None else sel_a.shape[0])
+    if st != OR_OK:
+        raise OracleError(st, "combine_bwd_w")
     return dA, dBt
 
 

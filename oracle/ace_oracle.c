@@ -26,6 +26,11 @@
  *   dB_g  = s * sum_{pairs p in g} dy_p (A_g x_p)^T          (stored transposed)
  *   dx_p  = s * A_g^T (B_g^T dy_p)   (summed over a token's pairs for gate/up)
  *
+ * The gate-weighted combine of the down projection (the oracle_combine_*
+ * functions) carries the router weight p_e(x) of Sec. 3.1 into the sum over
+ * a token's routed experts and returns token rows; its gradients are the
+ * adjoint of that sum, including the gradient of each gate weight.
+ *
  * The routing permutation is a stable sort of the (token, slot) pairs by the
  * key (g(e), e, t) -- the row order the library documents -- computed with
  * the C library's qsort on unique keys.
@@ -332,6 +337,165 @@ int oracle_bwd_w(int32_t T, int32_t k, int32_t E, int32_t G, const int32_t* topk
       for (int32_t c = 0; c < d_in; ++c) hv += bf16_to_f64(a[c]) * bf16_to_f64(x[c]);
       for (int32_t c = 0; c < d_in; ++c) da[c] += s * w * bf16_to_f64(x[c]);
       for (int32_t o = 0; o < d_out; ++o) db[o] += s * hv * bf16_to_f64(dyp[o]);
+    }
+  }
+  return OR_OK;
+}
+
+/* --------------------------------------------- gate-weighted combine (down) */
+
+/*
+ * The down projection's adapter delta taken through the router's combine
+ * (Sec. 3.1: y(x) = sum_{e in R(x)} p_e(x) (W_e h_e + B_e A_e h_e), with
+ * expert e using the group adapter of g(e) as in Sec. 3.4):
+ *   z_out[t] = z_in[t] + sum_j w_p * s * B_g (A_g h_p),   p = t*k + j, g = g(e_p)
+ * h is pair-ordered [T*k, d_in], w the gate weights [T*k] (fp32), z token
+ * rows [T, d_out].  z_in may be NULL.  sel lists the tokens to compute,
+ * output row i holding token sel[i]; NULL = all.  Pairs of a token are
+ * summed in ascending j.
+ */
+int oracle_combine_fwd(int32_t T, int32_t k, int32_t E, int32_t G, const int32_t* topk_idx, const int32_t* e2g,
+                       const int32_t* rank_off, int32_t d_in, int32_t d_out, const uint16_t* h, const float* w,
+                       const uint16_t* A_all, const uint16_t* Bt_all, double s, const uint16_t* z_in,
+                       double* z_out, const int32_t* sel, int64_t n_sel) {
+  if (T < 0 || k < 1 || d_in < 1 || d_out < 1) return OR_ERR_ARG;
+  for (int32_t g = 0; g < G; ++g)
+    if (rank_off[g + 1] - rank_off[g] < 0 || rank_off[g + 1] - rank_off[g] > 1024) return OR_ERR_ARG;
+  const int64_t R = (int64_t)T * k;
+  const int64_t n = sel ? n_sel : T;
+  for (int64_t i = 0; i < n; ++i) {
+    int64_t t = sel ? sel[i] : i;
+    if (t < 0 || t >= T) return OR_ERR_INDEX;
+  }
+  for (int64_t p = 0; p < R; ++p) {
+    int32_t e = topk_idx[p];
+    if (e < 0 || e >= E || e2g[e] < 0 || e2g[e] >= G) return OR_ERR_INDEX;
+  }
+#pragma omp parallel for schedule(dynamic, 8)
+  for (int64_t i = 0; i < n; ++i) {
+    int64_t t = sel ? sel[i] : i;
+    double* z = z_out + i * (int64_t)d_out;
+    for (int32_t o = 0; o < d_out; ++o) z[o] = z_in ? bf16_to_f64(z_in[t * (int64_t)d_out + o]) : 0.0;
+    for (int64_t p = t * k; p < t * k + k; ++p) {
+      int32_t g = e2g[topk_idx[p]];
+      int32_t r0 = rank_off[g], rg = rank_off[g + 1] - rank_off[g];
+      const uint16_t* x = h + p * (int64_t)d_in;
+      double H[1024];
+      for (int32_t i_r = 0; i_r < rg; ++i_r) {
+        const uint16_t* a = A_all + (int64_t)(r0 + i_r) * d_in;
+        double acc = 0.0;
+        for (int32_t c = 0; c < d_in; ++c) acc += bf16_to_f64(a[c]) * bf16_to_f64(x[c]);
+        H[i_r] = acc;
+      }
+      const double wp = (double)w[p];
+      for (int32_t o = 0; o < d_out; ++o) {
+        double acc = 0.0;
+        for (int32_t i_r = 0; i_r < rg; ++i_r) acc += bf16_to_f64(Bt_all[(int64_t)(r0 + i_r) * d_out + o]) * H[i_r];
+        z[o] += wp * s * acc;
+      }
+    }
+  }
+  return OR_OK;
+}
+
+/*
+ * Input and gate-weight gradients of oracle_combine_fwd for a token-space
+ * output gradient dz [T, d_out]:
+ *   dh_out[p] = dh_in[p] + w_p * s * A_g^T (B_g^T dz_t)     (pair rows [T*k, d_in])
+ *   dw[p]     = s * (B_g^T dz_t) . (A_g h_p)                  (only the adapter's share)
+ * dh_in may be NULL.  sel lists the pairs to compute, output row i holding
+ * pair sel[i]; NULL = all.
+ */
+int oracle_combine_bwd_dh(int32_t T, int32_t k, int32_t E, int32_t G, const int32_t* topk_idx,
+                          const int32_t* e2g, const int32_t* rank_off, int32_t d_in, int32_t d_out,
+                          const uint16_t* dz, const uint16_t* h, const float* w, const uint16_t* A_all,
+                          const uint16_t* Bt_all, double s, const uint16_t* dh_in, double* dh_out, double* dw,
+                          const int32_t* sel, int64_t n_sel) {
+  if (T < 0 || k < 1 || d_in < 1 || d_out < 1) return OR_ERR_ARG;
+  for (int32_t g = 0; g < G; ++g)
+    if (rank_off[g + 1] - rank_off[g] < 0 || rank_off[g + 1] - rank_off[g] > 1024) return OR_ERR_ARG;
+  const int64_t R = (int64_t)T * k;
+  const int64_t n = sel ? n_sel : R;
+  for (int64_t i = 0; i < n; ++i) {
+    int64_t p = sel ? sel[i] : i;
+    if (p < 0 || p >= R) return OR_ERR_INDEX;
+  }
+  for (int64_t p = 0; p < R; ++p) {
+    int32_t e = topk_idx[p];
+    if (e < 0 || e >= E || e2g[e] < 0 || e2g[e] >= G) return OR_ERR_INDEX;
+  }
+#pragma omp parallel for schedule(dynamic, 16)
+  for (int64_t i = 0; i < n; ++i) {
+    int64_t p = sel ? sel[i] : i;
+    int64_t t = p / k;
+    int32_t g = e2g[topk_idx[p]];
+    int32_t r0 = rank_off[g], rg = rank_off[g + 1] - rank_off[g];
+    const uint16_t* dzt = dz + t * (int64_t)d_out;
+    const uint16_t* x = h + p * (int64_t)d_in;
+    double* out = dh_out + i * (int64_t)d_in;
+    for (int32_t c = 0; c < d_in; ++c) out[c] = dh_in ? bf16_to_f64(dh_in[p * (int64_t)d_in + c]) : 0.0;
+    const double wp = (double)w[p];
+    double dwp = 0.0;
+    for (int32_t i_r = 0; i_r < rg; ++i_r) {
+      const uint16_t* bt = Bt_all + (int64_t)(r0 + i_r) * d_out;
+      const uint16_t* a = A_all + (int64_t)(r0 + i_r) * d_in;
+      double v = 0.0; /* (B_g^T dz_t)[i_r] */
+      for (int32_t o = 0; o < d_out; ++o) v += bf16_to_f64(bt[o]) * bf16_to_f64(dzt[o]);
+      double hv = 0.0; /* (A_g h_p)[i_r] */
+      for (int32_t c = 0; c < d_in; ++c) hv += bf16_to_f64(a[c]) * bf16_to_f64(x[c]);
+      for (int32_t c = 0; c < d_in; ++c) out[c] += wp * s * v * bf16_to_f64(a[c]);
+      dwp += s * v * hv;
+    }
+    if (dw) dw[i] = dwp;
+  }
+  return OR_OK;
+}
+
+/*
+ * Weight gradients of oracle_combine_fwd (shared adapter updates, Sec. 3.4):
+ *   dA[i][c]  = s * sum_{p: g(e_p)=g(i)} w_p (B_g^T dz_t)[i] * h_p[c]
+ *   dBt[i][o] = s * sum_{p: g(e_p)=g(i)} w_p (A_g h_p)[i]   * dz_t[o]
+ * Pairs are visited in ascending p; groups with no pairs get exact zeros.
+ * sel lists the rank rows to compute (output row ii = rank row sel[ii]).
+ */
+int oracle_combine_bwd_w(int32_t T, int32_t k, int32_t E, int32_t G, const int32_t* topk_idx,
+                         const int32_t* e2g, const int32_t* rank_off, int32_t d_in, int32_t d_out,
+                         const uint16_t* h, const uint16_t* dz, const float* w, const uint16_t* A_all,
+                         const uint16_t* Bt_all, double s, double* dA, double* dBt, const int32_t* sel,
+                         int64_t n_sel) {
+  if (T < 0 || k < 1 || d_in < 1 || d_out < 1) return OR_ERR_ARG;
+  const int64_t R = (int64_t)T * k;
+  const int32_t n_rank = rank_off[G];
+  const int64_t n = sel ? n_sel : n_rank;
+  for (int64_t i = 0; i < n; ++i) {
+    int64_t q = sel ? sel[i] : i;
+    if (q < 0 || q >= n_rank) return OR_ERR_INDEX;
+  }
+  for (int64_t p = 0; p < R; ++p) {
+    int32_t e = topk_idx[p];
+    if (e < 0 || e >= E || e2g[e] < 0 || e2g[e] >= G) return OR_ERR_INDEX;
+  }
+#pragma omp parallel for schedule(dynamic, 1)
+  for (int64_t ii = 0; ii < n; ++ii) {
+    int32_t i = (int32_t)(sel ? sel[ii] : ii);
+    int32_t g = 0;
+    while (!(rank_off[g] <= i && i < rank_off[g + 1])) ++g;
+    double* da = dA + ii * (int64_t)d_in;
+    double* db = dBt + ii * (int64_t)d_out;
+    for (int32_t c = 0; c < d_in; ++c) da[c] = 0.0;
+    for (int32_t o = 0; o < d_out; ++o) db[o] = 0.0;
+    const uint16_t* a = A_all + (int64_t)i * d_in;
+    const uint16_t* bt = Bt_all + (int64_t)i * d_out;
+    for (int64_t p = 0; p < R; ++p) {
+      if (e2g[topk_idx[p]] != g) continue;
+      const uint16_t* x = h + p * (int64_t)d_in;
+      const uint16_t* dzt = dz + (p / k) * (int64_t)d_out;
+      const double wp = (double)w[p];
+      double v = 0.0, hv = 0.0;
+      for (int32_t o = 0; o < d_out; ++o) v += bf16_to_f64(bt[o]) * bf16_to_f64(dzt[o]);
+      for (int32_t c = 0; c < d_in; ++c) hv += bf16_to_f64(a[c]) * bf16_to_f64(x[c]);
+      for (int32_t c = 0; c < d_in; ++c) da[c] += s * wp * v * bf16_to_f64(x[c]);
+      for (int32_t o = 0; o < d_out; ++o) db[o] += s * wp * hv * bf16_to_f64(dzt[o]);
     }
   }
   return OR_OK;

@@ -120,6 +120,10 @@ void ace_plan_destroy(ace_plan* plan);
  * buffer below. */
 int32_t ace_plan_rank_max(const ace_plan* plan);
 
+/* rank_off[G] rounded up to a multiple of 64: the row stride (in elements)
+ * of the token-major combined H of ace_fwd_combine / ace_bwd_combine. */
+int32_t ace_plan_rank_cols(const ace_plan* plan);
+
 /* Workspace bytes for T tokens:
  *   perm_bytes  -- ace_permute (lives as long as the ace_perm views are used)
  *   fwd_bytes   -- forward scratch, used only when the call's H argument is NULL:
@@ -127,7 +131,7 @@ int32_t ace_plan_rank_max(const ace_plan* plan);
  *                  of the rows of its last wave of tiles (computed first, so that
  *                  wave can run in column parts; with neither H nor scratch that
  *                  wave runs whole tiles)
- *   bwd_bytes   -- ace_bwd_shared / ace_bwd_row scratch
+ *   bwd_bytes   -- ace_bwd_shared / ace_bwd_row / ace_bwd_combine scratch
  * A NULL output pointer is skipped. */
 ace_status ace_workspace_size(const ace_plan* plan, int32_t T, size_t* perm_bytes, size_t* fwd_bytes,
                               size_t* bwd_bytes);
@@ -205,6 +209,42 @@ ace_status ace_bwd_shared(const ace_plan* plan, const ace_perm* perm, int32_t np
 ace_status ace_bwd_row(const ace_plan* plan, const ace_perm* perm, const uint16_t* dY, const uint16_t* Hin,
                        const float* H, const uint16_t* A, const uint16_t* Bt, float s, uint16_t* dHin, float* dA,
                        float* dBt, void* ws, size_t ws_bytes, void* stream);
+
+/* Gate-weighted combine of the down projection, forward.  Sec. 3.1's
+ * y(x) = sum_{e in R(x)} p_e(x) (W_e h_e + B_e A_e h_e) with expert e using the
+ * group adapter of g(e) (Sec. 3.4): the adapter's share of the combined
+ * output, in token rows.
+ *   Hin     [R, f] bf16 expert inputs h_e in row order
+ *   topk_w  [T, k] fp32 gate weights p, pair order (pair t*k + j)
+ *   A       [rank_off[G], f] bf16 (A_g);  Bt [rank_off[G], d] bf16 (B_g^T)
+ *   Z       [T, d] bf16 IN/OUT: Z[t] += sum_j p[t,j] s B_g (A_g Hin[pair_row[t*k+j]])
+ *   H       [R, rank_max] fp32 OUT: A_g Hin[row] (columns >= r_g zero)
+ *   Hx      [T, ace_plan_rank_cols] bf16 OUT, the combined H:
+ *           Hx[t][rank_off[g] + i] = s sum_{j: g(e_tj) = g} p[t,j] H[pair_row[t*k+j]][i]
+ *           for i < r_g, every other column zero
+ * By linearity the weighted sum over a token's experts of one group is taken
+ * before B_g, so each token needs one product with the stacked B^T (K =
+ * rank_off[G]) instead of one per routed expert.  H and Hx are the inputs
+ * ace_bwd_combine needs.  Pairs of a token are summed in ascending j
+ * (deterministic). */
+ace_status ace_fwd_combine(const ace_plan* plan, const ace_perm* perm, const uint16_t* Hin, const float* topk_w,
+                           const uint16_t* A, const uint16_t* Bt, float s, uint16_t* Z, float* H, uint16_t* Hx,
+                           void* stream);
+
+/* Backward of ace_fwd_combine for the token gradient dZ [T, d] bf16:
+ *   H, Hx    from ace_fwd_combine
+ *   dHin     [R, f] bf16 IN/OUT: dHin[row] += p s A_g^T (B_g^T dZ[t])
+ *   dtopk_w  [T, k] fp32 OUT (overwritten): s (B_g^T dZ[t]) . (A_g Hin[row]), the
+ *            adapter's share of the gate-weight gradient
+ *   dA       [rank_off[G], f] fp32 OUT: s sum_rows p (B_g^T dZ[t]) Hin[row]^T
+ *   dBt      [rank_off[G], d] fp32 OUT: sum_t Hx[t] dZ[t]^T over the group's columns
+ *   ws       backward scratch (ace_workspace_size bwd_bytes)
+ * B_g^T dZ[t] is formed once per unique (g, t) pair.  Groups with no routed
+ * pair get exact zeros. */
+ace_status ace_bwd_combine(const ace_plan* plan, const ace_perm* perm, const uint16_t* dZ, const uint16_t* Hin,
+                           const float* topk_w, const float* H, const uint16_t* Hx, const uint16_t* A,
+                           const uint16_t* Bt, float s, uint16_t* dHin, float* dtopk_w, float* dA, float* dBt,
+                           void* ws, size_t ws_bytes, void* stream);
 
 /* Row-order helpers (bf16, `cols` elements per row, cols multiple of 8):
  *   gather:  dst[row] = src[row_pair[row]]   (pair order -> row order)

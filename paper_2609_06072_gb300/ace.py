@@ -32,7 +32,7 @@ STATUS_NAMES = {0: "ACE_OK", 1: "ACE_ERR_ARG", 2: "ACE_ERR_SHAPE", 3: "ACE_ERR_W
 
 EXPORTED = ["ace_version", "ace_last_error_message", "ace_plan_create", "ace_plan_destroy", "ace_plan_rank_max",
             "ace_workspace_size", "ace_permute", "ace_fwd_shared", "ace_fwd_shared_noalloc", "ace_fwd_row",
-            "ace_bwd_shared", "ace_bwd_row",
+            "ace_bwd_shared", "ace_bwd_row", "ace_plan_rank_cols", "ace_fwd_combine", "ace_bwd_combine",
             "ace_gather_rows", "ace_scatter_rows", "ace_get_error"]
 
 
@@ -83,6 +83,8 @@ def load(build_if_missing: bool = False) -> ctypes.CDLL:
     lib.ace_plan_destroy.argtypes = [vp]
     lib.ace_plan_rank_max.restype = i32
     lib.ace_plan_rank_max.argtypes = [vp]
+    lib.ace_plan_rank_cols.restype = i32
+    lib.ace_plan_rank_cols.argtypes = [vp]
     lib.ace_workspace_size.restype = i32
     lib.ace_workspace_size.argtypes = [vp, i32, ctypes.POINTER(sz), ctypes.POINTER(sz), ctypes.POINTER(sz)]
     lib.ace_permute.restype = i32
@@ -99,6 +101,11 @@ def load(build_if_missing: bool = False) -> ctypes.CDLL:
     lib.ace_bwd_row.restype = i32
     lib.ace_bwd_row.argtypes = [vp, ctypes.POINTER(ace_perm), vp, vp, vp, vp, vp, ctypes.c_float, vp, vp, vp, vp, sz,
                                 vp]
+    lib.ace_fwd_combine.restype = i32
+    lib.ace_fwd_combine.argtypes = [vp, ctypes.POINTER(ace_perm), vp, vp, vp, vp, ctypes.c_float, vp, vp, vp, vp]
+    lib.ace_bwd_combine.restype = i32
+    lib.ace_bwd_combine.argtypes = [vp, ctypes.POINTER(ace_perm), vp, vp, vp, vp, vp, vp, vp, ctypes.c_float, vp, vp,
+                                    vp, vp, vp, sz, vp]
     lib.ace_gather_rows.restype = i32
     lib.ace_gather_rows.argtypes = [ctypes.POINTER(ace_perm), vp, vp, i32, vp]
     lib.ace_scatter_rows.restype = i32
@@ -236,6 +243,27 @@ class Plan:
                                     _ptr(dHin, torch.bfloat16, "dHin"), _ptr(dA, torch.float32, "dA"),
                                     _ptr(dBt, torch.float32, "dBt"), _ptr(ws), ws.numel(), _stream(stream)),
                "ace_bwd_row")
+
+    @property
+    def rank_cols(self) -> int:
+        """Row stride of the token-major combined H (stacked ranks rounded up to 64)."""
+        return int(self.lib.ace_plan_rank_cols(self.h))
+
+    def fwd_combine(self, perm: Perm, Hin, topk_w, A, Bt, s, Z, H, Hx, stream=None):
+        _check(self.lib.ace_fwd_combine(self.h, ctypes.byref(perm.c), _ptr(Hin, torch.bfloat16, "Hin"),
+                                        _ptr(topk_w, torch.float32, "topk_w"), _ptr(A, torch.bfloat16, "A"),
+                                        _ptr(Bt, torch.bfloat16, "Bt"), float(s), _ptr(Z, torch.bfloat16, "Z"),
+                                        _ptr(H, torch.float32, "H"), _ptr(Hx, torch.bfloat16, "Hx"),
+                                        _stream(stream)), "ace_fwd_combine")
+
+    def bwd_combine(self, perm: Perm, dZ, Hin, topk_w, H, Hx, A, Bt, s, dHin, dtopk_w, dA, dBt, ws, stream=None):
+        _check(self.lib.ace_bwd_combine(self.h, ctypes.byref(perm.c), _ptr(dZ, torch.bfloat16, "dZ"),
+                                        _ptr(Hin, torch.bfloat16, "Hin"), _ptr(topk_w, torch.float32, "topk_w"),
+                                        _ptr(H, torch.float32, "H"), _ptr(Hx, torch.bfloat16, "Hx"),
+                                        _ptr(A, torch.bfloat16, "A"), _ptr(Bt, torch.bfloat16, "Bt"), float(s),
+                                        _ptr(dHin, torch.bfloat16, "dHin"), _ptr(dtopk_w, torch.float32, "dtopk_w"),
+                                        _ptr(dA, torch.float32, "dA"), _ptr(dBt, torch.float32, "dBt"), _ptr(ws),
+                                        ws.numel(), _stream(stream)), "ace_bwd_combine")
 
     def gather_rows(self, perm: Perm, src_pairs, dst_rows, stream=None):
         _check(self.lib.ace_gather_rows(ctypes.byref(perm.c), _ptr(src_pairs), _ptr(dst_rows),

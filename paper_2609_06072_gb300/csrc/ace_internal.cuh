@@ -134,11 +134,13 @@ cudaError_t launch_zero(void* const* ptrs, const size_t* bytes, int n, cudaStrea
 cudaError_t launch_rows_copy(const int32_t* row_pair, const uint16_t* src, uint16_t* dst, int64_t R, int32_t cols,
                              bool gather, cudaStream_t st);
 
-// H = A_g x per unique (g, t) pair of gate/up (deduplicated; X rows gathered).
+// H = A_g x per unique (g, t) pair of gate/up (deduplicated; X rows gathered),
+// or with `rows` H = A_g h per row over the forward row tiles.
 struct FwdHLaunch {
-  const Tile* tiles;  // unique-pair tiles
+  const Tile* tiles;  // unique-pair tiles (rows: the forward row tiles)
   const int32_t* counts;
   int32_t max_tiles;
+  int32_t rows;       // 1: row tiles, source row = output row; 0: unique pairs, source row = uniq_tok[u]
   const int32_t* uniq_tok;
   const uint16_t* X;
   const uint16_t* A[2];
@@ -224,6 +226,12 @@ struct BwdLaunch {
   float* part_dA[2];     // deterministic dA partials (down) [max_splits, rank_pad, d_in]
   int32_t d_in, d_out, nproj, T;
   bool deterministic;
+  // gate-weighted combine of down (with shared == false): H[0] = dHc per
+  // unique pair, H[1] = the forward's H per row, dB^T left to the dense GEMM
+  bool comb;
+  const float* w;           // combine: gate weights [T*k], pair order
+  float* dw;                // combine: gate-weight gradient [T*k] out, pair order
+  const int32_t* row_pair;  // combine: pair of each row
   int32_t* err;
 };
 cudaError_t launch_bwd(const PlanTables& pt, const BwdLaunch& a, bool shared, cudaStream_t st);
@@ -244,5 +252,24 @@ struct DenseBwdLaunch {
 };
 // dA must be zero on entry (the GEMM adds its tiles into it).
 cudaError_t launch_dense_bwd(const DenseBwdLaunch& a, cudaStream_t st);
+// The two halves of launch_dense_bwd on their own: dX += dHx . A (tm_dhx,
+// tm_acat, tm_dx) and dA += dHx^T . X (tm_dhx_t, tm_x, tm_da).
+cudaError_t launch_dense_dx(const DenseBwdLaunch& a, cudaStream_t st);
+cudaError_t launch_dense_da(const DenseBwdLaunch& a, cudaStream_t st);
+
+// Token-major combined H of the gate-weighted combine of down (combine.cu):
+//   Hx[t][rank_off[g] + k] = s * sum_{j: g(e_tj) = g} w[t*k+j] * H[pair_row[t*k+j]][k]
+// for k < r_g, every other column of [0, n_rank_pad) zero; bf16, row stride
+// n_rank_pad.  Pairs are added in ascending j (deterministic).
+struct CombReduceLaunch {
+  const float* H;          // [R, rank_max] fp32 per row
+  const float* w;          // [T*k] gate weights, pair order
+  const int32_t* pair_row;
+  const int32_t* pair_g;
+  uint16_t* Hx;            // [T, n_rank_pad] bf16 out
+  float s;
+  int32_t T, n_rank_pad;
+};
+cudaError_t launch_comb_reduce(const PlanTables& pt, const CombReduceLaunch& a, cudaStream_t st);
 
 }  // namespace ace

@@ -208,6 +208,8 @@ void ace_plan_destroy(ace_plan* plan) { delete plan; }
 
 int32_t ace_plan_rank_max(const ace_plan* plan) { return plan ? plan->pt.rank_max : 0; }
 
+int32_t ace_plan_rank_cols(const ace_plan* plan) { return plan ? n_rank_pad_of(plan->pt) : 0; }
+
 ace_status ace_workspace_size(const ace_plan* plan, int32_t T, size_t* perm_bytes, size_t* fwd_bytes,
                               size_t* bwd_bytes) {
   if (!plan) return fail(ACE_ERR_ARG, "null plan");
@@ -515,6 +517,185 @@ ace_status ace_bwd_row(const ace_plan* plan, const ace_perm* perm, const uint16_
   a.deterministic = (plan->flags & ACE_FLAG_DETERMINISTIC) != 0;
   a.err = at<int32_t>(perm->ws, L.err);
   return cuda_status(launch_bwd(plan->pt, a, false, static_cast<cudaStream_t>(stream)), "backward launch");
+}
+
+// Gate-weighted combine of down, forward: H per row (the row-tile mode of
+// the H kernel), the token-major combined H, then Z += Hx . [B_g^T] with the
+// dense dX GEMM.
+ace_status ace_fwd_combine(const ace_plan* plan, const ace_perm* perm, const uint16_t* Hin, const float* topk_w,
+                           const uint16_t* A, const uint16_t* Bt, float s, uint16_t* Z, float* H, uint16_t* Hx,
+                           void* stream) {
+  ace_status st = check_perm(plan, perm);
+  if (st != ACE_OK) return st;
+  if (!A || !Bt || !H || !Hx || (perm->T > 0 && !Z) || (perm->R > 0 && (!Hin || !topk_w)))
+    return fail(ACE_ERR_ARG, "null argument");
+  if (!aligned16(A) || !aligned16(Bt) || !aligned16(H) || !aligned16(Hx) || (Z && !aligned16(Z)) ||
+      (Hin && !aligned16(Hin)) || (reinterpret_cast<uintptr_t>(topk_w) & 3u))
+    return fail(ACE_ERR_ARG, "tensor not 16-byte aligned (topk_w: 4-byte)");
+  if (perm->R == 0) return ACE_OK;
+  const PlanTables& pt = plan->pt;
+  const PermLayout L = perm_layout(pt, perm->T);
+  const int n_rank = pt.rank_off[pt.G], nrp = n_rank_pad_of(pt);
+  cudaStream_t cs = static_cast<cudaStream_t>(stream);
+  int32_t* err = at<int32_t>(perm->ws, L.err);
+  DenseBwdLaunch x{};
+  const uint64_t T = (uint64_t)perm->T;
+  bool ok = make_tmap_bf16(&x.tm_dhx, Hx, T, (uint64_t)nrp, kTileM) &&
+            make_tmap_bf16(&x.tm_acat[0], Bt, (uint64_t)n_rank, (uint64_t)pt.d, 64) &&
+            make_tmap_bf16(&x.tm_dx, Z, T, (uint64_t)pt.d, kTileM);
+  if (!ok) return fail(ACE_ERR_UNSUPPORTED, "tensor-map encoding failed for this layout");
+  FwdHLaunch h{};
+  h.tiles = at<Tile>(perm->ws, L.tiles_row);
+  h.counts = perm->counts;
+  h.max_tiles = L.max_tiles;
+  h.rows = 1;
+  h.X = Hin;
+  h.A[0] = h.A[1] = A;
+  h.H[0] = h.H[1] = H;
+  h.d_in = pt.f;
+  h.nproj = 1;
+  h.err = err;
+  st = cuda_status(launch_fwd_h(pt, h, cs), "combine H launch");
+  if (st != ACE_OK) return st;
+  CombReduceLaunch c{};
+  c.H = H;
+  c.w = topk_w;
+  c.pair_row = perm->pair_row;
+  c.pair_g = at<int32_t>(perm->ws, L.pair_g);
+  c.Hx = Hx;
+  c.s = s;
+  c.T = perm->T;
+  c.n_rank_pad = nrp;
+  st = cuda_status(launch_comb_reduce(pt, c, cs), "combine reduce launch");
+  if (st != ACE_OK) return st;
+  x.tm_acat[1] = x.tm_acat[0];
+  x.dX = Z;
+  x.T = perm->T;
+  x.d = pt.d;
+  x.n_rank = n_rank;
+  x.n_rank_pad = nrp;
+  x.nproj = 1;
+  x.grid = plan->num_sms;
+  x.err = err;
+  return cuda_status(launch_dense_dx(x, cs), "combine output launch");
+}
+
+// Gate-weighted combine of down, backward: dHc_u = B_g^T dZ[t] per unique
+// pair (the forward's H kernels on dZ and B^T), the row kernel in its combine
+// mode (dh, dA, the gate-weight gradient), then dB^T += Hx^T . dZ with the
+// dense dA GEMM.
+ace_status ace_bwd_combine(const ace_plan* plan, const ace_perm* perm, const uint16_t* dZ, const uint16_t* Hin,
+                           const float* topk_w, const float* H, const uint16_t* Hx, const uint16_t* A,
+                           const uint16_t* Bt, float s, uint16_t* dHin, float* dtopk_w, float* dA, float* dBt,
+                           void* ws, size_t ws_bytes, void* stream) {
+  ace_status st = check_perm(plan, perm);
+  if (st != ACE_OK) return st;
+  if (!A || !Bt || !dA || !dBt ||
+      (perm->R > 0 && (!dZ || !Hin || !topk_w || !H || !Hx || !dHin || !dtopk_w)))
+    return fail(ACE_ERR_ARG, "null argument");
+  if (!aligned16(A) || !aligned16(Bt) || !aligned16(dA) || !aligned16(dBt) || (dZ && !aligned16(dZ)) ||
+      (Hin && !aligned16(Hin)) || (H && !aligned16(H)) || (Hx && !aligned16(Hx)) || (dHin && !aligned16(dHin)) ||
+      (reinterpret_cast<uintptr_t>(topk_w) & 3u) || (reinterpret_cast<uintptr_t>(dtopk_w) & 3u))
+    return fail(ACE_ERR_ARG, "tensor not 16-byte aligned (topk_w, dtopk_w: 4-byte)");
+  const BwdWs need = bwd_layout(plan, perm->T, nullptr);
+  if (!ws || ws_bytes < need.total) return fail(ACE_ERR_WORKSPACE, "backward workspace %zu < %zu bytes", ws_bytes, need.total);
+  if (!aligned16(ws)) return fail(ACE_ERR_WORKSPACE, "backward workspace misaligned");
+  const PlanTables& pt = plan->pt;
+  const PermLayout L = perm_layout(pt, perm->T);
+  const BwdWs w = bwd_layout(plan, perm->T, ws);
+  const int n_rank = pt.rank_off[pt.G], nrp = n_rank_pad_of(pt);
+  const uint64_t R = (uint64_t)perm->R, T = (uint64_t)perm->T;
+  cudaStream_t cs = static_cast<cudaStream_t>(stream);
+  int32_t* err = at<int32_t>(perm->ws, L.err);
+  float* Hc = w.dHrow[0];  // dHc per unique pair, row stride rank_max
+  BwdLaunch a{};
+  DenseBwdLaunch x{};
+  if (perm->R > 0) {
+    bool ok = make_tmap_bf16(&a.tm_a, A, (uint64_t)n_rank, (uint64_t)pt.f, pt.rank_pad) &&
+              make_tmap_bf16(&a.tm_dh, dHin, R, (uint64_t)pt.f, kTileM) &&
+              make_tmap_bf16(&a.tm_h, Hin, R, (uint64_t)pt.f, kTileM) &&
+              make_tmap_bf16(&x.tm_dhx_t, Hx, T, (uint64_t)nrp, 64) && make_tmap_bf16(&x.tm_x, dZ, T, (uint64_t)pt.d, 64) &&
+              make_tmap_f32(&x.tm_da[0], dBt, (uint64_t)n_rank, (uint64_t)pt.d, 32);
+    if (!ok) return fail(ACE_ERR_UNSUPPORTED, "tensor-map encoding failed for this layout");
+    if (n_rank <= kDenseHMaxRank) {
+      DenseHLaunch h{};
+      ok = make_tmap_bf16(&h.tm_x, dZ, T, (uint64_t)pt.d, kTileM) &&
+           make_tmap_bf16(&h.tm_a[0], Bt, (uint64_t)n_rank, (uint64_t)pt.d, 256);
+      if (!ok) return fail(ACE_ERR_UNSUPPORTED, "tensor-map encoding failed for this layout");
+      h.tm_a[1] = h.tm_a[0];
+      h.tok_uniq = perm->tok_uniq;
+      h.uniq_off = perm->uniq_off;
+      h.H[0] = h.H[1] = Hc;
+      h.T = perm->T;
+      h.d = pt.d;
+      h.n_rank = n_rank;
+      h.nproj = 1;
+      h.rank_max = pt.rank_max;
+      h.grid = plan->num_sms;
+      h.err = err;
+      st = cuda_status(launch_dense_h(pt, h, cs), "combine dHc launch");
+    } else {
+      FwdHLaunch h{};
+      h.tiles = at<Tile>(perm->ws, L.tiles_sh);
+      h.counts = perm->counts;
+      h.max_tiles = L.max_tiles;
+      h.rows = 0;
+      h.uniq_tok = perm->uniq_tok;
+      h.X = dZ;
+      h.A[0] = h.A[1] = Bt;
+      h.H[0] = h.H[1] = Hc;
+      h.d_in = pt.d;
+      h.nproj = 1;
+      h.err = err;
+      st = cuda_status(launch_fwd_h(pt, h, cs), "combine dHc launch");
+    }
+    if (st != ACE_OK) return st;
+  }
+  a.splits_row = at<Tile>(perm->ws, L.splits_row);
+  a.tiles_sh = at<Tile>(perm->ws, L.tiles_sh);
+  a.counts = perm->counts;
+  a.max_splits_row = L.max_splits;
+  a.max_tiles_sh = L.max_tiles;
+  a.uniq_tok = perm->uniq_tok;
+  a.uniq_off = perm->uniq_off;
+  a.group_off = perm->group_off;
+  a.pair_row = perm->pair_row;
+  a.pair_g = at<int32_t>(perm->ws, L.pair_g);
+  a.row_uniq = at<int32_t>(perm->ws, L.row_uniq);
+  a.Xin = Hin;
+  a.H[0] = Hc;
+  a.H[1] = H;
+  for (int j = 0; j < 2; ++j) {
+    a.dA[j] = dA;
+    a.dBt[j] = dBt;
+    a.dHrow[j] = w.dHrow[0];
+    a.part_dBt[j] = w.part_dBt[0];
+    a.part_dA[j] = w.part_dA;
+  }
+  a.s = s;
+  a.dXin = dHin;
+  a.d_in = pt.f;
+  a.d_out = pt.d;
+  a.nproj = 1;
+  a.T = perm->T;
+  a.deterministic = (plan->flags & ACE_FLAG_DETERMINISTIC) != 0;
+  a.comb = true;
+  a.w = topk_w;
+  a.dw = dtopk_w;
+  a.row_pair = perm->row_pair;
+  a.err = err;
+  st = cuda_status(launch_bwd(pt, a, false, cs), "combine backward launch");
+  if (st != ACE_OK || perm->R == 0) return st;
+  x.tm_da[1] = x.tm_da[0];
+  x.dA[0] = x.dA[1] = dBt;
+  x.T = perm->T;
+  x.d = pt.d;
+  x.n_rank = n_rank;
+  x.n_rank_pad = nrp;
+  x.nproj = 1;
+  x.grid = plan->num_sms;
+  x.err = err;
+  return cuda_status(launch_dense_da(x, cs), "combine dB launch");
 }
 
 ace_status ace_gather_rows(const ace_perm* perm, const uint16_t* src_pairs, uint16_t* dst_rows, int32_t cols,

@@ -21,6 +21,13 @@
 //   in the fast mode each row adds its dH there with bf16 vector reductions;
 //   in the deterministic mode the rows go to fp32 scratch and
 // k_dh_reduce sums them per unique pair in a fixed slot order.
+// MODE_COMB (the down projection's delta taken through the gate-weighted
+//   combine) has no phase 1: the token gradient dz reaches the rows through
+//   the unique-pair product dHc_u = B_g^T dz_t (computed before, by the dense
+//   H GEMM on dz), so the epilogue stages dH_row = s p_row dHc_u directly as
+//   the phase-2 operand and writes the gate-weight gradient
+//   dp_row = s dHc_u . H_row on the way; phase 2 (dh, dA) is MODE_DOWN's.
+//   dB^T comes from the dense dA GEMM of gemm.cu on the token-major combined H.
 // k_splitk_reduce: deterministic stage 2 of dB^T / dA (split order); empty groups
 //   -> exact zeros.
 #include <cstdint>
@@ -33,7 +40,7 @@ namespace {
 
 constexpr int kNcB = 128;           // columns per chunk
 constexpr int kBlk = kTileM * 128;  // one [128 x 64] bf16 SW128 block (16 KB)
-constexpr int MODE_DOWN = 0, MODE_SHARED = 1;
+constexpr int MODE_DOWN = 0, MODE_SHARED = 1, MODE_COMB = 2;
 constexpr int kThreadsWS = 320;     // producer, MMA, 8 epilogue warps (two per TMEM lane quarter)
 constexpr int kEpiThreads = 256;
 constexpr int kEpiBar = 1;
@@ -121,7 +128,7 @@ struct RowsCfg {
   static constexpr int kWBlk = RP * 128;
   static constexpr int kSlotA = 2 * kBlk + 2 * kWBlk;  // dY tile + B^T chunk (down phase 2: A chunk + h tile)
   static constexpr int kSlotB = 2 * kBlk;                      // down: dh tile for the RMW
-  static constexpr int SB = MODE == MODE_DOWN ? 2 : 0;
+  static constexpr int SB = MODE != MODE_SHARED ? 2 : 0;
   static constexpr int kBudget = 220 * 1024;
   static constexpr int kSA0 = (kBudget - kOps - SB * kSlotB) / kSlotA;
   static constexpr int SA = kSA0 > 6 ? 6 : (kSA0 < 2 ? 2 : kSA0);
@@ -131,7 +138,7 @@ struct RowsCfg {
   static constexpr int kTB = NT * RP > 128 ? 256 : 128;
   static constexpr int ND = (RP > 64 || kTB > 128) ? 1 : 2;  // down: dh D buffers of 128 columns
   static constexpr int kDB = (RP > 64 || kTB > 128) ? 384 : 256;
-  static constexpr int kTmem = (MODE == MODE_DOWN || RP > 64 || kTB > 128) ? 512 : 256;
+  static constexpr int kTmem = (MODE != MODE_SHARED || RP > 64 || kTB > 128) ? 512 : 256;
 };
 
 template <int RP, int MODE>
@@ -158,8 +165,8 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
   const int g = sp.g, r0 = pt.rank_off[g], rg = pt.rank_off[g + 1] - r0;
   const int ntiles = (sp.cnt + kTileM - 1) / kTileM;
   const int d_in = a.d_in, d_out = a.d_out;
-  const int nch1 = (d_out + kNcB - 1) / kNcB;
-  const int nch2 = MODE == MODE_DOWN ? (d_in + kNcB - 1) / kNcB : 0;
+  const int nch1 = MODE == MODE_COMB ? 0 : (d_out + kNcB - 1) / kNcB;
+  const int nch2 = MODE != MODE_SHARED ? (d_in + kNcB - 1) / kNcB : 0;
   const int NI1 = nch1 * ntiles, NI2 = nch2 * ntiles;
   const uint32_t sOps = smem_u32(smem);
   const uint32_t sA0 = sOps + C::kOps;
@@ -269,7 +276,7 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
         if (i == ntiles - 1) tc_commit(&dbt_full[c & 1]);
       }
       if (!bad) tc_commit(&dh_full);
-      if (MODE == MODE_DOWN && !bad) {
+      if (MODE != MODE_SHARED && !bad) {
         constexpr uint32_t id_d = idesc_bf16_f32(128, kNcB, 0, 1);
         if (!mbar_wait(&hs_ready, 0)) bad = true;
         for (int j = 0; j < NI2 && !bad; ++j) {
@@ -313,46 +320,69 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
     const int fmode = a.deterministic ? kPartial : kAtomic;
     // H operand slots: bf16 of the saved H of each row, staged while the
     // producer already streams the first dY tiles.  The rows' lines are
-    // prefetched into L2 first, ahead of the stream.
+    // prefetched into L2 first, ahead of the stream.  MODE_COMB stages
+    // dH_row = s p_row dHc_u instead (H[0] = dHc per unique pair, H[1] = the
+    // forward's H per row) and writes dp_row = s dHc_u . H_row.
     {
       for (int idx = et; idx < sp.cnt; idx += kEpiThreads) {
-        const int hrow = MODE == MODE_SHARED ? a.row_uniq[sp.start + idx] : sp.start + idx;
+        const int hrow = MODE != MODE_DOWN ? a.row_uniq[sp.start + idx] : sp.start + idx;
         const float* hp = a.H[proj] + (int64_t)hrow * pt.rank_max;
         for (int c = 0; c < RP && c < pt.rank_max; c += 32) prefetch_l2(hp + c);
+        if (MODE == MODE_COMB) {
+          const float* hs = a.H[1] + (int64_t)(sp.start + idx) * pt.rank_max;
+          for (int c = 0; c < RP && c < pt.rank_max; c += 32) prefetch_l2(hs + c);
+        }
       }
       named_bar_arrive(kIssueBar, kEpiThreads + 32);
       const bool vec = (pt.rank_max & 3) == 0;
+      // v[0..32) = src[c0 .. c0 + 32), zero past rank_max or for a dead row
+      auto load32 = [&](const float* src, int c0, bool live, float* v) {
+        if (vec) {
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            const int c = c0 + 4 * q;
+            const float4 x = (live && c < pt.rank_max) ? *reinterpret_cast<const float4*>(src + c)
+                                                       : make_float4(0.f, 0.f, 0.f, 0.f);
+            v[4 * q] = x.x;
+            v[4 * q + 1] = x.y;
+            v[4 * q + 2] = x.z;
+            v[4 * q + 3] = x.w;
+          }
+        } else {
+#pragma unroll
+          for (int q = 0; q < 32; ++q) v[q] = (live && c0 + q < pt.rank_max) ? src[c0 + q] : 0.f;
+        }
+      };
       for (int idx = et; idx < ntiles * kTileM; idx += kEpiThreads) {
         const int i = idx / kTileM, mm = idx % kTileM;
         const int row = sp.start + idx;
-        const int hrow = idx >= sp.cnt ? -1 : (MODE == MODE_SHARED ? a.row_uniq[row] : row);
+        const int hrow = idx >= sp.cnt ? -1 : (MODE != MODE_DOWN ? a.row_uniq[row] : row);
         const float* hp = a.H[proj] + (int64_t)(hrow < 0 ? 0 : hrow) * pt.rank_max;
         if (MODE == MODE_SHARED) tok_s[idx] = hrow < 0 ? -1 : a.uniq_tok[hrow];
+        const int pair = (MODE == MODE_COMB && hrow >= 0) ? a.row_pair[row] : 0;
+        const float wscale = (MODE == MODE_COMB && hrow >= 0) ? a.s * a.w[pair] : 0.f;
+        float dp = 0.f;
 #pragma unroll
         for (int c0 = 0; c0 < RP; c0 += 32) {
           float v[32];
-          if (vec) {
-#pragma unroll
-            for (int q = 0; q < 8; ++q) {
-              const int c = c0 + 4 * q;
-              const float4 x = (hrow >= 0 && c < pt.rank_max) ? *reinterpret_cast<const float4*>(hp + c)
-                                                             : make_float4(0.f, 0.f, 0.f, 0.f);
-              v[4 * q] = x.x;
-              v[4 * q + 1] = x.y;
-              v[4 * q + 2] = x.z;
-              v[4 * q + 3] = x.w;
-            }
-          } else {
-#pragma unroll
-            for (int q = 0; q < 32; ++q) v[q] = (hrow >= 0 && c0 + q < pt.rank_max) ? hp[c0 + q] : 0.f;
-          }
+          load32(hp, c0, hrow >= 0, v);
 #pragma unroll
           for (int q = 0; q < 32; ++q)
             if (c0 + q >= rg) v[q] = 0.f;
+          if (MODE == MODE_COMB) {
+            float hs[32];
+            load32(a.H[1] + (int64_t)(hrow >= 0 ? row : 0) * pt.rank_max, c0, hrow >= 0, hs);
+#pragma unroll
+            for (int q = 0; q < 32; ++q) {
+              dp += v[q] * hs[q];
+              v[q] *= wscale;
+            }
+          }
 #pragma unroll
           for (int c8 = 0; c8 < 4; ++c8)
             if (c0 + 8 * c8 < RP) sts128(sOps + SL::elem(i, mm, c0 + 8 * c8), pack8(v + 8 * c8));
         }
+        if (MODE == MODE_COMB && hrow >= 0) a.dw[pair] = a.s * dp;
       }
       fence_proxy_async_smem();
       __syncwarp();
@@ -373,7 +403,8 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
     if (ok) {
       tc_fence_after();
       // dH (scaled by s): gate/up -> fp32 per row; down -> bf16 operand slots
-      for (int i = 0; i < ntiles; ++i) {
+      // (the combine staged its dH with the operand slots above)
+      for (int i = 0; i < (MODE == MODE_COMB ? 0 : ntiles); ++i) {
         const bool live = i * kTileM + m < sp.cnt;
         const int64_t row = sp.start + i * kTileM + m;
 #pragma unroll
@@ -420,7 +451,7 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
       named_bar(kEpiBar, kEpiThreads);
       if (et == 0) mbar_arrive(&hs_ready);
     }
-    if (MODE == MODE_DOWN) {
+    if (MODE != MODE_SHARED) {
       for (int j = 0; j < NI2 && ok; ++j) {
         const int c = j / ntiles, i = j % ntiles, b = j % C::ND, sb = j % SB, n0 = c * kNcB;
         bool w_ok = mbar_wait(&fullB[sb], (j / SB) & 1);
@@ -586,8 +617,29 @@ cudaError_t launch_rows(const PlanTables& pt, const BwdLaunch& a, int nproj, cud
   return launch_k(kern, dim3(a.max_splits_row, nproj), kThreadsWS, C::kSmem, st, pt, a);
 }
 
+// Combine backward: one launch zeroes dB^T (the dense dA GEMM of gemm.cu
+// adds its tiles into it afterwards) and, in the fast mode, dA; then the row
+// kernel and, in the deterministic mode, stage 2 of dA.
+template <int RP>
+cudaError_t launch_comb_t(const PlanTables& pt, const BwdLaunch& a, cudaStream_t st) {
+  const int n_rank = pt.rank_off[pt.G];
+  void* zp[kZeroMax] = {};
+  size_t zb[kZeroMax] = {};
+  int nz = 0;
+  zp[nz] = a.dBt[0], zb[nz++] = sizeof(float) * (size_t)n_rank * a.d_out;
+  if (!a.deterministic) zp[nz] = a.dA[0], zb[nz++] = sizeof(float) * (size_t)n_rank * a.d_in;
+  cudaError_t e = launch_zero(zp, zb, nz, st);
+  if (e != cudaSuccess) return e;
+  if ((e = launch_rows<RP, MODE_COMB>(pt, a, 1, st)) != cudaSuccess) return e;
+  if (!a.deterministic) return cudaSuccess;
+  dim3 grid(n_rank, (a.d_in / 4 + 255) / 256);
+  return launch_k(k_splitk_reduce, grid, 256, 0, st, pt, a.splits_row, a.counts, kCntSplitsRow, a.part_dA[0], (int)RP,
+                  a.d_in, a.dA[0]);
+}
+
 template <int RP>
 cudaError_t launch_bwd_t(const PlanTables& pt, const BwdLaunch& a, bool shared, cudaStream_t st) {
+  if (a.comb) return launch_comb_t<RP>(pt, a, st);
   cudaError_t e;
   const int n_rank = pt.rank_off[pt.G];
   const int nproj = shared ? a.nproj : 1;

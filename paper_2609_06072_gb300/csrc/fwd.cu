@@ -6,7 +6,10 @@
 //   H_u = A_g x_t is computed ONCE per active group of a token (Sec. 3.5):
 //   X rows gathered by token with cp.async into 128-byte-swizzled smem,
 //   tcgen05 MMA with N = nproj * rank_pad (gate and up share the gather),
-//   fp32 H written per unique pair.
+//   fp32 H written per unique pair.  With `rows` set the same kernel takes
+//   the forward row tiles instead (each split tile once) and computes
+//   H_row = A_g h_row for contiguous rows of h: the first step of the
+//   gate-weighted combine of down.
 // k_fwd_rows: persistent, one CTA per SM; tiles of <= 128 consecutive rows
 //   of one group (expert segments are contiguous inside group segments) are
 //   taken dynamically from a counter; the last wave's tiles come in column
@@ -56,16 +59,24 @@ __global__ void __launch_bounds__(kHThreads) k_fwd_h(const __grid_constant__ Pla
   __shared__ int32_t src_row[kTileM];
 
   pdl_wait();
-  const int n_tiles = a.counts[kCntTilesSh];
-  if ((int)blockIdx.x >= n_tiles) return;
-  const Tile tl = a.tiles[blockIdx.x];
+  Tile tl;
+  if (a.rows) {
+    // row tiles: whole tiles first, then kSplitParts entries per split tile
+    const int n_items = a.counts[kCntTilesRow], split0 = a.counts[kCntRowSplit];
+    const int b = blockIdx.x;
+    if (b >= split0 + (n_items - split0) / kSplitParts) return;
+    tl = a.tiles[b < split0 ? b : split0 + (b - split0) * kSplitParts];
+  } else {
+    if ((int)blockIdx.x >= a.counts[kCntTilesSh]) return;
+    tl = a.tiles[blockIdx.x];
+  }
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int quarter = warp & 3, half = warp >> 2;
   const int m = quarter * 32 + lane;
   const int g = tl.g, r0 = pt.rank_off[g], rg = pt.rank_off[g + 1] - r0;
   const int d_in = a.d_in;
 
-  if (tid < kTileM) src_row[tid] = tid < tl.cnt ? a.uniq_tok[tl.start + tid] : -1;
+  if (tid < kTileM) src_row[tid] = tid < tl.cnt ? (a.rows ? tl.start + tid : a.uniq_tok[tl.start + tid]) : -1;
   if (tid == 0) {
     for (int i = 0; i < kHStages; ++i) mbar_init(&bar_k[i], 1);
     fence_mbar_init();

@@ -542,18 +542,27 @@ cudaError_t launch_dense_h(const PlanTables& pt, const DenseHLaunch& a, cudaStre
   return launch_k(kern, std::min(tiles, a.grid), kThreads, kHSmem, st, pt, a);
 }
 
-cudaError_t launch_dense_bwd(const DenseBwdLaunch& a, cudaStream_t st) {
+cudaError_t launch_dense_dx(const DenseBwdLaunch& a, cudaStream_t st) {
   if (a.T == 0) return cudaSuccess;
   cudaError_t e = cudaFuncSetAttribute(k_gemm_dx, cudaFuncAttributeMaxDynamicSharedMemorySize, kDxSmem);
   if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(k_gemm_da, cudaFuncAttributeMaxDynamicSharedMemorySize, kDaSmem);
-  if (e != cudaSuccess) return e;
   const int dx_tiles = ((a.T + 127) / 128) * ((a.d + kDxN - 1) / kDxN);
-  if ((e = launch_k(k_gemm_dx, std::min(dx_tiles, a.grid), kThreads, kDxSmem, st, a)) != cudaSuccess) return e;
+  return launch_k(k_gemm_dx, std::min(dx_tiles, a.grid), kThreads, kDxSmem, st, a);
+}
+
+cudaError_t launch_dense_da(const DenseBwdLaunch& a, cudaStream_t st) {
+  if (a.T == 0) return cudaSuccess;
+  cudaError_t e = cudaFuncSetAttribute(k_gemm_da, cudaFuncAttributeMaxDynamicSharedMemorySize, kDaSmem);
+  if (e != cudaSuccess) return e;
   // dA accumulates bulk reduce-adds: the caller has zeroed it (with the
   // backward's other accumulation targets, in one launch)
   const int da_tiles = ((a.nproj * a.n_rank_pad + 127) / 128) * ((a.d + kDaN - 1) / kDaN);
   return launch_k(k_gemm_da, da_tiles * da_ksplit(da_tiles, a.grid), kThreads, kDaSmem, st, a);
+}
+
+cudaError_t launch_dense_bwd(const DenseBwdLaunch& a, cudaStream_t st) {
+  cudaError_t e = launch_dense_dx(a, st);
+  return e != cudaSuccess ? e : launch_dense_da(a, st);
 }
 
 }  // namespace ace

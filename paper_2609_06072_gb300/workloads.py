@@ -277,6 +277,14 @@ class Layer:
     def dh_base(self) -> np.ndarray:
         return self._normal_bf16("dhbase", (self.cfg.R, self.cfg.f))
 
+    def dZ(self) -> np.ndarray:
+        """Upstream gradient of the gate-weighted combined down output, [T, d]."""
+        return self._normal_bf16("dZ", (self.cfg.T, self.cfg.d))
+
+    def Z_base(self) -> np.ndarray:
+        """Base-path combined output (nonzero z_in), [T, d]."""
+        return self._normal_bf16("Zbase", (self.cfg.T, self.cfg.d))
+
     # -- descriptors -----------------------------------------------------
     def describe(self) -> Dict[str, float]:
         """Realised routing statistics (workload descriptors only)."""

@@ -78,3 +78,7 @@ def test_null_arguments_are_rejected(lib):
     assert lib.ace_workspace_size(None, 0, None, None, None) == ace.ACE_ERR_ARG
     assert lib.ace_permute(None, None, 0, None, 0, None, None) == ace.ACE_ERR_ARG
     assert lib.ace_get_error(None, None) == ace.ACE_ERR_ARG
+    assert lib.ace_plan_rank_cols(None) == 0
+    assert lib.ace_fwd_combine(None, None, None, None, None, None, 1.0, None, None, None, None) == ace.ACE_ERR_ARG
+    assert lib.ace_bwd_combine(None, None, None, None, None, None, None, None, None, 1.0, None, None, None, None, None,
+                               0, None) == ace.ACE_ERR_ARG

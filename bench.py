@@ -161,7 +161,7 @@ class ClockSampler:
 class Layer:
     """Device-resident tensors of one layer plus the plan and workspaces."""
 
-    def __init__(self, cfg_name, seed, expertwise, det, T=None):
+    def __init__(self, cfg_name, seed, expertwise, det, T=None, combine=False):
         import torch
         from paper_2609_06072_gb300 import ace, workloads as W
         over = {"T": T} if T else {}
@@ -203,13 +203,24 @@ class Layer:
         self.dBt = [torch.empty(nr, f, device=dev), torch.empty(nr, f, device=dev), torch.empty(nr, d, device=dev)]
         self.h_grads = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in self.dA + self.dBt]
         self.perm = None
+        # down through the gate-weighted combine: token-space output and gradient
+        self.combine = combine
+        if combine:
+            self.w = torch.from_numpy(np.ascontiguousarray(self.L.topk_w, dtype=np.float32)).to(dev)
+            self.Z = randn(c.T, d).to(dev)
+            self.dZ = randn(c.T, d).to(dev)
+            self.Hx = torch.empty(c.T, self.plan.rank_cols, dtype=torch.bfloat16, device=dev)
+            self.dw = torch.empty(c.T, c.k, device=dev)
 
     def kernels_per_step(self):
         # permute 3, fwd_shared 2 (H per unique pair, row stream), fwd_row 1,
         # bwd_row 2 (zeroing, row stream), bwd_shared 4 (zeroing, row stream, dX, dA);
         # deterministic mode: bwd_row has nothing to zero and adds a dB^T and a dA reduce,
-        # bwd_shared adds the fixed-order dH_u sum and one dB^T reduce per projection
-        return 12 + (4 if self.det else 0)
+        # bwd_shared adds the fixed-order dH_u sum and one dB^T reduce per projection.
+        # With the combine, down is fwd_combine 3 (H per row, combined H, output GEMM)
+        # and bwd_combine 4 (B^T dz per unique pair, zeroing, row stream, dB^T GEMM),
+        # plus a dA reduce in deterministic mode
+        return (16 if self.combine else 12) + (4 if self.det else 0)
 
     def step(self, ev=None):
         """One pass of the hot path.  ev: 6 CUDA events or None at the call
@@ -226,10 +237,16 @@ class Layer:
         mark(1)
         p.fwd_shared(self.perm, self.X, self.A[:2], self.Bt[:2], c.s, self.Y[:2], self.H[:2])
         mark(2)
-        p.fwd_row(self.perm, self.hin, self.A[2], self.Bt[2], c.s, self.Y[2], self.H[2])
-        mark(3)
-        p.bwd_row(self.perm, self.dY[2], self.hin, self.H[2], self.A[2], self.Bt[2], c.s, self.dh, self.dA[2],
-                  self.dBt[2], self.bws)
+        if self.combine:
+            p.fwd_combine(self.perm, self.hin, self.w, self.A[2], self.Bt[2], c.s, self.Z, self.H[2], self.Hx)
+            mark(3)
+            p.bwd_combine(self.perm, self.dZ, self.hin, self.w, self.H[2], self.Hx, self.A[2], self.Bt[2], c.s,
+                          self.dh, self.dw, self.dA[2], self.dBt[2], self.bws)
+        else:
+            p.fwd_row(self.perm, self.hin, self.A[2], self.Bt[2], c.s, self.Y[2], self.H[2])
+            mark(3)
+            p.bwd_row(self.perm, self.dY[2], self.hin, self.H[2], self.A[2], self.Bt[2], c.s, self.dh, self.dA[2],
+                      self.dBt[2], self.bws)
         mark(4)
         p.bwd_shared(self.perm, self.dY[:2], self.X, self.H[:2], self.A[:2], self.Bt[:2], c.s, self.dX,
                      self.dA[:2], self.dBt[:2], self.bws)
@@ -392,6 +409,14 @@ def run_variants(args, flush, main_layer):
         del lay
     ms = time_steps(main_layer, args.steps, args.warmup, None)
     out["unflushed"] = {"value": c_rows / (ms * 1e-3), "ms_per_step": ms}
+    if args.combine:
+        # down through the gate-weighted combine (token-space output) in place
+        # of the per-row down forward and backward
+        lay = Layer(args.config, args.seed, args.expertwise, args.det, combine=True)
+        ms = time_steps(lay, args.steps, args.warmup, flush)
+        out["down_via_gate_weighted_combine"] = {"value": c_rows / (ms * 1e-3), "ms_per_step": ms,
+                                                 "kernels_per_step": lay.kernels_per_step()}
+        del lay
     return out
 
 
@@ -660,6 +685,8 @@ def main():
     ap.add_argument("--expertwise", action="store_true", help="matched-budget expert-wise layout (G=E, rank r)")
     ap.add_argument("--det", action="store_true", help="deterministic two-stage split-K for dA / dB^T")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU-oracle baseline leg")
+    ap.add_argument("--combine", action="store_true",
+                    help="also time the step with down through the gate-weighted combine (a variant)")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-variants", action="store_true",
                     help="skip the expert-wise, deterministic-mode and unflushed timings")

@@ -246,6 +246,28 @@ ace_status ace_bwd_combine(const ace_plan* plan, const ace_perm* perm, const uin
                            const uint16_t* Bt, float s, uint16_t* dHin, float* dtopk_w, float* dA, float* dBt,
                            void* ws, size_t ws_bytes, void* stream);
 
+/* Grouping of one layer's experts from their pairwise similarities, for rank
+ * consolidation (Sec. 3.2; layer-wise graph construction, Louvain, fixed-
+ * threshold and group-anchor appendices).  HOST memory, no GPU work:
+ *   S        [E, E] fp32 host similarities (e.g. linear CKA of the adapters'
+ *            outputs on a probe set), symmetrised as (S + S^T) / 2
+ *   method   ACE_GROUP_LOUVAIN: Louvain on W = max(0, S' - median of the
+ *            off-diagonal S'), zero diagonal, resolution `param` (the paper
+ *            uses 0.8); ACE_GROUP_THRESHOLD: connected components of
+ *            {(i, j): i != j, S'_ij >= param} (the paper's variant uses 0.9)
+ *   e2g      [E] int32 host OUT: group of each expert, groups numbered in order
+ *            of their smallest expert
+ *   anchors  [E] int32 host OUT or NULL: the first G entries receive each
+ *            group's CKA-centre anchor, the member with the largest sum of
+ *            similarities to its group (ties to the lower index)
+ *   G_out    OUT: number of groups
+ * The consolidated ranks follow as r_g = sum of the members' ranks (rank_off
+ * of the group plan).  Deterministic; double-precision arithmetic. */
+#define ACE_GROUP_LOUVAIN 0
+#define ACE_GROUP_THRESHOLD 1
+ace_status ace_group_experts(const float* S, int32_t E, int32_t method, double param, int32_t* e2g,
+                             int32_t* anchors, int32_t* G_out);
+
 /* Row-order helpers (bf16, `cols` elements per row, cols multiple of 8):
  *   gather:  dst[row] = src[row_pair[row]]   (pair order -> row order)
  *   scatter: dst[row_pair[row]] = src[row]   (row order -> pair order) */

@@ -33,6 +33,7 @@ STATUS_NAMES = {0: "ACE_OK", 1: "ACE_ERR_ARG", 2: "ACE_ERR_SHAPE", 3: "ACE_ERR_W
 EXPORTED = ["ace_version", "ace_last_error_message", "ace_plan_create", "ace_plan_destroy", "ace_plan_rank_max",
             "ace_workspace_size", "ace_permute", "ace_fwd_shared", "ace_fwd_shared_noalloc", "ace_fwd_row",
             "ace_bwd_shared", "ace_bwd_row", "ace_plan_rank_cols", "ace_fwd_combine", "ace_bwd_combine",
+            "ace_group_experts",
             "ace_gather_rows", "ace_scatter_rows", "ace_get_error"]
 
 
@@ -106,6 +107,8 @@ def load(build_if_missing: bool = False) -> ctypes.CDLL:
     lib.ace_bwd_combine.restype = i32
     lib.ace_bwd_combine.argtypes = [vp, ctypes.POINTER(ace_perm), vp, vp, vp, vp, vp, vp, vp, ctypes.c_float, vp, vp,
                                     vp, vp, vp, sz, vp]
+    lib.ace_group_experts.restype = i32
+    lib.ace_group_experts.argtypes = [vp, i32, i32, ctypes.c_double, vp, vp, vp]
     lib.ace_gather_rows.restype = i32
     lib.ace_gather_rows.argtypes = [ctypes.POINTER(ace_perm), vp, vp, i32, vp]
     lib.ace_scatter_rows.restype = i32
@@ -276,6 +279,25 @@ class Plan:
     def get_error(self, perm: Perm, stream=None) -> int:
         """Synchronise, read and clear the device flag; returns the status code."""
         return self.lib.ace_get_error(ctypes.byref(perm.c), _stream(stream))
+
+
+GROUP_LOUVAIN, GROUP_THRESHOLD = 0, 1
+
+
+def group_experts(S, method: int = GROUP_LOUVAIN, param: float = 0.8):
+    """ace_group_experts on a host [E, E] similarity matrix: returns
+    (e2g [E] int32, anchors [G] int32, G).  No GPU work."""
+    import numpy as np
+    S = np.ascontiguousarray(S, dtype=np.float32)
+    if S.ndim != 2 or S.shape[0] != S.shape[1]:
+        raise ValueError("S must be a square matrix")
+    E = S.shape[0]
+    e2g = np.empty(E, np.int32)
+    anchors = np.empty(E, np.int32)
+    G = ctypes.c_int32()
+    _check(load().ace_group_experts(S.ctypes.data, E, int(method), float(param), e2g.ctypes.data,
+                                    anchors.ctypes.data, ctypes.byref(G)), "ace_group_experts")
+    return e2g, anchors[: G.value].copy(), G.value
 
 
 def perm_arrays(plan: Plan, perm: Perm) -> dict:

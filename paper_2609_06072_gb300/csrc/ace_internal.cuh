@@ -124,6 +124,9 @@ inline T* at(void* base, size_t off) {
   return reinterpret_cast<T*>(static_cast<char*>(base) + off);
 }
 
+// Sets the message ace_last_error_message returns and passes st through.
+ace_status report(ace_status st, const char* msg);
+
 // Launchers implemented in the .cu files (host side).  Each returns the
 // cudaError_t of its launches.
 cudaError_t launch_permute(const PlanTables& pt, const int32_t* topk_idx, int32_t T, void* ws, const PermLayout& L,

@@ -75,6 +75,16 @@ ace_status fail(ace_status st, const char* fmt, ...) {
   return st;
 }
 
+}  // namespace
+
+// The thread's last host-side error message, for the other translation units.
+ace_status ace::report(ace_status st, const char* msg) {
+  snprintf(g_msg, sizeof(g_msg), "%s", msg);
+  return st;
+}
+
+namespace {
+
 ace_status cuda_status(cudaError_t e, const char* what) {
   if (e == cudaSuccess) return ACE_OK;
   return fail(ACE_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));

@@ -263,6 +263,22 @@ ace_status ace_bwd_combine(const ace_plan* plan, const ace_perm* perm, const uin
  *   G_out    OUT: number of groups
  * The consolidated ranks follow as r_g = sum of the members' ranks (rank_off
  * of the group plan).  Deterministic; double-precision arithmetic. */
+/* Linear CKA similarity of a layer's expert-wise adapters on a probe set
+ * (Sec. 3.2): s_ij = ||Zc_i^T Zc_j||_F^2 / (||Zc_i^T Zc_i||_F ||Zc_j^T Zc_j||_F)
+ * with Z_e = X A_e^T B_e^T and Zc_e = H Z_e, H = I - 11^T / N (center != 0) or
+ * Zc_e = Z_e (center == 0; the centering appendix's other variant).
+ *   X      [N, d_in] bf16 probe inputs (the same for every expert)
+ *   A      [E * r, d_in] bf16, rows e*r.. hold A_e;  Bt [E * r, d_out] bf16 (B_e^T)
+ *   S      [E, E] fp32 OUT
+ *   ws     device workspace of ace_cka_workspace_size bytes
+ * d_in a multiple of 64, r <= 32.  The representation matrices are never
+ * formed: with M_ij = A_i (Xc^T Xc) A_j^T, every norm is an r x r trace.  If
+ * a bounded device wait gives up, S is filled with NaN.  Device pointers;
+ * asynchronous on `stream`. */
+ace_status ace_cka_workspace_size(int32_t N, int32_t d_in, int32_t d_out, int32_t E, int32_t r, size_t* bytes);
+ace_status ace_cka(int32_t N, int32_t d_in, int32_t d_out, int32_t E, int32_t r, const uint16_t* X, const uint16_t* A,
+                   const uint16_t* Bt, int32_t center, float* S, void* ws, size_t ws_bytes, void* stream);
+
 #define ACE_GROUP_LOUVAIN 0
 #define ACE_GROUP_THRESHOLD 1
 ace_status ace_group_experts(const float* S, int32_t E, int32_t method, double param, int32_t* e2g,

@@ -33,7 +33,7 @@ STATUS_NAMES = {0: "ACE_OK", 1: "ACE_ERR_ARG", 2: "ACE_ERR_SHAPE", 3: "ACE_ERR_W
 EXPORTED = ["ace_version", "ace_last_error_message", "ace_plan_create", "ace_plan_destroy", "ace_plan_rank_max",
             "ace_workspace_size", "ace_permute", "ace_fwd_shared", "ace_fwd_shared_noalloc", "ace_fwd_row",
             "ace_bwd_shared", "ace_bwd_row", "ace_plan_rank_cols", "ace_fwd_combine", "ace_bwd_combine",
-            "ace_group_experts",
+            "ace_group_experts", "ace_cka_workspace_size", "ace_cka",
             "ace_gather_rows", "ace_scatter_rows", "ace_get_error"]
 
 
@@ -107,6 +107,10 @@ def load(build_if_missing: bool = False) -> ctypes.CDLL:
     lib.ace_bwd_combine.restype = i32
     lib.ace_bwd_combine.argtypes = [vp, ctypes.POINTER(ace_perm), vp, vp, vp, vp, vp, vp, vp, ctypes.c_float, vp, vp,
                                     vp, vp, vp, sz, vp]
+    lib.ace_cka_workspace_size.restype = i32
+    lib.ace_cka_workspace_size.argtypes = [i32, i32, i32, i32, i32, ctypes.POINTER(sz)]
+    lib.ace_cka.restype = i32
+    lib.ace_cka.argtypes = [i32, i32, i32, i32, i32, vp, vp, vp, i32, vp, vp, sz, vp]
     lib.ace_group_experts.restype = i32
     lib.ace_group_experts.argtypes = [vp, i32, i32, ctypes.c_double, vp, vp, vp]
     lib.ace_gather_rows.restype = i32
@@ -282,6 +286,25 @@ class Plan:
 
 
 GROUP_LOUVAIN, GROUP_THRESHOLD = 0, 1
+
+
+def cka(X, A, Bt, E: int, r: int, center: bool = True, S=None, ws=None, stream=None):
+    """ace_cka: the E x E linear-CKA matrix of expert adapters (A [E*r, d_in],
+    Bt [E*r, d_out], bf16) on the probe inputs X [N, d_in] (bf16), all on the
+    GPU.  Returns S (fp32 [E, E], allocated when not given)."""
+    lib = load()
+    N, d_in = int(X.shape[0]), int(X.shape[1])
+    d_out = int(Bt.shape[1])
+    if ws is None:
+        nb = ctypes.c_size_t()
+        _check(lib.ace_cka_workspace_size(N, d_in, d_out, int(E), int(r), ctypes.byref(nb)), "ace_cka_workspace_size")
+        ws = torch.empty(max(nb.value, 16), dtype=torch.uint8, device=X.device)
+    if S is None:
+        S = torch.empty(E, E, dtype=torch.float32, device=X.device)
+    _check(lib.ace_cka(N, d_in, d_out, int(E), int(r), _ptr(X, torch.bfloat16, "X"), _ptr(A, torch.bfloat16, "A"),
+                       _ptr(Bt, torch.bfloat16, "Bt"), int(bool(center)), _ptr(S, torch.float32, "S"), _ptr(ws),
+                       ws.numel(), _stream(stream)), "ace_cka")
+    return S
 
 
 def group_experts(S, method: int = GROUP_LOUVAIN, param: float = 0.8):

@@ -82,3 +82,15 @@ def test_null_arguments_are_rejected(lib):
     assert lib.ace_fwd_combine(None, None, None, None, None, None, 1.0, None, None, None, None) == ace.ACE_ERR_ARG
     assert lib.ace_bwd_combine(None, None, None, None, None, None, None, None, None, 1.0, None, None, None, None, None,
                                0, None) == ace.ACE_ERR_ARG
+
+
+def test_cka_shape_checks_without_gpu(lib):
+    import ctypes
+    from paper_2609_06072_gb300 import ace
+    nb = ctypes.c_size_t()
+    assert lib.ace_cka_workspace_size(10000, 2048, 1024, 64, 8, ctypes.byref(nb)) == ace.ACE_OK
+    # covariance 16 MiB + stacked-rank products, and more for more experts
+    assert nb.value >= 4 * 2048 * 2048 + 4 * 512 * 2048 + 4 * 512 * 512
+    assert lib.ace_cka_workspace_size(10000, 2000, 1024, 64, 8, ctypes.byref(nb)) == ace.ACE_ERR_SHAPE
+    assert lib.ace_cka_workspace_size(10000, 2048, 1024, 64, 33, ctypes.byref(nb)) == ace.ACE_ERR_SHAPE
+    assert lib.ace_cka(16, 64, 8, 2, 2, None, None, None, 1, None, None, 0, None) == ace.ACE_ERR_ARG

@@ -279,6 +279,23 @@ ace_status ace_cka_workspace_size(int32_t N, int32_t d_in, int32_t d_out, int32_
 ace_status ace_cka(int32_t N, int32_t d_in, int32_t d_out, int32_t E, int32_t r, const uint16_t* X, const uint16_t* A,
                    const uint16_t* Bt, int32_t center, float* S, void* ws, size_t ws_bytes, void* stream);
 
+/* The groups' shared adapters at the consolidation step (Sec. 3.2, group-anchor
+ * appendix), from expert-wise adapters of rank r:
+ *   e2g      [E] int32 HOST group of each expert (e.g. from ace_group_experts), G groups
+ *   anchors  [G] int32 HOST anchor expert of each group (a member of it)
+ *   A_e [E*r, d_in], Bt_e [E*r, d_out] bf16 device: the expert-wise adapters
+ *   A_init   [E*r, d_in] bf16 device: LoRA initialisation rows for A (the caller's draw)
+ *   A_g, Bt_g [E*r, d_in] / [E*r, d_out] bf16 device OUT: group g's rank rows
+ *            rank_off[g].. start with its anchor's r rows of A_e / B_e^T; the
+ *            rest take A_init's rows at the same positions and zero B^T rows
+ *   rank_off [G+1] int32 HOST OUT: r_g = r |g|, the plan's rank offsets
+ * At the consolidation step each group's Delta W_g therefore equals its
+ * anchor's Delta W_e.  The budget is unchanged: sum_g r_g = E r. */
+ace_status ace_consolidate_adapters(int32_t E, int32_t r, int32_t d_in, int32_t d_out, const int32_t* e2g,
+                                    const int32_t* anchors, int32_t G, const uint16_t* A_e, const uint16_t* Bt_e,
+                                    const uint16_t* A_init, uint16_t* A_g, uint16_t* Bt_g, int32_t* rank_off,
+                                    void* stream);
+
 #define ACE_GROUP_LOUVAIN 0
 #define ACE_GROUP_THRESHOLD 1
 ace_status ace_group_experts(const float* S, int32_t E, int32_t method, double param, int32_t* e2g,

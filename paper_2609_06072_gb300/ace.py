@@ -33,7 +33,7 @@ STATUS_NAMES = {0: "ACE_OK", 1: "ACE_ERR_ARG", 2: "ACE_ERR_SHAPE", 3: "ACE_ERR_W
 EXPORTED = ["ace_version", "ace_last_error_message", "ace_plan_create", "ace_plan_destroy", "ace_plan_rank_max",
             "ace_workspace_size", "ace_permute", "ace_fwd_shared", "ace_fwd_shared_noalloc", "ace_fwd_row",
             "ace_bwd_shared", "ace_bwd_row", "ace_plan_rank_cols", "ace_fwd_combine", "ace_bwd_combine",
-            "ace_group_experts", "ace_cka_workspace_size", "ace_cka",
+            "ace_group_experts", "ace_cka_workspace_size", "ace_cka", "ace_consolidate_adapters",
             "ace_gather_rows", "ace_scatter_rows", "ace_get_error"]
 
 
@@ -111,6 +111,8 @@ def load(build_if_missing: bool = False) -> ctypes.CDLL:
     lib.ace_cka_workspace_size.argtypes = [i32, i32, i32, i32, i32, ctypes.POINTER(sz)]
     lib.ace_cka.restype = i32
     lib.ace_cka.argtypes = [i32, i32, i32, i32, i32, vp, vp, vp, i32, vp, vp, sz, vp]
+    lib.ace_consolidate_adapters.restype = i32
+    lib.ace_consolidate_adapters.argtypes = [i32, i32, i32, i32, vp, vp, i32, vp, vp, vp, vp, vp, vp, vp]
     lib.ace_group_experts.restype = i32
     lib.ace_group_experts.argtypes = [vp, i32, i32, ctypes.c_double, vp, vp, vp]
     lib.ace_gather_rows.restype = i32
@@ -321,6 +323,38 @@ def group_experts(S, method: int = GROUP_LOUVAIN, param: float = 0.8):
     _check(load().ace_group_experts(S.ctypes.data, E, int(method), float(param), e2g.ctypes.data,
                                     anchors.ctypes.data, ctypes.byref(G)), "ace_group_experts")
     return e2g, anchors[: G.value].copy(), G.value
+
+
+def consolidate_adapters(e2g, anchors, A_e, Bt_e, A_init, r: int, stream=None):
+    """ace_consolidate_adapters: the groups' shared adapters (bf16, on the
+    device of A_e) and the plan's rank offsets (numpy) from expert-wise
+    adapters of rank r, a grouping and its anchors."""
+    import numpy as np
+    e2g = np.ascontiguousarray(e2g, dtype=np.int32)
+    anchors = np.ascontiguousarray(anchors, dtype=np.int32)
+    E, G = int(e2g.shape[0]), int(anchors.shape[0])
+    d_in, d_out = int(A_e.shape[1]), int(Bt_e.shape[1])
+    A_g = torch.empty_like(A_e)
+    Bt_g = torch.empty_like(Bt_e)
+    rank_off = np.empty(G + 1, np.int32)
+    _check(load().ace_consolidate_adapters(E, int(r), d_in, d_out, e2g.ctypes.data, anchors.ctypes.data, G,
+                                           _ptr(A_e, torch.bfloat16, "A_e"), _ptr(Bt_e, torch.bfloat16, "Bt_e"),
+                                           _ptr(A_init, torch.bfloat16, "A_init"), _ptr(A_g), _ptr(Bt_g),
+                                           rank_off.ctypes.data, _stream(stream)), "ace_consolidate_adapters")
+    return A_g, Bt_g, rank_off
+
+
+def consolidate(X_probe, A_e, Bt_e, E: int, r: int, A_init, method: int = 0, param: float = 0.8,
+                center: bool = True, stream=None):
+    """Rank consolidation of one layer and projection (Sec. 3.2): CKA of the
+    expert-wise adapters on the probe (GPU), grouping and anchors (host),
+    then the shared adapters.  Returns (e2g, rank_off, A_g, Bt_g, S) ready
+    for a group plan."""
+    S = cka(X_probe, A_e, Bt_e, E, r, center=center, stream=stream)
+    S_host = S.cpu().numpy()  # synchronises the stream
+    e2g, anchors, _ = group_experts(S_host, method, param)
+    A_g, Bt_g, rank_off = consolidate_adapters(e2g, anchors, A_e, Bt_e, A_init, r, stream=stream)
+    return e2g, rank_off, A_g, Bt_g, S_host
 
 
 def perm_arrays(plan: Plan, perm: Perm) -> dict:

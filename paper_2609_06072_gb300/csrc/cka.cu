@@ -163,6 +163,38 @@ __global__ void __launch_bounds__(256) k_cka_norm(float* __restrict__ S, const f
   S[idx] = *err ? __int_as_float(0x7fc00000) : (den > 0.f ? S[idx] / den : 0.f);
 }
 
+// The groups' shared adapters at the consolidation step (Sec. 3.2, group-
+// anchor appendix): rank row i of group g (k = i - rank_off[g]) copies row
+// anchor_g * r + k of the expert-wise adapters when k < r, else A takes the
+// caller's initialisation row i and B^T is zero.  One CTA per rank row.
+struct ConsolidateParams {
+  int32_t G, r, d_in, d_out;
+  int32_t rank_off[ACE_MAX_EXPERTS + 1];
+  int32_t anchor[ACE_MAX_EXPERTS];
+};
+
+__global__ void __launch_bounds__(256) k_consolidate(const __grid_constant__ ConsolidateParams p,
+                                                     const uint16_t* __restrict__ A_e, const uint16_t* __restrict__ Bt_e,
+                                                     const uint16_t* __restrict__ A_init, uint16_t* __restrict__ A_g,
+                                                     uint16_t* __restrict__ Bt_g) {
+  const int i = blockIdx.x;
+  int lo = 0, hi = p.G;  // the group holding row i: largest g with rank_off[g] <= i
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (p.rank_off[mid] <= i)
+      lo = mid;
+    else
+      hi = mid;
+  }
+  const int k = i - p.rank_off[lo];
+  const bool anchor_row = k < p.r;
+  const int64_t src = (int64_t)p.anchor[lo] * p.r + k;
+  for (int c = threadIdx.x; c < p.d_in; c += 256)
+    A_g[(int64_t)i * p.d_in + c] = anchor_row ? A_e[src * p.d_in + c] : A_init[(int64_t)i * p.d_in + c];
+  for (int c = threadIdx.x; c < p.d_out; c += 256)
+    Bt_g[(int64_t)i * p.d_out + c] = anchor_row ? Bt_e[src * p.d_out + c] : (uint16_t)0;
+}
+
 struct CkaWs {
   float *C, *part, *colsum, *P, *Mx, *Gb, *diag;
   int32_t* err;
@@ -274,6 +306,39 @@ ace_status ace_cka(int32_t N, int32_t d_in, int32_t d_out, int32_t E, int32_t r,
   }
   if (e != cudaSuccess) return report(ACE_ERR_CUDA, cudaGetErrorString(e));
   return ACE_OK;
+}
+
+ace_status ace_consolidate_adapters(int32_t E, int32_t r, int32_t d_in, int32_t d_out, const int32_t* e2g,
+                                    const int32_t* anchors, int32_t G, const uint16_t* A_e, const uint16_t* Bt_e,
+                                    const uint16_t* A_init, uint16_t* A_g, uint16_t* Bt_g, int32_t* rank_off,
+                                    void* stream) {
+  if (!e2g || !anchors || !rank_off || !A_e || !Bt_e || !A_init || !A_g || !Bt_g)
+    return report(ACE_ERR_ARG, "ace_consolidate_adapters: null argument");
+  if (E < 1 || E > ACE_MAX_EXPERTS || G < 1 || G > E || r < 1 || d_in < 1 || d_out < 1)
+    return report(ACE_ERR_SHAPE, "ace_consolidate_adapters: need 1 <= G <= E <= ACE_MAX_EXPERTS, r, d_in, d_out >= 1");
+  ConsolidateParams p{};
+  p.G = G;
+  p.r = r;
+  p.d_in = d_in;
+  p.d_out = d_out;
+  int members[ACE_MAX_EXPERTS] = {0};
+  for (int e = 0; e < E; ++e) {
+    if (e2g[e] < 0 || e2g[e] >= G) return report(ACE_ERR_INDEX, "ace_consolidate_adapters: group out of range");
+    ++members[e2g[e]];
+  }
+  p.rank_off[0] = 0;
+  for (int g = 0; g < G; ++g) {
+    if (members[g] == 0) return report(ACE_ERR_INDEX, "ace_consolidate_adapters: empty group");
+    if (anchors[g] < 0 || anchors[g] >= E || e2g[anchors[g]] != g)
+      return report(ACE_ERR_INDEX, "ace_consolidate_adapters: anchor is not a member of its group");
+    p.anchor[g] = anchors[g];
+    p.rank_off[g + 1] = p.rank_off[g] + r * members[g];
+  }
+  for (int g = 0; g <= G; ++g) rank_off[g] = p.rank_off[g];
+  cudaStream_t cs = static_cast<cudaStream_t>(stream);
+  k_consolidate<<<E * r, 256, 0, cs>>>(p, A_e, Bt_e, A_init, A_g, Bt_g);
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? ACE_OK : report(ACE_ERR_CUDA, cudaGetErrorString(e));
 }
 
 }  // extern "C"

@@ -94,3 +94,20 @@ def test_cka_shape_checks_without_gpu(lib):
     assert lib.ace_cka_workspace_size(10000, 2000, 1024, 64, 8, ctypes.byref(nb)) == ace.ACE_ERR_SHAPE
     assert lib.ace_cka_workspace_size(10000, 2048, 1024, 64, 33, ctypes.byref(nb)) == ace.ACE_ERR_SHAPE
     assert lib.ace_cka(16, 64, 8, 2, 2, None, None, None, 1, None, None, 0, None) == ace.ACE_ERR_ARG
+
+
+def test_consolidate_adapters_host_checks_without_gpu(lib):
+    import ctypes
+    import numpy as np
+    from paper_2609_06072_gb300 import ace
+    e2g = np.array([0, 1, 0, 1], np.int32)
+    ro = np.zeros(3, np.int32)
+    dummy = ctypes.c_void_p(16)  # never dereferenced: the checks fail before any launch
+
+    def call(e2g_, anchors_, G):
+        return lib.ace_consolidate_adapters(4, 2, 8, 8, e2g_.ctypes.data, anchors_.ctypes.data, G, dummy, dummy,
+                                            dummy, dummy, dummy, ro.ctypes.data, None)
+    assert call(e2g, np.array([1, 1], np.int32), 2) == ace.ACE_ERR_INDEX  # anchor 1 is not in group 0
+    assert call(np.array([0, 2, 0, 1], np.int32), np.array([0, 1], np.int32), 2) == ace.ACE_ERR_INDEX
+    assert call(np.array([0, 0, 0, 0], np.int32), np.array([0, 1], np.int32), 2) == ace.ACE_ERR_INDEX  # empty group
+    assert call(e2g, np.array([0, 1], np.int32), 0) == ace.ACE_ERR_SHAPE

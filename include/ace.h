@@ -301,6 +301,38 @@ ace_status ace_consolidate_adapters(int32_t E, int32_t r, int32_t d_in, int32_t 
 ace_status ace_group_experts(const float* S, int32_t E, int32_t method, double param, int32_t* e2g,
                              int32_t* anchors, int32_t* G_out);
 
+/* Routed expert FFN forward with the group-shared adapters (App. "Implementation
+ * and Profiling of Grouped Adapter Execution"): for every row (pair t, e)
+ *   u = (W_e^up + s B_g A_g) x_t,  v = (W_e^gate + s B_g A_g) x_t,
+ *   h = SiLU(v) * u,  y = (W_e^down + s B_g A_g) h
+ * with the plan's map for all three projections.  Composed from per-expert
+ * base GEMMs and the adapter calls above (ace_fwd_shared for gate/up,
+ * ace_fwd_row for down); u, v, h and y are rounded to bf16 between steps.
+ *   X        [T, d] bf16 token inputs
+ *   W_gate, W_up [E, f, d] bf16; W_down [E, d, f] bf16: frozen base weights
+ *   A[3], Bt[3]  gate, up, down adapters (layouts as in ace_fwd_shared / ace_fwd_row)
+ *   U, V, Hh [R, f] bf16 OUT (row order): u, v and h;  Y [R, d] bf16 OUT: y
+ *   Hgu[2]   [R, rank_max] fp32 OUT: H of gate and up per unique pair
+ *   Hd       [R, rank_max] fp32 OUT: H of down per row
+ *   ws       ace_ffn_workspace_size bytes (the token rows in row order) */
+/* Backward of ace_ffn_fwd with frozen base weights, for the per-row output
+ * gradient dY [R, d] bf16 (row order):
+ *   dX       [T, d] bf16 OUT (overwritten): the token-input gradient through
+ *            the three projections and the gating
+ *   dA[3], dBt[3]  fp32 OUT: adapter gradients of gate, up, down
+ *   U, V, Hh, Hgu, Hd  from ace_ffn_fwd;  ws: ace_ffn_workspace_size bytes;
+ *   bws: the adapter backward workspace (ace_workspace_size bwd_bytes) */
+ace_status ace_ffn_bwd(const ace_plan* plan, const ace_perm* perm, const uint16_t* dY, const uint16_t* X,
+                       const uint16_t* W_gate, const uint16_t* W_up, const uint16_t* W_down, const uint16_t* const* A,
+                       const uint16_t* const* Bt, float s, const uint16_t* U, const uint16_t* V, const uint16_t* Hh,
+                       const float* const* Hgu, const float* Hd, uint16_t* dX, float* const* dA, float* const* dBt,
+                       void* ws, size_t ws_bytes, void* bws, size_t bws_bytes, void* stream);
+ace_status ace_ffn_workspace_size(const ace_plan* plan, int32_t T, size_t* bytes);
+ace_status ace_ffn_fwd(const ace_plan* plan, const ace_perm* perm, const uint16_t* X, const uint16_t* W_gate,
+                       const uint16_t* W_up, const uint16_t* W_down, const uint16_t* const* A,
+                       const uint16_t* const* Bt, float s, uint16_t* U, uint16_t* V, uint16_t* Hh, uint16_t* Y,
+                       float* const* Hgu, float* Hd, void* ws, size_t ws_bytes, void* stream);
+
 /* Row-order helpers (bf16, `cols` elements per row, cols multiple of 8):
  *   gather:  dst[row] = src[row_pair[row]]   (pair order -> row order)
  *   scatter: dst[row_pair[row]] = src[row]   (row order -> pair order) */

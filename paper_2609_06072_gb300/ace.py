@@ -33,7 +33,7 @@ STATUS_NAMES = {0: "ACE_OK", 1: "ACE_ERR_ARG", 2: "ACE_ERR_SHAPE", 3: "ACE_ERR_W
 EXPORTED = ["ace_version", "ace_last_error_message", "ace_plan_create", "ace_plan_destroy", "ace_plan_rank_max",
             "ace_workspace_size", "ace_permute", "ace_fwd_shared", "ace_fwd_shared_noalloc", "ace_fwd_row",
             "ace_bwd_shared", "ace_bwd_row", "ace_plan_rank_cols", "ace_fwd_combine", "ace_bwd_combine",
-            "ace_group_experts", "ace_cka_workspace_size", "ace_cka", "ace_consolidate_adapters",
+            "ace_group_experts", "ace_ffn_workspace_size", "ace_ffn_fwd", "ace_ffn_bwd", "ace_cka_workspace_size", "ace_cka", "ace_consolidate_adapters",
             "ace_gather_rows", "ace_scatter_rows", "ace_get_error"]
 
 
@@ -113,6 +113,14 @@ def load(build_if_missing: bool = False) -> ctypes.CDLL:
     lib.ace_cka.argtypes = [i32, i32, i32, i32, i32, vp, vp, vp, i32, vp, vp, sz, vp]
     lib.ace_consolidate_adapters.restype = i32
     lib.ace_consolidate_adapters.argtypes = [i32, i32, i32, i32, vp, vp, i32, vp, vp, vp, vp, vp, vp, vp]
+    lib.ace_ffn_workspace_size.restype = i32
+    lib.ace_ffn_workspace_size.argtypes = [vp, i32, ctypes.POINTER(sz)]
+    lib.ace_ffn_fwd.restype = i32
+    lib.ace_ffn_fwd.argtypes = [vp, ctypes.POINTER(ace_perm), vp, vp, vp, vp, vp, vp, ctypes.c_float, vp, vp, vp, vp,
+                                vp, vp, vp, sz, vp]
+    lib.ace_ffn_bwd.restype = i32
+    lib.ace_ffn_bwd.argtypes = [vp, ctypes.POINTER(ace_perm), vp, vp, vp, vp, vp, vp, vp, ctypes.c_float, vp, vp, vp,
+                                vp, vp, vp, vp, vp, vp, sz, vp, sz, vp]
     lib.ace_group_experts.restype = i32
     lib.ace_group_experts.argtypes = [vp, i32, i32, ctypes.c_double, vp, vp, vp]
     lib.ace_gather_rows.restype = i32
@@ -252,6 +260,38 @@ class Plan:
                                     _ptr(dHin, torch.bfloat16, "dHin"), _ptr(dA, torch.float32, "dA"),
                                     _ptr(dBt, torch.float32, "dBt"), _ptr(ws), ws.numel(), _stream(stream)),
                "ace_bwd_row")
+
+    def ffn_workspace(self, T: int, device="cuda"):
+        n = ctypes.c_size_t()
+        _check(self.lib.ace_ffn_workspace_size(self.h, int(T), ctypes.byref(n)), "ace_ffn_workspace_size")
+        return torch.empty(max(n.value, 16), dtype=torch.uint8, device=device)
+
+    def ffn_fwd(self, perm: Perm, X, W_gate, W_up, W_down, A, Bt, s, U, V, Hh, Y, Hgu, Hd, ws, stream=None):
+        """ace_ffn_fwd: A / Bt are (gate, up, down); Hgu is (gate, up)."""
+        _check(self.lib.ace_ffn_fwd(self.h, ctypes.byref(perm.c), _ptr(X, torch.bfloat16, "X"),
+                                    _ptr(W_gate, torch.bfloat16, "W_gate"), _ptr(W_up, torch.bfloat16, "W_up"),
+                                    _ptr(W_down, torch.bfloat16, "W_down"),
+                                    _arr([_ptr(t, torch.bfloat16, "A") for t in A]),
+                                    _arr([_ptr(t, torch.bfloat16, "Bt") for t in Bt]), float(s),
+                                    _ptr(U, torch.bfloat16, "U"), _ptr(V, torch.bfloat16, "V"),
+                                    _ptr(Hh, torch.bfloat16, "Hh"), _ptr(Y, torch.bfloat16, "Y"),
+                                    _arr([_ptr(t, torch.float32, "Hgu") for t in Hgu]), _ptr(Hd, torch.float32, "Hd"),
+                                    _ptr(ws), ws.numel(), _stream(stream)), "ace_ffn_fwd")
+
+    def ffn_bwd(self, perm: Perm, dY, X, W_gate, W_up, W_down, A, Bt, s, U, V, Hh, Hgu, Hd, dX, dA, dBt, ws, bws,
+                stream=None):
+        """ace_ffn_bwd: A / Bt / dA / dBt are (gate, up, down); Hgu is (gate, up)."""
+        _check(self.lib.ace_ffn_bwd(self.h, ctypes.byref(perm.c), _ptr(dY, torch.bfloat16, "dY"),
+                                    _ptr(X, torch.bfloat16, "X"), _ptr(W_gate, torch.bfloat16, "W_gate"),
+                                    _ptr(W_up, torch.bfloat16, "W_up"), _ptr(W_down, torch.bfloat16, "W_down"),
+                                    _arr([_ptr(t, torch.bfloat16, "A") for t in A]),
+                                    _arr([_ptr(t, torch.bfloat16, "Bt") for t in Bt]), float(s),
+                                    _ptr(U, torch.bfloat16, "U"), _ptr(V, torch.bfloat16, "V"),
+                                    _ptr(Hh, torch.bfloat16, "Hh"),
+                                    _arr([_ptr(t, torch.float32, "Hgu") for t in Hgu]), _ptr(Hd, torch.float32, "Hd"),
+                                    _ptr(dX, torch.bfloat16, "dX"), _arr([_ptr(t, torch.float32, "dA") for t in dA]),
+                                    _arr([_ptr(t, torch.float32, "dBt") for t in dBt]), _ptr(ws), ws.numel(),
+                                    _ptr(bws), bws.numel(), _stream(stream)), "ace_ffn_bwd")
 
     @property
     def rank_cols(self) -> int:

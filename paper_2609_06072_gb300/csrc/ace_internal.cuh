@@ -275,4 +275,23 @@ struct CombReduceLaunch {
 };
 cudaError_t launch_comb_reduce(const PlanTables& pt, const CombReduceLaunch& a, cudaStream_t st);
 
+// Expert FFN pieces (ffn.cu).
+// out[row] (+)= in[row] . W_e^T over the rows of each expert e; W is [E * N, K]
+// (W_e^T rows), or with w_kn [E * K, N] (W_e itself: the input gradient).
+cudaError_t launch_expert_gemm(const void* in, const void* W, const int32_t* expert_off, const int32_t* expert_cnt,
+                               uint16_t* out, int E, int64_t R, int N, int K, int grid, int32_t* err,
+                               cudaStream_t st, bool w_kn = false, bool accumulate = false);
+cudaError_t launch_gather_tokens(const int32_t* row_pair, const int32_t* counts, int k, int T, const uint16_t* X,
+                                 uint16_t* dst, int64_t R, int cols, cudaStream_t st);
+cudaError_t launch_swiglu(const uint16_t* u, const uint16_t* v, uint16_t* h, int64_t n, cudaStream_t st);
+
 }  // namespace ace
+
+// The plan behind the opaque ace_plan handle (host memory).
+struct ace_plan {
+  ace::PlanTables pt;
+  int32_t T_max;
+  uint32_t flags;
+  int device;
+  int num_sms;  // persistent kernels launch one CTA per SM
+};

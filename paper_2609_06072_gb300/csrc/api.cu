@@ -55,14 +55,6 @@ bool ace::make_tmap_f32(CUtensorMap* m, const void* base, uint64_t rows, uint64_
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-struct ace_plan {
-  PlanTables pt;
-  int32_t T_max;
-  uint32_t flags;
-  int device;
-  int num_sms;  // persistent kernels launch one CTA per SM
-};
-
 namespace {
 
 thread_local char g_msg[512] = "";

@@ -277,6 +277,13 @@ class Layer:
     def dh_base(self) -> np.ndarray:
         return self._normal_bf16("dhbase", (self.cfg.R, self.cfg.f))
 
+    def W_base(self, proj: str) -> np.ndarray:
+        """Frozen base expert weights: gate / up [E, f, d], down [E, d, f],
+        N(0, 1/fan_in) in bf16."""
+        c = self.cfg
+        d_in, d_out = self.dims(proj)
+        return self._normal_bf16(f"Wbase_{proj}", (c.E, d_out, d_in), 1.0 / np.sqrt(d_in))
+
     def dZ(self) -> np.ndarray:
         """Upstream gradient of the gate-weighted combined down output, [T, d]."""
         return self._normal_bf16("dZ", (self.cfg.T, self.cfg.d))

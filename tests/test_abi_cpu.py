@@ -111,3 +111,12 @@ def test_consolidate_adapters_host_checks_without_gpu(lib):
     assert call(np.array([0, 2, 0, 1], np.int32), np.array([0, 1], np.int32), 2) == ace.ACE_ERR_INDEX
     assert call(np.array([0, 0, 0, 0], np.int32), np.array([0, 1], np.int32), 2) == ace.ACE_ERR_INDEX  # empty group
     assert call(e2g, np.array([0, 1], np.int32), 0) == ace.ACE_ERR_SHAPE
+
+
+def test_ffn_null_arguments_without_gpu(lib):
+    from paper_2609_06072_gb300 import ace
+    assert lib.ace_ffn_workspace_size(None, 0, None) == ace.ACE_ERR_ARG
+    assert lib.ace_ffn_fwd(None, None, None, None, None, None, None, None, 1.0, None, None, None, None, None, None,
+                           None, 0, None) == ace.ACE_ERR_ARG
+    assert lib.ace_ffn_bwd(None, None, None, None, None, None, None, None, None, 1.0, None, None, None, None, None,
+                           None, None, None, None, 0, None, 0, None) == ace.ACE_ERR_ARG

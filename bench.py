@@ -505,11 +505,14 @@ def run_gpu(args, rank, world, local):
     dom = "fwd_row"
     achieved = bytes_[dom] / (fwd_row_ms * 1e-3) / 1e9
     traffic = None
+    traffic_sha = None  # kernel sources the stored counters were taken from
+    sources_sha = csrc_sha()
     tf = os.path.join(ROOT, "profiles", "traffic.json")
     if os.path.exists(tf):
         tj = json.load(open(tf))
+        traffic_sha = tj.get("csrc_sha")
         ent = tj.get(f"{args.config}{'_ew' if args.expertwise else ''}{'_det' if args.det else ''}", {}).get(dom)
-        if ent and tj.get("csrc_sha") == csrc_sha():
+        if ent and traffic_sha == sources_sha:
             traffic = ent
     total_bytes = sum(bytes_.values())
     total_flops = sum(flops.values())
@@ -529,6 +532,7 @@ def run_gpu(args, rank, world, local):
         "roofline": {"bound": "hbm", "kernel": SINGLE_KERNEL[dom], "call": dom, "achieved": achieved,
                      "launch_ms": fwd_row_ms, "peak": peaks["hbm_gbs"],
                      "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"], "traffic": traffic,
+                     "traffic_counters_csrc_sha": traffic_sha, "csrc_sha": sources_sha,
                      "algorithmic_bytes": bytes_[dom], "peak_source": peaks["source"]},
         "step_roofline": {"algorithmic_bytes": total_bytes, "algorithmic_flops": total_flops,
                           "achieved_GBps": total_bytes / (ms_per_step * 1e-3) / 1e9,

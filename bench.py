@@ -396,6 +396,80 @@ def time_steps(lay, steps, warmup, flush):
     return float(np.mean([e[0].elapsed_time(e[5]) for e in evs]))
 
 
+def time_expert_ffn(args, lay, flush):
+    """Opt-in (--ffn): the routed expert FFN with frozen base weights and the
+    group-shared adapters, forward and backward (ace_ffn_fwd / ace_ffn_bwd), on
+    the main layer's routing and adapters, with synthetic base weights."""
+    import torch
+    c, p = lay.c, lay.plan
+    gen = torch.Generator().manual_seed(2000 + args.seed)
+    w = lambda *s_, fan: (torch.randn(*s_, generator=gen) / fan ** 0.5).to(torch.bfloat16).cuda()
+    Wg, Wu, Wd = w(c.E, c.f, c.d, fan=c.d), w(c.E, c.f, c.d, fan=c.d), w(c.E, c.d, c.f, fan=c.f)
+    bf = lambda *s_: torch.empty(*s_, dtype=torch.bfloat16, device="cuda")
+    U, V, Hh, Y = bf(c.R, c.f), bf(c.R, c.f), bf(c.R, c.f), bf(c.R, c.d)
+    Hgu = [torch.empty(c.R, p.rank_max, device="cuda") for _ in range(2)]
+    Hd = torch.empty(c.R, p.rank_max, device="cuda")
+    dX = bf(c.T, c.d)
+    ws = p.ffn_workspace(c.T)
+    A, Bt = lay.A, lay.Bt  # gate, up, down
+
+    def step():
+        lay.perm = p.permute(lay.topk, lay.pws)
+        p.ffn_fwd(lay.perm, lay.X, Wg, Wu, Wd, A, Bt, c.s, U, V, Hh, Y, Hgu, Hd, ws)
+        p.ffn_bwd(lay.perm, lay.dY[2], lay.X, Wg, Wu, Wd, A, Bt, c.s, U, V, Hh, Hgu, Hd, dX, lay.dA, lay.dBt, ws,
+                  lay.bws)
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    for e0, e1 in ev:
+        flush()
+        e0.record()
+        step()
+        e1.record()
+    torch.cuda.synchronize()
+    assert p.get_error(lay.perm) == 0
+    ms = float(np.mean([a.elapsed_time(b) for a, b in ev]))
+    flops = 2 * (2 * c.R * c.d * 2 * c.f + 2 * c.R * c.f * c.d)  # base GEMMs, forward + input gradients
+    return {"ms_per_step": ms, "value": c.R / (ms * 1e-3), "unit": UNIT,
+            "base_tflops": flops / (ms * 1e-3) / 1e12, "note": "composed (unfused) base + adapter layer step"}
+
+
+def time_cka(args, lay):
+    """Opt-in (--cka): rank consolidation of the gate projection -- the CKA
+    matrix of the expert-wise adapters (rank r each) on a 10 000-token probe
+    (ace_cka), then the grouping on the host (ace_group_experts)."""
+    import time as _time
+    import torch
+    from paper_2609_06072_gb300 import ace
+    c = lay.c
+    gen = torch.Generator().manual_seed(3000 + args.seed)
+    N = 10000
+    X = torch.randn(N, c.d, generator=gen).to(torch.bfloat16).cuda()
+    A = ((torch.rand(c.E * c.r, c.d, generator=gen) * 2 - 1) / c.d ** 0.5).to(torch.bfloat16).cuda()
+    Bt = (torch.randn(c.E * c.r, c.f, generator=gen) * 0.02).to(torch.bfloat16).cuda()
+    S = torch.empty(c.E, c.E, device="cuda")
+    nb = ace.ctypes.c_size_t()
+    ace._check(ace.load().ace_cka_workspace_size(N, c.d, c.f, c.E, c.r, ace.ctypes.byref(nb)), "workspace")
+    ws = torch.empty(nb.value, dtype=torch.uint8, device="cuda")
+    for _ in range(args.warmup):
+        ace.cka(X, A, Bt, c.E, c.r, S=S, ws=ws)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(args.steps):
+        ace.cka(X, A, Bt, c.E, c.r, S=S, ws=ws)
+    e1.record()
+    torch.cuda.synchronize()
+    cka_ms = e0.elapsed_time(e1) / args.steps
+    S_host = S.cpu().numpy()
+    t0 = _time.perf_counter()
+    _, _, G = ace.group_experts(S_host, ace.GROUP_LOUVAIN, 0.8)
+    group_ms = (_time.perf_counter() - t0) * 1e3
+    return {"cka_ms": cka_ms, "grouping_ms_host": group_ms, "groups": int(G), "probe_tokens": N,
+            "experts": c.E, "rank": c.r, "d_in": c.d, "d_out": c.f}
+
+
 def run_variants(args, flush, main_layer):
     """The other timings of the same workload: the expert-wise layout at the
     matched adapter budget, the deterministic split-K mode, and no L2 flush."""
@@ -549,6 +623,10 @@ def run_gpu(args, rank, world, local):
     }
     if not args.no_variants:
         out["variants"] = run_variants(args, flush, lay)
+    if args.ffn:
+        out.setdefault("variants", {})["expert_ffn_composed"] = time_expert_ffn(args, lay, flush)
+    if args.cka:
+        out["consolidation"] = time_cka(args, lay)
     return out, lay
 
 
@@ -691,6 +769,10 @@ def main():
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU-oracle baseline leg")
     ap.add_argument("--combine", action="store_true",
                     help="also time the step with down through the gate-weighted combine (a variant)")
+    ap.add_argument("--ffn", action="store_true",
+                    help="also time the routed expert FFN with base weights and adapters, forward and backward")
+    ap.add_argument("--cka", action="store_true",
+                    help="also time rank consolidation: the CKA matrix on a 10k-token probe and the grouping")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-variants", action="store_true",
                     help="skip the expert-wise, deterministic-mode and unflushed timings")

@@ -16,6 +16,12 @@
  *   App. "Implementation and Profiling of Grouped Adapter Execution":
  *             gate/up take x, down takes the expert-specific h_e
  *
+ * Beyond that path: the down delta taken through the router's gate-weighted
+ * combine (ace_fwd_combine / ace_bwd_combine); rank consolidation, the step
+ * that produces the expert -> group map (ace_cka, ace_group_experts,
+ * ace_consolidate_adapters); and the routed expert FFN with frozen base
+ * weights and the adapters together (ace_ffn_fwd / ace_ffn_bwd).
+ *
  * Terms used below.  T tokens, top-k routing, pair p = t*k + j (token t,
  * slot j), R = T*k pairs.  E experts, G groups, e2g the expert->group map,
  * rank_off[G+1] the packed rank offsets (r_g = rank_off[g+1] - rank_off[g]).

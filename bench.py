@@ -491,6 +491,18 @@ def run_variants(args, flush, main_layer):
         out["down_via_gate_weighted_combine"] = {"value": c_rows / (ms * 1e-3), "ms_per_step": ms,
                                                  "kernels_per_step": lay.kernels_per_step()}
         del lay
+        if not args.no_cpu:
+            # the oracle of the same step on a bounded sample, beside it
+            os.environ.setdefault("OMP_NUM_THREADS", str(cpu_cores()))
+            f1, f2 = 1.0 / 1024, 1.0 / 256
+            t1, _ = combine_oracle_sample(args.config, args.seed, f1)
+            t2, _ = combine_oracle_sample(args.config, args.seed, f2)
+            slope = max((t2 - t1) / (f2 - f1), 1e-6)
+            frac = float(min(1.0, max(f1, (min(args.cpu_seconds, 10.0) - max(t1 - slope * f1, 0.0)) / slope)))
+            dt, rows = combine_oracle_sample(args.config, args.seed, frac)
+            out["down_via_gate_weighted_combine"]["cpu_baseline"] = {
+                "value": rows / dt, "unit": UNIT, "cores": int(os.environ["OMP_NUM_THREADS"]), "kind": "oracle",
+                "sample": f"permutation plus {frac:.4f} of the pairs, tokens and rank rows; {dt:.1f} s"}
     return out
 
 
@@ -631,6 +643,39 @@ def run_gpu(args, rank, world, local):
 
 
 # ------------------------------------------------------------------ CPU oracle
+def combine_oracle_sample(cfg_name, seed, frac, rng_seed=0):
+    """The oracle on a sample of the step with down through the gate-weighted
+    combine: gate/up as in oracle_sample, and for down the combined output of
+    a fraction of the tokens, dh and the gate-weight gradient of that fraction
+    of the pairs and dA / dB^T of that fraction of the rank rows.  Returns
+    (seconds, sampled rows)."""
+    import oracle
+    from paper_2609_06072_gb300 import workloads as W
+    L = W.Layer(W.get_config(cfg_name), seed=seed)
+    c = L.cfg
+    rng = np.random.default_rng(rng_seed)
+    n_p = max(1, int(round(frac * c.R)))
+    n_t = max(1, int(round(frac * c.T)))
+    n_r = max(1, int(round(frac * int(L.rank_off[-1]))))
+    sel_p = np.sort(rng.choice(c.R, n_p, replace=False)).astype(np.int32)
+    sel_t = np.sort(rng.choice(c.T, n_t, replace=False)).astype(np.int32)
+    sel_r = np.sort(rng.choice(int(L.rank_off[-1]), n_r, replace=False)).astype(np.int32)
+    X, h, w, dZ = L.X(), L.h(), L.topk_w, L.dZ()
+    A = {p: L.A(p) for p in ("gate", "up", "down")}
+    Bt = {p: L.Bt(p) for p in ("gate", "up", "down")}
+    dY = {p: L.dY(p) for p in ("gate", "up")}
+    t0 = time.perf_counter()
+    oracle.permute(L.topk_idx, L.e2g, L.G)
+    for p in ("gate", "up"):
+        oracle.fwd(L.topk_idx, L.e2g, L.rank_off, X, A[p], Bt[p], c.s, sel=sel_p)
+        oracle.bwd_dx(L.topk_idx, L.e2g, L.rank_off, dY[p], A[p], Bt[p], c.s, sel=sel_t)
+        oracle.bwd_w(L.topk_idx, L.e2g, L.rank_off, X, dY[p], A[p], Bt[p], c.s, sel=sel_r)
+    oracle.combine_fwd(L.topk_idx, L.e2g, L.rank_off, h, w, A["down"], Bt["down"], c.s, sel=sel_t)
+    oracle.combine_bwd_dh(L.topk_idx, L.e2g, L.rank_off, dZ, h, w, A["down"], Bt["down"], c.s, sel=sel_p)
+    oracle.combine_bwd_w(L.topk_idx, L.e2g, L.rank_off, h, dZ, w, A["down"], Bt["down"], c.s, sel=sel_r)
+    return time.perf_counter() - t0, frac * c.R
+
+
 def oracle_sample(cfg_name, seed, expertwise, frac, rng_seed=0):
     """Time the fp64 oracle on a sample of one step: the full permutation, the
     forward of a fraction `frac` of the pairs, input gradients of the same

@@ -63,3 +63,11 @@ def test_source_hash_ignores_comments(tmp_path, monkeypatch):
     assert bench.csrc_sha() == h0
     (src / "a.cu").write_text("int f() { return 2; }\n")
     assert bench.csrc_sha() != h0
+
+
+def test_combine_oracle_sample_runs_on_cpu():
+    """The CPU baseline beside the combine variant: every oracle call of the
+    sample accepts its selections (no GPU needed)."""
+    dt, rows = bench.combine_oracle_sample("tiny", 0, 0.25)
+    c = W.get_config("tiny")
+    assert dt > 0 and abs(rows - 0.25 * c.R) < 1e-9

@@ -636,9 +636,22 @@ def run_gpu(args, rank, world, local):
     if not args.no_variants:
         out["variants"] = run_variants(args, flush, lay)
     if args.ffn:
-        out.setdefault("variants", {})["expert_ffn_composed"] = time_expert_ffn(args, lay, flush)
+        ffn = time_expert_ffn(args, lay, flush)
+        if not args.no_cpu:
+            dt, rows = ffn_oracle_sample(args.config, args.seed, 4)
+            ffn["cpu_baseline"] = {"value": rows / dt, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+                                   "sample": f"4 tokens ({int(rows)} rows), forward and backward; {dt:.1f} s"}
+        out.setdefault("variants", {})["expert_ffn_composed"] = ffn
     if args.cka:
-        out["consolidation"] = time_cka(args, lay)
+        cons = time_cka(args, lay)
+        if not args.no_cpu:
+            n = 4
+            dt, _ = cka_oracle_sample(args.config, args.seed, n)
+            cons["cpu_baseline"] = {"value": dt / n * lay.c.E ** 2 * 1e3, "unit": "ms per CKA matrix (estimated)",
+                                    "cores": cpu_cores(), "kind": "oracle",
+                                    "sample": f"{n} expert pairs by the definition on the 10k probe, "
+                                              f"scaled to {lay.c.E}^2 pairs; {dt:.1f} s"}
+        out["consolidation"] = cons
     return out, lay
 
 
@@ -674,6 +687,56 @@ def combine_oracle_sample(cfg_name, seed, frac, rng_seed=0):
     oracle.combine_bwd_dh(L.topk_idx, L.e2g, L.rank_off, dZ, h, w, A["down"], Bt["down"], c.s, sel=sel_p)
     oracle.combine_bwd_w(L.topk_idx, L.e2g, L.rank_off, h, dZ, w, A["down"], Bt["down"], c.s, sel=sel_r)
     return time.perf_counter() - t0, frac * c.R
+
+
+def ffn_oracle_sample(cfg_name, seed, n_tokens, rng_seed=0):
+    """The expert-FFN oracle (forward and backward, frozen base weights) on
+    n_tokens sampled tokens of the layer (all their pairs).  Returns
+    (seconds, sampled rows)."""
+    from oracle import ffn as F
+    from paper_2609_06072_gb300 import workloads as W
+    L = W.Layer(W.get_config(cfg_name), seed=seed)
+    c = L.cfg
+    rng = np.random.default_rng(rng_seed)
+    toks = np.sort(rng.choice(c.T, n_tokens, replace=False))
+    dec = lambda b: W.bf16_bits_to_f32(b).astype(np.float64)
+    projs = ("gate", "up", "down")
+    # only the experts the sampled tokens route to, renumbered compactly, with
+    # base weights of the same distribution drawn for them alone (the timing
+    # does not depend on their values)
+    used, idx = np.unique(L.topk_idx[toks], return_inverse=True)
+    idx = idx.reshape(n_tokens, c.k).astype(np.int32)
+    maps = {q: (L.e2g[used], L.rank_off) for q in projs}
+    shapes = {"gate": (c.f, c.d), "up": (c.f, c.d), "down": (c.d, c.f)}
+    Wb = {q: rng.standard_normal((len(used),) + shapes[q]) / np.sqrt(shapes[q][1]) for q in projs}
+    A = {q: dec(L.A(q)) for q in projs}
+    Bt = {q: dec(L.Bt(q)) for q in projs}
+    X = dec(L.X())[toks]
+    dy = dec(L.dY("down")).reshape(c.T, c.k, c.d)[toks].reshape(-1, c.d)
+    t0 = time.perf_counter()
+    F.ffn_fwd(idx, maps, X, Wb, A, Bt, c.s)
+    F.ffn_bwd(idx, maps, X, Wb, A, Bt, c.s, dy=dy)
+    return time.perf_counter() - t0, n_tokens * c.k
+
+
+def cka_oracle_sample(cfg_name, seed, n_pairs, rng_seed=0):
+    """Linear CKA by its definition (explicit representation matrices on a
+    10 000-token probe) for n_pairs sampled expert pairs of the gate
+    projection.  Returns (seconds, pairs)."""
+    from oracle import consolidation as C
+    from paper_2609_06072_gb300 import workloads as W
+    L = W.Layer(W.get_config(cfg_name), seed=seed, expertwise=True)
+    c = L.cfg
+    rng = np.random.default_rng(rng_seed)
+    X = W.f32_to_bf16_bits(rng.standard_normal((10000, c.d)).astype(np.float32))
+    A, Bt = L.A("gate"), L.Bt("gate")
+    pairs = rng.integers(0, c.E, (n_pairs, 2))
+    t0 = time.perf_counter()
+    for i, j in pairs:
+        Zi, Zj = C.adapter_outputs(X, [A[i * c.r:(i + 1) * c.r], A[j * c.r:(j + 1) * c.r]],
+                                   [Bt[i * c.r:(i + 1) * c.r], Bt[j * c.r:(j + 1) * c.r]])
+        C.cka(Zi, Zj)
+    return time.perf_counter() - t0, n_pairs
 
 
 def oracle_sample(cfg_name, seed, expertwise, frac, rng_seed=0):

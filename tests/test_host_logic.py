@@ -71,3 +71,10 @@ def test_combine_oracle_sample_runs_on_cpu():
     dt, rows = bench.combine_oracle_sample("tiny", 0, 0.25)
     c = W.get_config("tiny")
     assert dt > 0 and abs(rows - 0.25 * c.R) < 1e-9
+
+
+def test_ffn_and_cka_oracle_samples_run_on_cpu():
+    dt, rows = bench.ffn_oracle_sample("tiny", 0, 4)
+    assert dt > 0 and rows == 4 * W.get_config("tiny").k
+    dt, n = bench.cka_oracle_sample("tiny", 0, 2)
+    assert dt > 0 and n == 2

@@ -56,3 +56,28 @@ def test_cka_olmoe_probe_sampled_pairs():
         Zi, Zj = C.adapter_outputs(X, [A[i * r:(i + 1) * r], A[j * r:(j + 1) * r]],
                                    [Bt[i * r:(i + 1) * r], Bt[j * r:(j + 1) * r]])
         assert abs(S[i, j] - C.cka(Zi, Zj)) <= 2e-3, (i, j)
+
+
+def test_consolidation_pipeline_against_oracle():
+    """Probe -> CKA -> Louvain groups and anchors -> shared adapters: the
+    library's result equals the oracle's consolidation of the same grouping
+    bit for bit (a copy), with the budget kept."""
+    import torch
+    from paper_2609_06072_gb300 import ace
+    rng = np.random.default_rng(5)
+    E, N, d_in, d_out, r = 16, 1500, 128, 96, 4
+    X, A, Bt, proto = planted(rng, E, N, d_in, d_out, r, 4, 0.2)
+    A_init = bits(rng.standard_normal((E * r, d_in)) / np.sqrt(d_in))
+    e2g, rank_off, A_g, Bt_g, S = ace.consolidate(dev_bf16(X), dev_bf16(A), dev_bf16(Bt), E, r, dev_bf16(A_init))
+    torch.cuda.synchronize()
+    Sd = S.astype(np.float64)
+    labels = C.louvain(C.similarity_graph(Sd), 0.8)
+    assert np.array_equal(e2g, labels) and np.array_equal(labels, C._relabel(proto))
+    anchors = C.cka_center_anchor(Sd, labels)
+    _, ro, rA, rB = C.consolidate(labels, [r] * E, anchors, [A[e * r:(e + 1) * r] for e in range(E)],
+                                  [Bt[e * r:(e + 1) * r] for e in range(E)],
+                                  W.bf16_bits_to_f32(A_init).astype(np.float64))
+    assert np.array_equal(rank_off, ro) and rank_off[-1] == E * r
+    got_A = W.bf16_bits_to_f32(A_g.view(torch.int16).cpu().numpy().view(np.uint16)).astype(np.float64)
+    got_B = W.bf16_bits_to_f32(Bt_g.view(torch.int16).cpu().numpy().view(np.uint16)).astype(np.float64)
+    assert np.array_equal(got_A, rA) and np.array_equal(got_B, rB)

@@ -1,0 +1,94 @@
+"""GPU parity of the routed expert FFN forward with the group-shared
+adapters (base expert GEMMs, adapter deltas, SiLU gating) against the FFN
+oracle.  The composed path rounds u, v, h and y to bf16 between its steps
+(two roundings on u and v, whose base part is stored before the adapter
+delta is added), so the bar is a relative Frobenius error of 1e-2 and a
+maximum error of 3e-2 of the largest reference value."""
+import numpy as np
+import pytest
+
+import oracle
+from oracle import ffn as F
+from paper_2609_06072_gb300 import workloads as W
+from ace_testlib import check_close, dev_bf16, host_f64
+from test_gpu_fwd import compare_perm, make_plan, run_perm
+
+pytestmark = pytest.mark.gpu
+
+
+def _dec(b):
+    return W.bf16_bits_to_f32(b).astype(np.float64)
+
+
+# the OLMoE-shaped routing and groupings at a reduced hidden / expert width,
+# so that the oracle's base weights stay small
+@pytest.mark.parametrize("name,seed,over", [("tiny", 0, {}), ("tiny", 1, {"T": 300}),
+                                            ("olmoe", 0, {"T": 256, "d": 512, "f": 256}),
+                                            ("olmoe_uneven", 0, {"T": 128, "d": 512, "f": 256})])
+def test_ffn_forward_parity(name, seed, over):
+    import torch
+    L = W.Layer(W.get_config(name, **over), seed=seed)
+    c = L.cfg
+    plan = make_plan(L)
+    perm, P = run_perm(L, plan)
+    O = oracle.permute(L.topk_idx, L.e2g, L.G)
+    compare_perm(P, O)
+    rp = O["row_pair"]
+    projs = ("gate", "up", "down")
+    Wb = {q: L.W_base(q) for q in projs}
+    A = [dev_bf16(L.A(q)) for q in projs]
+    Bt = [dev_bf16(L.Bt(q)) for q in projs]
+    X = dev_bf16(L.X())
+    bf = lambda *s: torch.empty(*s, dtype=torch.bfloat16, device="cuda")
+    U, V, Hh, Y = bf(c.R, c.f), bf(c.R, c.f), bf(c.R, c.f), bf(c.R, c.d)
+    Hgu = [torch.empty(c.R, plan.rank_max, device="cuda") for _ in range(2)]
+    Hd = torch.empty(c.R, plan.rank_max, device="cuda")
+    plan.ffn_fwd(perm, X, dev_bf16(Wb["gate"]), dev_bf16(Wb["up"]), dev_bf16(Wb["down"]), A, Bt, c.s, U, V, Hh, Y,
+                 Hgu, Hd, plan.ffn_workspace(c.T))
+    assert plan.get_error(perm) == 0
+    maps = {q: (L.e2g, L.rank_off) for q in projs}
+    ref = F.ffn_fwd(L.topk_idx, maps, _dec(L.X()), {q: _dec(Wb[q]) for q in projs},
+                    {q: _dec(L.A(q)) for q in projs}, {q: _dec(L.Bt(q)) for q in projs}, c.s)
+    for name_, t in (("u", U), ("v", V), ("h", Hh), ("y", Y)):
+        got = np.empty_like(ref[name_])
+        got[rp] = host_f64(t)
+        check_close(got, ref[name_], name_, max_rel=3e-2, fro_rel=1e-2)
+
+
+@pytest.mark.parametrize("name,seed,over", [("tiny", 0, {}), ("tiny", 4, {"r": 3}),
+                                            ("olmoe_uneven", 0, {"T": 128, "d": 512, "f": 256})])
+def test_ffn_backward_parity(name, seed, over):
+    import torch
+    L = W.Layer(W.get_config(name, **over), seed=seed)
+    c = L.cfg
+    plan = make_plan(L)
+    perm, P = run_perm(L, plan)
+    rp = oracle.permute(L.topk_idx, L.e2g, L.G)["row_pair"]
+    projs = ("gate", "up", "down")
+    Wb = {q: L.W_base(q) for q in projs}
+    Wd = {q: dev_bf16(Wb[q]) for q in projs}
+    A = [dev_bf16(L.A(q)) for q in projs]
+    Bt = [dev_bf16(L.Bt(q)) for q in projs]
+    X = dev_bf16(L.X())
+    bf = lambda *s: torch.empty(*s, dtype=torch.bfloat16, device="cuda")
+    U, V, Hh, Y = bf(c.R, c.f), bf(c.R, c.f), bf(c.R, c.f), bf(c.R, c.d)
+    Hgu = [torch.empty(c.R, plan.rank_max, device="cuda") for _ in range(2)]
+    Hd = torch.empty(c.R, plan.rank_max, device="cuda")
+    ws = plan.ffn_workspace(c.T)
+    plan.ffn_fwd(perm, X, Wd["gate"], Wd["up"], Wd["down"], A, Bt, c.s, U, V, Hh, Y, Hgu, Hd, ws)
+    dY_pairs = L.dY("down")  # [R, d] per pair
+    dY = dev_bf16(dY_pairs[rp])
+    dX = bf(c.T, c.d)
+    nan = lambda *s: torch.full(s, float("nan"), device="cuda")
+    dA = [nan(plan.n_rank, c.d), nan(plan.n_rank, c.d), nan(plan.n_rank, c.f)]
+    dBt = [nan(plan.n_rank, c.f), nan(plan.n_rank, c.f), nan(plan.n_rank, c.d)]
+    _, _, bws = plan.alloc_workspaces(c.T)
+    plan.ffn_bwd(perm, dY, X, Wd["gate"], Wd["up"], Wd["down"], A, Bt, c.s, U, V, Hh, Hgu, Hd, dX, dA, dBt, ws, bws)
+    assert plan.get_error(perm) == 0
+    maps = {q: (L.e2g, L.rank_off) for q in projs}
+    ref = F.ffn_bwd(L.topk_idx, maps, _dec(L.X()), {q: _dec(Wb[q]) for q in projs}, {q: _dec(L.A(q)) for q in projs},
+                    {q: _dec(L.Bt(q)) for q in projs}, c.s, dy=_dec(dY_pairs))
+    check_close(host_f64(dX), ref["dX"], "dX", max_rel=3e-2, fro_rel=1e-2)
+    for j, q in enumerate(projs):
+        check_close(host_f64(dA[j]), ref["dA"][q], f"dA_{q}", max_rel=3e-2, fro_rel=1e-2)
+        check_close(host_f64(dBt[j]), ref["dBt"][q], f"dBt_{q}", max_rel=3e-2, fro_rel=1e-2)

@@ -84,8 +84,6 @@ ace_status cuda_status(cudaError_t e, const char* what) {
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-// Row tiles per backward split: (tiles + 2) * rank_pad TMEM columns <= 256.
-
 ace_status check_perm(const ace_plan* plan, const ace_perm* perm) {
   if (!plan || !perm || !perm->ws) return fail(ACE_ERR_ARG, "null plan or perm");
   if (perm->T < 0 || perm->T > plan->T_max) return fail(ACE_ERR_SHAPE, "perm T=%d outside [0, %d]", perm->T, plan->T_max);
@@ -93,7 +91,12 @@ ace_status check_perm(const ace_plan* plan, const ace_perm* perm) {
   return ACE_OK;
 }
 
+// Row tiles per backward split.  A split's dH accumulators (tiles x rank_pad
+// TMEM columns) sit below its double-buffered weight-gradient accumulators
+// (2 x rank_pad); down also keeps 128 columns of dh buffers, so at rank_pad
+// 128 down takes one tile per split and gate/up two.
 int pt_nt_split(int rank_pad) { return rank_pad <= 64 ? 4 : 1; }
+int pt_nt_split_sh(int rank_pad) { return rank_pad <= 64 ? 4 : 2; }
 
 struct BwdWs {
   float* dHrow[2];
@@ -113,7 +116,8 @@ BwdWs bwd_layout(const ace_plan* plan, int32_t T, void* base) {
   const PermLayout L = perm_layout(pt, T);
   const int64_t R = (int64_t)T * pt.k;
   const size_t dhrow = align_up(4 * (size_t)R * pt.rank_pad, 256);
-  const size_t pa = align_up(4 * (size_t)L.max_splits * pt.rank_pad * (size_t)(pt.d > pt.f ? pt.d : pt.f), 256);
+  const size_t n_part = (size_t)(L.max_splits > L.max_splits_sh ? L.max_splits : L.max_splits_sh);
+  const size_t pa = align_up(4 * n_part * pt.rank_pad * (size_t)(pt.d > pt.f ? pt.d : pt.f), 256);
   BwdWs w{};
   char* b = static_cast<char*>(base);
   size_t off = 0;
@@ -193,6 +197,7 @@ ace_status ace_plan_create(ace_plan** out, const ace_layer_desc* desc) {
   p->pt.rank_max = rank_max;
   p->pt.rank_pad = rank_max <= 16 ? 16 : rank_max <= 32 ? 32 : rank_max <= 64 ? 64 : 128;
   p->pt.nt_split = pt_nt_split(p->pt.rank_pad);
+  p->pt.nt_split_sh = pt_nt_split_sh(p->pt.rank_pad);
   p->pt.nsm = num_sms;
   for (int e = 0; e < D.E; ++e) p->pt.e2g[e] = (int16_t)D.e2g[e];
   {
@@ -413,9 +418,11 @@ ace_status ace_bwd_shared(const ace_plan* plan, const ace_perm* perm, int32_t np
   }
   if (perm->R > 0 && !ok) return fail(ACE_ERR_UNSUPPORTED, "tensor-map encoding failed for this layout");
   a.splits_row = at<Tile>(perm->ws, L.splits_row);
+  a.splits_sh = at<Tile>(perm->ws, L.splits_sh);
   a.tiles_sh = at<Tile>(perm->ws, L.tiles_sh);
   a.counts = perm->counts;
   a.max_splits_row = L.max_splits;
+  a.max_splits_sh = L.max_splits_sh;
   a.max_tiles_sh = L.max_tiles;
   a.uniq_tok = perm->uniq_tok;
   a.uniq_off = perm->uniq_off;
@@ -497,9 +504,11 @@ ace_status ace_bwd_row(const ace_plan* plan, const ace_perm* perm, const uint16_
   a.tm_dy[1] = a.tm_dy[0];
   a.tm_bt[1] = a.tm_bt[0];
   a.splits_row = at<Tile>(perm->ws, L.splits_row);
+  a.splits_sh = at<Tile>(perm->ws, L.splits_sh);
   a.tiles_sh = at<Tile>(perm->ws, L.tiles_sh);
   a.counts = perm->counts;
   a.max_splits_row = L.max_splits;
+  a.max_splits_sh = L.max_splits_sh;
   a.max_tiles_sh = L.max_tiles;
   a.uniq_tok = perm->uniq_tok;
   a.uniq_off = perm->uniq_off;
@@ -660,9 +669,11 @@ ace_status ace_bwd_combine(const ace_plan* plan, const ace_perm* perm, const uin
     if (st != ACE_OK) return st;
   }
   a.splits_row = at<Tile>(perm->ws, L.splits_row);
+  a.splits_sh = at<Tile>(perm->ws, L.splits_sh);
   a.tiles_sh = at<Tile>(perm->ws, L.tiles_sh);
   a.counts = perm->counts;
   a.max_splits_row = L.max_splits;
+  a.max_splits_sh = L.max_splits_sh;
   a.max_tiles_sh = L.max_tiles;
   a.uniq_tok = perm->uniq_tok;
   a.uniq_off = perm->uniq_off;

@@ -123,7 +123,10 @@ __device__ __forceinline__ void flush_wgrad(uint32_t taddr, int n0, int ld, int 
 // ----------------------------------------------------------------- k_bwd_rows
 template <int RP, int MODE>
 struct RowsCfg {
-  static constexpr int NT = RP <= 64 ? 4 : 1;
+  // row tiles per split: the split's dH accumulators (NT x RP TMEM columns)
+  // sit below the weight-gradient accumulators (2 x RP from kTB); gate/up
+  // needs no phase-2 buffers, so at RP = 128 two tiles fill the 512 columns
+  static constexpr int NT = RP <= 64 ? 4 : (MODE == MODE_SHARED ? 2 : 1);
   static constexpr int kOps = Slots<RP>::bytes(NT);
   static constexpr int kWBlk = RP * 128;
   static constexpr int kSlotA = 2 * kBlk + 2 * kWBlk;  // dY tile + B^T chunk (down phase 2: A chunk + h tile)
@@ -157,10 +160,10 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
   static_assert(NT * RP <= C::kTB, "dH accumulators must fit below the dB^T columns");
 
   pdl_wait();
-  const int n_splits = a.counts[kCntSplitsRow];
+  const int n_splits = a.counts[MODE == MODE_SHARED ? kCntSplitsSh : kCntSplitsRow];
   if ((int)blockIdx.x >= n_splits) return;
   const int proj = blockIdx.y;
-  const Tile sp = a.splits_row[blockIdx.x];
+  const Tile sp = (MODE == MODE_SHARED ? a.splits_sh : a.splits_row)[blockIdx.x];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = sp.g, r0 = pt.rank_off[g], rg = pt.rank_off[g + 1] - r0;
   const int ntiles = (sp.cnt + kTileM - 1) / kTileM;
@@ -614,7 +617,8 @@ cudaError_t launch_rows(const PlanTables& pt, const BwdLaunch& a, int nproj, cud
   auto kern = k_bwd_rows<RP, MODE>;
   cudaError_t e = set_smem(kern, C::kSmem);
   if (e != cudaSuccess) return e;
-  return launch_k(kern, dim3(a.max_splits_row, nproj), kThreadsWS, C::kSmem, st, pt, a);
+  const int grid = MODE == MODE_SHARED ? a.max_splits_sh : a.max_splits_row;
+  return launch_k(kern, dim3(grid, nproj), kThreadsWS, C::kSmem, st, pt, a);
 }
 
 // Combine backward: one launch zeroes dB^T (the dense dA GEMM of gemm.cu
@@ -666,10 +670,12 @@ cudaError_t launch_bwd_t(const PlanTables& pt, const BwdLaunch& a, bool shared, 
       return e;
   }
   if (a.deterministic) {
+    const Tile* splits = shared ? a.splits_sh : a.splits_row;
+    const int slot = shared ? kCntSplitsSh : kCntSplitsRow;
     for (int j = 0; j < nproj; ++j) {
       dim3 grid(n_rank, (a.d_out / 4 + 255) / 256);
-      if ((e = launch_k(k_splitk_reduce, grid, 256, 0, st, pt, a.splits_row, a.counts, kCntSplitsRow, a.part_dBt[j],
-                        (int)RP, a.d_out, a.dBt[j])) != cudaSuccess)
+      if ((e = launch_k(k_splitk_reduce, grid, 256, 0, st, pt, splits, a.counts, slot, a.part_dBt[j], (int)RP,
+                        a.d_out, a.dBt[j])) != cudaSuccess)
         return e;
     }
     if (!shared) {

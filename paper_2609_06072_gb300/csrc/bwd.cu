@@ -171,6 +171,10 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
   const int nch1 = MODE == MODE_COMB ? 0 : (d_out + kNcB - 1) / kNcB;
   const int nch2 = MODE != MODE_SHARED ? (d_in + kNcB - 1) / kNcB : 0;
   const int NI1 = nch1 * ntiles, NI2 = nch2 * ntiles;
+  // Each split walks the column chunks starting at its own offset, so the
+  // splits of one group that run at the same time flush their weight
+  // gradients into different columns (fewer same-address atomics in L2).
+  auto chunk_col = [&](int c, int nch) { return ((c + sp.id) % nch) * kNcB; };
   const uint32_t sOps = smem_u32(smem);
   const uint32_t sA0 = sOps + C::kOps;
   const uint32_t sB0 = sA0 + SA * C::kSlotA;
@@ -223,14 +227,14 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
         }
         const uint32_t base = sA0 + s * C::kSlotA;
         if (q < NI1) {
-          const int c = q / ntiles, i = q % ntiles, n0 = c * kNcB, row0 = sp.start + i * kTileM;
+          const int c = q / ntiles, i = q % ntiles, n0 = chunk_col(c, nch1), row0 = sp.start + i * kTileM;
           mbar_arrive_expect_tx(&fullA[s], 2 * kBlk + 2 * C::kWBlk);
           tma_load_2d(base, &a.tm_dy[proj], n0, row0, &fullA[s]);
           tma_load_2d(base + kBlk, &a.tm_dy[proj], n0 + 64, row0, &fullA[s]);
           tma_load_2d(base + 2 * kBlk, &a.tm_bt[proj], n0, r0, &fullA[s]);
           tma_load_2d(base + 2 * kBlk + C::kWBlk, &a.tm_bt[proj], n0 + 64, r0, &fullA[s]);
         } else {
-          const int j = q - NI1, c = j / ntiles, i = j % ntiles, n0 = c * kNcB, row0 = sp.start + i * kTileM;
+          const int j = q - NI1, c = j / ntiles, i = j % ntiles, n0 = chunk_col(c, nch2), row0 = sp.start + i * kTileM;
           mbar_arrive_expect_tx(&fullA[s], 2 * C::kWBlk + 2 * kBlk);
           tma_load_2d(base, &a.tm_a, n0, r0, &fullA[s]);
           tma_load_2d(base + C::kWBlk, &a.tm_a, n0 + 64, r0, &fullA[s]);
@@ -396,7 +400,7 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
       ok = named_bar_and(kEpiBar, kEpiThreads, mbar_wait(&dbt_full[c & 1], (c >> 1) & 1));
       if (!ok) break;
       tc_fence_after();
-      flush_wgrad<RP>(tmem + lane_base + C::kTB + (c & 1) * RP, c * kNcB, d_out, rg, r0, a.s, fmode,
+      flush_wgrad<RP>(tmem + lane_base + C::kTB + (c & 1) * RP, chunk_col(c, nch1), d_out, rg, r0, a.s, fmode,
                       a.part_dBt[proj], sp.id, a.dBt[proj], m, false, ehalf * 16, 32);
       tc_fence_before();
       named_bar(kEpiBar, kEpiThreads);
@@ -456,7 +460,7 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
     }
     if (MODE != MODE_SHARED) {
       for (int j = 0; j < NI2 && ok; ++j) {
-        const int c = j / ntiles, i = j % ntiles, b = j % C::ND, sb = j % SB, n0 = c * kNcB;
+        const int c = j / ntiles, i = j % ntiles, b = j % C::ND, sb = j % SB, n0 = chunk_col(c, nch2);
         bool w_ok = mbar_wait(&fullB[sb], (j / SB) & 1);
         w_ok = w_ok && mbar_wait(&d_full[b], (j / C::ND) & 1);
         ok = named_bar_and(kEpiBar, kEpiThreads, w_ok);

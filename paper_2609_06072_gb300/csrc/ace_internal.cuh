@@ -16,6 +16,7 @@ constexpr int kMaxK = 32;          // largest top-k the kernels accept
 // Device error-flag bits (the flag lives at perm workspace word 0).
 constexpr int kErrIndex = 1;
 constexpr int kErrTimeout = 2;
+constexpr int kErrValue = 4;  // a non-finite gate weight reached the combine
 
 // Plan tables passed by value (__grid_constant__) to every kernel.
 struct PlanTables {
@@ -280,6 +281,7 @@ struct CombReduceLaunch {
   uint16_t* Hx;            // [T, n_rank_pad] bf16 out
   float s;
   int32_t T, n_rank_pad;
+  int32_t* err;            // device error flag (kErrValue on a non-finite gate weight)
 };
 cudaError_t launch_comb_reduce(const PlanTables& pt, const CombReduceLaunch& a, cudaStream_t st);
 

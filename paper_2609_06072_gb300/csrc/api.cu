@@ -583,6 +583,7 @@ ace_status ace_fwd_combine(const ace_plan* plan, const ace_perm* perm, const uin
   c.s = s;
   c.T = perm->T;
   c.n_rank_pad = nrp;
+  c.err = err;
   st = cuda_status(launch_comb_reduce(pt, c, cs), "combine reduce launch");
   if (st != ACE_OK) return st;
   x.tm_acat[1] = x.tm_acat[0];
@@ -749,6 +750,7 @@ ace_status ace_get_error(const ace_perm* perm, void* stream) {
   if (s != ACE_OK) return s;
   if (flag & kErrTimeout) return fail(ACE_ERR_DEVICE_TIMEOUT, "a bounded device wait gave up");
   if (flag & kErrIndex) return fail(ACE_ERR_INDEX, "invalid routing: expert id out of range or repeated in a token");
+  if (flag & kErrValue) return fail(ACE_ERR_ARG, "a gate weight given to the combine is not finite");
   return ACE_OK;
 }
 

@@ -270,8 +270,8 @@ static ace_status fwd_common(const ace_plan* plan, const ace_perm* perm, const u
   if (perm->R > 0 && !X) return fail(ACE_ERR_ARG, "null input");
   if (X && !aligned16(X)) return fail(ACE_ERR_ARG, "input not 16-byte aligned");
   for (int j = 0; j < nproj; ++j) {
-    if (!A[j] || !Bt[j] || !Y[j]) return fail(ACE_ERR_ARG, "null A / Bt / Y of projection %d", j);
-    if (!aligned16(A[j]) || !aligned16(Bt[j]) || !aligned16(Y[j]) || (H && H[j] && !aligned16(H[j])))
+    if (!A[j] || !Bt[j] || (perm->R > 0 && !Y[j])) return fail(ACE_ERR_ARG, "null A / Bt / Y of projection %d", j);
+    if (!aligned16(A[j]) || !aligned16(Bt[j]) || (Y[j] && !aligned16(Y[j])) || (H && H[j] && !aligned16(H[j])))
       return fail(ACE_ERR_ARG, "tensor of projection %d not 16-byte aligned", j);
   }
   if (perm->R == 0) return ACE_OK;
@@ -395,12 +395,14 @@ ace_status ace_bwd_shared(const ace_plan* plan, const ace_perm* perm, int32_t np
   ace_status st = check_perm(plan, perm);
   if (st != ACE_OK) return st;
   if (nproj < 1 || nproj > 2) return fail(ACE_ERR_ARG, "nproj=%d must be 1 or 2", nproj);
-  if (!dY || !H || !A || !Bt || !dA || !dBt || !dX || !X) return fail(ACE_ERR_ARG, "null argument");
-  if (!aligned16(X) || !aligned16(dX)) return fail(ACE_ERR_ARG, "X / dX not 16-byte aligned");
+  // token and row tensors may be null (empty) when the call has no tokens
+  if (!dY || !H || !A || !Bt || !dA || !dBt || (perm->T > 0 && (!dX || !X))) return fail(ACE_ERR_ARG, "null argument");
+  if ((X && !aligned16(X)) || (dX && !aligned16(dX))) return fail(ACE_ERR_ARG, "X / dX not 16-byte aligned");
   for (int j = 0; j < nproj; ++j) {
-    if (!dY[j] || !H[j] || !A[j] || !Bt[j] || !dA[j] || !dBt[j]) return fail(ACE_ERR_ARG, "null tensor of projection %d", j);
-    if (!aligned16(dY[j]) || !aligned16(H[j]) || !aligned16(A[j]) || !aligned16(Bt[j]) || !aligned16(dA[j]) ||
-        !aligned16(dBt[j]))
+    if (!A[j] || !Bt[j] || !dA[j] || !dBt[j] || (perm->R > 0 && (!dY[j] || !H[j])))
+      return fail(ACE_ERR_ARG, "null tensor of projection %d", j);
+    if ((dY[j] && !aligned16(dY[j])) || (H[j] && !aligned16(H[j])) || !aligned16(A[j]) || !aligned16(Bt[j]) ||
+        !aligned16(dA[j]) || !aligned16(dBt[j]))
       return fail(ACE_ERR_ARG, "tensor of projection %d not 16-byte aligned", j);
   }
   const BwdWs need = bwd_layout(plan, perm->T, nullptr);
@@ -483,9 +485,11 @@ ace_status ace_bwd_row(const ace_plan* plan, const ace_perm* perm, const uint16_
                        float* dBt, void* ws, size_t ws_bytes, void* stream) {
   ace_status st = check_perm(plan, perm);
   if (st != ACE_OK) return st;
-  if (!dY || !Hin || !H || !A || !Bt || !dHin || !dA || !dBt) return fail(ACE_ERR_ARG, "null argument");
-  if (!aligned16(dY) || !aligned16(Hin) || !aligned16(H) || !aligned16(A) || !aligned16(Bt) || !aligned16(dHin) ||
-      !aligned16(dA) || !aligned16(dBt))
+  // row tensors may be null (empty) when the call has no rows
+  if (!A || !Bt || !dA || !dBt || (perm->R > 0 && (!dY || !Hin || !H || !dHin)))
+    return fail(ACE_ERR_ARG, "null argument");
+  if ((dY && !aligned16(dY)) || (Hin && !aligned16(Hin)) || (H && !aligned16(H)) || !aligned16(A) ||
+      !aligned16(Bt) || (dHin && !aligned16(dHin)) || !aligned16(dA) || !aligned16(dBt))
     return fail(ACE_ERR_ARG, "tensor not 16-byte aligned");
   const BwdWs need = bwd_layout(plan, perm->T, nullptr);
   if (!ws || ws_bytes < need.total) return fail(ACE_ERR_WORKSPACE, "backward workspace %zu < %zu bytes", ws_bytes, need.total);
@@ -544,9 +548,9 @@ ace_status ace_fwd_combine(const ace_plan* plan, const ace_perm* perm, const uin
                            void* stream) {
   ace_status st = check_perm(plan, perm);
   if (st != ACE_OK) return st;
-  if (!A || !Bt || !H || !Hx || (perm->T > 0 && !Z) || (perm->R > 0 && (!Hin || !topk_w)))
+  if (!A || !Bt || (perm->T > 0 && (!Z || !Hx)) || (perm->R > 0 && (!Hin || !topk_w || !H)))
     return fail(ACE_ERR_ARG, "null argument");
-  if (!aligned16(A) || !aligned16(Bt) || !aligned16(H) || !aligned16(Hx) || (Z && !aligned16(Z)) ||
+  if (!aligned16(A) || !aligned16(Bt) || (H && !aligned16(H)) || (Hx && !aligned16(Hx)) || (Z && !aligned16(Z)) ||
       (Hin && !aligned16(Hin)) || (reinterpret_cast<uintptr_t>(topk_w) & 3u))
     return fail(ACE_ERR_ARG, "tensor not 16-byte aligned (topk_w: 4-byte)");
   if (perm->R == 0) return ACE_OK;

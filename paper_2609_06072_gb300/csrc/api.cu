@@ -169,12 +169,6 @@ ace_status ace_plan_create(ace_plan** out, const ace_layer_desc* desc) {
     if (rg > ACE_MAX_RANK) return fail(ACE_ERR_UNSUPPORTED, "r_%d=%d > %d", g, rg, ACE_MAX_RANK);
     rank_max = rg > rank_max ? rg : rank_max;
   }
-  // The forward row kernel cuts the last wave's tiles into column parts (a
-  // quarter of the 64-column chunks for down, half for gate/up); below four
-  // chunks of d or two of f a part would be empty, a case the kernels are not
-  // validated for.
-  if ((D.d + 63) / 64 < kSplitParts || (D.f + 63) / 64 < 2)
-    return fail(ACE_ERR_UNSUPPORTED, "d=%d, f=%d: need d > %d and f > 64", D.d, D.f, 64 * (kSplitParts - 1));
   int dev = 0;
   cudaError_t ce = cudaGetDevice(&dev);
   if (ce != cudaSuccess) return cuda_status(ce, "cudaGetDevice");

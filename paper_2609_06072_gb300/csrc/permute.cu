@@ -393,7 +393,11 @@ __global__ void __launch_bounds__(kPermTB) k_perm_scatter(const __grid_constant_
       const int n = build_tiles(totU, uoff, G, kTileM, o.tiles_sh, scratch);
       if (tid == 0) o.counts[kCntTilesSh] = n;
     } else if (job == 1) {
-      const int n = build_row_tiles(rows_g, goff, G, min(pt.nsm, 8 * (int)blockDim.x), o.tiles_row, scratch,
+      // the last wave's tiles are cut into column parts only when every part
+      // gets at least one 64-column chunk (a quarter of d's chunks for down,
+      // half of f's for gate/up)
+      const bool parts = (pt.d + 63) / 64 >= kSplitParts && (pt.f + 63) / 64 >= 2;
+      const int n = build_row_tiles(rows_g, goff, G, parts ? min(pt.nsm, 8 * (int)blockDim.x) : 0, o.tiles_row, scratch,
                                     o.counts + kCntRowSplit);
       if (tid == 0) o.counts[kCntTilesRow] = n;
     } else {

@@ -221,7 +221,8 @@ ace_status ace_bwd_row(const ace_plan* plan, const ace_perm* perm, const uint16_
  * group adapter of g(e) (Sec. 3.4): the adapter's share of the combined
  * output, in token rows.
  *   Hin     [R, f] bf16 expert inputs h_e in row order
- *   topk_w  [T, k] fp32 gate weights p, pair order (pair t*k + j)
+ *   topk_w  [T, k] fp32 gate weights p, pair order (pair t*k + j); a non-finite
+ *           weight sets the device flag (ACE_ERR_ARG from ace_get_error)
  *   A       [rank_off[G], f] bf16 (A_g);  Bt [rank_off[G], d] bf16 (B_g^T)
  *   Z       [T, d] bf16 IN/OUT: Z[t] += sum_j p[t,j] s B_g (A_g Hin[pair_row[t*k+j]])
  *   H       [R, rank_max] fp32 OUT: A_g Hin[row] (columns >= r_g zero)
@@ -348,8 +349,9 @@ ace_status ace_scatter_rows(const ace_perm* perm, const uint16_t* src_rows, uint
                             void* stream);
 
 /* Synchronises `stream`, then reads and clears the device error flag of the
- * permutation workspace: ACE_OK, ACE_ERR_INDEX (invalid routing) or
- * ACE_ERR_DEVICE_TIMEOUT (a bounded wait gave up; results unspecified). */
+ * permutation workspace: ACE_OK, ACE_ERR_INDEX (invalid routing),
+ * ACE_ERR_DEVICE_TIMEOUT (a bounded wait gave up; results unspecified) or
+ * ACE_ERR_ARG (a non-finite gate weight reached ace_fwd_combine). */
 ace_status ace_get_error(const ace_perm* perm, void* stream);
 
 #ifdef __cplusplus

@@ -16,13 +16,15 @@ constexpr int kMaxK = 32;          // largest top-k the kernels accept
 // Device error-flag bits (the flag lives at perm workspace word 0).
 constexpr int kErrIndex = 1;
 constexpr int kErrTimeout = 2;
+constexpr int kErrValue = 4;  // a non-finite gate weight reached the combine
 
 // Plan tables passed by value (__grid_constant__) to every kernel.
 struct PlanTables {
   int32_t E, G, k, d, f;
   int32_t rank_max;  // max_g r_g
   int32_t rank_pad;  // MMA N of one projection's rank block (16/32/64/128)
-  int32_t nt_split;  // tiles per backward split
+  int32_t nt_split;     // tiles per backward split (down and the combine)
+  int32_t nt_split_sh;  // tiles per backward split of gate/up (no phase-2 buffers in TMEM)
   int32_t nsm;       // SMs of the plan's device (the last nsm forward row tiles are split in column halves)
   int16_t e2g[ACE_MAX_EXPERTS];
   int16_t eorder[ACE_MAX_EXPERTS];  // experts in (g, e) order
@@ -43,14 +45,15 @@ struct PermLayout {
   size_t err, counts, sched, group_off, expert_off, expert_cnt, uniq_off, tot_u, row_pair, pair_row, pair_g, row_uniq,
       uniq_tok, tok_uniq;
   size_t chunk_cntE, chunk_cntU, chunk_baseE, chunk_baseU, chunk_err;
-  size_t tiles_sh, tiles_row, splits_row;
+  size_t tiles_sh, tiles_row, splits_row, splits_sh;
   size_t total;
-  int32_t n_chunks, max_tiles, max_splits;
+  int32_t n_chunks, max_tiles, max_splits, max_splits_sh;
 };
 
 // counts[] slots
 constexpr int kCntU = 0, kCntRows = 1, kCntTilesSh = 2, kCntTilesRow = 3, kCntSplitsRow = 4;
 constexpr int kCntRowSplit = 5;  // index of the first split entry of the row tiles
+constexpr int kCntSplitsSh = 6;  // backward splits of gate/up
 constexpr int kSplitParts = 4;   // column parts of each split row tile (the last wave's tiles)
 // sched[] slots: work counter and finished-CTA counter of the dynamically
 // scheduled forward row kernel; the permutation zeroes them and the last CTA
@@ -64,10 +67,14 @@ inline PermLayout perm_layout(const PlanTables& pt, int32_t T) {
   const int64_t R = (int64_t)T * pt.k;
   L.n_chunks = (T + kPermTB - 1) / kPermTB;
   L.max_tiles = (int32_t)((R + kTileM - 1) / kTileM + pt.G);
-  const int64_t split_rows = (int64_t)kTileM * pt.nt_split;
-  // pieces of split_rows rows, rounded up to whole waves of nsm CTAs
-  const int64_t min_splits = (R + split_rows - 1) / split_rows + pt.G;
-  L.max_splits = (int32_t)((min_splits + pt.nsm - 1) / pt.nsm * pt.nsm);
+  // pieces of kTileM * nt rows, rounded up to whole waves of nsm CTAs
+  auto max_pieces = [&](int nt) {
+    const int64_t split_rows = (int64_t)kTileM * nt;
+    const int64_t min_splits = (R + split_rows - 1) / split_rows + pt.G;
+    return (int32_t)((min_splits + pt.nsm - 1) / pt.nsm * pt.nsm);
+  };
+  L.max_splits = max_pieces(pt.nt_split);
+  L.max_splits_sh = max_pieces(pt.nt_split_sh);
   size_t off = 0;
   auto take = [&](size_t bytes) {
     size_t o = off;
@@ -96,6 +103,7 @@ inline PermLayout perm_layout(const PlanTables& pt, int32_t T) {
   L.tiles_sh = take(sizeof(Tile) * (size_t)L.max_tiles);
   L.tiles_row = take(sizeof(Tile) * (size_t)(L.max_tiles + (kSplitParts - 1) * pt.nsm));
   L.splits_row = take(sizeof(Tile) * (size_t)L.max_splits);
+  L.splits_sh = take(sizeof(Tile) * (size_t)L.max_splits_sh);
   L.total = off;
   return L;
 }
@@ -206,10 +214,11 @@ struct BwdLaunch {
   CUtensorMap tm_a;        // down: A [n_rank, d_in], box 64 x rank_pad
   CUtensorMap tm_dh;       // down: dHin [R, d_in], box 64 x 128
   CUtensorMap tm_h;        // down: Hin [R, d_in], box 64 x 128
-  const Tile* splits_row;  // row splits (the dY streaming kernel)
+  const Tile* splits_row;  // row splits (the dY streaming kernel: down, combine)
+  const Tile* splits_sh;   // row splits of gate/up (nt_split_sh tiles each)
   const Tile* tiles_sh;    // unique-pair tiles (dH per unique pair)
   const int32_t* counts;
-  int32_t max_splits_row, max_tiles_sh;
+  int32_t max_splits_row, max_splits_sh, max_tiles_sh;
   const int32_t* uniq_tok;
   const int32_t* uniq_off;
   const int32_t* group_off;
@@ -272,6 +281,7 @@ struct CombReduceLaunch {
   uint16_t* Hx;            // [T, n_rank_pad] bf16 out
   float s;
   int32_t T, n_rank_pad;
+  int32_t* err;            // device error flag (kErrValue on a non-finite gate weight)
 };
 cudaError_t launch_comb_reduce(const PlanTables& pt, const CombReduceLaunch& a, cudaStream_t st);
 

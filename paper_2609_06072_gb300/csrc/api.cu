@@ -84,8 +84,6 @@ ace_status cuda_status(cudaError_t e, const char* what) {
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-// Row tiles per backward split: (tiles + 2) * rank_pad TMEM columns <= 256.
-
 ace_status check_perm(const ace_plan* plan, const ace_perm* perm) {
   if (!plan || !perm || !perm->ws) return fail(ACE_ERR_ARG, "null plan or perm");
   if (perm->T < 0 || perm->T > plan->T_max) return fail(ACE_ERR_SHAPE, "perm T=%d outside [0, %d]", perm->T, plan->T_max);
@@ -93,7 +91,12 @@ ace_status check_perm(const ace_plan* plan, const ace_perm* perm) {
   return ACE_OK;
 }
 
+// Row tiles per backward split.  A split's dH accumulators (tiles x rank_pad
+// TMEM columns) sit below its double-buffered weight-gradient accumulators
+// (2 x rank_pad); down also keeps 128 columns of dh buffers, so at rank_pad
+// 128 down takes one tile per split and gate/up two.
 int pt_nt_split(int rank_pad) { return rank_pad <= 64 ? 4 : 1; }
+int pt_nt_split_sh(int rank_pad) { return rank_pad <= 64 ? 4 : 2; }
 
 struct BwdWs {
   float* dHrow[2];
@@ -113,7 +116,8 @@ BwdWs bwd_layout(const ace_plan* plan, int32_t T, void* base) {
   const PermLayout L = perm_layout(pt, T);
   const int64_t R = (int64_t)T * pt.k;
   const size_t dhrow = align_up(4 * (size_t)R * pt.rank_pad, 256);
-  const size_t pa = align_up(4 * (size_t)L.max_splits * pt.rank_pad * (size_t)(pt.d > pt.f ? pt.d : pt.f), 256);
+  const size_t n_part = (size_t)(L.max_splits > L.max_splits_sh ? L.max_splits : L.max_splits_sh);
+  const size_t pa = align_up(4 * n_part * pt.rank_pad * (size_t)(pt.d > pt.f ? pt.d : pt.f), 256);
   BwdWs w{};
   char* b = static_cast<char*>(base);
   size_t off = 0;
@@ -165,12 +169,6 @@ ace_status ace_plan_create(ace_plan** out, const ace_layer_desc* desc) {
     if (rg > ACE_MAX_RANK) return fail(ACE_ERR_UNSUPPORTED, "r_%d=%d > %d", g, rg, ACE_MAX_RANK);
     rank_max = rg > rank_max ? rg : rank_max;
   }
-  // The forward row kernel cuts the last wave's tiles into column parts (a
-  // quarter of the 64-column chunks for down, half for gate/up); below four
-  // chunks of d or two of f a part would be empty, a case the kernels are not
-  // validated for.
-  if ((D.d + 63) / 64 < kSplitParts || (D.f + 63) / 64 < 2)
-    return fail(ACE_ERR_UNSUPPORTED, "d=%d, f=%d: need d > %d and f > 64", D.d, D.f, 64 * (kSplitParts - 1));
   int dev = 0;
   cudaError_t ce = cudaGetDevice(&dev);
   if (ce != cudaSuccess) return cuda_status(ce, "cudaGetDevice");
@@ -193,6 +191,7 @@ ace_status ace_plan_create(ace_plan** out, const ace_layer_desc* desc) {
   p->pt.rank_max = rank_max;
   p->pt.rank_pad = rank_max <= 16 ? 16 : rank_max <= 32 ? 32 : rank_max <= 64 ? 64 : 128;
   p->pt.nt_split = pt_nt_split(p->pt.rank_pad);
+  p->pt.nt_split_sh = pt_nt_split_sh(p->pt.rank_pad);
   p->pt.nsm = num_sms;
   for (int e = 0; e < D.E; ++e) p->pt.e2g[e] = (int16_t)D.e2g[e];
   {
@@ -265,8 +264,8 @@ static ace_status fwd_common(const ace_plan* plan, const ace_perm* perm, const u
   if (perm->R > 0 && !X) return fail(ACE_ERR_ARG, "null input");
   if (X && !aligned16(X)) return fail(ACE_ERR_ARG, "input not 16-byte aligned");
   for (int j = 0; j < nproj; ++j) {
-    if (!A[j] || !Bt[j] || !Y[j]) return fail(ACE_ERR_ARG, "null A / Bt / Y of projection %d", j);
-    if (!aligned16(A[j]) || !aligned16(Bt[j]) || !aligned16(Y[j]) || (H && H[j] && !aligned16(H[j])))
+    if (!A[j] || !Bt[j] || (perm->R > 0 && !Y[j])) return fail(ACE_ERR_ARG, "null A / Bt / Y of projection %d", j);
+    if (!aligned16(A[j]) || !aligned16(Bt[j]) || (Y[j] && !aligned16(Y[j])) || (H && H[j] && !aligned16(H[j])))
       return fail(ACE_ERR_ARG, "tensor of projection %d not 16-byte aligned", j);
   }
   if (perm->R == 0) return ACE_OK;
@@ -390,12 +389,14 @@ ace_status ace_bwd_shared(const ace_plan* plan, const ace_perm* perm, int32_t np
   ace_status st = check_perm(plan, perm);
   if (st != ACE_OK) return st;
   if (nproj < 1 || nproj > 2) return fail(ACE_ERR_ARG, "nproj=%d must be 1 or 2", nproj);
-  if (!dY || !H || !A || !Bt || !dA || !dBt || !dX || !X) return fail(ACE_ERR_ARG, "null argument");
-  if (!aligned16(X) || !aligned16(dX)) return fail(ACE_ERR_ARG, "X / dX not 16-byte aligned");
+  // token and row tensors may be null (empty) when the call has no tokens
+  if (!dY || !H || !A || !Bt || !dA || !dBt || (perm->T > 0 && (!dX || !X))) return fail(ACE_ERR_ARG, "null argument");
+  if ((X && !aligned16(X)) || (dX && !aligned16(dX))) return fail(ACE_ERR_ARG, "X / dX not 16-byte aligned");
   for (int j = 0; j < nproj; ++j) {
-    if (!dY[j] || !H[j] || !A[j] || !Bt[j] || !dA[j] || !dBt[j]) return fail(ACE_ERR_ARG, "null tensor of projection %d", j);
-    if (!aligned16(dY[j]) || !aligned16(H[j]) || !aligned16(A[j]) || !aligned16(Bt[j]) || !aligned16(dA[j]) ||
-        !aligned16(dBt[j]))
+    if (!A[j] || !Bt[j] || !dA[j] || !dBt[j] || (perm->R > 0 && (!dY[j] || !H[j])))
+      return fail(ACE_ERR_ARG, "null tensor of projection %d", j);
+    if ((dY[j] && !aligned16(dY[j])) || (H[j] && !aligned16(H[j])) || !aligned16(A[j]) || !aligned16(Bt[j]) ||
+        !aligned16(dA[j]) || !aligned16(dBt[j]))
       return fail(ACE_ERR_ARG, "tensor of projection %d not 16-byte aligned", j);
   }
   const BwdWs need = bwd_layout(plan, perm->T, nullptr);
@@ -413,9 +414,11 @@ ace_status ace_bwd_shared(const ace_plan* plan, const ace_perm* perm, int32_t np
   }
   if (perm->R > 0 && !ok) return fail(ACE_ERR_UNSUPPORTED, "tensor-map encoding failed for this layout");
   a.splits_row = at<Tile>(perm->ws, L.splits_row);
+  a.splits_sh = at<Tile>(perm->ws, L.splits_sh);
   a.tiles_sh = at<Tile>(perm->ws, L.tiles_sh);
   a.counts = perm->counts;
   a.max_splits_row = L.max_splits;
+  a.max_splits_sh = L.max_splits_sh;
   a.max_tiles_sh = L.max_tiles;
   a.uniq_tok = perm->uniq_tok;
   a.uniq_off = perm->uniq_off;
@@ -476,9 +479,11 @@ ace_status ace_bwd_row(const ace_plan* plan, const ace_perm* perm, const uint16_
                        float* dBt, void* ws, size_t ws_bytes, void* stream) {
   ace_status st = check_perm(plan, perm);
   if (st != ACE_OK) return st;
-  if (!dY || !Hin || !H || !A || !Bt || !dHin || !dA || !dBt) return fail(ACE_ERR_ARG, "null argument");
-  if (!aligned16(dY) || !aligned16(Hin) || !aligned16(H) || !aligned16(A) || !aligned16(Bt) || !aligned16(dHin) ||
-      !aligned16(dA) || !aligned16(dBt))
+  // row tensors may be null (empty) when the call has no rows
+  if (!A || !Bt || !dA || !dBt || (perm->R > 0 && (!dY || !Hin || !H || !dHin)))
+    return fail(ACE_ERR_ARG, "null argument");
+  if ((dY && !aligned16(dY)) || (Hin && !aligned16(Hin)) || (H && !aligned16(H)) || !aligned16(A) ||
+      !aligned16(Bt) || (dHin && !aligned16(dHin)) || !aligned16(dA) || !aligned16(dBt))
     return fail(ACE_ERR_ARG, "tensor not 16-byte aligned");
   const BwdWs need = bwd_layout(plan, perm->T, nullptr);
   if (!ws || ws_bytes < need.total) return fail(ACE_ERR_WORKSPACE, "backward workspace %zu < %zu bytes", ws_bytes, need.total);
@@ -497,9 +502,11 @@ ace_status ace_bwd_row(const ace_plan* plan, const ace_perm* perm, const uint16_
   a.tm_dy[1] = a.tm_dy[0];
   a.tm_bt[1] = a.tm_bt[0];
   a.splits_row = at<Tile>(perm->ws, L.splits_row);
+  a.splits_sh = at<Tile>(perm->ws, L.splits_sh);
   a.tiles_sh = at<Tile>(perm->ws, L.tiles_sh);
   a.counts = perm->counts;
   a.max_splits_row = L.max_splits;
+  a.max_splits_sh = L.max_splits_sh;
   a.max_tiles_sh = L.max_tiles;
   a.uniq_tok = perm->uniq_tok;
   a.uniq_off = perm->uniq_off;
@@ -535,9 +542,9 @@ ace_status ace_fwd_combine(const ace_plan* plan, const ace_perm* perm, const uin
                            void* stream) {
   ace_status st = check_perm(plan, perm);
   if (st != ACE_OK) return st;
-  if (!A || !Bt || !H || !Hx || (perm->T > 0 && !Z) || (perm->R > 0 && (!Hin || !topk_w)))
+  if (!A || !Bt || (perm->T > 0 && (!Z || !Hx)) || (perm->R > 0 && (!Hin || !topk_w || !H)))
     return fail(ACE_ERR_ARG, "null argument");
-  if (!aligned16(A) || !aligned16(Bt) || !aligned16(H) || !aligned16(Hx) || (Z && !aligned16(Z)) ||
+  if (!aligned16(A) || !aligned16(Bt) || (H && !aligned16(H)) || (Hx && !aligned16(Hx)) || (Z && !aligned16(Z)) ||
       (Hin && !aligned16(Hin)) || (reinterpret_cast<uintptr_t>(topk_w) & 3u))
     return fail(ACE_ERR_ARG, "tensor not 16-byte aligned (topk_w: 4-byte)");
   if (perm->R == 0) return ACE_OK;
@@ -574,6 +581,7 @@ ace_status ace_fwd_combine(const ace_plan* plan, const ace_perm* perm, const uin
   c.s = s;
   c.T = perm->T;
   c.n_rank_pad = nrp;
+  c.err = err;
   st = cuda_status(launch_comb_reduce(pt, c, cs), "combine reduce launch");
   if (st != ACE_OK) return st;
   x.tm_acat[1] = x.tm_acat[0];
@@ -660,9 +668,11 @@ ace_status ace_bwd_combine(const ace_plan* plan, const ace_perm* perm, const uin
     if (st != ACE_OK) return st;
   }
   a.splits_row = at<Tile>(perm->ws, L.splits_row);
+  a.splits_sh = at<Tile>(perm->ws, L.splits_sh);
   a.tiles_sh = at<Tile>(perm->ws, L.tiles_sh);
   a.counts = perm->counts;
   a.max_splits_row = L.max_splits;
+  a.max_splits_sh = L.max_splits_sh;
   a.max_tiles_sh = L.max_tiles;
   a.uniq_tok = perm->uniq_tok;
   a.uniq_off = perm->uniq_off;
@@ -738,6 +748,7 @@ ace_status ace_get_error(const ace_perm* perm, void* stream) {
   if (s != ACE_OK) return s;
   if (flag & kErrTimeout) return fail(ACE_ERR_DEVICE_TIMEOUT, "a bounded device wait gave up");
   if (flag & kErrIndex) return fail(ACE_ERR_INDEX, "invalid routing: expert id out of range or repeated in a token");
+  if (flag & kErrValue) return fail(ACE_ERR_ARG, "a gate weight given to the combine is not finite");
   return ACE_OK;
 }
 

@@ -123,7 +123,10 @@ __device__ __forceinline__ void flush_wgrad(uint32_t taddr, int n0, int ld, int 
 // ----------------------------------------------------------------- k_bwd_rows
 template <int RP, int MODE>
 struct RowsCfg {
-  static constexpr int NT = RP <= 64 ? 4 : 1;
+  // row tiles per split: the split's dH accumulators (NT x RP TMEM columns)
+  // sit below the weight-gradient accumulators (2 x RP from kTB); gate/up
+  // needs no phase-2 buffers, so at RP = 128 two tiles fill the 512 columns
+  static constexpr int NT = RP <= 64 ? 4 : (MODE == MODE_SHARED ? 2 : 1);
   static constexpr int kOps = Slots<RP>::bytes(NT);
   static constexpr int kWBlk = RP * 128;
   static constexpr int kSlotA = 2 * kBlk + 2 * kWBlk;  // dY tile + B^T chunk (down phase 2: A chunk + h tile)
@@ -157,10 +160,10 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
   static_assert(NT * RP <= C::kTB, "dH accumulators must fit below the dB^T columns");
 
   pdl_wait();
-  const int n_splits = a.counts[kCntSplitsRow];
+  const int n_splits = a.counts[MODE == MODE_SHARED ? kCntSplitsSh : kCntSplitsRow];
   if ((int)blockIdx.x >= n_splits) return;
   const int proj = blockIdx.y;
-  const Tile sp = a.splits_row[blockIdx.x];
+  const Tile sp = (MODE == MODE_SHARED ? a.splits_sh : a.splits_row)[blockIdx.x];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = sp.g, r0 = pt.rank_off[g], rg = pt.rank_off[g + 1] - r0;
   const int ntiles = (sp.cnt + kTileM - 1) / kTileM;
@@ -168,6 +171,10 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
   const int nch1 = MODE == MODE_COMB ? 0 : (d_out + kNcB - 1) / kNcB;
   const int nch2 = MODE != MODE_SHARED ? (d_in + kNcB - 1) / kNcB : 0;
   const int NI1 = nch1 * ntiles, NI2 = nch2 * ntiles;
+  // Each split walks the column chunks starting at its own offset, so the
+  // splits of one group that run at the same time flush their weight
+  // gradients into different columns (fewer same-address atomics in L2).
+  auto chunk_col = [&](int c, int nch) { return ((c + sp.id) % nch) * kNcB; };
   const uint32_t sOps = smem_u32(smem);
   const uint32_t sA0 = sOps + C::kOps;
   const uint32_t sB0 = sA0 + SA * C::kSlotA;
@@ -220,14 +227,14 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
         }
         const uint32_t base = sA0 + s * C::kSlotA;
         if (q < NI1) {
-          const int c = q / ntiles, i = q % ntiles, n0 = c * kNcB, row0 = sp.start + i * kTileM;
+          const int c = q / ntiles, i = q % ntiles, n0 = chunk_col(c, nch1), row0 = sp.start + i * kTileM;
           mbar_arrive_expect_tx(&fullA[s], 2 * kBlk + 2 * C::kWBlk);
           tma_load_2d(base, &a.tm_dy[proj], n0, row0, &fullA[s]);
           tma_load_2d(base + kBlk, &a.tm_dy[proj], n0 + 64, row0, &fullA[s]);
           tma_load_2d(base + 2 * kBlk, &a.tm_bt[proj], n0, r0, &fullA[s]);
           tma_load_2d(base + 2 * kBlk + C::kWBlk, &a.tm_bt[proj], n0 + 64, r0, &fullA[s]);
         } else {
-          const int j = q - NI1, c = j / ntiles, i = j % ntiles, n0 = c * kNcB, row0 = sp.start + i * kTileM;
+          const int j = q - NI1, c = j / ntiles, i = j % ntiles, n0 = chunk_col(c, nch2), row0 = sp.start + i * kTileM;
           mbar_arrive_expect_tx(&fullA[s], 2 * C::kWBlk + 2 * kBlk);
           tma_load_2d(base, &a.tm_a, n0, r0, &fullA[s]);
           tma_load_2d(base + C::kWBlk, &a.tm_a, n0 + 64, r0, &fullA[s]);
@@ -393,7 +400,7 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
       ok = named_bar_and(kEpiBar, kEpiThreads, mbar_wait(&dbt_full[c & 1], (c >> 1) & 1));
       if (!ok) break;
       tc_fence_after();
-      flush_wgrad<RP>(tmem + lane_base + C::kTB + (c & 1) * RP, c * kNcB, d_out, rg, r0, a.s, fmode,
+      flush_wgrad<RP>(tmem + lane_base + C::kTB + (c & 1) * RP, chunk_col(c, nch1), d_out, rg, r0, a.s, fmode,
                       a.part_dBt[proj], sp.id, a.dBt[proj], m, false, ehalf * 16, 32);
       tc_fence_before();
       named_bar(kEpiBar, kEpiThreads);
@@ -453,7 +460,7 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
     }
     if (MODE != MODE_SHARED) {
       for (int j = 0; j < NI2 && ok; ++j) {
-        const int c = j / ntiles, i = j % ntiles, b = j % C::ND, sb = j % SB, n0 = c * kNcB;
+        const int c = j / ntiles, i = j % ntiles, b = j % C::ND, sb = j % SB, n0 = chunk_col(c, nch2);
         bool w_ok = mbar_wait(&fullB[sb], (j / SB) & 1);
         w_ok = w_ok && mbar_wait(&d_full[b], (j / C::ND) & 1);
         ok = named_bar_and(kEpiBar, kEpiThreads, w_ok);
@@ -614,7 +621,8 @@ cudaError_t launch_rows(const PlanTables& pt, const BwdLaunch& a, int nproj, cud
   auto kern = k_bwd_rows<RP, MODE>;
   cudaError_t e = set_smem(kern, C::kSmem);
   if (e != cudaSuccess) return e;
-  return launch_k(kern, dim3(a.max_splits_row, nproj), kThreadsWS, C::kSmem, st, pt, a);
+  const int grid = MODE == MODE_SHARED ? a.max_splits_sh : a.max_splits_row;
+  return launch_k(kern, dim3(grid, nproj), kThreadsWS, C::kSmem, st, pt, a);
 }
 
 // Combine backward: one launch zeroes dB^T (the dense dA GEMM of gemm.cu
@@ -666,10 +674,12 @@ cudaError_t launch_bwd_t(const PlanTables& pt, const BwdLaunch& a, bool shared, 
       return e;
   }
   if (a.deterministic) {
+    const Tile* splits = shared ? a.splits_sh : a.splits_row;
+    const int slot = shared ? kCntSplitsSh : kCntSplitsRow;
     for (int j = 0; j < nproj; ++j) {
       dim3 grid(n_rank, (a.d_out / 4 + 255) / 256);
-      if ((e = launch_k(k_splitk_reduce, grid, 256, 0, st, pt, a.splits_row, a.counts, kCntSplitsRow, a.part_dBt[j],
-                        (int)RP, a.d_out, a.dBt[j])) != cudaSuccess)
+      if ((e = launch_k(k_splitk_reduce, grid, 256, 0, st, pt, splits, a.counts, slot, a.part_dBt[j], (int)RP,
+                        a.d_out, a.dBt[j])) != cudaSuccess)
         return e;
     }
     if (!shared) {

@@ -42,6 +42,7 @@ __global__ void __launch_bounds__(kReduceThreads) k_comb_reduce(const __grid_con
       const int r0 = pt.rank_off[g], r1 = pt.rank_off[g + 1];
       if (c + 8 <= r0 || c >= r1) continue;
       const float wv = a.w[p];
+      if (!isfinite(wv)) atomicOr(a.err, kErrValue);
       const float* h = a.H + (int64_t)a.pair_row[p] * pt.rank_max - r0;
 #pragma unroll
       for (int q = 0; q < 8; ++q)

@@ -291,7 +291,7 @@ __device__ __forceinline__ int prefix_bits(const uint32_t* mask, int tid) {
   return r + __popc(mask[w] & ((1u << (tid & 31)) - 1u));
 }
 
-constexpr int kTableCtas = 3;  // scatter CTAs that build the offsets and tile tables
+constexpr int kTableCtas = 4;  // scatter CTAs that build the offsets and tile tables
 
 struct ScatterOut {
   int32_t* row_pair;
@@ -307,6 +307,7 @@ struct ScatterOut {
   Tile* tiles_sh;
   Tile* tiles_row;
   Tile* splits_row;
+  Tile* splits_sh;
 };
 
 template <int KB>
@@ -392,13 +393,20 @@ __global__ void __launch_bounds__(kPermTB) k_perm_scatter(const __grid_constant_
       const int n = build_tiles(totU, uoff, G, kTileM, o.tiles_sh, scratch);
       if (tid == 0) o.counts[kCntTilesSh] = n;
     } else if (job == 1) {
-      const int n = build_row_tiles(rows_g, goff, G, min(pt.nsm, 8 * (int)blockDim.x), o.tiles_row, scratch,
+      // the last wave's tiles are cut into column parts only when every part
+      // gets at least one 64-column chunk (a quarter of d's chunks for down,
+      // half of f's for gate/up)
+      const bool parts = (pt.d + 63) / 64 >= kSplitParts && (pt.f + 63) / 64 >= 2;
+      const int n = build_row_tiles(rows_g, goff, G, parts ? min(pt.nsm, 8 * (int)blockDim.x) : 0, o.tiles_row, scratch,
                                     o.counts + kCntRowSplit);
       if (tid == 0) o.counts[kCntTilesRow] = n;
     } else {
+      // backward splits: down / combine (job 2), gate/up (job 3)
       __shared__ int32_t red[32];
-      const int n = build_splits(rows_g, goff, G, kTileM * pt.nt_split, pt.nsm, o.splits_row, scratch, red);
-      if (tid == 0) o.counts[kCntSplitsRow] = n;
+      const bool sh = job == 3;
+      const int n = build_splits(rows_g, goff, G, kTileM * (sh ? pt.nt_split_sh : pt.nt_split), pt.nsm,
+                                 sh ? o.splits_sh : o.splits_row, scratch, red);
+      if (tid == 0) o.counts[sh ? kCntSplitsSh : kCntSplitsRow] = n;
     }
     return;
   }
@@ -508,6 +516,7 @@ cudaError_t launch_permute(const PlanTables& pt, const int32_t* topk_idx, int32_
   o.tiles_sh = at<Tile>(ws, L.tiles_sh);
   o.tiles_row = at<Tile>(ws, L.tiles_row);
   o.splits_row = at<Tile>(ws, L.splits_row);
+  o.splits_sh = at<Tile>(ws, L.splits_sh);
   size_t sm3 = sizeof(uint32_t) * (size_t)(pt.E + pt.G) * (kPermTB / 32);
   // one CTA per chunk, plus the ones that write the offsets and tables
   return launch_k(pt.k <= 8 ? k_perm_scatter<8> : k_perm_scatter<kMaxK>, C + kTableCtas, kPermTB, sm3, st, pt, topk_idx, T, at<int32_t>(ws, L.chunk_baseE),

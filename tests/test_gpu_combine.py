@@ -93,3 +93,25 @@ def test_combine_deterministic_mode_is_bitwise_reproducible():
     b = _combine_case(L, True)
     for key in a:
         assert np.array_equal(a[key], b[key]), key
+
+
+def test_combine_flags_non_finite_gate_weights():
+    """A non-finite gate weight is reported through the device flag (read and
+    cleared by ace_get_error) instead of passing silently."""
+    import torch
+    from paper_2609_06072_gb300 import ace
+    L = W.Layer(W.get_config("tiny"), seed=0)
+    c = L.cfg
+    plan = make_plan(L)
+    perm, P = run_perm(L, plan)
+    rp = P["row_pair"]
+    hin = dev_bf16(L.h()[rp])
+    A, Bt = dev_bf16(L.A("down")), dev_bf16(L.Bt("down"))
+    w = torch.from_numpy(np.ascontiguousarray(L.topk_w, dtype=np.float32)).cuda()
+    w[3, 1] = float("inf")
+    Z = torch.zeros(c.T, c.d, dtype=torch.bfloat16, device="cuda")
+    H = torch.empty(c.R, plan.rank_max, device="cuda")
+    Hx = torch.empty(c.T, plan.rank_cols, dtype=torch.bfloat16, device="cuda")
+    plan.fwd_combine(perm, hin, w, A, Bt, c.s, Z, H, Hx)
+    assert plan.get_error(perm) == ace.ACE_ERR_ARG
+    assert plan.get_error(perm) == ace.ACE_OK

@@ -191,3 +191,35 @@ def test_fwd_row_without_saved_h(with_ws):
 def test_fwd_row_parity(name, seed, over, base):
     L = W.Layer(W.get_config(name, **over), seed=seed)
     _fwd_row_case(L, L.cfg.s, with_base=base)
+
+
+def test_no_tokens():
+    """T = 0: every call succeeds with empty (null) token and row tensors,
+    launches no row work, and leaves exact-zero weight gradients."""
+    import torch
+    L = W.Layer(W.get_config("tiny"), seed=0)
+    c = L.cfg
+    plan = make_plan(L)
+    pws, _, bws = plan.alloc_workspaces(0)
+    perm = plan.permute(torch.zeros(0, c.k, dtype=torch.int32, device="cuda"), pws)
+    assert perm.T == 0 and perm.R == 0
+    bf = lambda *s: torch.empty(*s, dtype=torch.bfloat16, device="cuda")
+    f32 = lambda *s: torch.empty(*s, dtype=torch.float32, device="cuda")
+    rm = plan.rank_max
+    A = [dev_bf16(L.A(p)) for p in ("gate", "up", "down")]
+    Bt = [dev_bf16(L.Bt(p)) for p in ("gate", "up", "down")]
+    plan.fwd_shared(perm, bf(0, c.d), A[:2], Bt[:2], c.s, [bf(0, c.f), bf(0, c.f)], [f32(0, rm), f32(0, rm)])
+    plan.fwd_row(perm, bf(0, c.f), A[2], Bt[2], c.s, bf(0, c.d), f32(0, rm))
+    nan = lambda *s: torch.full(s, float("nan"), device="cuda")
+    dA = [nan(plan.n_rank, c.d), nan(plan.n_rank, c.d), nan(plan.n_rank, c.f)]
+    dBt = [nan(plan.n_rank, c.f), nan(plan.n_rank, c.f), nan(plan.n_rank, c.d)]
+    plan.bwd_shared(perm, [bf(0, c.f), bf(0, c.f)], bf(0, c.d), [f32(0, rm), f32(0, rm)], A[:2], Bt[:2], c.s,
+                    bf(0, c.d), dA[:2], dBt[:2], bws)
+    plan.bwd_row(perm, bf(0, c.d), bf(0, c.f), f32(0, rm), A[2], Bt[2], c.s, bf(0, c.f), dA[2], dBt[2], bws)
+    dAc, dBc = nan(plan.n_rank, c.f), nan(plan.n_rank, c.d)
+    plan.fwd_combine(perm, bf(0, c.f), f32(0, c.k), A[2], Bt[2], c.s, bf(0, c.d), f32(0, rm), bf(0, plan.rank_cols))
+    plan.bwd_combine(perm, bf(0, c.d), bf(0, c.f), f32(0, c.k), f32(0, rm), bf(0, plan.rank_cols), A[2], Bt[2], c.s,
+                     bf(0, c.f), f32(0, c.k), dAc, dBc, bws)
+    assert plan.get_error(perm) == 0
+    for t in dA + dBt + [dAc, dBc]:
+        assert bool((t == 0).all())

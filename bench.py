@@ -378,6 +378,18 @@ def load_stats(expert_cnt, R, U):
             "load_entropy_bits": h, "load_entropy_ratio": float(h / np.log2(len(cnt))) if len(cnt) > 1 else 1.0}
 
 
+def workload_config(args, L, U, expert_cnt, world, l2):
+    """The `config` object of both arms: the workload's shape, grouping and
+    realised routing (U and the expert loads), plus how L2 was handled."""
+    c = L.cfg
+    return {"workload": f"{args.config}-shaped MoE layer"
+                        f"{' (expert-wise, matched budget)' if args.expertwise else ' (grouped)'}",
+            "T": c.T, "d": c.d, "f": c.f, "E": c.E, "k": c.k, "G": L.G, "r": c.r,
+            "rank_g": int(np.max(np.diff(L.rank_off))), "s": c.s, "routing": f"{c.routing}({c.alpha})",
+            "rows_per_step": c.R, "U": int(U), **load_stats(expert_cnt, c.R, int(U)),
+            "deterministic": bool(args.det), "l2": l2, "parallelism": f"replicas x{world}"}
+
+
 def time_steps(lay, steps, warmup, flush):
     """Mean step time (ms) of `steps` steps, events at step boundaries only;
     flush: an L2Flush run before each step, or None."""
@@ -606,15 +618,9 @@ def run_gpu(args, rank, world, local):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": f"{args.config}-shaped MoE layer"
-                               f"{' (expert-wise, matched budget)' if args.expertwise else ' (grouped)'}",
-                   "T": c.T, "d": c.d, "f": c.f, "E": c.E, "k": c.k, "G": lay.L.G, "r": c.r,
-                   "rank_g": int(np.max(np.diff(lay.L.rank_off))), "s": c.s, "routing": f"{c.routing}({c.alpha})",
-                   "rows_per_step": c.R, "U": int(P["U"]), **load_stats(P["expert_cnt"], c.R, int(P["U"])),
-                   "deterministic": bool(args.det),
-                   "l2": "flushed between timed steps (256 MB write, then 256 MB read so no dirty line "
-                         "is left; outside the event pair)",
-                   "parallelism": f"replicas x{world}"},
+        "config": workload_config(args, lay.L, P["U"], P["expert_cnt"], world,
+                                  "flushed between timed steps (256 MB write, then 256 MB read so no dirty line "
+                                  "is left; outside the event pair)"),
         "roofline": {"bound": "hbm", "kernel": SINGLE_KERNEL[dom], "call": dom, "achieved": achieved,
                      "launch_ms": fwd_row_ms, "peak": peaks["hbm_gbs"],
                      "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"], "traffic": traffic,
@@ -836,7 +842,10 @@ def run_reference(args, rank, world):
         return None
     from paper_2609_06072_gb300 import workloads as W
     os.environ.setdefault("OMP_NUM_THREADS", str(cpu_cores()))
-    c = W.get_config(args.config)
+    L = W.Layer(W.get_config(args.config), seed=args.seed, expertwise=args.expertwise)
+    c = L.cfg
+    # realised routing, for the config object: distinct (token, group) pairs
+    U = len(np.unique(np.arange(c.T)[:, None] * L.G + np.asarray(L.e2g)[L.topk_idx]))
     # per step: a bounded sample sized so that warmup + steps end within minutes
     per_step_s = max(2.0, min(20.0, 120.0 / max(1, args.steps + args.warmup)))
     frac = calibrate_fraction(args.config, args.seed, args.expertwise, per_step_s)
@@ -854,8 +863,8 @@ def run_reference(args, rank, world):
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": 1e3 * c.R / value, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": f"{args.config}-shaped MoE layer{' (expert-wise)' if args.expertwise else ' (grouped)'}",
-                   "T": c.T, "d": c.d, "f": c.f, "E": c.E, "k": c.k},
+        "config": workload_config(args, L, U, np.bincount(L.topk_idx.ravel(), minlength=c.E), world,
+                                  "not applicable: the fp64 CPU oracle on host cores"),
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
                          "sample": f"per step: permutation plus {frac:.4f} of the pairs and rank rows of one step"},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},

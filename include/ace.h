@@ -175,8 +175,10 @@ ace_status ace_fwd_shared(const ace_plan* plan, const ace_perm* perm, const uint
  * without the workspace: H is not returned, and the scratch it needs (2 x
  * T*k x rank_max fp32) lives in a 32 MiB array inside the library that every
  * GPU loading the library holds until the process exits.  Larger sizes fail
- * with ACE_ERR_WORKSPACE and launch nothing.  The first call on a device
- * looks up the array's device address (make it before any stream capture).
+ * with ACE_ERR_WORKSPACE and launch nothing.  The first call in a CUDA
+ * context (per device; again after cudaDeviceReset or when another context
+ * is current) looks up the array's device address: make that call before
+ * any stream capture.
  * All calls share the array: calls that overlap on the GPU race, so issue
  * them on one stream or otherwise order them.  Nothing in the array has to
  * start at zero: each call writes every scratch word it reads before reading
@@ -253,23 +255,6 @@ ace_status ace_bwd_combine(const ace_plan* plan, const ace_perm* perm, const uin
                            const uint16_t* Bt, float s, uint16_t* dHin, float* dtopk_w, float* dA, float* dBt,
                            void* ws, size_t ws_bytes, void* stream);
 
-/* Grouping of one layer's experts from their pairwise similarities, for rank
- * consolidation (Sec. 3.2; layer-wise graph construction, Louvain, fixed-
- * threshold and group-anchor appendices).  HOST memory, no GPU work:
- *   S        [E, E] fp32 host similarities (e.g. linear CKA of the adapters'
- *            outputs on a probe set), symmetrised as (S + S^T) / 2
- *   method   ACE_GROUP_LOUVAIN: Louvain on W = max(0, S' - median of the
- *            off-diagonal S'), zero diagonal, resolution `param` (the paper
- *            uses 0.8); ACE_GROUP_THRESHOLD: connected components of
- *            {(i, j): i != j, S'_ij >= param} (the paper's variant uses 0.9)
- *   e2g      [E] int32 host OUT: group of each expert, groups numbered in order
- *            of their smallest expert
- *   anchors  [E] int32 host OUT or NULL: the first G entries receive each
- *            group's CKA-centre anchor, the member with the largest sum of
- *            similarities to its group (ties to the lower index)
- *   G_out    OUT: number of groups
- * The consolidated ranks follow as r_g = sum of the members' ranks (rank_off
- * of the group plan).  Deterministic; double-precision arithmetic. */
 /* Linear CKA similarity of a layer's expert-wise adapters on a probe set
  * (Sec. 3.2): s_ij = ||Zc_i^T Zc_j||_F^2 / (||Zc_i^T Zc_i||_F ||Zc_j^T Zc_j||_F)
  * with Z_e = X A_e^T B_e^T and Zc_e = H Z_e, H = I - 11^T / N (center != 0) or
@@ -303,6 +288,23 @@ ace_status ace_consolidate_adapters(int32_t E, int32_t r, int32_t d_in, int32_t 
                                     const uint16_t* A_init, uint16_t* A_g, uint16_t* Bt_g, int32_t* rank_off,
                                     void* stream);
 
+/* Grouping of one layer's experts from their pairwise similarities, for rank
+ * consolidation (Sec. 3.2; layer-wise graph construction, Louvain, fixed-
+ * threshold and group-anchor appendices).  HOST memory, no GPU work:
+ *   S        [E, E] fp32 host similarities (e.g. linear CKA of the adapters'
+ *            outputs on a probe set), symmetrised as (S + S^T) / 2
+ *   method   ACE_GROUP_LOUVAIN: Louvain on W = max(0, S' - median of the
+ *            off-diagonal S'), zero diagonal, resolution `param` (the paper
+ *            uses 0.8); ACE_GROUP_THRESHOLD: connected components of
+ *            {(i, j): i != j, S'_ij >= param} (the paper's variant uses 0.9)
+ *   e2g      [E] int32 host OUT: group of each expert, groups numbered in order
+ *            of their smallest expert
+ *   anchors  [E] int32 host OUT or NULL: the first G entries receive each
+ *            group's CKA-centre anchor, the member with the largest sum of
+ *            similarities to its group (ties to the lower index)
+ *   G_out    OUT: number of groups
+ * The consolidated ranks follow as r_g = sum of the members' ranks (rank_off
+ * of the group plan).  Deterministic; double-precision arithmetic. */
 #define ACE_GROUP_LOUVAIN 0
 #define ACE_GROUP_THRESHOLD 1
 ace_status ace_group_experts(const float* S, int32_t E, int32_t method, double param, int32_t* e2g,
@@ -322,6 +324,12 @@ ace_status ace_group_experts(const float* S, int32_t E, int32_t method, double p
  *   Hgu[2]   [R, rank_max] fp32 OUT: H of gate and up per unique pair
  *   Hd       [R, rank_max] fp32 OUT: H of down per row
  *   ws       ace_ffn_workspace_size bytes (the token rows in row order) */
+ace_status ace_ffn_workspace_size(const ace_plan* plan, int32_t T, size_t* bytes);
+ace_status ace_ffn_fwd(const ace_plan* plan, const ace_perm* perm, const uint16_t* X, const uint16_t* W_gate,
+                       const uint16_t* W_up, const uint16_t* W_down, const uint16_t* const* A,
+                       const uint16_t* const* Bt, float s, uint16_t* U, uint16_t* V, uint16_t* Hh, uint16_t* Y,
+                       float* const* Hgu, float* Hd, void* ws, size_t ws_bytes, void* stream);
+
 /* Backward of ace_ffn_fwd with frozen base weights, for the per-row output
  * gradient dY [R, d] bf16 (row order):
  *   dX       [T, d] bf16 OUT (overwritten): the token-input gradient through
@@ -334,11 +342,6 @@ ace_status ace_ffn_bwd(const ace_plan* plan, const ace_perm* perm, const uint16_
                        const uint16_t* const* Bt, float s, const uint16_t* U, const uint16_t* V, const uint16_t* Hh,
                        const float* const* Hgu, const float* Hd, uint16_t* dX, float* const* dA, float* const* dBt,
                        void* ws, size_t ws_bytes, void* bws, size_t bws_bytes, void* stream);
-ace_status ace_ffn_workspace_size(const ace_plan* plan, int32_t T, size_t* bytes);
-ace_status ace_ffn_fwd(const ace_plan* plan, const ace_perm* perm, const uint16_t* X, const uint16_t* W_gate,
-                       const uint16_t* W_up, const uint16_t* W_down, const uint16_t* const* A,
-                       const uint16_t* const* Bt, float s, uint16_t* U, uint16_t* V, uint16_t* Hh, uint16_t* Y,
-                       float* const* Hgu, float* Hd, void* ws, size_t ws_bytes, void* stream);
 
 /* Row-order helpers (bf16, `cols` elements per row, cols multiple of 8):
  *   gather:  dst[row] = src[row_pair[row]]   (pair order -> row order)

@@ -769,7 +769,26 @@ constexpr size_t kNoAllocScratchBytes = size_t(32) << 20;  // 32 MiB
 __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 constexpr int kNoAllocMaxDevices = 64;
 std::mutex g_noalloc_mu;
-void* g_noalloc_ptr[kNoAllocMaxDevices] = {};
+// The array's device address, looked up once per (device, context): a
+// context created after cudaDeviceReset, or another context made current on
+// the same device, holds its own copy of the array at another address.
+struct NoAllocAddr {
+  void* ctx;
+  void* ptr;
+};
+NoAllocAddr g_noalloc_addr[kNoAllocMaxDevices] = {};
+using CtxGetCurrentFn = int (*)(void**);  // CUresult cuCtxGetCurrent(CUcontext*)
+CtxGetCurrentFn ctx_get_current() {
+  static CtxGetCurrentFn fn = [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      return reinterpret_cast<CtxGetCurrentFn>(p);
+    return static_cast<CtxGetCurrentFn>(nullptr);
+  }();
+  return fn;
+}
 }  // namespace
 
 extern "C" ace_status ace_fwd_shared_noalloc(const ace_plan* plan, const ace_perm* perm, const uint16_t* X,
@@ -787,17 +806,24 @@ extern "C" ace_status ace_fwd_shared_noalloc(const ace_plan* plan, const ace_per
   if (ce != cudaSuccess) return cuda_status(ce, "cudaGetDevice");
   if (dev != plan->device) return fail(ACE_ERR_ARG, "current device %d is not the plan's device %d", dev, plan->device);
   if (dev < 0 || dev >= kNoAllocMaxDevices) return fail(ACE_ERR_UNSUPPORTED, "device index %d too large", dev);
+  // cudaGetDevice above made the runtime's context of `dev` current
+  CtxGetCurrentFn get_ctx = ctx_get_current();
+  if (!get_ctx) return fail(ACE_ERR_UNSUPPORTED, "cuCtxGetCurrent is unavailable from the driver");
+  void* ctx = nullptr;
+  if (get_ctx(&ctx) != 0 || !ctx) return fail(ACE_ERR_CUDA, "no current CUDA context on device %d", dev);
   void* scratch = nullptr;
   {
     std::lock_guard<std::mutex> lock(g_noalloc_mu);
-    if (!g_noalloc_ptr[dev]) {
-      // once per device, with that device current: the device address of the array
+    NoAllocAddr& slot = g_noalloc_addr[dev];
+    if (slot.ctx != ctx || !slot.ptr) {
+      // first call in this context, with its device current: the array's device address
       void* p = nullptr;
       ce = cudaGetSymbolAddress(&p, g_noalloc_scratch);
       if (ce != cudaSuccess) return cuda_status(ce, "cudaGetSymbolAddress");
-      g_noalloc_ptr[dev] = p;
+      slot.ctx = ctx;
+      slot.ptr = p;
     }
-    scratch = g_noalloc_ptr[dev];
+    scratch = slot.ptr;
   }
   return ace_fwd_shared(plan, perm, X, nproj, A, Bt, s, Y, nullptr, scratch, kNoAllocScratchBytes, stream);
 }

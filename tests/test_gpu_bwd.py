@@ -88,7 +88,11 @@ CASES = [("tiny", 0, {}), ("tiny", 1, {"T": 300}), ("olmoe", 0, {"T": 1024}), ("
          # r_g = 12: rank offsets that are not multiples of 8 (unaligned dH_u columns)
          ("tiny", 4, {"r": 3}),
          # paper-like uneven groups, r_g from 2 to 86 (128-wide rank tiles), and E = 256
-         ("olmoe_uneven", 0, {"T": 512}), ("kimi", 0, {"T": 256})]
+         ("olmoe_uneven", 0, {"T": 512}), ("kimi", 0, {"T": 256}),
+         # the grouping sweep's uniform points (r_g = 16 and r_g = 64)
+         ("deepseek_g32", 0, {"T": 1024}), ("deepseek_g8", 0, {"T": 1024}),
+         # full Mixtral widths (d = 4096, f = 14336) at a reduced token count
+         ("mixtral", 0, {"T": 256})]
 
 
 @pytest.mark.parametrize("det", [True, False])

@@ -1,5 +1,6 @@
 """Full-size parity: the workloads at their full token counts, run through the
-same calls and launch configuration as the benchmark (fast split-K mode), with
+same calls and launch configuration as the benchmark (fast split-K mode; one
+case per workload family also in the deterministic mode), with
 sampled outputs checked one by one against the oracle (which computes just
 the sampled pairs, tokens and rank rows)."""
 import numpy as np
@@ -15,11 +16,11 @@ pytestmark = pytest.mark.gpu
 N_PAIRS, N_TOK, N_RANK = 256, 96, 48
 
 
-def _full_case(name, seed):
+def _full_case(name, seed, det=False):
     import torch
     L = W.Layer(W.get_config(name), seed=seed)
     c = L.cfg
-    plan = make_plan(L)
+    plan = make_plan(L, deterministic=det)
     perm, P = run_perm(L, plan)
     O = oracle.permute(L.topk_idx, L.e2g, L.G)
     compare_perm(P, O)
@@ -81,6 +82,13 @@ def _full_case(name, seed):
         check_close(host_f64(dBt[p][ri]), rdBt, f"dBt_{p}[sampled]")
 
 
-@pytest.mark.parametrize("name", ["olmoe", "qwen", "deepseek_g16", "olmoe_uneven", "kimi"])
+@pytest.mark.parametrize("name", ["olmoe", "qwen", "deepseek_g16", "deepseek_g32", "deepseek_g8", "olmoe_uneven",
+                                  "kimi", "mixtral"])
 def test_full_size_sampled_parity(name):
     _full_case(name, 0)
+
+
+@pytest.mark.parametrize("name", ["olmoe", "olmoe_uneven"])
+def test_full_size_sampled_parity_deterministic(name):
+    """The deterministic two-stage split-K mode at full size."""
+    _full_case(name, 1, det=True)

@@ -118,7 +118,10 @@ def _fwd_shared_case(L, s, with_base, nproj=2):
 @pytest.mark.parametrize("name,seed,over", [("tiny", 0, {}), ("tiny", 1, {"T": 300}), ("olmoe", 0, {"T": 1024}),
                                             ("olmoe", 2, {"T": 4096}), ("qwen", 0, {"T": 1024}),
                                             ("deepseek_g16", 0, {"T": 1024}), ("tiny", 4, {"r": 3}),
-                                            ("olmoe_uneven", 0, {"T": 512}), ("kimi", 0, {"T": 256})])
+                                            ("olmoe_uneven", 0, {"T": 512}), ("kimi", 0, {"T": 256}),
+                                            ("deepseek_g32", 0, {"T": 1024}), ("deepseek_g8", 0, {"T": 1024}),
+                                            # full Mixtral widths: 224 column chunks of f, a 64-step K loop
+                                            ("mixtral", 0, {"T": 256})])
 def test_fwd_shared_parity(name, seed, over):
     L = W.Layer(W.get_config(name, **over), seed=seed)
     _fwd_shared_case(L, L.cfg.s, with_base=False)
@@ -187,7 +190,11 @@ def test_fwd_row_without_saved_h(with_ws):
                                                  ("olmoe", 0, {"T": 512}, False), ("olmoe", 2, {"T": 4096}, True),
                                                  ("qwen", 1, {"T": 512}, False),
                                                  ("deepseek_g16", 0, {"T": 512}, True), ("tiny", 4, {"r": 3}, False),
-                                                 ("olmoe_uneven", 0, {"T": 512}, True), ("kimi", 0, {"T": 256}, False)])
+                                                 ("olmoe_uneven", 0, {"T": 512}, True), ("kimi", 0, {"T": 256}, False),
+                                                 ("deepseek_g32", 0, {"T": 1024}, False),
+                                                 ("deepseek_g8", 0, {"T": 1024}, True),
+                                                 # full Mixtral widths: a 224-step K loop over f, 64 chunks of d
+                                                 ("mixtral", 0, {"T": 256}, True)])
 def test_fwd_row_parity(name, seed, over, base):
     L = W.Layer(W.get_config(name, **over), seed=seed)
     _fwd_row_case(L, L.cfg.s, with_base=base)

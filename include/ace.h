@@ -77,6 +77,13 @@ typedef int32_t ace_status;
 /* plan flags */
 #define ACE_FLAG_DETERMINISTIC 1u /* dA / dB^T via fixed-order two-stage split-K (bitwise reproducible);
                                      otherwise fp32 atomics (any summation order) */
+/* Test only, never for production use: exercises the bounded-wait failure
+ * path.  With it, ace_fwd_row (when it computes the split row tiles' H up
+ * front, i.e. with a saved H or forward scratch) never raises the ready flags
+ * of that H, and the row kernel's wait on them gives up after 2 ms instead of
+ * 1 s.  The call then ends early: ace_get_error returns
+ * ACE_ERR_DEVICE_TIMEOUT, Y is unspecified, and the context stays usable. */
+#define ACE_FLAG_TEST_WAIT_EXPIRY 2u
 
 /* Limits. */
 #define ACE_MAX_EXPERTS 512

@@ -26,6 +26,7 @@ ACE_ERR_UNSUPPORTED = 5
 ACE_ERR_CUDA = 6
 ACE_ERR_DEVICE_TIMEOUT = 7
 ACE_FLAG_DETERMINISTIC = 1
+ACE_FLAG_TEST_WAIT_EXPIRY = 2  # test only: makes the down forward's bounded flag wait give up
 
 STATUS_NAMES = {0: "ACE_OK", 1: "ACE_ERR_ARG", 2: "ACE_ERR_SHAPE", 3: "ACE_ERR_WORKSPACE", 4: "ACE_ERR_INDEX",
                 5: "ACE_ERR_UNSUPPORTED", 6: "ACE_ERR_CUDA", 7: "ACE_ERR_DEVICE_TIMEOUT"}
@@ -180,12 +181,13 @@ class Perm:
 class Plan:
     """One layer description (ace_plan) on the current CUDA device."""
 
-    def __init__(self, T_max: int, k: int, E: int, G: int, e2g, rank_off, d: int, f: int, deterministic=False):
+    def __init__(self, T_max: int, k: int, E: int, G: int, e2g, rank_off, d: int, f: int, deterministic=False,
+                 flags=0):
         self.lib = load()
         self._e2g = (ctypes.c_int32 * E)(*[int(x) for x in e2g])
         self._ro = (ctypes.c_int32 * (G + 1))(*[int(x) for x in rank_off])
         desc = ace_layer_desc(int(T_max), int(k), int(E), int(G), self._e2g, self._ro, int(d), int(f),
-                              ACE_FLAG_DETERMINISTIC if deterministic else 0)
+                              (ACE_FLAG_DETERMINISTIC if deterministic else 0) | int(flags))
         h = ctypes.c_void_p()
         _check(self.lib.ace_plan_create(ctypes.byref(h), ctypes.byref(desc)), "ace_plan_create")
         self.h = h

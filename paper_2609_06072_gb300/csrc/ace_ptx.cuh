@@ -132,15 +132,13 @@ __device__ __forceinline__ void named_bar_arrive(int id, int nthreads) {
   asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
-// Relaxed, gpu-scope reductions into bf16 global memory: 8 values at a
-// 16-byte aligned address, or one value.
+// Relaxed, gpu-scope reduction of 8 bf16 values into global memory at a
+// 16-byte aligned address.  (No scalar 16-bit form is offered: it would run
+// as a compare-and-swap loop.)
 __device__ __forceinline__ void red_add_bf16x8(void* p, uint4 v) {
   asm volatile("red.global.add.noftz.v4.bf16x2 [%0], {%1, %2, %3, %4};" ::"l"(p), "r"(v.x), "r"(v.y), "r"(v.z),
                "r"(v.w)
                : "memory");
-}
-__device__ __forceinline__ void red_add_bf16(void* p, uint16_t h) {
-  asm volatile("red.global.add.noftz.bf16 [%0], %1;" ::"l"(p), "h"(h) : "memory");
 }
 
 // Load with acquire semantics at gpu scope (pairs with a writer's fence +

@@ -357,6 +357,7 @@ static ace_status fwd_common(const ace_plan* plan, const ace_perm* perm, const u
     r.Hpre = r.Hsave;
     if (!r.Hpre && ws && aligned16(ws) && ws_bytes >= 4 * (size_t)R * pt.rank_max) r.Hpre = static_cast<float*>(ws);
     r.pre = r.Hpre != nullptr;
+    r.test_expiry = (plan->flags & ACE_FLAG_TEST_WAIT_EXPIRY) != 0;
   }
   r.s = s;
   r.d_in = d_in;

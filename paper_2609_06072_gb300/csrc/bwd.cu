@@ -89,6 +89,30 @@ __device__ __forceinline__ uint4 pack8(const float* v) {
   return w;
 }
 
+// Adds v[0..16), the values of 16 consecutive bf16 columns starting O
+// columns past an 8-column boundary (win0 = that boundary), into global
+// memory with 16-byte vector reductions only: one per aligned 8-column
+// window that meets the first `nvalid` columns.  Window positions outside
+// them receive +0, which leaves a neighbour's bf16 value unchanged (x + 0 = x),
+// so a group whose rank offset is not a multiple of 8 needs no 16-bit
+// atomics (those would run as compare-and-swap loops).
+template <int O>
+__device__ __forceinline__ void red_windows(uint16_t* win0, const float* v, int nvalid) {
+#pragma unroll
+  for (int w = 0; w < (O == 0 ? 2 : 3); ++w) {
+    const int qlo = 8 * w - O;  // index into v of the window's first column
+    const int lo = qlo < 0 ? 0 : qlo;
+    if (lo >= nvalid) continue;
+    float u[8];
+#pragma unroll
+    for (int p = 0; p < 8; ++p) {
+      const int q = qlo + p;
+      u[p] = (q >= 0 && q < 16 && q < nvalid) ? v[q] : 0.f;
+    }
+    red_add_bf16x8(win0 + 8 * w, pack8(u));
+  }
+}
+
 // Flush one [128 cols x RP] fp32 accumulator of a weight gradient (TMEM lane
 // `col_lane` = column n0 + col_lane): atomics into out, a per-split partial,
 // or a plain store of the final value.
@@ -429,22 +453,21 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
 #pragma unroll
               for (int q = 0; q < 4; ++q) dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
             } else if (live) {
-              // dHx[t][proj * n_rank_pad + r0 + k] += dH_row[k], k < r_g
-              uint16_t* dst = a.dHx + (int64_t)tok_s[i * kTileM + m] * (a.nproj * a.n_rank_pad) +
-                              proj * a.n_rank_pad + r0 + c0;
-#pragma unroll
-              for (int h8 = 0; h8 < 2; ++h8) {
-                const int k0 = c0 + h8 * 8;
-                if (((r0 & 7) == 0) && k0 + 8 <= rg) {
-                  red_add_bf16x8(dst + h8 * 8, pack8(v + h8 * 8));
-                } else {
-#pragma unroll
-                  for (int q = 0; q < 8; ++q)
-                    if (k0 + q < rg) {
-                      const __nv_bfloat16 b = __float2bfloat16_rn(v[h8 * 8 + q]);
-                      red_add_bf16(dst + h8 * 8 + q, *reinterpret_cast<const uint16_t*>(&b));
-                    }
-                }
+              // dHx[t][proj * n_rank_pad + r0 + k] += dH_row[k], k < r_g, by
+              // 16-byte vector reductions over the aligned 8-column windows
+              uint16_t* row_dst = a.dHx + (int64_t)tok_s[i * kTileM + m] * (a.nproj * a.n_rank_pad) +
+                                  proj * a.n_rank_pad;
+              const int col0 = r0 + c0, o = col0 & 7;
+              uint16_t* win0 = row_dst + (col0 - o);
+              switch (o) {
+                case 0: red_windows<0>(win0, v, rg - c0); break;
+                case 1: red_windows<1>(win0, v, rg - c0); break;
+                case 2: red_windows<2>(win0, v, rg - c0); break;
+                case 3: red_windows<3>(win0, v, rg - c0); break;
+                case 4: red_windows<4>(win0, v, rg - c0); break;
+                case 5: red_windows<5>(win0, v, rg - c0); break;
+                case 6: red_windows<6>(win0, v, rg - c0); break;
+                default: red_windows<7>(win0, v, rg - c0); break;
               }
             }
           } else {

@@ -225,6 +225,8 @@ __device__ __forceinline__ int chunk_hi(const Tile& t, int nch, int merge) {
 // Up-front H of the split row tiles (down): ready once every epilogue warp of
 // the CTA that computed it has added 1.
 constexpr int kPreWriters = 4 * 4;
+// the H-ready wait's bound under ACE_FLAG_TEST_WAIT_EXPIRY
+constexpr uint64_t kTestWaitLimitNs = 2000000ull;
 __device__ __forceinline__ uint32_t rows_bytes(int cnt) {
   return cnt == kTileM ? (uint32_t)kBlk : (uint32_t)((cnt + kQuant - 1) / kQuant) * kQuant * 128;
 }
@@ -567,9 +569,9 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
       if (!SHARED && kt < 0) {  // split tile: wait for its up-front H
         bool w2 = true;
         if (lane == 0) {
-          const uint64_t t0 = globaltimer_ns();
+          const uint64_t t0 = globaltimer_ns(), limit = a.test_expiry ? kTestWaitLimitNs : kWaitLimitNs;
           while (ld_acquire(hflag + split_index(t)) < kPreWriters)
-            if (globaltimer_ns() - t0 > kWaitLimitNs) {
+            if (globaltimer_ns() - t0 > limit) {
               w2 = false;
               break;
             }
@@ -606,7 +608,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
       tc_fence_before();
       __threadfence();
       __syncwarp();
-      if (lane == 0) atomicAdd(hflag + blockIdx.x, 1);
+      if (lane == 0 && !a.test_expiry) atomicAdd(hflag + blockIdx.x, 1);
       return true;
     };
     int q = 0, ib = 0, cc0 = 0, ci = 0, kc = 0;

@@ -195,6 +195,7 @@ struct FwdRowsLaunch {
   float* Hsave;          // down: H per row out (may be null)
   float* Hpre;           // down: where the split row tiles' H is computed first (Hsave or scratch), or null
   int32_t pre;           // down: split row tiles take their H from Hpre (computed up front), not a K loop
+  int32_t proj_split;    // gate/up: the two projections are separate work items (NPROJ = 1 kernel)
   int32_t test_expiry;   // ACE_FLAG_TEST_WAIT_EXPIRY: the up-front H's ready flags are never raised and
                          // the wait on them gives up after 2 ms
   float s;

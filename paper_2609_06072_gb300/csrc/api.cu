@@ -93,9 +93,9 @@ ace_status check_perm(const ace_plan* plan, const ace_perm* perm) {
 
 // Row tiles per backward split.  A split's dH accumulators (tiles x rank_pad
 // TMEM columns) sit below its double-buffered weight-gradient accumulators
-// (2 x rank_pad); down also keeps 128 columns of dh buffers, so at rank_pad
-// 128 down takes one tile per split and gate/up two.
-int pt_nt_split(int rank_pad) { return rank_pad <= 64 ? 4 : 1; }
+// (2 x rank_pad), so at rank_pad 128 a split takes two tiles (down's phase-2
+// dh buffer reuses the dH columns).
+int pt_nt_split(int rank_pad) { return rank_pad <= 64 ? 4 : 2; }
 int pt_nt_split_sh(int rank_pad) { return rank_pad <= 64 ? 4 : 2; }
 
 struct BwdWs {

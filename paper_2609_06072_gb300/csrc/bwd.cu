@@ -148,14 +148,17 @@ __device__ __forceinline__ void flush_wgrad(uint32_t taddr, int n0, int ld, int 
 template <int RP, int MODE>
 struct RowsCfg {
   // row tiles per split: the split's dH accumulators (NT x RP TMEM columns)
-  // sit below the weight-gradient accumulators (2 x RP from kTB); gate/up
-  // needs no phase-2 buffers, so at RP = 128 two tiles fill the 512 columns
-  static constexpr int NT = RP <= 64 ? 4 : (MODE == MODE_SHARED ? 2 : 1);
+  // sit below the weight-gradient accumulators (2 x RP from kTB); at RP = 128
+  // two tiles fill the 512 columns, and the phase-2 dh buffer of down and the
+  // combine takes the dH columns once dH is staged as the phase-2 operand
+  static constexpr int NT = RP <= 64 ? 4 : 2;
   static constexpr int kOps = Slots<RP>::bytes(NT);
   static constexpr int kWBlk = RP * 128;
   static constexpr int kSlotA = 2 * kBlk + 2 * kWBlk;  // dY tile + B^T chunk (down phase 2: A chunk + h tile)
   static constexpr int kSlotB = 2 * kBlk;                      // down: dh tile for the RMW
-  static constexpr int SB = MODE != MODE_SHARED ? 2 : 0;
+  // down / combine: dh tiles of the RMW (one at RP = 128, where two would not
+  // fit beside the ring)
+  static constexpr int SB = MODE != MODE_SHARED ? (RP > 64 ? 1 : 2) : 0;
   static constexpr int kBudget = 220 * 1024;
   static constexpr int kSA0 = (kBudget - kOps - SB * kSlotB) / kSlotA;
   static constexpr int SA = kSA0 > 6 ? 6 : (kSA0 < 2 ? 2 : kSA0);
@@ -164,8 +167,10 @@ struct RowsCfg {
   // (phase 2) accumulators, 2 x RP columns, from kTB
   static constexpr int kTB = NT * RP > 128 ? 256 : 128;
   static constexpr int ND = (RP > 64 || kTB > 128) ? 1 : 2;  // down: dh D buffers of 128 columns
-  static constexpr int kDB = (RP > 64 || kTB > 128) ? 384 : 256;
+  static constexpr int kDB = RP > 64 ? 0 : (kTB > 128 ? 384 : 256);
   static constexpr int kTmem = (MODE != MODE_SHARED || RP > 64 || kTB > 128) ? 512 : 256;
+  static_assert(kSmem <= 227 * 1024, "shared memory per CTA");
+  static_assert(ND * kNcB + (kDB == 0 ? 0 : kDB) <= 512 && (kDB != 0 || ND * kNcB <= kTB), "TMEM: dh buffers");
 };
 
 template <int RP, int MODE>

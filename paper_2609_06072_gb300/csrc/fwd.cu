@@ -181,7 +181,8 @@ struct RowsFwdCfg {
   static constexpr int kSlot = NPROJ * (kBlk + kWBlk);      // Y tiles + B^T blocks (down K-step: h + A)
   static constexpr int kHs = ((NPROJ * RP + 63) / 64) * kBlk;  // bf16 H operand of one tile
   static constexpr int kBudget = 210 * 1024;
-  static constexpr int NBH = 2 * kHs + 4 * kSlot <= kBudget ? 2 : 1;  // H operand buffers
+  // H operand buffers: two wherever they fit beside three ring slots
+  static constexpr int NBH = 2 * kHs + 3 * kSlot <= kBudget ? 2 : 1;
   static constexpr int kS0 = (kBudget - NBH * kHs) / kSlot;
   // ring slots: down keeps at most 6 (7 or 8 measured slower, 6 the fastest)
   static constexpr int kSmax = SHARED ? 8 : 6;
@@ -245,7 +246,7 @@ struct TileQueue {
 // Consumer side: the next tile (false at the end or if a wait gave up; *ok
 // tells which).  Every lane of a warp calls it; lane 0 releases the entry.
 __device__ __forceinline__ bool queue_next(TileQueue& tq, int& q, const Tile* tiles, Tile& t, bool single_lane,
-                                           bool* ok) {
+                                           bool* ok, int psplit, int& pj) {
   const int e = q % kQ;
   bool w = mbar_wait(&tq.full[e], (q / kQ) & 1);
   if (!single_lane) w = __all_sync(0xffffffffu, w);
@@ -258,7 +259,8 @@ __device__ __forceinline__ bool queue_next(TileQueue& tq, int& q, const Tile* ti
   if (single_lane || (threadIdx.x & 31) == 0) mbar_arrive(&tq.empty[e]);
   ++q;
   if (item < 0) return false;
-  t = tiles[item];
+  t = tiles[item >> psplit];
+  pj = item & psplit;
   return true;
 }
 // Persistent: one CTA per SM; tiles of <= 128 consecutive rows of one group
@@ -324,6 +326,9 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
   // instead of repeating the K loop, so the last work comes in halves
   const bool pre = !SHARED && a.pre != 0;
   const int merge = SHARED ? 2 : (pre ? 1 : kSplitParts);  // parts of a split tile taken together
+  // gate/up with the two projections as separate work items (one projection
+  // per kernel instance, NPROJ == 1): 1, else 0
+  const int psplit = (SHARED && NPROJ == 1 && a.proj_split) ? 1 : 0;
   const int split0 = a.counts[kCntRowSplit], n_split = (n_items - split0) / kSplitParts;
   const bool has_pre = pre && (int)blockIdx.x < n_split;
   Tile pre_t{};
@@ -347,8 +352,10 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
       // take the next tile (the counter runs over the entries this kernel
       // takes: every unsplit tile, then every merge-th part entry), or the
       // end; hand it on
-      const int n_take = split0 + (n_items - split0) / merge;
-      auto grab = [&](Tile& t) -> bool {
+      // with the projections split, counter value v names projection v & 1
+      // of entry v >> 1, and the queue carries (entry << 1) | projection
+      const int n_take = (split0 + (n_items - split0) / merge) << psplit;
+      auto grab = [&](Tile& t, int& pj) -> bool {
         int item;
         while (true) {
           const int v = atomicAdd(a.sched + kSchedFwdRows, 1);
@@ -356,8 +363,10 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
             item = -1;
             break;
           }
-          item = v < split0 ? v : split0 + (v - split0) * merge;
+          const int vt = v >> psplit;
+          item = vt < split0 ? vt : split0 + (vt - split0) * merge;
           t = a.tiles[item];
+          pj = v & psplit;
           if (tile_live(t, merge)) break;
         }
         const int e = q % kQ;
@@ -365,7 +374,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
           bad = true;
           return false;
         }
-        tq.item[e] = item;
+        tq.item[e] = item < 0 ? -1 : (item << psplit) | pj;
         mbar_arrive(&tq.full[e]);
         ++q;
         return item >= 0;
@@ -388,7 +397,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
         tma_load_2d(base + NPROJ * kBlk, &a.tm_a, k * 64, pt.rank_off[t.g], &full[s]);
         ++i;
       };
-      auto load_c = [&](const Tile& t, int c) {
+      auto load_c = [&](const Tile& t, int pj, int c) {
         const uint32_t s = acquire(false);
         if (bad) return;
         const uint32_t base = slot0 + s * C::kSlot;
@@ -396,23 +405,26 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
         mbar_arrive_expect_tx(&full[s], NPROJ * (rows_bytes(t.cnt) + C::kWBlk));
 #pragma unroll
         for (int j = 0; j < NPROJ; ++j) {
-          load_rows(base + j * kBlk, &a.tm_y[j], &a.tm_y16[j], n0, t.start, t.cnt, &full[s]);
-          tma_load_2d(base + NPROJ * kBlk + j * C::kWBlk, &a.tm_bt[j], n0, pt.rank_off[t.g], &full[s]);
+          const int jj = j + pj;  // the tensors' projection (pj = 0 unless the projections are split)
+          load_rows(base + j * kBlk, &a.tm_y[jj], &a.tm_y16[jj], n0, t.start, t.cnt, &full[s]);
+          tma_load_2d(base + NPROJ * kBlk + j * C::kWBlk, &a.tm_bt[jj], n0, pt.rank_off[t.g], &full[s]);
         }
         ++i;
       };
       Tile cur, nxt;
+      int pcur = 0, pnxt = 0;
       if (has_pre)
         for (int k = 0; k < NK && !bad; ++k) load_k(pre_t, k);
-      bool has_cur = grab(cur);
+      bool has_cur = grab(cur, pcur);
       if (has_cur && needs_k(cur))
         for (int k = 0; k < NK && !bad; ++k) load_k(cur, k);
       while (has_cur && !bad) {
-        const bool has_nxt = grab(nxt);
-        for (int c = chunk_lo(cur, nch, merge); c < chunk_hi(cur, nch, merge) && !bad; ++c) load_c(cur, c);
+        const bool has_nxt = grab(nxt, pnxt);
+        for (int c = chunk_lo(cur, nch, merge); c < chunk_hi(cur, nch, merge) && !bad; ++c) load_c(cur, pcur, c);
         if (has_nxt && needs_k(nxt))
           for (int k = 0; k < NK && !bad; ++k) load_k(nxt, k);
         cur = nxt;
+        pcur = pnxt;
         has_cur = has_nxt;
       }
       // every copy issued has landed before the CTA can exit
@@ -470,18 +482,19 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
         ++i;
       };
       Tile cur, nxt;
+      int pdummy = 0;
       bool qok = true;
       if (has_pre) {
         for (int k = 0; k < NK && !bad; ++k) mma_k(kc & 1, k);
         ++kc;
       }
-      bool has_cur = queue_next(tq, q, a.tiles, cur, true, &qok);
+      bool has_cur = queue_next(tq, q, a.tiles, cur, true, &qok, psplit, pdummy);
       if (has_cur && needs_k(cur)) {
         for (int k = 0; k < NK && !bad; ++k) mma_k(kc & 1, k);
         ++kc;
       }
       while (has_cur && !bad) {
-        const bool has_nxt = queue_next(tq, q, a.tiles, nxt, true, &qok);
+        const bool has_nxt = queue_next(tq, q, a.tiles, nxt, true, &qok, psplit, pdummy);
         const int lo = chunk_lo(cur, nch, merge), hi = chunk_hi(cur, nch, merge);
         for (int c = lo; c < hi && !bad; ++c) mma_c(c == lo, c == hi - 1);
         ++ci;
@@ -506,7 +519,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
     const float s = a.s;
     // H operand of chunk-tile ci (tile t, K-tile kt or -1) into buffer
     // ci % NBH: this warp's rows, its group's share of the columns
-    auto stage_h = [&](const Tile& t, int ci, int kt) {
+    auto stage_h = [&](const Tile& t, int pj, int ci, int kt) {
       const uint32_t sHs = sHs0 + (ci % NBH) * C::kHs;
       if (quarter * 32 >= t.cnt) return;  // no live row: these H rows feed only D rows nobody reads
       const bool live = m < t.cnt;
@@ -542,7 +555,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
         const int u = live ? (SHARED ? a.row_uniq[t.start + m] : t.start + m) : -1;
 #pragma unroll
         for (int j = 0; j < NPROJ; ++j) {
-          const float* hp = (SHARED ? a.Hu[j] : a.Hpre) + (int64_t)(u < 0 ? 0 : u) * pt.rank_max;
+          const float* hp = (SHARED ? a.Hu[j + pj] : a.Hpre) + (int64_t)(u < 0 ? 0 : u) * pt.rank_max;
           for (int c8 = grp * 8; c8 < RP; c8 += 8 * kNGrp) {
             float v[8];
 #pragma unroll
@@ -562,7 +575,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
     // loop): wait until the buffer's previous tile is done with it and the H
     // exists (down: the K loop, or the up-front H of a split tile), stage,
     // publish
-    auto prepare_h = [&](const Tile& t, int ci, int kt) -> bool {
+    auto prepare_h = [&](const Tile& t, int pj, int ci, int kt) -> bool {
       bool w = true;
       if (ci >= NBH) w = mbar_wait(&hs_free[ci % NBH], ((ci - NBH) / NBH) & 1);
       if (kt >= 0) w = w && mbar_wait(&hacc[kt & 1], (kt >> 1) & 1);
@@ -580,7 +593,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
         if (w) (void)ld_acquire(hflag + split_index(t));  // every lane's H loads follow an acquire
       }
       if (!__all_sync(0xffffffffu, w)) return false;
-      stage_h(t, ci, kt);
+      stage_h(t, pj, ci, kt);
       fence_proxy_async_smem();
       tc_fence_before();
       __syncwarp();
@@ -614,27 +627,28 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
     int q = 0, ib = 0, cc0 = 0, ci = 0, kc = 0;
     bool ok = true;
     Tile cur, nxt;
+    int pcur = 0, pnxt = 0;
     if (has_pre) {
       ok = drain_pre(pre_t, kc);
       ++kc;
       ib += NK;
     }
-    bool has_cur = ok && queue_next(tq, q, a.tiles, cur, false, &ok);
+    bool has_cur = ok && queue_next(tq, q, a.tiles, cur, false, &ok, psplit, pcur);
     if (has_cur) {
       int kt = -1;
       if (needs_k(cur)) {
         kt = kc++;
         ib += NK;
       }
-      ok = prepare_h(cur, ci, kt);
+      ok = prepare_h(cur, pcur, ci, kt);
     }
     while (has_cur && ok) {
-      const bool has_nxt = queue_next(tq, q, a.tiles, nxt, false, &ok);
+      const bool has_nxt = queue_next(tq, q, a.tiles, nxt, false, &ok, psplit, pnxt);
       if (!ok) break;
       const bool inter = has_nxt && needs_k(nxt);
       // gate/up with two H buffers: gather the next tile's H now, while this tile streams
       const bool early = SHARED && NBH == 2 && has_nxt;
-      if (early && !(ok = prepare_h(nxt, ci + 1, -1))) break;
+      if (early && !(ok = prepare_h(nxt, pnxt, ci + 1, -1))) break;
       const bool qlive = quarter * 32 < cur.cnt;  // this warp has live rows (warp-uniform)
       const int lo = chunk_lo(cur, nch, merge), hi = chunk_hi(cur, nch, merge);
       for (int c = lo + ((grp - cc0) % kNGrp + kNGrp) % kNGrp; c < hi; c += kNGrp) {
@@ -683,7 +697,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
               const int row = quarter * 32 + it * 4 + (lane >> 3), ch = lane & 7, col = n0 + ch * 8;
               if (row < cur.cnt && col < d_out) {
                 const uint4 v = lds128(base + j * kBlk + sw128_off(row, ch));
-                *reinterpret_cast<uint4*>(a.Y[j] + (int64_t)(cur.start + row) * d_out + col) = v;
+                *reinterpret_cast<uint4*>(a.Y[j + pcur] + (int64_t)(cur.start + row) * d_out + col) = v;
               }
             }
         }
@@ -692,11 +706,12 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
         if (lane == 0) mbar_arrive(&emptyC[sl]);
       }
       if (!ok) break;
-      if (has_nxt && !early && !(ok = prepare_h(nxt, ci + 1, inter ? kc++ : -1))) break;
+      if (has_nxt && !early && !(ok = prepare_h(nxt, pnxt, ci + 1, inter ? kc++ : -1))) break;
       ib += (hi - lo) + (inter ? NK : 0);
       cc0 += hi - lo;
       ++ci;
       cur = nxt;
+      pcur = pnxt;
       has_cur = has_nxt;
     }
     if (!ok) bad = true;
@@ -771,11 +786,18 @@ cudaError_t launch_fwd_rows(const PlanTables& pt, const FwdRowsLaunch& a, bool s
       case 128: return launch_rows_t<128, 1, false>(pt, a, st);
     }
   } else if (a.nproj == 2) {
+    // at rank_pad 128 a tile's two projections go out as separate work
+    // items: their shared-memory budget then leaves room for two H operand
+    // buffers and four ring slots (both projections in one item: one H
+    // buffer and two slots).  At rank_pad 64 one item holding both
+    // projections measured faster.
+    FwdRowsLaunch b = a;
+    b.proj_split = 1;
     switch (pt.rank_pad) {
       case 16: return launch_rows_t<16, 2, true>(pt, a, st);
       case 32: return launch_rows_t<32, 2, true>(pt, a, st);
       case 64: return launch_rows_t<64, 2, true>(pt, a, st);
-      case 128: return launch_rows_t<128, 2, true>(pt, a, st);
+      case 128: return launch_rows_t<128, 1, true>(pt, b, st);
     }
   } else {
     switch (pt.rank_pad) {

@@ -174,6 +174,14 @@ struct DenseHLaunch {
   int32_t* err;
 };
 cudaError_t launch_dense_h(const PlanTables& pt, const DenseHLaunch& a, cudaStream_t st);
+}  // namespace ace
+struct ace_plan;
+namespace ace {
+// H_u of gate/up per unique pair into Hbuf[j] (api.cu): the token-major dense
+// H GEMM when a projection's stacked ranks are at most kDenseHMaxRank, else
+// the gathering H kernel.  Host-side status; launches on `st`.
+ace_status launch_gate_up_h(const ace_plan* plan, const ace_perm* perm, const uint16_t* X, int nproj,
+                            const uint16_t* const* A, float* const* Hbuf, cudaStream_t st);
 
 // Row-tile forward: Y[row] += s * B_g H_row over contiguous rows of a group.
 // MODE down: H_row = A_g h_row computed here (K loop over h);  gate/up:
@@ -294,6 +302,25 @@ cudaError_t launch_comb_reduce(const PlanTables& pt, const CombReduceLaunch& a, 
 cudaError_t launch_expert_gemm(const void* in, const void* W, const int32_t* expert_off, const int32_t* expert_cnt,
                                uint16_t* out, int E, int64_t R, int N, int K, int grid, int32_t* err,
                                cudaStream_t st, bool w_kn = false, bool accumulate = false);
+// Expert FFN forward with the adapters fused into the base GEMMs
+// (ffn_fused.cu): gate/up writes u, v, h = SiLU(v) u; down writes y.
+struct FfnFusedLaunch {
+  CUtensorMap tm_in;     // gate/up: x [R, d], down: h [R, f], in row order; box 64 x 128
+  CUtensorMap tm_w[2];   // gate/up: W_up, W_gate [E*f, d], box 64 x 128; down: W_down [E*d, f], box 64 x 256
+  CUtensorMap tm_bt[2];  // gate/up: B^T of up, gate [n_rank, f]; down: [n_rank, d]; box 64 x rank_pad
+  const int32_t* row_uniq;
+  const int32_t* expert_off;
+  const int32_t* expert_cnt;
+  const float* Hs[2];    // gate/up: H of up, gate per unique pair; down: H per row; stride rank_max
+  uint16_t* U;           // gate/up outputs [R, f] bf16 (row order): u, v, h
+  uint16_t* V;
+  uint16_t* Hh;
+  uint16_t* Y;           // down output [R, d] bf16
+  float s;
+  int32_t N, K, grid;    // output columns, reduction length, persistent CTAs
+  int32_t* err;
+};
+cudaError_t launch_ffn_fused(const PlanTables& pt, const FfnFusedLaunch& a, bool gate_up, cudaStream_t st);
 cudaError_t launch_gather_tokens(const int32_t* row_pair, const int32_t* counts, int k, int T, const uint16_t* X,
                                  uint16_t* dst, int64_t R, int cols, cudaStream_t st);
 cudaError_t launch_swiglu(const uint16_t* u, const uint16_t* v, uint16_t* h, int64_t n, cudaStream_t st);

@@ -137,6 +137,57 @@ BwdWs bwd_layout(const ace_plan* plan, int32_t T, void* base) {
 
 }  // namespace
 
+// H_u = A_g x_t per unique pair (g, t) of gate/up into Hbuf[j] (fp32, stride
+// rank_max): token-major dense tiles when the stacked ranks of a projection
+// are few (the MMA then also forms the products of the groups a token skips,
+// cheaper than gathering X once per active group), else gathered per unique
+// pair.
+namespace ace {
+ace_status launch_gate_up_h(const ace_plan* plan, const ace_perm* perm, const uint16_t* X, int nproj,
+                            const uint16_t* const* A, float* const* Hbuf, cudaStream_t cs) {
+  const PlanTables& pt = plan->pt;
+  const PermLayout L = perm_layout(pt, perm->T);
+  const int n_rank = pt.rank_off[pt.G];
+  const int d_in = pt.d;
+  int32_t* err = at<int32_t>(perm->ws, L.err);
+  ace_status st = ACE_OK;
+  if (n_rank <= kDenseHMaxRank) {
+    DenseHLaunch h{};
+    bool okh = make_tmap_bf16(&h.tm_x, X, (uint64_t)perm->T, (uint64_t)d_in, kTileM);
+    for (int j = 0; j < nproj; ++j) okh = okh && make_tmap_bf16(&h.tm_a[j], A[j], (uint64_t)n_rank, (uint64_t)d_in, 256);
+    if (!okh) return fail(ACE_ERR_UNSUPPORTED, "tensor-map encoding failed for this layout");
+    h.tok_uniq = perm->tok_uniq;
+    h.uniq_off = perm->uniq_off;
+    for (int j = 0; j < 2; ++j) h.H[j] = Hbuf[j < nproj ? j : 0];
+    h.T = perm->T;
+    h.d = d_in;
+    h.n_rank = n_rank;
+    h.nproj = nproj;
+    h.rank_max = pt.rank_max;
+    h.grid = plan->num_sms;
+    h.err = err;
+    st = cuda_status(launch_dense_h(pt, h, cs), "forward H launch");
+  } else {
+    FwdHLaunch h{};
+    h.tiles = at<Tile>(perm->ws, L.tiles_sh);
+    h.counts = perm->counts;
+    h.max_tiles = L.max_tiles;
+    h.uniq_tok = perm->uniq_tok;
+    h.X = X;
+    for (int j = 0; j < 2; ++j) {
+      const int jj = j < nproj ? j : 0;
+      h.A[j] = A[jj];
+      h.H[j] = Hbuf[jj];
+    }
+    h.d_in = d_in;
+    h.nproj = nproj;
+    h.err = err;
+    st = cuda_status(launch_fwd_h(pt, h, cs), "forward H launch");
+  }
+  return st;
+}
+}  // namespace ace
+
 extern "C" {
 
 int32_t ace_version(void) { return ACE_VERSION; }
@@ -287,44 +338,8 @@ static ace_status fwd_common(const ace_plan* plan, const ace_perm* perm, const u
     for (int j = 0; j < nproj; ++j)
       if (!Hbuf[j]) Hbuf[j] = reinterpret_cast<float*>(static_cast<char*>(ws) + j * align_up(4 * (size_t)R * pt.rank_max, 256));
   }
-  // H_u of gate/up: token-major dense tiles when the stacked ranks of a
-  // projection are few (the MMA then also forms the products of the groups a
-  // token skips, cheaper than gathering X once per active group), else
-  // gathered per unique pair
-  const bool dense_h = shared && n_rank <= kDenseHMaxRank;
-  if (dense_h) {
-    DenseHLaunch h{};
-    bool okh = make_tmap_bf16(&h.tm_x, X, (uint64_t)perm->T, (uint64_t)d_in, kTileM);
-    for (int j = 0; j < nproj; ++j) okh = okh && make_tmap_bf16(&h.tm_a[j], A[j], (uint64_t)n_rank, (uint64_t)d_in, 256);
-    if (!okh) return fail(ACE_ERR_UNSUPPORTED, "tensor-map encoding failed for this layout");
-    h.tok_uniq = perm->tok_uniq;
-    h.uniq_off = perm->uniq_off;
-    for (int j = 0; j < 2; ++j) h.H[j] = Hbuf[j < nproj ? j : 0];
-    h.T = perm->T;
-    h.d = d_in;
-    h.n_rank = n_rank;
-    h.nproj = nproj;
-    h.rank_max = pt.rank_max;
-    h.grid = plan->num_sms;
-    h.err = err;
-    st = cuda_status(launch_dense_h(pt, h, cs), "forward H launch");
-    if (st != ACE_OK) return st;
-  } else if (shared) {
-    FwdHLaunch h{};
-    h.tiles = at<Tile>(perm->ws, L.tiles_sh);
-    h.counts = perm->counts;
-    h.max_tiles = L.max_tiles;
-    h.uniq_tok = perm->uniq_tok;
-    h.X = X;
-    for (int j = 0; j < 2; ++j) {
-      const int jj = j < nproj ? j : 0;
-      h.A[j] = A[jj];
-      h.H[j] = Hbuf[jj];
-    }
-    h.d_in = d_in;
-    h.nproj = nproj;
-    h.err = err;
-    st = cuda_status(launch_fwd_h(pt, h, cs), "forward H launch");
+  if (shared) {
+    st = launch_gate_up_h(plan, perm, X, nproj, A, Hbuf, cs);
     if (st != ACE_OK) return st;
   }
   FwdRowsLaunch r{};

@@ -394,31 +394,75 @@ ace_status ace_ffn_fwd(const ace_plan* plan, const ace_perm* perm, const uint16_
   cudaStream_t cs = static_cast<cudaStream_t>(stream);
   const PermLayout L = perm_layout(pt, perm->T);
   int32_t* err = at<int32_t>(perm->ws, L.err);
-  uint16_t* Xr = static_cast<uint16_t*>(ws);
   auto cuda = [](cudaError_t e, const char* what) {
     return e == cudaSuccess ? ACE_OK : report(ACE_ERR_CUDA, what);
   };
-  ace_status st = cuda(launch_gather_tokens(perm->row_pair, perm->counts, pt.k, perm->T, X, Xr, R, pt.d, cs),
-                       "ace_ffn_fwd: gather launch");
-  if (st != ACE_OK) return st;
-  st = cuda(launch_expert_gemm(Xr, W_up, perm->expert_off, perm->expert_cnt, U, pt.E, R, pt.f, pt.d, plan->num_sms,
-                               err, cs), "ace_ffn_fwd: up GEMM launch");
-  if (st != ACE_OK) return st;
-  st = cuda(launch_expert_gemm(Xr, W_gate, perm->expert_off, perm->expert_cnt, V, pt.E, R, pt.f, pt.d,
-                               plan->num_sms, err, cs), "ace_ffn_fwd: gate GEMM launch");
-  if (st != ACE_OK) return st;
-  // gate and up adapter deltas onto v and u (shared input, deduplicated A_g x)
+  const int n_rank = pt.rank_off[pt.G];
+  // 1. H of gate and up per unique pair, A_g x once per active group of a token
   const uint16_t* Agu[2] = {A[0], A[1]};
-  const uint16_t* Bgu[2] = {Bt[0], Bt[1]};
-  uint16_t* Ygu[2] = {V, U};
-  st = ace_fwd_shared(plan, perm, X, 2, Agu, Bgu, s, Ygu, Hgu, nullptr, 0, stream);
+  float* Hgu_buf[2] = {Hgu[0], Hgu[1]};
+  ace_status st = launch_gate_up_h(plan, perm, X, 2, Agu, Hgu_buf, cs);
   if (st != ACE_OK) return st;
-  st = cuda(launch_swiglu(U, V, Hh, R * pt.f, cs), "ace_ffn_fwd: SiLU gating launch");
+  // 2. the token rows in row order, then u, v (base + adapter) and
+  // h = SiLU(v) u in one kernel
+  uint16_t* Xr = static_cast<uint16_t*>(ws);
+  st = cuda(launch_gather_tokens(perm->row_pair, perm->counts, pt.k, perm->T, X, Xr, R, pt.d, cs),
+            "ace_ffn_fwd: gather launch");
   if (st != ACE_OK) return st;
-  st = cuda(launch_expert_gemm(Hh, W_down, perm->expert_off, perm->expert_cnt, Y, pt.E, R, pt.d, pt.f,
-                               plan->num_sms, err, cs), "ace_ffn_fwd: down GEMM launch");
+  FfnFusedLaunch g{};
+  bool ok = make_tmap_bf16(&g.tm_in, Xr, (uint64_t)R, (uint64_t)pt.d, 128) &&
+            make_tmap_bf16(&g.tm_w[0], W_up, (uint64_t)pt.E * pt.f, (uint64_t)pt.d, 128) &&
+            make_tmap_bf16(&g.tm_w[1], W_gate, (uint64_t)pt.E * pt.f, (uint64_t)pt.d, 128) &&
+            make_tmap_bf16(&g.tm_bt[0], Bt[1], (uint64_t)n_rank, (uint64_t)pt.f, pt.rank_pad) &&
+            make_tmap_bf16(&g.tm_bt[1], Bt[0], (uint64_t)n_rank, (uint64_t)pt.f, pt.rank_pad);
+  if (!ok) return report(ACE_ERR_UNSUPPORTED, "ace_ffn_fwd: tensor-map encoding failed");
+  g.row_uniq = at<int32_t>(perm->ws, L.row_uniq);
+  g.expert_off = perm->expert_off;
+  g.expert_cnt = perm->expert_cnt;
+  g.Hs[0] = Hgu[1];  // TMEM half 0: up
+  g.Hs[1] = Hgu[0];  // TMEM half 1: gate
+  g.U = U;
+  g.V = V;
+  g.Hh = Hh;
+  g.s = s;
+  g.N = pt.f;
+  g.K = pt.d;
+  g.grid = plan->num_sms;
+  g.err = err;
+  st = cuda(launch_ffn_fused(pt, g, true, cs), "ace_ffn_fwd: gate/up launch");
   if (st != ACE_OK) return st;
-  return ace_fwd_row(plan, perm, Hh, A[2], Bt[2], s, Y, Hd, nullptr, 0, stream);
+  // 3. H of down per row, A_g h
+  FwdHLaunch hd{};
+  hd.tiles = at<Tile>(perm->ws, L.tiles_row);
+  hd.counts = perm->counts;
+  hd.max_tiles = L.max_tiles;
+  hd.rows = 1;
+  hd.X = Hh;
+  hd.A[0] = hd.A[1] = A[2];
+  hd.H[0] = hd.H[1] = Hd;
+  hd.d_in = pt.f;
+  hd.nproj = 1;
+  hd.err = err;
+  st = cuda(launch_fwd_h(pt, hd, cs), "ace_ffn_fwd: down H launch");
+  if (st != ACE_OK) return st;
+  // 4. y (base + adapter)
+  FfnFusedLaunch dn{};
+  ok = make_tmap_bf16(&dn.tm_in, Hh, (uint64_t)R, (uint64_t)pt.f, 128) &&
+       make_tmap_bf16(&dn.tm_w[0], W_down, (uint64_t)pt.E * pt.d, (uint64_t)pt.f, 256) &&
+       make_tmap_bf16(&dn.tm_bt[0], Bt[2], (uint64_t)n_rank, (uint64_t)pt.d, pt.rank_pad);
+  if (!ok) return report(ACE_ERR_UNSUPPORTED, "ace_ffn_fwd: tensor-map encoding failed");
+  dn.tm_w[1] = dn.tm_w[0];
+  dn.tm_bt[1] = dn.tm_bt[0];
+  dn.expert_off = perm->expert_off;
+  dn.expert_cnt = perm->expert_cnt;
+  dn.Hs[0] = dn.Hs[1] = Hd;
+  dn.Y = Y;
+  dn.s = s;
+  dn.N = pt.d;
+  dn.K = pt.f;
+  dn.grid = plan->num_sms;
+  dn.err = err;
+  return cuda(launch_ffn_fused(pt, dn, false, cs), "ace_ffn_fwd: down launch");
 }
 
 ace_status ace_ffn_bwd(const ace_plan* plan, const ace_perm* perm, const uint16_t* dY, const uint16_t* X,

@@ -1,9 +1,16 @@
-"""GPU parity of the routed expert FFN forward with the group-shared
-adapters (base expert GEMMs, adapter deltas, SiLU gating) against the FFN
-oracle.  The composed path rounds u, v, h and y to bf16 between its steps
-(two roundings on u and v, whose base part is stored before the adapter
-delta is added), so the bar is a relative Frobenius error of 1e-2 and a
-maximum error of 3e-2 of the largest reference value."""
+"""GPU parity of the routed expert FFN with the group-shared adapters
+against the FFN oracle.
+
+Forward (ace_ffn_fwd): the base expert GEMMs with the adapter deltas fused in
+as extra K steps of the same accumulators, and the SiLU gating in the gate/up
+epilogue, so u, v, h and y are each rounded to bf16 once; held to the per-
+tensor bar of the other parity tests (max|err| <= 2e-2 max|ref|, relative
+Frobenius error <= 5e-3).  y is formed from the bf16 h, the oracle's from the
+exact h.
+Backward (ace_ffn_bwd): composed from the base input-gradient GEMMs and the
+adapter backward calls, which round dh, du and dv to bf16 between steps; its
+bar is a relative Frobenius error of 1e-2 and a maximum error of 3e-2 of the
+largest reference value."""
 import numpy as np
 import pytest
 
@@ -24,7 +31,13 @@ def _dec(b):
 # so that the oracle's base weights stay small
 @pytest.mark.parametrize("name,seed,over", [("tiny", 0, {}), ("tiny", 1, {"T": 300}),
                                             ("olmoe", 0, {"T": 256, "d": 512, "f": 256}),
-                                            ("olmoe_uneven", 0, {"T": 128, "d": 512, "f": 256})])
+                                            # rank_pad 64, f = 3 chunks of 128
+                                            ("qwen", 0, {"T": 128, "d": 512, "f": 384}),
+                                            # rank_pad 128 (r_g 2 .. 86)
+                                            ("olmoe_uneven", 0, {"T": 128, "d": 512, "f": 256}),
+                                            # d and f not multiples of the 64-column K steps or the
+                                            # 128 / 256-column output chunks; top-1 routing
+                                            ("tiny", 11, {"d": 200, "f": 120, "T": 77}), ("tiny", 8, {"k": 1})])
 def test_ffn_forward_parity(name, seed, over):
     import torch
     L = W.Layer(W.get_config(name, **over), seed=seed)
@@ -52,7 +65,7 @@ def test_ffn_forward_parity(name, seed, over):
     for name_, t in (("u", U), ("v", V), ("h", Hh), ("y", Y)):
         got = np.empty_like(ref[name_])
         got[rp] = host_f64(t)
-        check_close(got, ref[name_], name_, max_rel=3e-2, fro_rel=1e-2)
+        check_close(got, ref[name_], name_)
 
 
 @pytest.mark.parametrize("name,seed,over", [("tiny", 0, {}), ("tiny", 4, {"r": 3}),

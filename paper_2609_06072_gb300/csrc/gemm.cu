@@ -238,6 +238,218 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemm_dx(const __grid_constant__
   if (warp == 0) tmem_dealloc(tmem, 2 * kDxN);
 }
 
+// ------------------------------------------------------------------ dX on CTA pairs
+// The same product on clusters of two CTAs whose tensor cores share one
+// M = 256 MMA (cta_group::2): a pair computes a [256-token x 256-column] tile,
+// each CTA holding the dHx rows of its 128 tokens and 128 of the 256 weight
+// columns, so a CTA receives 32 KB per K step for the work that takes 48 KB
+// on a single CTA, and six stages fit in flight.  Both CTAs' loads count on
+// the leader's stage barrier; the leader issues the MMAs and its commits
+// arrive in both CTAs; each CTA's epilogue reads its own 128 accumulator rows
+// and tells the leader when they are read.  Two accumulators of 256 columns,
+// so a tile's epilogue overlaps the next tile's K loop; the tiles left after
+// the last whole round go out as column halves (N = 128).
+constexpr int kD2S = 6;
+constexpr int kD2Stage = kBlk + 2 * kHalfBlk;  // dHx [128 t x 64 k] + A [64 k x 128 d]
+constexpr int kD2Smem = kD2S * kD2Stage + 8 * kDxWarpBlk + 1024;
+constexpr uint32_t kD2Tmem = 512;
+
+// Work item `it` of pair `pair` (of npair): as dx_item, over pair tiles.
+__device__ __forceinline__ bool d2_item(int it, int ntile, int pair, int npair, int& tile, int& half) {
+  const int full = ntile / npair, rem = ntile % npair;
+  if (it < full) {
+    tile = it * npair + pair;
+    half = -1;
+    return true;
+  }
+  const int h = (it - full) * npair + pair;
+  if (h >= 2 * rem) return false;
+  tile = full * npair + h / 2;
+  half = h & 1;
+  return true;
+}
+
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+    k_gemm2_dx(const __grid_constant__ DenseBwdLaunch a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  __shared__ __align__(8) uint64_t full[kD2S], empty[kD2S], acc_full[2], acc_empty[2];
+  __shared__ uint32_t tslot;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const uint32_t rank = cluster_ctarank();
+  const int npair = gridDim.x / 2, pair = blockIdx.x / 2;
+  const int ncol = (a.d + kDxN - 1) / kDxN, ntile = ((a.T + 255) / 256) * ncol;
+  const int ksteps = a.n_rank_pad / 64;
+  const int NK = a.nproj * ksteps;
+  const uint32_t s0 = smem_u32(smem);
+  if (tid == 0) {
+    for (int i = 0; i < kD2S; ++i) {
+      mbar_init(&full[i], 1);   // the leader's arm; both CTAs' bytes
+      mbar_init(&empty[i], 1);  // the leader's commit
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&acc_full[i], 1);
+      mbar_init(&acc_empty[i], 16);  // every epilogue warp of both CTAs
+    }
+    fence_mbar_init();
+  }
+  if (warp == 0) tmem_alloc_pair(&tslot, kD2Tmem);
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // the peer's barriers exist before anything arrives on them
+  tc_fence_after();
+  pdl_wait();
+  const uint32_t tmem = tslot;
+  bool bad = false;
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer (both CTAs)
+    if (lane == 0) {
+      int i = 0, tile, half;
+      for (int it = 0; d2_item(it, ntile, pair, npair, tile, half) && !bad; ++it) {
+        const int t0 = (tile / ncol) * 256 + (int)rank * 128;
+        // this CTA's half of the item's columns (a whole tile: 128 of 256; a column half: 64 of 128)
+        const int cw = half < 0 ? 128 : 64;
+        const int c0 = (tile % ncol) * kDxN + (half > 0 ? kDxN / 2 : 0) + (int)rank * cw;
+        for (int kb = 0; kb < NK; ++kb, ++i) {
+          const int s = i % kD2S, u = i / kD2S;
+          if (u >= 1 && !mbar_wait(&empty[s], (u - 1) & 1)) {
+            bad = true;
+            break;
+          }
+          const int j = kb / ksteps, ks = kb % ksteps;
+          const uint32_t base = s0 + s * kD2Stage;
+          const uint32_t bar = mapa_shared(smem_u32(&full[s]), 0);
+          if (rank == 0) mbar_arrive_expect_tx(&full[s], 2 * (kBlk + (cw / 64) * kHalfBlk));
+          tma_load_2d_pair(base, &a.tm_dhx, j * a.n_rank_pad + ks * 64, t0, bar);
+          tma_load_2d_pair(base + kBlk, &a.tm_acat[j], c0, ks * 64, bar);
+          if (cw == 128) tma_load_2d_pair(base + kBlk + kHalfBlk, &a.tm_acat[j], c0 + 64, ks * 64, bar);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer (leader)
+    if (lane == 0 && rank == 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(256, kDxN, 0, 1);
+      constexpr uint32_t idesc_half = idesc_bf16_f32(256, kDxN / 2, 0, 1);
+      int i = 0, tile, half;
+      for (int it = 0; d2_item(it, ntile, pair, npair, tile, half) && !bad; ++it) {
+        const int b = it & 1;
+        const uint32_t id = half < 0 ? idesc : idesc_half;
+        if (it >= 2 && !mbar_wait(&acc_empty[b], ((it - 2) >> 1) & 1)) {
+          bad = true;
+          break;
+        }
+        tc_fence_after();
+        for (int kb = 0; kb < NK; ++kb, ++i) {
+          const int s = i % kD2S;
+          if (!mbar_wait(&full[s], (i / kD2S) & 1)) {
+            bad = true;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t base = s0 + s * kD2Stage;
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            tc_mma_bf16_pair(tmem + b * kDxN, sdesc_sw128(base + kk * 32, 16, 1024),
+                             sdesc_sw128(base + kBlk + kk * 2048, kHalfBlk, 1024), id, (kb > 0 || kk > 0) ? 1u : 0u);
+          tc_commit_pair(&empty[s]);
+        }
+        if (!bad) tc_commit_pair(&acc_full[b]);
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue (both CTAs): this CTA's 128 tokens
+    const int quarter = warp & 3, ehalf = (warp - 2) >> 2;  // this warp: 32 rows x 128 columns
+    const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
+    const uint32_t wb = s0 + kD2S * kD2Stage + (warp - 2) * kDxWarpBlk;
+    const uint32_t acc_empty_leader[2] = {mapa_shared(smem_u32(&acc_empty[0]), 0),
+                                          mapa_shared(smem_u32(&acc_empty[1]), 0)};
+    int tile, half;
+    for (int it = 0; d2_item(it, ntile, pair, npair, tile, half); ++it) {
+      const int b = it & 1;
+      const int tq = (tile / ncol) * 256 + (int)rank * 128 + quarter * 32;  // first token of this warp's rows
+      // first column of this warp's block; of a column half only the ehalf 0
+      // warps have one (the accumulator's first 128 columns)
+      const int cb = (tile % ncol) * kDxN + (half < 0 ? ehalf : half) * 128;
+      if (half >= 0 && ehalf == 1) {
+        if (!__all_sync(0xffffffffu, mbar_wait(&acc_full[b], (it >> 1) & 1))) {
+          bad = true;
+          break;
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_cluster(acc_empty_leader[b]);
+        continue;
+      }
+      uint4 later[8];
+#pragma unroll
+      for (int k2 = 0; k2 < 8; ++k2) {
+        const int r = k2 * 4 + (lane >> 3), c = lane & 7, t = tq + r, col = cb + c * 8;
+        const uint4 v = (t < a.T && col < a.d) ? *reinterpret_cast<const uint4*>(a.dX + (int64_t)t * a.d + col)
+                                               : make_uint4(0, 0, 0, 0);
+        later[k2] = (t < a.T && col + 64 < a.d) ? *reinterpret_cast<const uint4*>(a.dX + (int64_t)t * a.d + col + 64)
+                                                : make_uint4(0, 0, 0, 0);
+        sts128(wb + dx_off(r, c), v);
+      }
+      if (!__all_sync(0xffffffffu, mbar_wait(&acc_full[b], (it >> 1) & 1))) {
+        bad = true;
+        break;
+      }
+      tc_fence_after();
+#pragma unroll
+      for (int pass = 0; pass < 2; ++pass) {
+        if (pass == 1) {
+#pragma unroll
+          for (int k2 = 0; k2 < 8; ++k2) sts128(wb + dx_off(k2 * 4 + (lane >> 3), lane & 7), later[k2]);
+          __syncwarp();
+        }
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          uint32_t r[32];
+          const uint32_t ta = tmem + lane_base + b * kDxN + ehalf * 128 + pass * 64 + h * 32;
+          tmem_ld16(ta, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
+          tmem_ld16(ta + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
+          tmem_ld_wait();
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const uint32_t addr = wb + dx_off(lane, h * 4 + q);
+            const uint4 y = lds128(addr);
+            const uint32_t* dq = &r[q * 8];
+            const float2 f0 = unpack_bf16x2(y.x), f1 = unpack_bf16x2(y.y), f2 = unpack_bf16x2(y.z),
+                         f3 = unpack_bf16x2(y.w);
+            uint4 o;
+            o.x = pack_bf16x2(f0.x + __uint_as_float(dq[0]), f0.y + __uint_as_float(dq[1]));
+            o.y = pack_bf16x2(f1.x + __uint_as_float(dq[2]), f1.y + __uint_as_float(dq[3]));
+            o.z = pack_bf16x2(f2.x + __uint_as_float(dq[4]), f2.y + __uint_as_float(dq[5]));
+            o.w = pack_bf16x2(f3.x + __uint_as_float(dq[6]), f3.y + __uint_as_float(dq[7]));
+            sts128(addr, o);
+          }
+        }
+        if (pass == 1) {  // this warp's accumulator rows are read out: tell the leader
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive_cluster(acc_empty_leader[b]);
+        }
+        __syncwarp();
+#pragma unroll
+        for (int k2 = 0; k2 < 8; ++k2) {
+          const int r = k2 * 4 + (lane >> 3), c = lane & 7, t = tq + r, col = cb + pass * 64 + c * 8;
+          if (t < a.T && col < a.d)
+            *reinterpret_cast<uint4*>(a.dX + (int64_t)t * a.d + col) = lds128(wb + dx_off(r, c));
+        }
+        __syncwarp();
+      }
+      __syncwarp();
+    }
+  }
+  __syncwarp();
+  tc_fence_before();
+  if (__syncthreads_or(bad) && tid == 0) atomicOr(a.err, kErrTimeout);
+  cluster_sync();  // no arrival or copy of the pair is still headed for this CTA
+  pdl_trigger();
+  if (warp == 0) tmem_dealloc_pair(tmem, kD2Tmem);
+}
+
 // ------------------------------------------------------------------ dA
 // Output tiles of [128 stacked rank rows x 256 columns]; when the tiles alone
 // leave SMs idle the token (K) loop is split in two halves, and each CTA adds
@@ -544,6 +756,13 @@ cudaError_t launch_dense_h(const PlanTables& pt, const DenseHLaunch& a, cudaStre
 
 cudaError_t launch_dense_dx(const DenseBwdLaunch& a, cudaStream_t st) {
   if (a.T == 0) return cudaSuccess;
+  if (a.T >= 256 && a.grid >= 2) {
+    // CTA pairs: one per two SMs
+    cudaError_t e = cudaFuncSetAttribute(k_gemm2_dx, cudaFuncAttributeMaxDynamicSharedMemorySize, kD2Smem);
+    if (e != cudaSuccess) return e;
+    const int pairs = std::min(((a.T + 255) / 256) * ((a.d + kDxN - 1) / kDxN), a.grid / 2);
+    return launch_k(k_gemm2_dx, 2 * pairs, kThreads, kD2Smem, st, a);
+  }
   cudaError_t e = cudaFuncSetAttribute(k_gemm_dx, cudaFuncAttributeMaxDynamicSharedMemorySize, kDxSmem);
   if (e != cudaSuccess) return e;
   const int dx_tiles = ((a.T + 127) / 128) * ((a.d + kDxN - 1) / kDxN);

@@ -203,6 +203,7 @@ class Layer:
         self.dBt = [torch.empty(nr, f, device=dev), torch.empty(nr, f, device=dev), torch.empty(nr, d, device=dev)]
         self.h_grads = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in self.dA + self.dBt]
         self.perm = None
+        self._randn = randn
         # down through the gate-weighted combine: token-space output and gradient
         self.combine = combine
         if combine:
@@ -222,12 +223,14 @@ class Layer:
         # plus a dA reduce in deterministic mode
         return (16 if self.combine else 12) + (4 if self.det else 0)
 
-    def step(self, ev=None):
+    def step(self, ev=None, only=None):
         """One pass of the hot path.  ev: 6 CUDA events or None at the call
         boundaries (before permute, ..., after bwd_shared); None entries are
-        not recorded."""
+        not recorded.  only: a set of call names to run (the permutation
+        always runs), or None for all."""
         c, p = self.c, self.plan
         ev = ev or [None] * 6
+        run = lambda n: only is None or n in only
 
         def mark(j):
             if ev[j] is not None:
@@ -235,22 +238,75 @@ class Layer:
         mark(0)
         self.perm = p.permute(self.topk, self.pws)
         mark(1)
-        p.fwd_shared(self.perm, self.X, self.A[:2], self.Bt[:2], c.s, self.Y[:2], self.H[:2])
+        if run("fwd_shared"):
+            p.fwd_shared(self.perm, self.X, self.A[:2], self.Bt[:2], c.s, self.Y[:2], self.H[:2])
         mark(2)
         if self.combine:
-            p.fwd_combine(self.perm, self.hin, self.w, self.A[2], self.Bt[2], c.s, self.Z, self.H[2], self.Hx)
+            if run("fwd_row"):
+                p.fwd_combine(self.perm, self.hin, self.w, self.A[2], self.Bt[2], c.s, self.Z, self.H[2], self.Hx)
             mark(3)
-            p.bwd_combine(self.perm, self.dZ, self.hin, self.w, self.H[2], self.Hx, self.A[2], self.Bt[2], c.s,
-                          self.dh, self.dw, self.dA[2], self.dBt[2], self.bws)
+            if run("bwd_row"):
+                p.bwd_combine(self.perm, self.dZ, self.hin, self.w, self.H[2], self.Hx, self.A[2], self.Bt[2], c.s,
+                              self.dh, self.dw, self.dA[2], self.dBt[2], self.bws)
         else:
-            p.fwd_row(self.perm, self.hin, self.A[2], self.Bt[2], c.s, self.Y[2], self.H[2])
+            if run("fwd_row"):
+                p.fwd_row(self.perm, self.hin, self.A[2], self.Bt[2], c.s, self.Y[2], self.H[2])
             mark(3)
-            p.bwd_row(self.perm, self.dY[2], self.hin, self.H[2], self.A[2], self.Bt[2], c.s, self.dh, self.dA[2],
-                      self.dBt[2], self.bws)
+            if run("bwd_row"):
+                p.bwd_row(self.perm, self.dY[2], self.hin, self.H[2], self.A[2], self.Bt[2], c.s, self.dh,
+                          self.dA[2], self.dBt[2], self.bws)
         mark(4)
-        p.bwd_shared(self.perm, self.dY[:2], self.X, self.H[:2], self.A[:2], self.Bt[:2], c.s, self.dX,
-                     self.dA[:2], self.dBt[:2], self.bws)
+        if run("bwd_shared"):
+            p.bwd_shared(self.perm, self.dY[:2], self.X, self.H[:2], self.A[:2], self.Bt[:2], c.s, self.dX,
+                         self.dA[:2], self.dBt[:2], self.bws)
         mark(5)
+
+    # ---- end to end: every input of a step comes from pinned host memory and
+    # every result goes back, through two device sets so that one step's
+    # copies overlap the other's compute
+    _IN = ("topk", "X", "hin", "dY", "Y", "dX", "dh")   # routing, activations, upstream gradients, base outputs
+    _OUT = ("Y", "dX", "dh", "dA", "dBt")               # outputs with the deltas added, input and weight gradients
+
+    def e2e_setup(self):
+        import torch
+        dev = "cuda"
+        # host copies of the base outputs / input gradients the deltas accumulate onto, and of every result
+        self.h_Y = [self._randn(*t.shape).pin_memory() for t in self.Y]
+        self.h_dX = self._randn(*self.dX.shape).pin_memory()
+        self.h_dh = self._randn(*self.dh.shape).pin_memory()
+        self.h_out = {"Y": [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in self.Y],
+                      "dX": torch.empty(self.dX.shape, dtype=self.dX.dtype).pin_memory(),
+                      "dh": torch.empty(self.dh.shape, dtype=self.dh.dtype).pin_memory(),
+                      "dA": [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in self.dA],
+                      "dBt": [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in self.dBt]}
+        mk = lambda t: torch.empty(t.shape, dtype=t.dtype, device=dev)
+        self.sets = []
+        for _ in range(2):
+            st = {n: ([mk(x) for x in getattr(self, n)] if isinstance(getattr(self, n), list) else mk(getattr(self, n)))
+                  for n in set(self._IN) | set(self._OUT)}
+            self.sets.append(st)
+        self.h_in = {"topk": self.h_topk, "X": self.h_X, "hin": self.h_hin, "dY": self.h_dY, "Y": self.h_Y,
+                     "dX": self.h_dX, "dh": self.h_dh}
+
+    def use_set(self, st):
+        for n, v in st.items():
+            setattr(self, n, v)
+
+    def e2e_h2d(self, st):
+        for n in self._IN:
+            d, h = st[n], self.h_in[n]
+            for a, b in (zip(d, h) if isinstance(d, list) else [(d, h)]):
+                a.copy_(b, non_blocking=True)
+
+    def e2e_d2h(self, st):
+        for n in self._OUT:
+            d, h = st[n], self.h_out[n]
+            for a, b in (zip(h, d) if isinstance(d, list) else [(h, d)]):
+                a.copy_(b, non_blocking=True)
+
+    def e2e_bytes(self):
+        nb = lambda t: sum(x.numel() * x.element_size() for x in (t if isinstance(t, list) else [t]))
+        return sum(nb(self.h_in[n]) for n in self._IN), sum(nb(self.h_out[n]) for n in self._OUT)
 
     def h2d_inputs(self):
         self.topk.copy_(self.h_topk, non_blocking=True)
@@ -499,6 +555,58 @@ def time_cka(args, lay):
             "experts": c.E, "rank": c.r, "d_in": c.d, "d_out": c.f}
 
 
+def e2e_pipeline(args, lay, world):
+    """End-to-end rows/s through pinned host buffers (see run_gpu): host to
+    device copies on one stream, device to host on another (both directions of
+    the link at once), compute on the current stream."""
+    import torch
+    lay.e2e_setup()
+    main = torch.cuda.current_stream()
+    up, down = torch.cuda.Stream(), torch.cuda.Stream()
+    ev = lambda: torch.cuda.Event()
+    in_ready, done, freed = [ev(), ev()], [ev(), ev()], [ev(), ev()]
+    started = [False, False]
+
+    def run(n):
+        for i in range(n + 1):
+            if i < n:  # inputs of step i into set i % 2, once that set's previous results are back
+                b = i % 2
+                with torch.cuda.stream(up):
+                    if started[b]:
+                        up.wait_event(freed[b])
+                    lay.e2e_h2d(lay.sets[b])
+                    in_ready[b].record(up)
+            if i >= 1:  # compute step i - 1, then read its results back
+                b = (i - 1) % 2
+                main.wait_event(in_ready[b])
+                lay.use_set(lay.sets[b])
+                lay.step()
+                done[b].record(main)
+                with torch.cuda.stream(down):
+                    down.wait_event(done[b])
+                    lay.e2e_d2h(lay.sets[b])
+                    freed[b].record(down)
+                started[b] = True
+        main.wait_stream(up)
+        main.wait_stream(down)
+
+    run(2)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(main)
+    run(args.steps)
+    e1.record(main)
+    torch.cuda.synchronize()
+    assert lay.plan.get_error(lay.perm) == 0
+    ms = e0.elapsed_time(e1)
+    if world > 1:
+        ms = reduce_max(ms, "cuda")
+    h2d, d2h = lay.e2e_bytes()
+    return world * lay.c.R * args.steps / (ms * 1e-3), h2d, d2h
+
+
 def run_variants(args, flush, main_layer):
     """The other timings of the same workload: the expert-wise layout at the
     matched adapter budget, the deterministic split-K mode, and no L2 flush."""
@@ -591,26 +699,13 @@ def run_gpu(args, rank, world, local):
     ms_per_step = ms / args.steps
     value = world * c.R / (ms_per_step * 1e-3)
 
-    # ---- end to end through host buffers (same calls, pinned H2D in, grads D2H out)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    for _ in range(2):
-        lay.h2d_inputs()
-        lay.step()
-        lay.d2h_result()
-    torch.cuda.synchronize()
-    if world > 1:
-        torch.distributed.barrier()
-    e0.record()
-    for _ in range(args.steps):
-        lay.h2d_inputs()
-        lay.step()
-        lay.d2h_result()
-    e1.record()
-    torch.cuda.synchronize()
-    e2e_ms = e0.elapsed_time(e1)
-    if world > 1:
-        e2e_ms = reduce_max(e2e_ms, "cuda")
-    e2e_value = world * c.R * args.steps / (e2e_ms * 1e-3)
+    # ---- end to end through host buffers: every step copies all of its inputs
+    # in from pinned host memory (routing, X, h, the three dY, the three base
+    # outputs and the base dX / dh that the deltas accumulate onto) and reads all
+    # of its results back (the three outputs, dX, dh, the six weight
+    # gradients); two device sets, the copies on a second stream, so step i's
+    # copies overlap step i - 1's compute
+    e2e_value, e2e_h2d, e2e_d2h = e2e_pipeline(args, lay, world)
 
     peaks = load_peaks()
     call_ms = {n: float(np.mean(v)) for n, v in per_call.items()}
@@ -650,8 +745,9 @@ def run_gpu(args, rank, world, local):
         "step_ms_stats": step_stats,
         "per_call_ms": call_ms,
         "per_call_frac_hbm": {n: bytes_[n] / (call_ms[n] * 1e-3) / 1e9 / peaks["hbm_gbs"] for n in CALLS},
-        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": lay.h2d_bytes(),
-                "d2h_bytes_per_step": lay.d2h_bytes()},
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": e2e_h2d, "d2h_bytes_per_step": e2e_d2h,
+                "overlap": "two device sets; H2D on one stream, D2H on another, beside the compute of the "
+                           "neighbouring steps"},
         "gpu_launches": lay.kernels_per_step() * args.steps,
         "clocks": clocks,
         "wall_s_timed": t_wall,
@@ -888,6 +984,36 @@ def run_reference(args, rank, world):
     }
 
 
+def run_once(args):
+    """--once: the calls of one layer step, each run --repeat times in step
+    order with no timing (the launch pattern a profiler captures); with --ffn
+    the expert FFN forward (base GEMMs with the adapters fused in) follows."""
+    import torch
+    from paper_2609_06072_gb300 import ace
+    ace.load()
+    lay = Layer(args.config, args.seed, args.expertwise, args.det, combine=args.combine)
+    only = set(args.only.split(",")) if args.only else None
+    for _ in range(args.repeat):
+        lay.step(only=only)
+    if args.ffn:
+        import torch as _t
+        c, p = lay.c, lay.plan
+        gen = _t.Generator().manual_seed(2000 + args.seed)
+        w = lambda *s_, fan: (_t.randn(*s_, generator=gen) / fan ** 0.5).to(_t.bfloat16).cuda()
+        Wg, Wu, Wd = w(c.E, c.f, c.d, fan=c.d), w(c.E, c.f, c.d, fan=c.d), w(c.E, c.d, c.f, fan=c.f)
+        bf = lambda *s_: _t.empty(*s_, dtype=_t.bfloat16, device="cuda")
+        U, V, Hh, Y = bf(c.R, c.f), bf(c.R, c.f), bf(c.R, c.f), bf(c.R, c.d)
+        Hgu = [_t.empty(c.R, p.rank_max, device="cuda") for _ in range(2)]
+        Hd = _t.empty(c.R, p.rank_max, device="cuda")
+        ws = p.ffn_workspace(c.T)
+        for _ in range(args.repeat):
+            p.ffn_fwd(lay.perm, lay.X, Wg, Wu, Wd, lay.A, lay.Bt, c.s, U, V, Hh, Y, Hgu, Hd, ws)
+    torch.cuda.synchronize()
+    assert lay.plan.get_error(lay.perm) == 0
+    print(json.dumps({"mode": "once", "config": args.config, "repeat": args.repeat, "only": args.only,
+                      "deterministic": bool(args.det), "combine": bool(args.combine), "ffn": bool(args.ffn)}))
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -908,9 +1034,16 @@ def main():
     ap.add_argument("--cka", action="store_true",
                     help="also time rank consolidation: the CKA matrix on a 10k-token probe and the grouping")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--once", action="store_true",
+                    help="untimed: run the step's calls --repeat times and exit (for profilers)")
+    ap.add_argument("--repeat", type=int, default=1)
+    ap.add_argument("--only", default="", help="with --once: comma-separated calls to run after the permutation")
     ap.add_argument("--no-variants", action="store_true",
                     help="skip the expert-wise, deterministic-mode and unflushed timings")
     args = ap.parse_args()
+    if args.once:
+        run_once(args)
+        return
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     rank, world, local = dist_env()

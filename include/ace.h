@@ -271,7 +271,8 @@ ace_status ace_bwd_combine(const ace_plan* plan, const ace_perm* perm, const uin
  *   S      [E, E] fp32 OUT
  *   ws     device workspace of ace_cka_workspace_size bytes
  * d_in a multiple of 64, r <= 32.  The representation matrices are never
- * formed: with M_ij = A_i (Xc^T Xc) A_j^T, every norm is an r x r trace.  If
+ * formed: with M_ij = A_i (Xc^T Xc) A_j^T, every norm is an r x r trace; the
+ * probe is centred (fp32 column means, bf16 Xc) before the product.  If
  * a bounded device wait gives up, S is filled with NaN.  Device pointers;
  * asynchronous on `stream`. */
 ace_status ace_cka_workspace_size(int32_t N, int32_t d_in, int32_t d_out, int32_t E, int32_t r, size_t* bytes);

@@ -6,7 +6,8 @@
 // so every Frobenius norm in CKA reduces to r x r products:
 //   ||Zc_i^T Zc_j||_F^2 = tr(M_ij^T Gb_i M_ij Gb_j),  Gb_e = B_e^T B_e (r x r).
 // The work is one K = N product Xc^T Xc (tensor cores: the dense dA GEMM of
-// gemm.cu with X as both operands, then a rank-one centring correction),
+// gemm.cu with the centred probe as both operands; the column means are
+// taken out of X before the product, so a large mean cancels nothing),
 // P = A (Xc^T Xc) and M = P A^T over the stacked expert ranks (fp32), the
 // E Gram blocks Gb_e, and one small trace per expert pair.
 #include <cmath>
@@ -42,12 +43,23 @@ __global__ void __launch_bounds__(256) k_colsum_total(const float* __restrict__ 
   colsum[col] = s;
 }
 
-// Cc = C - N mu mu^T = C - colsum colsum^T / N
-__global__ void __launch_bounds__(256) k_center(float* __restrict__ C, const float* __restrict__ colsum, int N, int d) {
+// Xc = X - 1 mu^T with mu = colsum / N (fp32 arithmetic, bf16 out), 8 columns a thread
+__global__ void __launch_bounds__(256) k_center_x(const uint16_t* __restrict__ X, const float* __restrict__ colsum,
+                                                  int N, int d, uint16_t* __restrict__ Xc) {
   const int64_t idx = (int64_t)blockIdx.x * 256 + threadIdx.x;
-  if (idx >= (int64_t)d * d) return;
-  const int a = (int)(idx / d), b = (int)(idx % d);
-  C[idx] -= colsum[a] * colsum[b] / (float)N;
+  if (idx >= (int64_t)N * (d / 8)) return;
+  const int64_t row = idx / (d / 8);
+  const int c0 = (int)(idx % (d / 8)) * 8;
+  const uint4 v = *reinterpret_cast<const uint4*>(X + row * d + c0);
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  uint32_t o[4];
+  const float inv_n = 1.f / (float)N;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const float2 f = unpack_bf16x2(w[q]);
+    o[q] = pack_bf16x2(f.x - colsum[c0 + 2 * q] * inv_n, f.y - colsum[c0 + 2 * q + 1] * inv_n);
+  }
+  *reinterpret_cast<uint4*>(Xc + row * d + c0) = make_uint4(o[0], o[1], o[2], o[3]);
 }
 
 // C[M x N] = A[M x K] . B with A row-major (lda) and B row-major [K x N]
@@ -197,12 +209,12 @@ __global__ void __launch_bounds__(256) k_consolidate(const __grid_constant__ Con
 
 struct CkaWs {
   float *C, *part, *colsum, *P, *Mx, *Gb, *diag;
+  uint16_t* Xc;  // the centred probe [N, d_in] bf16
   int32_t* err;
   size_t total;
 };
 
 CkaWs cka_layout(int N, int d_in, int E, int r, void* base) {
-  (void)N;
   CkaWs w{};
   char* b = static_cast<char*>(base);
   size_t off = 0;
@@ -220,6 +232,7 @@ CkaWs cka_layout(int N, int d_in, int E, int r, void* base) {
   w.Gb = reinterpret_cast<float*>(take(4 * (size_t)E * r * r));
   w.diag = reinterpret_cast<float*>(take(4 * (size_t)E));
   w.err = reinterpret_cast<int32_t*>(take(16));
+  w.Xc = reinterpret_cast<uint16_t*>(take(2 * (size_t)N * d_in));
   w.total = off;
   return w;
 }
@@ -267,10 +280,22 @@ ace_status ace_cka(int32_t N, int32_t d_in, int32_t d_out, int32_t E, int32_t r,
   cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
   if (!(major == 10 && minor == 3)) return report(ACE_ERR_UNSUPPORTED, "ace_cka: this library is built for sm_103a only");
   cudaStream_t cs = static_cast<cudaStream_t>(stream);
-  // Xc^T Xc = X^T X - N mu mu^T: the dense dA GEMM with X as both operands
+  // Xc^T Xc: the dense dA GEMM with the probe, centred first (center != 0),
+  // as both operands
+  cudaError_t e = cudaMemsetAsync(w.C, 0, 4 * (size_t)d_in * d_in, cs);
+  if (e == cudaSuccess) e = cudaMemsetAsync(w.err, 0, 16, cs);
+  const uint16_t* Xg = X;
+  if (e == cudaSuccess && center) {
+    k_colsum<<<dim3((d_in + 255) / 256, kColChunks), 256, 0, cs>>>(X, N, d_in, w.part);
+    k_colsum_total<<<(d_in + 255) / 256, 256, 0, cs>>>(w.part, d_in, w.colsum);
+    const int64_t nv = (int64_t)N * (d_in / 8);
+    k_center_x<<<(unsigned)((nv + 255) / 256), 256, 0, cs>>>(X, w.colsum, N, d_in, w.Xc);
+    e = cudaGetLastError();
+    Xg = w.Xc;
+  }
   DenseBwdLaunch g{};
   const uint64_t n = (uint64_t)N, di = (uint64_t)d_in;
-  if (!make_tmap_bf16(&g.tm_dhx_t, X, n, di, 64) || !make_tmap_bf16(&g.tm_x, X, n, di, 64) ||
+  if (!make_tmap_bf16(&g.tm_dhx_t, Xg, n, di, 64) || !make_tmap_bf16(&g.tm_x, Xg, n, di, 64) ||
       !make_tmap_f32(&g.tm_da[0], w.C, di, di, 32))
     return report(ACE_ERR_UNSUPPORTED, "ace_cka: tensor-map encoding failed");
   g.tm_da[1] = g.tm_da[0];
@@ -282,16 +307,7 @@ ace_status ace_cka(int32_t N, int32_t d_in, int32_t d_out, int32_t E, int32_t r,
   g.nproj = 1;
   g.grid = nsm;
   g.err = w.err;
-  cudaError_t e = cudaMemsetAsync(w.C, 0, 4 * (size_t)d_in * d_in, cs);
-  if (e == cudaSuccess) e = cudaMemsetAsync(w.err, 0, 16, cs);
   if (e == cudaSuccess) e = launch_dense_da(g, cs);
-  if (e == cudaSuccess && center) {
-    k_colsum<<<dim3((d_in + 255) / 256, kColChunks), 256, 0, cs>>>(X, N, d_in, w.part);
-    k_colsum_total<<<(d_in + 255) / 256, 256, 0, cs>>>(w.part, d_in, w.colsum);
-    const int64_t dd = (int64_t)d_in * d_in;
-    k_center<<<(unsigned)((dd + 255) / 256), 256, 0, cs>>>(w.C, w.colsum, N, d_in);
-    e = cudaGetLastError();
-  }
   const int er = E * r;
   if (e == cudaSuccess) {
     // P = A . Cc  [er x d_in],  M = P . A^T  [er x er]

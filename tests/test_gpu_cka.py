@@ -43,6 +43,23 @@ def test_cka_matrix_parity(E, N, d_in, d_out, r, center):
     assert np.array_equal(g_gpu, g_ref)
 
 
+@pytest.mark.parametrize("mean", [16.0, 64.0])
+def test_cka_probe_with_a_large_mean(mean):
+    """Probe activations whose mean dwarfs their spread: centring must not
+    cancel (the covariance of the centred probe, not X^T X minus a rank-one
+    correction)."""
+    from paper_2609_06072_gb300 import ace
+    rng = np.random.default_rng(int(mean))
+    E, N, d_in, d_out, r = 12, 1500, 128, 96, 4
+    X, A, Bt, proto = planted(rng, E, N, d_in, d_out, r, 3, 0.3)
+    X = bits(W.bf16_bits_to_f32(X).astype(np.float64) + mean)
+    S = ace.cka(dev_bf16(X), dev_bf16(A), dev_bf16(Bt), E, r, center=True).cpu().numpy().astype(np.float64)
+    Z = C.adapter_outputs(X, [A[e * r:(e + 1) * r] for e in range(E)], [Bt[e * r:(e + 1) * r] for e in range(E)])
+    ref = C.cka_matrix(Z, center=True)
+    assert np.all(np.isfinite(S))
+    assert np.abs(S - ref).max() <= 2e-3, np.abs(S - ref).max()
+
+
 def test_cka_olmoe_probe_sampled_pairs():
     """OLMoE gate shapes (d 2048 -> f 1024, 64 experts of rank 8) on the
     paper's 10k-token probe: sampled pairs against the oracle's definition."""

@@ -197,10 +197,19 @@ __device__ int build_splits(const int32_t* n_g, const int32_t* off_g, int G, int
   const int min_total = count_pieces(n_g, G, cap, red);
   const int target = (min_total + nsm - 1) / nsm * nsm;
   int per = cap;
-  if (min_total > 0 && 10 * (min_total - (target - nsm)) < 9 * nsm && target > G) {
-    int rows = 0;
-    for (int g = 0; g < G; ++g) rows += n_g[g];  // (every thread; G <= 512)
-    per = min(cap, max(1, (rows + target - G - 1) / (target - G)));
+  if (min_total > 0 && 10 * (min_total - (target - nsm)) < 9 * nsm) {
+    // the shortest pieces whose count still fits the whole waves of the
+    // target (the count only falls as the pieces lengthen); every thread
+    // takes the same branches, so the block reductions stay aligned
+    int lo = 1, hi = cap;
+    while (lo < hi) {
+      const int mid = (lo + hi) / 2;
+      if (count_pieces(n_g, G, mid, red) <= target)
+        hi = mid;
+      else
+        lo = mid + 1;
+    }
+    per = hi;
   }
   const int tid = threadIdx.x;
   for (int g = tid; g < G; g += blockDim.x) scratch[g + 1] = (n_g[g] + per - 1) / per;
@@ -404,7 +413,10 @@ __global__ void __launch_bounds__(kPermTB) k_perm_scatter(const __grid_constant_
       // backward splits: down / combine (job 2), gate/up (job 3)
       __shared__ int32_t red[32];
       const bool sh = job == 3;
-      const int n = build_splits(rows_g, goff, G, kTileM * (sh ? pt.nt_split_sh : pt.nt_split), pt.nsm,
+      // gate/up runs its two projections side by side (grid.y = 2), so its
+      // splits fill whole waves in units of half the SMs
+      const int wave = sh ? (pt.nsm > 1 ? pt.nsm / 2 : 1) : pt.nsm;
+      const int n = build_splits(rows_g, goff, G, kTileM * (sh ? pt.nt_split_sh : pt.nt_split), wave,
                                  sh ? o.splits_sh : o.splits_row, scratch, red);
       if (tid == 0) o.counts[sh ? kCntSplitsSh : kCntSplitsRow] = n;
     }

@@ -649,38 +649,10 @@ ace_status ace_bwd_combine(const ace_plan* plan, const ace_perm* perm, const uin
               make_tmap_bf16(&x.tm_dhx_t, Hx, T, (uint64_t)nrp, 64) && make_tmap_bf16(&x.tm_x, dZ, T, (uint64_t)pt.d, 64) &&
               make_tmap_f32(&x.tm_da[0], dBt, (uint64_t)n_rank, (uint64_t)pt.d, 32);
     if (!ok) return fail(ACE_ERR_UNSUPPORTED, "tensor-map encoding failed for this layout");
-    if (n_rank <= kDenseHMaxRank) {
-      DenseHLaunch h{};
-      ok = make_tmap_bf16(&h.tm_x, dZ, T, (uint64_t)pt.d, kTileM) &&
-           make_tmap_bf16(&h.tm_a[0], Bt, (uint64_t)n_rank, (uint64_t)pt.d, 256);
-      if (!ok) return fail(ACE_ERR_UNSUPPORTED, "tensor-map encoding failed for this layout");
-      h.tm_a[1] = h.tm_a[0];
-      h.tok_uniq = perm->tok_uniq;
-      h.uniq_off = perm->uniq_off;
-      h.H[0] = h.H[1] = Hc;
-      h.T = perm->T;
-      h.d = pt.d;
-      h.n_rank = n_rank;
-      h.nproj = 1;
-      h.rank_max = pt.rank_max;
-      h.grid = plan->num_sms;
-      h.err = err;
-      st = cuda_status(launch_dense_h(pt, h, cs), "combine dHc launch");
-    } else {
-      FwdHLaunch h{};
-      h.tiles = at<Tile>(perm->ws, L.tiles_sh);
-      h.counts = perm->counts;
-      h.max_tiles = L.max_tiles;
-      h.rows = 0;
-      h.uniq_tok = perm->uniq_tok;
-      h.X = dZ;
-      h.A[0] = h.A[1] = Bt;
-      h.H[0] = h.H[1] = Hc;
-      h.d_in = pt.d;
-      h.nproj = 1;
-      h.err = err;
-      st = cuda_status(launch_fwd_h(pt, h, cs), "combine dHc launch");
-    }
+    // B_g^T dz once per unique (g, t) pair: the same product as the gate/up H
+    const uint16_t* Bts[1] = {Bt};
+    float* Hcs[1] = {Hc};
+    st = launch_gate_up_h(plan, perm, dZ, 1, Bts, Hcs, cs);
     if (st != ACE_OK) return st;
   }
   a.splits_row = at<Tile>(perm->ws, L.splits_row);

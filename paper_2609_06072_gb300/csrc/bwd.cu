@@ -370,10 +370,19 @@ __global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constan
         }
       }
       named_bar_arrive(kIssueBar, kEpiThreads + 32);
-      const bool vec = (pt.rank_max & 3) == 0;
-      // v[0..32) = src[c0 .. c0 + 32), zero past rank_max or for a dead row
+      const bool vec = (pt.rank_max & 3) == 0, vec2 = (pt.rank_max & 1) == 0;
+      // v[0..32) = src[c0 .. c0 + 32), zero past rank_max or for a dead row;
+      // 16- or 8-byte loads where the row stride rank_max keeps them aligned
       auto load32 = [&](const float* src, int c0, bool live, float* v) {
-        if (vec) {
+        if (vec2 && !vec) {
+#pragma unroll
+          for (int q = 0; q < 16; ++q) {
+            const int c = c0 + 2 * q;
+            const float2 x = (live && c < pt.rank_max) ? *reinterpret_cast<const float2*>(src + c) : make_float2(0.f, 0.f);
+            v[2 * q] = x.x;
+            v[2 * q + 1] = x.y;
+          }
+        } else if (vec) {
 #pragma unroll
           for (int q = 0; q < 8; ++q) {
             const int c = c0 + 4 * q;

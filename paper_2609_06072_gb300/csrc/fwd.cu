@@ -144,17 +144,38 @@ __global__ void __launch_bounds__(kHThreads) k_fwd_h(const __grid_constant__ Pla
   aborted = __syncthreads_or(bad || aborted);
   tc_fence_after();
   if (!aborted) {
-    constexpr int kHcols = NPROJ * RP;
+    // the tile goes through the (now idle) stage buffers: its rows are rows
+    // [start, start + cnt) of H_j, one contiguous range of cnt * rank_max
+    // floats, which the CTA then writes with consecutive threads on
+    // consecutive addresses (a thread per row would write 32 rows per store)
+    constexpr int kHcols = NPROJ * RP, kLd = kHcols + 4;  // smem row stride in floats (bank-conflict free)
+    static_assert(kTileM * kLd * 4 <= kHStages * C::kStage, "H tile fits the stage buffers");
+    float* sH = reinterpret_cast<float*>(smem);
     for (int c0 = half * 16; c0 < kHcols; c0 += 32) {
       uint32_t r[16];
       tmem_ld16(tmem + lane_base + c0, r);
       tmem_ld_wait();
-      const int j = c0 / RP, kb = c0 % RP;
-      if (m < tl.cnt) {
-        float* hrow = a.H[j] + (int64_t)(tl.start + m) * pt.rank_max;
+      float4* dst = reinterpret_cast<float4*>(sH + m * kLd + c0);
 #pragma unroll
-        for (int q = 0; q < 16; ++q)
-          if (kb + q < pt.rank_max) hrow[kb + q] = __uint_as_float(r[q]);
+      for (int q = 0; q < 4; ++q)
+        dst[q] = make_float4(__uint_as_float(r[4 * q]), __uint_as_float(r[4 * q + 1]), __uint_as_float(r[4 * q + 2]),
+                             __uint_as_float(r[4 * q + 3]));
+    }
+    __syncthreads();
+    const int W = pt.rank_max, n = tl.cnt * W;
+#pragma unroll
+    for (int j = 0; j < NPROJ; ++j) {
+      float* dst = a.H[j] + (int64_t)tl.start * W;
+      if ((W & 3) == 0) {
+        for (int e = 4 * tid; e < n; e += 4 * kHThreads) {
+          const int row = e / W, col = e - row * W;
+          *reinterpret_cast<float4*>(dst + e) = *reinterpret_cast<const float4*>(sH + row * kLd + j * RP + col);
+        }
+      } else {
+        for (int e = tid; e < n; e += kHThreads) {
+          const int row = e / W, col = e - row * W;
+          dst[e] = sH[row * kLd + j * RP + col];
+        }
       }
     }
   }
@@ -165,6 +186,20 @@ __global__ void __launch_bounds__(kHThreads) k_fwd_h(const __grid_constant__ Pla
   // as this grid's CTAs finish (an early launch measured slower)
   pdl_trigger();
   if (warp == 0) tmem_dealloc(tmem, C::kTmem);
+}
+
+// Columns [c0, c0 + 16) of an fp32 H row of rank_max columns (those below
+// rank_max): 16-byte stores where the row stride keeps them aligned.
+__device__ __forceinline__ void store_row16(float* hrow, int c0, int rank_max, const float* v) {
+  if ((rank_max & 3) == 0 && c0 + 16 <= rank_max) {
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      *reinterpret_cast<float4*>(hrow + c0 + 4 * q) = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+  } else {
+#pragma unroll
+    for (int q = 0; q < 16; ++q)
+      if (c0 + q < rank_max) hrow[c0 + q] = v[q];
+  }
 }
 
 // --------------------------------------------------------------- k_fwd_rows
@@ -533,12 +568,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
           float v[16];
 #pragma unroll
           for (int qq = 0; qq < 16; ++qq) v[qq] = (live && c0 + qq < rg) ? __uint_as_float(r[qq]) : 0.f;
-          if (live && a.Hsave != nullptr) {
-            float* hrow = a.Hsave + (int64_t)(t.start + m) * pt.rank_max;
-#pragma unroll
-            for (int qq = 0; qq < 16; ++qq)
-              if (c0 + qq < pt.rank_max) hrow[c0 + qq] = v[qq];
-          }
+          if (live && a.Hsave != nullptr) store_row16(a.Hsave + (int64_t)(t.start + m) * pt.rank_max, c0, pt.rank_max, v);
 #pragma unroll
           for (int h = 0; h < 2; ++h) {
             const int col = c0 + h * 8;
@@ -657,10 +687,10 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
         tmem_ld16(tmem + lane_base + (kt & 1) * C::kHcol + c0, r);
         tmem_ld_wait();
         if (live) {
-          float* hrow = a.Hpre + (int64_t)(t.start + m) * pt.rank_max;
+          float v[16];
 #pragma unroll
-          for (int qq = 0; qq < 16; ++qq)
-            if (c0 + qq < pt.rank_max) hrow[c0 + qq] = c0 + qq < rg ? __uint_as_float(r[qq]) : 0.f;
+          for (int qq = 0; qq < 16; ++qq) v[qq] = c0 + qq < rg ? __uint_as_float(r[qq]) : 0.f;
+          store_row16(a.Hpre + (int64_t)(t.start + m) * pt.rank_max, c0, pt.rank_max, v);
         }
       }
       tc_fence_before();

@@ -724,9 +724,17 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemm_h(const __grid_constant__ 
           if (u < 0) continue;
           const int off = roff_s[gg], end = roff_s[gg + 1];
           float* hrow = Hj + (int64_t)u * a.rank_max - off;
+          if (c >= off && c + 16 <= end && ((a.rank_max | off) & 3) == 0) {  // 16-byte aligned, all in the group
 #pragma unroll
-          for (int q = 0; q < 16; ++q)
-            if (c + q >= off && c + q < end) hrow[c + q] = __uint_as_float(r[q]);
+            for (int q = 0; q < 4; ++q)
+              *reinterpret_cast<float4*>(hrow + c + 4 * q) =
+                  make_float4(__uint_as_float(r[4 * q]), __uint_as_float(r[4 * q + 1]), __uint_as_float(r[4 * q + 2]),
+                              __uint_as_float(r[4 * q + 3]));
+          } else {
+#pragma unroll
+            for (int q = 0; q < 16; ++q)
+              if (c + q >= off && c + q < end) hrow[c + q] = __uint_as_float(r[q]);
+          }
           if (end <= c + 16)  // the group ends here: zero its row's columns past r_g
             for (int q = end - off; q < a.rank_max; ++q) hrow[off + q] = 0.f;
         }

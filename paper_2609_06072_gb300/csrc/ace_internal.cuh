@@ -18,6 +18,15 @@ constexpr int kErrIndex = 1;
 constexpr int kErrTimeout = 2;
 constexpr int kErrValue = 4;  // a non-finite gate weight reached the combine
 
+// Backward row kernel of gate/up at a padded rank of at most 32: two CTAs
+// per SM (half the shared-memory budget each, two-tile splits), so one CTA's
+// H staging and final dH epilogue overlap the other's dY stream.
+__host__ __device__ constexpr int bwd_sh_ctas_per_sm(int rank_pad) { return rank_pad <= 32 ? 2 : 1; }
+// row tiles per backward split (gate/up: shared; down and the combine: not)
+__host__ __device__ constexpr int bwd_nt_split(int rank_pad, bool shared) {
+  return shared && bwd_sh_ctas_per_sm(rank_pad) == 2 ? 2 : rank_pad <= 64 ? 4 : 2;
+}
+
 // Plan tables passed by value (__grid_constant__) to every kernel.
 struct PlanTables {
   int32_t E, G, k, d, f;

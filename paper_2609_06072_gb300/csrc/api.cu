@@ -95,8 +95,8 @@ ace_status check_perm(const ace_plan* plan, const ace_perm* perm) {
 // TMEM columns) sit below its double-buffered weight-gradient accumulators
 // (2 x rank_pad), so at rank_pad 128 a split takes two tiles (down's phase-2
 // dh buffer reuses the dH columns).
-int pt_nt_split(int rank_pad) { return rank_pad <= 64 ? 4 : 2; }
-int pt_nt_split_sh(int rank_pad) { return rank_pad <= 64 ? 4 : 2; }
+int pt_nt_split(int rank_pad) { return bwd_nt_split(rank_pad, false); }
+int pt_nt_split_sh(int rank_pad) { return bwd_nt_split(rank_pad, true); }
 
 struct BwdWs {
   float* dHrow[2];

@@ -151,7 +151,8 @@ struct RowsCfg {
   // sit below the weight-gradient accumulators (2 x RP from kTB); at RP = 128
   // two tiles fill the 512 columns, and the phase-2 dh buffer of down and the
   // combine takes the dH columns once dH is staged as the phase-2 operand
-  static constexpr int NT = RP <= 64 ? 4 : 2;
+  static constexpr int NT = bwd_nt_split(RP, MODE == MODE_SHARED);
+  static constexpr int kPerSM = MODE == MODE_SHARED ? bwd_sh_ctas_per_sm(RP) : 1;  // resident CTAs per SM
   static constexpr int kOps = Slots<RP>::bytes(NT);
   static constexpr int kWBlk = RP * 128;
   static constexpr int kSlotA = 2 * kBlk + 2 * kWBlk;  // dY tile + B^T chunk (down phase 2: A chunk + h tile)
@@ -159,7 +160,7 @@ struct RowsCfg {
   // down / combine: dh tiles of the RMW (one at RP = 128, where two would not
   // fit beside the ring)
   static constexpr int SB = MODE != MODE_SHARED ? (RP > 64 ? 1 : 2) : 0;
-  static constexpr int kBudget = 220 * 1024;
+  static constexpr int kBudget = 220 * 1024 / kPerSM;
   static constexpr int kSA0 = (kBudget - kOps - SB * kSlotB) / kSlotA;
   static constexpr int SA = kSA0 > 6 ? 6 : (kSA0 < 2 ? 2 : kSA0);
   static constexpr int kSmem = kOps + SA * kSlotA + SB * kSlotB + 1024;
@@ -170,11 +171,12 @@ struct RowsCfg {
   static constexpr int kDB = RP > 64 ? 0 : (kTB > 128 ? 384 : 256);
   static constexpr int kTmem = (MODE != MODE_SHARED || RP > 64 || kTB > 128) ? 512 : 256;
   static_assert(kSmem <= 227 * 1024, "shared memory per CTA");
+  static_assert(kPerSM == 1 || kPerSM * (kSmem + 3 * 1024) <= 228 * 1024, "resident CTAs per SM");
   static_assert(ND * kNcB + (kDB == 0 ? 0 : kDB) <= 512 && (kDB != 0 || ND * kNcB <= kTB), "TMEM: dh buffers");
 };
 
 template <int RP, int MODE>
-__global__ void __launch_bounds__(kThreadsWS, 1) k_bwd_rows(const __grid_constant__ PlanTables pt,
+__global__ void __launch_bounds__(kThreadsWS, RowsCfg<RP, MODE>::kPerSM) k_bwd_rows(const __grid_constant__ PlanTables pt,
                                                             const __grid_constant__ BwdLaunch a) {
   using C = RowsCfg<RP, MODE>;
   using SL = Slots<RP>;

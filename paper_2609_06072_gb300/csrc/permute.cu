@@ -414,8 +414,9 @@ __global__ void __launch_bounds__(kPermTB) k_perm_scatter(const __grid_constant_
       __shared__ int32_t red[32];
       const bool sh = job == 3;
       // gate/up runs its two projections side by side (grid.y = 2), so its
-      // splits fill whole waves in units of half the SMs
-      const int wave = sh ? (pt.nsm > 1 ? pt.nsm / 2 : 1) : pt.nsm;
+      // splits fill whole waves: gate/up's two projections run side by side,
+      // so a wave holds ctas_per_sm * nsm / 2 splits of each
+      const int wave = sh ? max(1, bwd_sh_ctas_per_sm(pt.rank_pad) * pt.nsm / 2) : pt.nsm;
       const int n = build_splits(rows_g, goff, G, kTileM * (sh ? pt.nt_split_sh : pt.nt_split), wave,
                                  sh ? o.splits_sh : o.splits_row, scratch, red);
       if (tid == 0) o.counts[sh ? kCntSplitsSh : kCntSplitsRow] = n;

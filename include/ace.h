@@ -73,6 +73,10 @@ typedef int32_t ace_status;
 #define ACE_ERR_UNSUPPORTED 5    /* device is not sm_103, or rank too large */
 #define ACE_ERR_CUDA 6           /* a CUDA runtime call failed */
 #define ACE_ERR_DEVICE_TIMEOUT 7 /* a bounded device-side wait gave up */
+#define ACE_ERR_CHECK 8          /* libace_checks.so only: an index read from the
+                                    permutation arrays, or a tile of a tile table,
+                                    was outside its range; the access went to a safe
+                                    index instead and the results are unspecified */
 
 /* plan flags */
 #define ACE_FLAG_DETERMINISTIC 1u /* dA / dB^T via fixed-order two-stage split-K (bitwise reproducible);
@@ -118,6 +122,7 @@ typedef struct ace_perm {
   int32_t* uniq_off;      /* [G+1] first unique pair of each group */
   int32_t* uniq_tok;      /* [R] token of unique pair u (first U entries valid) */
   int32_t* tok_uniq;      /* [T*k] unique pairs of token t, ascending g, then -1 */
+  int32_t* row_uniq;      /* [R] unique pair (g, t) of the pair held by row r */
   void* ws;               /* the workspace these views point into */
 } ace_perm;
 
@@ -361,9 +366,18 @@ ace_status ace_scatter_rows(const ace_perm* perm, const uint16_t* src_rows, uint
 
 /* Synchronises `stream`, then reads and clears the device error flag of the
  * permutation workspace: ACE_OK, ACE_ERR_INDEX (invalid routing),
- * ACE_ERR_DEVICE_TIMEOUT (a bounded wait gave up; results unspecified) or
- * ACE_ERR_ARG (a non-finite gate weight reached ace_fwd_combine). */
+ * ACE_ERR_DEVICE_TIMEOUT (a bounded wait gave up; results unspecified),
+ * ACE_ERR_ARG (a non-finite gate weight reached ace_fwd_combine) or, in the
+ * checked build, ACE_ERR_CHECK. */
 ace_status ace_get_error(const ace_perm* perm, void* stream);
+
+/* 1 in libace_checks.so, the debug build of the same sources compiled with
+ * ACE_CHECKS: every kernel range-checks each index it reads from the
+ * permutation arrays and each tile it takes from a tile table before using
+ * it, and reports a violation as ACE_ERR_CHECK (the access goes to a safe
+ * index; nothing faults or traps).  0 in libace.so, where the checks compile
+ * away.  The two libraries export the same calls with the same semantics. */
+int32_t ace_build_checks(void);
 
 #ifdef __cplusplus
 }

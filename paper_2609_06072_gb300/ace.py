@@ -25,17 +25,19 @@ ACE_ERR_INDEX = 4
 ACE_ERR_UNSUPPORTED = 5
 ACE_ERR_CUDA = 6
 ACE_ERR_DEVICE_TIMEOUT = 7
+ACE_ERR_CHECK = 8  # libace_checks.so: an index or a tile outside its range
 ACE_FLAG_DETERMINISTIC = 1
 ACE_FLAG_TEST_WAIT_EXPIRY = 2  # test only: makes the down forward's bounded flag wait give up
 
 STATUS_NAMES = {0: "ACE_OK", 1: "ACE_ERR_ARG", 2: "ACE_ERR_SHAPE", 3: "ACE_ERR_WORKSPACE", 4: "ACE_ERR_INDEX",
-                5: "ACE_ERR_UNSUPPORTED", 6: "ACE_ERR_CUDA", 7: "ACE_ERR_DEVICE_TIMEOUT"}
+                5: "ACE_ERR_UNSUPPORTED", 6: "ACE_ERR_CUDA", 7: "ACE_ERR_DEVICE_TIMEOUT",
+                8: "ACE_ERR_CHECK"}
 
 EXPORTED = ["ace_version", "ace_last_error_message", "ace_plan_create", "ace_plan_destroy", "ace_plan_rank_max",
             "ace_workspace_size", "ace_permute", "ace_fwd_shared", "ace_fwd_shared_noalloc", "ace_fwd_row",
             "ace_bwd_shared", "ace_bwd_row", "ace_plan_rank_cols", "ace_fwd_combine", "ace_bwd_combine",
             "ace_group_experts", "ace_ffn_workspace_size", "ace_ffn_fwd", "ace_ffn_bwd", "ace_cka_workspace_size", "ace_cka", "ace_consolidate_adapters",
-            "ace_gather_rows", "ace_scatter_rows", "ace_get_error"]
+            "ace_gather_rows", "ace_scatter_rows", "ace_get_error", "ace_build_checks"]
 
 
 class AceError(RuntimeError):
@@ -54,25 +56,26 @@ class ace_perm(ctypes.Structure):
     _fields_ = [("T", ctypes.c_int32), ("R", ctypes.c_int32), ("counts", ctypes.c_void_p),
                 ("group_off", ctypes.c_void_p), ("expert_off", ctypes.c_void_p), ("expert_cnt", ctypes.c_void_p),
                 ("row_pair", ctypes.c_void_p), ("pair_row", ctypes.c_void_p), ("uniq_off", ctypes.c_void_p),
-                ("uniq_tok", ctypes.c_void_p), ("tok_uniq", ctypes.c_void_p), ("ws", ctypes.c_void_p)]
+                ("uniq_tok", ctypes.c_void_p), ("tok_uniq", ctypes.c_void_p), ("row_uniq", ctypes.c_void_p),
+                ("ws", ctypes.c_void_p)]
 
 
-_lib = None
+_libs = {}
 
 
-def lib_path() -> str:
-    return _build.LIB
+def lib_path(checks: bool = False) -> str:
+    return _build.lib_path(checks)
 
 
-def load(build_if_missing: bool = False) -> ctypes.CDLL:
-    """Load libace.so (in-tree).  Raises if it has not been built."""
-    global _lib
-    if _lib is not None:
-        return _lib
-    path = _build.LIB
+def load(build_if_missing: bool = False, checks: bool = False) -> ctypes.CDLL:
+    """Load libace.so (in-tree), or with checks=True its range-checked debug
+    build libace_checks.so.  Raises if it has not been built."""
+    if checks in _libs:
+        return _libs[checks]
+    path = _build.lib_path(checks)
     if not os.path.exists(path):
         if build_if_missing:
-            _build.build()
+            _build.build(checks=checks)
         else:
             raise RuntimeError(f"ACE CUDA library not built ({path}); run __graft_entry__.build()")
     lib = ctypes.CDLL(path)
@@ -130,13 +133,17 @@ def load(build_if_missing: bool = False) -> ctypes.CDLL:
     lib.ace_scatter_rows.argtypes = [ctypes.POINTER(ace_perm), vp, vp, i32, vp]
     lib.ace_get_error.restype = i32
     lib.ace_get_error.argtypes = [ctypes.POINTER(ace_perm), vp]
-    _lib = lib
+    lib.ace_build_checks.restype = i32
+    want = 1 if checks else 0
+    if lib.ace_build_checks() != want:
+        raise RuntimeError(f"{path} reports ace_build_checks() = {lib.ace_build_checks()}, expected {want}")
+    _libs[checks] = lib
     return lib
 
 
-def _check(st: int, what: str):
+def _check(st: int, what: str, lib=None):
     if st != ACE_OK:
-        msg = load().ace_last_error_message()
+        msg = (lib or load()).ace_last_error_message()
         raise AceError(st, what, msg.decode() if msg else "")
 
 
@@ -182,18 +189,22 @@ class Plan:
     """One layer description (ace_plan) on the current CUDA device."""
 
     def __init__(self, T_max: int, k: int, E: int, G: int, e2g, rank_off, d: int, f: int, deterministic=False,
-                 flags=0):
-        self.lib = load()
+                 flags=0, checks=False):
+        # checks=True: every call of this plan goes to libace_checks.so
+        self.lib = load(checks=checks)
         self._e2g = (ctypes.c_int32 * E)(*[int(x) for x in e2g])
         self._ro = (ctypes.c_int32 * (G + 1))(*[int(x) for x in rank_off])
         desc = ace_layer_desc(int(T_max), int(k), int(E), int(G), self._e2g, self._ro, int(d), int(f),
                               (ACE_FLAG_DETERMINISTIC if deterministic else 0) | int(flags))
         h = ctypes.c_void_p()
-        _check(self.lib.ace_plan_create(ctypes.byref(h), ctypes.byref(desc)), "ace_plan_create")
+        self._check(self.lib.ace_plan_create(ctypes.byref(h), ctypes.byref(desc)), "ace_plan_create")
         self.h = h
         self.T_max, self.k, self.E, self.G, self.d, self.f = T_max, k, E, G, d, f
         self.rank_max = self.lib.ace_plan_rank_max(h)
         self.n_rank = int(rank_off[-1])
+
+    def _check(self, st: int, what: str):
+        _check(st, what, self.lib)
 
     def __del__(self):
         h = getattr(self, "h", None)
@@ -203,7 +214,7 @@ class Plan:
 
     def workspace_size(self, T: int):
         p, fw, bw = ctypes.c_size_t(), ctypes.c_size_t(), ctypes.c_size_t()
-        _check(self.lib.ace_workspace_size(self.h, int(T), ctypes.byref(p), ctypes.byref(fw), ctypes.byref(bw)),
+        self._check(self.lib.ace_workspace_size(self.h, int(T), ctypes.byref(p), ctypes.byref(fw), ctypes.byref(bw)),
                "ace_workspace_size")
         return p.value, fw.value, bw.value
 
@@ -215,14 +226,14 @@ class Plan:
     def permute(self, topk_idx: torch.Tensor, perm_ws: torch.Tensor, stream=None) -> Perm:
         T = int(topk_idx.shape[0]) if topk_idx.numel() else 0
         c = ace_perm()
-        _check(self.lib.ace_permute(self.h, _ptr(topk_idx, torch.int32, "topk_idx"), T, _ptr(perm_ws),
+        self._check(self.lib.ace_permute(self.h, _ptr(topk_idx, torch.int32, "topk_idx"), T, _ptr(perm_ws),
                                     perm_ws.numel(), ctypes.byref(c), _stream(stream)), "ace_permute")
         return Perm(c, perm_ws)
 
     def fwd_shared(self, perm: Perm, X, A, Bt, s, Y, H=None, ws=None, stream=None):
         n = len(A)
         Hp = _arr([_ptr(h, torch.float32, "H") for h in H]) if H is not None else None
-        _check(self.lib.ace_fwd_shared(self.h, ctypes.byref(perm.c), _ptr(X, torch.bfloat16, "X"), n,
+        self._check(self.lib.ace_fwd_shared(self.h, ctypes.byref(perm.c), _ptr(X, torch.bfloat16, "X"), n,
                                        _arr([_ptr(a, torch.bfloat16, "A") for a in A]),
                                        _arr([_ptr(b, torch.bfloat16, "Bt") for b in Bt]), float(s),
                                        _arr([_ptr(y, torch.bfloat16, "Y") for y in Y]), Hp,
@@ -231,14 +242,14 @@ class Plan:
 
     def fwd_shared_noalloc(self, perm: Perm, X, A, Bt, s, Y, stream=None):
         """ace_fwd_shared_noalloc: no H output, scratch inside the library."""
-        _check(self.lib.ace_fwd_shared_noalloc(self.h, ctypes.byref(perm.c), _ptr(X, torch.bfloat16, "X"), len(A),
+        self._check(self.lib.ace_fwd_shared_noalloc(self.h, ctypes.byref(perm.c), _ptr(X, torch.bfloat16, "X"), len(A),
                                                _arr([_ptr(a, torch.bfloat16, "A") for a in A]),
                                                _arr([_ptr(b, torch.bfloat16, "Bt") for b in Bt]), float(s),
                                                _arr([_ptr(y, torch.bfloat16, "Y") for y in Y]), _stream(stream)),
                "ace_fwd_shared_noalloc")
 
     def fwd_row(self, perm: Perm, Hin, A, Bt, s, Y, H=None, ws=None, stream=None):
-        _check(self.lib.ace_fwd_row(self.h, ctypes.byref(perm.c), _ptr(Hin, torch.bfloat16, "Hin"),
+        self._check(self.lib.ace_fwd_row(self.h, ctypes.byref(perm.c), _ptr(Hin, torch.bfloat16, "Hin"),
                                     _ptr(A, torch.bfloat16, "A"), _ptr(Bt, torch.bfloat16, "Bt"), float(s),
                                     _ptr(Y, torch.bfloat16, "Y"), _ptr(H, torch.float32, "H"),
                                     _ptr(ws) if ws is not None else None, 0 if ws is None else ws.numel(),
@@ -246,7 +257,7 @@ class Plan:
 
     def bwd_shared(self, perm: Perm, dY, X, H, A, Bt, s, dX, dA, dBt, ws, stream=None):
         n = len(dY)
-        _check(self.lib.ace_bwd_shared(self.h, ctypes.byref(perm.c), n,
+        self._check(self.lib.ace_bwd_shared(self.h, ctypes.byref(perm.c), n,
                                        _arr([_ptr(t, torch.bfloat16, "dY") for t in dY]),
                                        _ptr(X, torch.bfloat16, "X"), _arr([_ptr(t, torch.float32, "H") for t in H]),
                                        _arr([_ptr(t, torch.bfloat16, "A") for t in A]),
@@ -256,7 +267,7 @@ class Plan:
                                        _stream(stream)), "ace_bwd_shared")
 
     def bwd_row(self, perm: Perm, dY, Hin, H, A, Bt, s, dHin, dA, dBt, ws, stream=None):
-        _check(self.lib.ace_bwd_row(self.h, ctypes.byref(perm.c), _ptr(dY, torch.bfloat16, "dY"),
+        self._check(self.lib.ace_bwd_row(self.h, ctypes.byref(perm.c), _ptr(dY, torch.bfloat16, "dY"),
                                     _ptr(Hin, torch.bfloat16, "Hin"), _ptr(H, torch.float32, "H"),
                                     _ptr(A, torch.bfloat16, "A"), _ptr(Bt, torch.bfloat16, "Bt"), float(s),
                                     _ptr(dHin, torch.bfloat16, "dHin"), _ptr(dA, torch.float32, "dA"),
@@ -265,12 +276,12 @@ class Plan:
 
     def ffn_workspace(self, T: int, device="cuda"):
         n = ctypes.c_size_t()
-        _check(self.lib.ace_ffn_workspace_size(self.h, int(T), ctypes.byref(n)), "ace_ffn_workspace_size")
+        self._check(self.lib.ace_ffn_workspace_size(self.h, int(T), ctypes.byref(n)), "ace_ffn_workspace_size")
         return torch.empty(max(n.value, 16), dtype=torch.uint8, device=device)
 
     def ffn_fwd(self, perm: Perm, X, W_gate, W_up, W_down, A, Bt, s, U, V, Hh, Y, Hgu, Hd, ws, stream=None):
         """ace_ffn_fwd: A / Bt are (gate, up, down); Hgu is (gate, up)."""
-        _check(self.lib.ace_ffn_fwd(self.h, ctypes.byref(perm.c), _ptr(X, torch.bfloat16, "X"),
+        self._check(self.lib.ace_ffn_fwd(self.h, ctypes.byref(perm.c), _ptr(X, torch.bfloat16, "X"),
                                     _ptr(W_gate, torch.bfloat16, "W_gate"), _ptr(W_up, torch.bfloat16, "W_up"),
                                     _ptr(W_down, torch.bfloat16, "W_down"),
                                     _arr([_ptr(t, torch.bfloat16, "A") for t in A]),
@@ -283,7 +294,7 @@ class Plan:
     def ffn_bwd(self, perm: Perm, dY, X, W_gate, W_up, W_down, A, Bt, s, U, V, Hh, Hgu, Hd, dX, dA, dBt, ws, bws,
                 stream=None):
         """ace_ffn_bwd: A / Bt / dA / dBt are (gate, up, down); Hgu is (gate, up)."""
-        _check(self.lib.ace_ffn_bwd(self.h, ctypes.byref(perm.c), _ptr(dY, torch.bfloat16, "dY"),
+        self._check(self.lib.ace_ffn_bwd(self.h, ctypes.byref(perm.c), _ptr(dY, torch.bfloat16, "dY"),
                                     _ptr(X, torch.bfloat16, "X"), _ptr(W_gate, torch.bfloat16, "W_gate"),
                                     _ptr(W_up, torch.bfloat16, "W_up"), _ptr(W_down, torch.bfloat16, "W_down"),
                                     _arr([_ptr(t, torch.bfloat16, "A") for t in A]),
@@ -301,14 +312,14 @@ class Plan:
         return int(self.lib.ace_plan_rank_cols(self.h))
 
     def fwd_combine(self, perm: Perm, Hin, topk_w, A, Bt, s, Z, H, Hx, stream=None):
-        _check(self.lib.ace_fwd_combine(self.h, ctypes.byref(perm.c), _ptr(Hin, torch.bfloat16, "Hin"),
+        self._check(self.lib.ace_fwd_combine(self.h, ctypes.byref(perm.c), _ptr(Hin, torch.bfloat16, "Hin"),
                                         _ptr(topk_w, torch.float32, "topk_w"), _ptr(A, torch.bfloat16, "A"),
                                         _ptr(Bt, torch.bfloat16, "Bt"), float(s), _ptr(Z, torch.bfloat16, "Z"),
                                         _ptr(H, torch.float32, "H"), _ptr(Hx, torch.bfloat16, "Hx"),
                                         _stream(stream)), "ace_fwd_combine")
 
     def bwd_combine(self, perm: Perm, dZ, Hin, topk_w, H, Hx, A, Bt, s, dHin, dtopk_w, dA, dBt, ws, stream=None):
-        _check(self.lib.ace_bwd_combine(self.h, ctypes.byref(perm.c), _ptr(dZ, torch.bfloat16, "dZ"),
+        self._check(self.lib.ace_bwd_combine(self.h, ctypes.byref(perm.c), _ptr(dZ, torch.bfloat16, "dZ"),
                                         _ptr(Hin, torch.bfloat16, "Hin"), _ptr(topk_w, torch.float32, "topk_w"),
                                         _ptr(H, torch.float32, "H"), _ptr(Hx, torch.bfloat16, "Hx"),
                                         _ptr(A, torch.bfloat16, "A"), _ptr(Bt, torch.bfloat16, "Bt"), float(s),
@@ -317,11 +328,11 @@ class Plan:
                                         ws.numel(), _stream(stream)), "ace_bwd_combine")
 
     def gather_rows(self, perm: Perm, src_pairs, dst_rows, stream=None):
-        _check(self.lib.ace_gather_rows(ctypes.byref(perm.c), _ptr(src_pairs), _ptr(dst_rows),
+        self._check(self.lib.ace_gather_rows(ctypes.byref(perm.c), _ptr(src_pairs), _ptr(dst_rows),
                                         int(src_pairs.shape[-1]), _stream(stream)), "ace_gather_rows")
 
     def scatter_rows(self, perm: Perm, src_rows, dst_pairs, stream=None):
-        _check(self.lib.ace_scatter_rows(ctypes.byref(perm.c), _ptr(src_rows), _ptr(dst_pairs),
+        self._check(self.lib.ace_scatter_rows(ctypes.byref(perm.c), _ptr(src_rows), _ptr(dst_pairs),
                                          int(src_rows.shape[-1]), _stream(stream)), "ace_scatter_rows")
 
     def get_error(self, perm: Perm, stream=None) -> int:
@@ -418,4 +429,5 @@ def perm_arrays(plan: Plan, perm: Perm) -> dict:
     return {"U": U, "rows": int(counts[1]), "group_off": view(c.group_off, G + 1),
             "expert_off": view(c.expert_off, E), "expert_cnt": view(c.expert_cnt, E),
             "row_pair": view(c.row_pair, R), "pair_row": view(c.pair_row, R), "uniq_off": view(c.uniq_off, G + 1),
-            "uniq_tok": view(c.uniq_tok, U), "tok_uniq": view(c.tok_uniq, R).reshape(T, k)}
+            "uniq_tok": view(c.uniq_tok, U), "tok_uniq": view(c.tok_uniq, R).reshape(T, k),
+            "row_uniq": view(c.row_uniq, R)}

@@ -17,6 +17,32 @@ constexpr int kMaxK = 32;          // largest top-k the kernels accept
 constexpr int kErrIndex = 1;
 constexpr int kErrTimeout = 2;
 constexpr int kErrValue = 4;  // a non-finite gate weight reached the combine
+constexpr int kErrCheck = 8;  // ACE_CHECKS build: an index or a tile outside its range
+
+// ACE_CHECKS (a debug build of the same sources, libace_checks.so): every
+// index a kernel reads from the permutation arrays (a token, a row, a pair,
+// a unique pair) and every tile or split it takes from a tile table is
+// checked against its range before it is used.  A value outside raises
+// kErrCheck in the device flag (ace_get_error: ACE_ERR_CHECK) and the access
+// goes to a safe index instead (a bad tile is dropped), so nothing faults or
+// traps.  Shared-memory and TMEM coordinates are fixed at compile time and
+// checked there (static_assert).  In the normal build the checks compile away.
+#ifdef ACE_CHECKS
+constexpr bool kChecks = true;
+#else
+constexpr bool kChecks = false;
+#endif
+// i when lo <= i < hi; else (ACE_CHECKS) raises kErrCheck and returns `safe`
+__device__ __forceinline__ int chk_idx(int i, int lo, int hi, int safe, int32_t* err) {
+  if (i < lo || i >= hi) {
+    atomicOr(err, kErrCheck);
+    return safe;
+  }
+  return i;
+}
+// ACE_CHK(i, lo, hi, safe, err): chk_idx in the ACE_CHECKS build; the plain
+// index otherwise (lo, hi and safe are then not evaluated)
+#define ACE_CHK(i, lo, hi, safe, err) (::ace::kChecks ? ::ace::chk_idx((i), (lo), (hi), (safe), (err)) : (i))
 
 // Backward row kernel of gate/up at a padded rank of at most 32: two CTAs
 // per SM (half the shared-memory budget each, two-tile splits), so one CTA's
@@ -48,6 +74,16 @@ struct PlanTables {
 struct Tile {
   int32_t g, start, cnt, id;
 };
+// ACE_CHECKS: true when the tile lies in group range [0, G), has at most
+// max_cnt items and its items lie in [0, limit); else raises kErrCheck.  The
+// normal build always returns true.
+__device__ __forceinline__ bool chk_tile(const Tile& t, int G, int max_cnt, int limit, int32_t* err) {
+  if (kChecks && (t.g < 0 || t.g >= G || t.cnt < 0 || t.cnt > max_cnt || t.start < 0 || t.start > limit - t.cnt)) {
+    atomicOr(err, kErrCheck);
+    return false;
+  }
+  return true;
+}
 
 // Byte layout of the permutation workspace for T tokens.
 struct PermLayout {
@@ -152,7 +188,7 @@ cudaError_t launch_permute(const PlanTables& pt, const int32_t* topk_idx, int32_
 constexpr int kZeroMax = 6;
 cudaError_t launch_zero(void* const* ptrs, const size_t* bytes, int n, cudaStream_t st);
 cudaError_t launch_rows_copy(const int32_t* row_pair, const uint16_t* src, uint16_t* dst, int64_t R, int32_t cols,
-                             bool gather, cudaStream_t st);
+                             bool gather, int32_t* err, cudaStream_t st);
 
 // H = A_g x per unique (g, t) pair of gate/up (deduplicated; X rows gathered),
 // or with `rows` H = A_g h per row over the forward row tiles.
@@ -166,6 +202,7 @@ struct FwdHLaunch {
   const uint16_t* A[2];
   float* H[2];        // [R, rank_max] fp32, row u
   int32_t d_in, nproj;
+  int32_t n_src;      // rows of X (T for unique pairs, R for row tiles)
   int32_t* err;
 };
 cudaError_t launch_fwd_h(const PlanTables& pt, const FwdHLaunch& a, cudaStream_t st);
@@ -320,6 +357,7 @@ struct FfnFusedLaunch {
   const int32_t* row_uniq;
   const int32_t* expert_off;
   const int32_t* expert_cnt;
+  const int32_t* counts;  // the permutation's counts (ACE_CHECKS bounds)
   const float* Hs[2];    // gate/up: H of up, gate per unique pair; down: H per row; stride rank_max
   uint16_t* U;           // gate/up outputs [R, f] bf16 (row order): u, v, h
   uint16_t* V;

@@ -181,6 +181,7 @@ ace_status launch_gate_up_h(const ace_plan* plan, const ace_perm* perm, const ui
     }
     h.d_in = d_in;
     h.nproj = nproj;
+    h.n_src = perm->T;
     h.err = err;
     st = cuda_status(launch_fwd_h(pt, h, cs), "forward H launch");
   }
@@ -191,6 +192,8 @@ ace_status launch_gate_up_h(const ace_plan* plan, const ace_perm* perm, const ui
 extern "C" {
 
 int32_t ace_version(void) { return ACE_VERSION; }
+
+int32_t ace_build_checks(void) { return kChecks ? 1 : 0; }
 
 const char* ace_last_error_message(void) { return g_msg; }
 
@@ -301,6 +304,7 @@ ace_status ace_permute(const ace_plan* plan, const int32_t* topk_idx, int32_t T,
   out->uniq_off = at<int32_t>(perm_ws, L.uniq_off);
   out->uniq_tok = at<int32_t>(perm_ws, L.uniq_tok);
   out->tok_uniq = at<int32_t>(perm_ws, L.tok_uniq);
+  out->row_uniq = at<int32_t>(perm_ws, L.row_uniq);
   out->ws = perm_ws;
   return ACE_OK;
 }
@@ -585,6 +589,7 @@ ace_status ace_fwd_combine(const ace_plan* plan, const ace_perm* perm, const uin
   h.H[0] = h.H[1] = H;
   h.d_in = pt.f;
   h.nproj = 1;
+  h.n_src = perm->R;
   h.err = err;
   st = cuda_status(launch_fwd_h(pt, h, cs), "combine H launch");
   if (st != ACE_OK) return st;
@@ -710,7 +715,7 @@ ace_status ace_gather_rows(const ace_perm* perm, const uint16_t* src_pairs, uint
   if (cols < 8 || cols % 8) return fail(ACE_ERR_SHAPE, "cols=%d must be a positive multiple of 8", cols);
   if (!aligned16(src_pairs) || !aligned16(dst_rows)) return fail(ACE_ERR_ARG, "misaligned tensor");
   return cuda_status(launch_rows_copy(perm->row_pair, src_pairs, dst_rows, perm->R, cols, true,
-                                      static_cast<cudaStream_t>(stream)),
+                                      static_cast<int32_t*>(perm->ws), static_cast<cudaStream_t>(stream)),
                      "gather launch");
 }
 
@@ -720,7 +725,7 @@ ace_status ace_scatter_rows(const ace_perm* perm, const uint16_t* src_rows, uint
   if (cols < 8 || cols % 8) return fail(ACE_ERR_SHAPE, "cols=%d must be a positive multiple of 8", cols);
   if (!aligned16(src_rows) || !aligned16(dst_pairs)) return fail(ACE_ERR_ARG, "misaligned tensor");
   return cuda_status(launch_rows_copy(perm->row_pair, src_rows, dst_pairs, perm->R, cols, false,
-                                      static_cast<cudaStream_t>(stream)),
+                                      static_cast<int32_t*>(perm->ws), static_cast<cudaStream_t>(stream)),
                      "scatter launch");
 }
 
@@ -737,6 +742,7 @@ ace_status ace_get_error(const ace_perm* perm, void* stream) {
   if (flag & kErrTimeout) return fail(ACE_ERR_DEVICE_TIMEOUT, "a bounded device wait gave up");
   if (flag & kErrIndex) return fail(ACE_ERR_INDEX, "invalid routing: expert id out of range or repeated in a token");
   if (flag & kErrValue) return fail(ACE_ERR_ARG, "a gate weight given to the combine is not finite");
+  if (flag & kErrCheck) return fail(ACE_ERR_CHECK, "ACE_CHECKS: an index or a tile outside its range (the access was skipped)");
   return ACE_OK;
 }
 

@@ -195,6 +195,7 @@ __global__ void __launch_bounds__(kThreadsWS, RowsCfg<RP, MODE>::kPerSM) k_bwd_r
   if ((int)blockIdx.x >= n_splits) return;
   const int proj = blockIdx.y;
   const Tile sp = (MODE == MODE_SHARED ? a.splits_sh : a.splits_row)[blockIdx.x];
+  if (kChecks && !chk_tile(sp, pt.G, RowsCfg<RP, MODE>::NT * kTileM, a.counts[kCntRows], a.err)) return;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = sp.g, r0 = pt.rank_off[g], rg = pt.rank_off[g + 1] - r0;
   const int ntiles = (sp.cnt + kTileM - 1) / kTileM;
@@ -363,7 +364,8 @@ __global__ void __launch_bounds__(kThreadsWS, RowsCfg<RP, MODE>::kPerSM) k_bwd_r
     // forward's H per row) and writes dp_row = s dHc_u . H_row.
     {
       for (int idx = et; idx < sp.cnt; idx += kEpiThreads) {
-        const int hrow = MODE != MODE_DOWN ? a.row_uniq[sp.start + idx] : sp.start + idx;
+        const int hrow =
+            MODE != MODE_DOWN ? ACE_CHK(a.row_uniq[sp.start + idx], 0, a.counts[kCntU], 0, a.err) : sp.start + idx;
         const float* hp = a.H[proj] + (int64_t)hrow * pt.rank_max;
         for (int c = 0; c < RP && c < pt.rank_max; c += 32) prefetch_l2(hp + c);
         if (MODE == MODE_COMB) {
@@ -403,10 +405,12 @@ __global__ void __launch_bounds__(kThreadsWS, RowsCfg<RP, MODE>::kPerSM) k_bwd_r
       for (int idx = et; idx < ntiles * kTileM; idx += kEpiThreads) {
         const int i = idx / kTileM, mm = idx % kTileM;
         const int row = sp.start + idx;
-        const int hrow = idx >= sp.cnt ? -1 : (MODE != MODE_DOWN ? a.row_uniq[row] : row);
+        const int hrow =
+            idx >= sp.cnt ? -1 : (MODE != MODE_DOWN ? ACE_CHK(a.row_uniq[row], 0, a.counts[kCntU], 0, a.err) : row);
         const float* hp = a.H[proj] + (int64_t)(hrow < 0 ? 0 : hrow) * pt.rank_max;
-        if (MODE == MODE_SHARED) tok_s[idx] = hrow < 0 ? -1 : a.uniq_tok[hrow];
-        const int pair = (MODE == MODE_COMB && hrow >= 0) ? a.row_pair[row] : 0;
+        if (MODE == MODE_SHARED) tok_s[idx] = hrow < 0 ? -1 : ACE_CHK(a.uniq_tok[hrow], 0, a.T, 0, a.err);
+        const int pair =
+            (MODE == MODE_COMB && hrow >= 0) ? ACE_CHK(a.row_pair[row], 0, a.counts[kCntRows], 0, a.err) : 0;
         const float wscale = (MODE == MODE_COMB && hrow >= 0) ? a.s * a.w[pair] : 0.f;
         float dp = 0.f;
 #pragma unroll
@@ -583,14 +587,16 @@ __global__ void __launch_bounds__(128) k_dh_reduce(const __grid_constant__ PlanT
   if (tile >= n_tiles) return;
   const int proj = blockIdx.y;
   const Tile tl = a.tiles_sh[tile];
+  if (kChecks && !chk_tile(tl, pt.G, kTileM, a.counts[kCntU], a.err)) return;
   const int m = (blockIdx.x % CH) * (128 / CH) + threadIdx.x / CH, q = threadIdx.x % CH;
   if (m >= tl.cnt) return;
-  const int u = tl.start + m, t = a.uniq_tok[u], k = pt.k, g = tl.g;
+  const int u = tl.start + m, t = ACE_CHK(a.uniq_tok[u], 0, a.T, 0, a.err), k = pt.k, g = tl.g;
   const int r0 = pt.rank_off[g], rg = pt.rank_off[g + 1] - r0;
   int rows[kMaxK];
   int n = 0;
   for (int j = 0; j < k; ++j)
-    if (a.pair_g[(int64_t)t * k + j] == g) rows[n++] = a.pair_row[(int64_t)t * k + j];
+    if (a.pair_g[(int64_t)t * k + j] == g)
+      rows[n++] = ACE_CHK(a.pair_row[(int64_t)t * k + j], 0, a.counts[kCntRows], 0, a.err);
   float acc[8];
 #pragma unroll
   for (int c = 0; c < 8; ++c) acc[c] = 0.f;

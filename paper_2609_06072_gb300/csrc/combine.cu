@@ -37,13 +37,13 @@ __global__ void __launch_bounds__(kReduceThreads) k_comb_reduce(const __grid_con
     for (int q = 0; q < 8; ++q) acc[q] = 0.f;
     for (int j = 0; j < k; ++j) {
       const int64_t p = (int64_t)t * k + j;
-      const int g = a.pair_g[p];
+      const int g = ACE_CHK(a.pair_g[p], -1, pt.G, -1, a.err);
       if (g < 0) continue;  // invalid token: no rows (the error flag is set)
       const int r0 = pt.rank_off[g], r1 = pt.rank_off[g + 1];
       if (c + 8 <= r0 || c >= r1) continue;
       const float wv = a.w[p];
       if (!isfinite(wv)) atomicOr(a.err, kErrValue);
-      const float* h = a.H + (int64_t)a.pair_row[p] * pt.rank_max - r0;
+      const float* h = a.H + (int64_t)ACE_CHK(a.pair_row[p], 0, a.T * k, 0, a.err) * pt.rank_max - r0;
 #pragma unroll
       for (int q = 0; q < 8; ++q)
         if (c + q >= r0 && c + q < r1) acc[q] += wv * h[c + q];

@@ -287,7 +287,7 @@ __global__ void __launch_bounds__(256) k_swiglu_bwd(const uint16_t* __restrict__
 // ascending j (fp32 sum, one rounding); 8 columns a thread
 __global__ void __launch_bounds__(256) k_token_sum(const uint16_t* __restrict__ rows, const int32_t* __restrict__ pair_row,
                                                    const int32_t* __restrict__ pair_g, int k, int T, int cols,
-                                                   uint16_t* __restrict__ dX) {
+                                                   uint16_t* __restrict__ dX, int32_t* err) {
   pdl_wait();
   pdl_trigger();
   const int per = cols / 8;
@@ -299,7 +299,8 @@ __global__ void __launch_bounds__(256) k_token_sum(const uint16_t* __restrict__ 
   for (int j = 0; j < k; ++j) {
     const int64_t p = t * k + j;
     if (pair_g[p] < 0) continue;  // invalid token: no rows
-    const uint4 w = *reinterpret_cast<const uint4*>(rows + (int64_t)pair_row[p] * cols + c);
+    const uint4 w =
+        *reinterpret_cast<const uint4*>(rows + (int64_t)ACE_CHK(pair_row[p], 0, T * k, 0, err) * cols + c);
     const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
@@ -419,6 +420,7 @@ ace_status ace_ffn_fwd(const ace_plan* plan, const ace_perm* perm, const uint16_
   g.row_uniq = at<int32_t>(perm->ws, L.row_uniq);
   g.expert_off = perm->expert_off;
   g.expert_cnt = perm->expert_cnt;
+  g.counts = perm->counts;
   g.Hs[0] = Hgu[1];  // TMEM half 0: up
   g.Hs[1] = Hgu[0];  // TMEM half 1: gate
   g.U = U;
@@ -442,6 +444,7 @@ ace_status ace_ffn_fwd(const ace_plan* plan, const ace_perm* perm, const uint16_
   hd.H[0] = hd.H[1] = Hd;
   hd.d_in = pt.f;
   hd.nproj = 1;
+  hd.n_src = R;
   hd.err = err;
   st = cuda(launch_fwd_h(pt, hd, cs), "ace_ffn_fwd: down H launch");
   if (st != ACE_OK) return st;
@@ -455,6 +458,7 @@ ace_status ace_ffn_fwd(const ace_plan* plan, const ace_perm* perm, const uint16_
   dn.tm_bt[1] = dn.tm_bt[0];
   dn.expert_off = perm->expert_off;
   dn.expert_cnt = perm->expert_cnt;
+  dn.counts = perm->counts;
   dn.Hs[0] = dn.Hs[1] = Hd;
   dn.Y = Y;
   dn.s = s;
@@ -529,7 +533,7 @@ ace_status ace_ffn_bwd(const ace_plan* plan, const ace_perm* perm, const uint16_
   const int64_t nt = (int64_t)perm->T * (pt.d / 8);
   st = cuda(launch_k(k_token_sum, (unsigned)((nt + 255) / 256), 256, 0, cs, (const uint16_t*)dxr,
                      (const int32_t*)perm->pair_row, (const int32_t*)at<int32_t>(perm->ws, L.pair_g), pt.k, perm->T,
-                     pt.d, dX),
+                     pt.d, dX, err),
             "ace_ffn_bwd: token sum launch");
   if (st != ACE_OK) return st;
   // the gate and up adapters: dX += their input gradient, dA, dB

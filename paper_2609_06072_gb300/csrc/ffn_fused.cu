@@ -114,6 +114,11 @@ __global__ void __launch_bounds__(kXThreads, 1) k_ffn_fused(const __grid_constan
     const int i = rt - tpre[e];
     row0 = a.expert_off[e] + i * 128;
     cnt = min(128, a.expert_cnt[e] - i * 128);
+    if (kChecks && (row0 < 0 || cnt < 0 || row0 > a.counts[kCntRows] - cnt)) {
+      atomicOr(a.err, kErrCheck);  // an expert segment outside the rows: the item is dropped
+      row0 = 0;
+      cnt = 0;
+    }
   };
   const uint32_t tmem = tslot;
   bool bad = false;
@@ -299,7 +304,7 @@ __global__ void __launch_bounds__(kXThreads, 1) k_ffn_fused(const __grid_constan
         break;
       }
       tc_fence_after();
-      const int hrow = live ? (GU ? a.row_uniq[row0 + t] : row0 + t) : -1;
+      const int hrow = live ? (GU ? ACE_CHK(a.row_uniq[row0 + t], 0, a.counts[kCntU], 0, a.err) : row0 + t) : -1;
 #pragma unroll
       for (int j = 0; j < (GU ? 2 : 1); ++j) {
         const float* hp = a.Hs[j] + (int64_t)(hrow < 0 ? 0 : hrow) * pt.rank_max;

@@ -70,13 +70,16 @@ __global__ void __launch_bounds__(kHThreads) k_fwd_h(const __grid_constant__ Pla
     if ((int)blockIdx.x >= a.counts[kCntTilesSh]) return;
     tl = a.tiles[blockIdx.x];
   }
+  if (kChecks && !chk_tile(tl, pt.G, kTileM, a.counts[a.rows ? kCntRows : kCntU], a.err)) return;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int quarter = warp & 3, half = warp >> 2;
   const int m = quarter * 32 + lane;
   const int g = tl.g, r0 = pt.rank_off[g], rg = pt.rank_off[g + 1] - r0;
   const int d_in = a.d_in;
 
-  if (tid < kTileM) src_row[tid] = tid < tl.cnt ? (a.rows ? tl.start + tid : a.uniq_tok[tl.start + tid]) : -1;
+  if (tid < kTileM)
+    src_row[tid] = tid < tl.cnt ? (a.rows ? tl.start + tid : ACE_CHK(a.uniq_tok[tl.start + tid], 0, a.n_src, 0, a.err))
+                                : -1;
   if (tid == 0) {
     for (int i = 0; i < kHStages; ++i) mbar_init(&bar_k[i], 1);
     fence_mbar_init();
@@ -365,9 +368,10 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
   // per kernel instance, NPROJ == 1): 1, else 0
   const int psplit = (SHARED && NPROJ == 1 && a.proj_split) ? 1 : 0;
   const int split0 = a.counts[kCntRowSplit], n_split = (n_items - split0) / kSplitParts;
-  const bool has_pre = pre && (int)blockIdx.x < n_split;
+  bool has_pre = pre && (int)blockIdx.x < n_split;
   Tile pre_t{};
   if (has_pre) pre_t = a.tiles[split0 + kSplitParts * (int)blockIdx.x];
+  if (kChecks && has_pre) has_pre = chk_tile(pre_t, pt.G, kTileM, a.counts[kCntRows], a.err);
   int32_t* const hflag = a.sched + 8;
   auto needs_k = [&](const Tile& t) { return !SHARED && !(pre && t.id > 0); };
   const int d_in = a.d_in, d_out = a.d_out;
@@ -402,7 +406,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
           item = vt < split0 ? vt : split0 + (vt - split0) * merge;
           t = a.tiles[item];
           pj = v & psplit;
-          if (tile_live(t, merge)) break;
+          if (tile_live(t, merge) && (!kChecks || chk_tile(t, pt.G, kTileM, a.counts[kCntRows], a.err))) break;
         }
         const int e = q % kQ;
         if (q >= kQ && !mbar_wait(&tq.empty[e], ((q - kQ) / kQ) & 1)) {
@@ -582,7 +586,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1) k_fwd_rows(const __grid_const
         }
       } else {
         // gate/up: H of the row's unique pair; down split tile: its up-front H row
-        const int u = live ? (SHARED ? a.row_uniq[t.start + m] : t.start + m) : -1;
+        const int u = live ? (SHARED ? ACE_CHK(a.row_uniq[t.start + m], 0, a.counts[kCntU], 0, a.err) : t.start + m) : -1;
         if ((pt.rank_max & 3) != 0) {
           // rows not 16-byte aligned: 8 columns at a time (measured faster
           // here than all loads up front)

@@ -699,7 +699,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemm_h(const __grid_constant__ 
       int uu[KB], gu[KB];
 #pragma unroll
       for (int n = 0; n < KB; ++n) {
-        uu[n] = (t < a.T && n < k) ? a.tok_uniq[(int64_t)t * k + n] : -1;
+        uu[n] = (t < a.T && n < k) ? ACE_CHK(a.tok_uniq[(int64_t)t * k + n], -1, uoff_s[G], -1, a.err) : -1;
         gu[n] = uu[n] >= 0 ? upper_idx(uoff_s, G, uu[n]) : -1;
       }
       if (!__all_sync(0xffffffffu, mbar_wait(&acc_full[b], (it >> 1) & 1))) {

@@ -485,13 +485,13 @@ __global__ void __launch_bounds__(256) k_zero(const __grid_constant__ ZeroList z
 }
 
 __global__ void k_rows_copy(const int32_t* __restrict__ row_pair, const uint4* __restrict__ src,
-                            uint4* __restrict__ dst, int64_t R, int vec_per_row, bool gather) {
+                            uint4* __restrict__ dst, int64_t R, int vec_per_row, bool gather, int32_t* err) {
   pdl_wait();
   pdl_trigger();
   const int64_t n = R * vec_per_row;
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
     const int64_t row = i / vec_per_row, v = i % vec_per_row;
-    const int64_t p = row_pair[row];
+    const int64_t p = ACE_CHK(row_pair[row], 0, (int)R, 0, err);
     if (gather)
       dst[row * vec_per_row + v] = src[p * vec_per_row + v];
     else
@@ -552,13 +552,13 @@ cudaError_t launch_zero(void* const* ptrs, const size_t* bytes, int n, cudaStrea
 }
 
 cudaError_t launch_rows_copy(const int32_t* row_pair, const uint16_t* src, uint16_t* dst, int64_t R, int32_t cols,
-                             bool gather, cudaStream_t st) {
+                             bool gather, int32_t* err, cudaStream_t st) {
   if (R == 0) return cudaSuccess;
   const int vpr = cols / 8;
   const int64_t n = R * vpr;
   int blocks = (int)std::min<int64_t>((n + 255) / 256, 152 * 16);
   return launch_k(k_rows_copy, blocks, 256, 0, st, row_pair, reinterpret_cast<const uint4*>(src),
-                  reinterpret_cast<uint4*>(dst), R, vpr, gather);
+                  reinterpret_cast<uint4*>(dst), R, vpr, gather, err);
 }
 
 }  // namespace ace

@@ -23,6 +23,23 @@ def lib():
     return ace.load()
 
 
+@pytest.fixture(scope="module")
+def lib_checks():
+    from paper_2609_06072_gb300 import _build, ace
+    _build.build(checks=True)
+    return ace.load(checks=True)
+
+
+def test_checked_build_exports_the_same_boundary(lib, lib_checks):
+    # libace_checks.so: the same sources with ACE_CHECKS; same symbols, and
+    # each library reports which build it is
+    for s in declared_symbols():
+        assert hasattr(lib_checks, s), f"libace_checks.so does not export {s}"
+    assert lib.ace_build_checks() == 0
+    assert lib_checks.ace_build_checks() == 1
+    assert lib_checks.ace_version() == lib.ace_version()
+
+
 def test_header_declares_the_boundary():
     syms = declared_symbols()
     from paper_2609_06072_gb300 import ace

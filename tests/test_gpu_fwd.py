@@ -35,7 +35,8 @@ def run_perm(L, plan):
 
 def compare_perm(G_arr, O):
     assert G_arr["U"] == O["U"]
-    for key in ("group_off", "expert_off", "expert_cnt", "row_pair", "pair_row", "uniq_off", "uniq_tok", "tok_uniq"):
+    for key in ("group_off", "expert_off", "expert_cnt", "row_pair", "pair_row", "uniq_off", "uniq_tok", "tok_uniq",
+                "row_uniq"):
         assert np.array_equal(G_arr[key], O[key]), key
 
 

@@ -369,7 +369,7 @@ struct FfnFusedLaunch {
 };
 cudaError_t launch_ffn_fused(const PlanTables& pt, const FfnFusedLaunch& a, bool gate_up, cudaStream_t st);
 cudaError_t launch_gather_tokens(const int32_t* row_pair, const int32_t* counts, int k, int T, const uint16_t* X,
-                                 uint16_t* dst, int64_t R, int cols, cudaStream_t st);
+                                 uint16_t* dst, int64_t R, int cols, int nsm, cudaStream_t st);
 cudaError_t launch_swiglu(const uint16_t* u, const uint16_t* v, uint16_t* h, int64_t n, cudaStream_t st);
 
 }  // namespace ace

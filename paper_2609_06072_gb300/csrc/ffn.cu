@@ -221,24 +221,39 @@ __global__ void __launch_bounds__(kFThreads, 1) k_expert_gemm(const __grid_const
   if (warp == 0) tmem_dealloc(tmem, 2 * kFN);
 }
 
-// dst[row] = X[row_pair[row] / k]: token rows into row order, 16 bytes a
-// thread, over the rows the permutation wrote (counts[kCntRows]; the rows of
-// invalid tokens are never written and are skipped)
+// dst[row] = X[row_pair[row] / k]: token rows into row order over the rows
+// the permutation wrote (counts[kCntRows]; the rows of invalid tokens are
+// never written and are skipped).  A warp copies a row, each lane eight
+// 16-byte pieces at a time, all eight loads issued before the first store.
 __global__ void __launch_bounds__(256) k_gather_tokens(const int32_t* __restrict__ row_pair,
                                                        const int32_t* __restrict__ counts, int k, int T,
                                                        const uint16_t* __restrict__ X, uint16_t* __restrict__ dst,
                                                        int64_t R, int cols) {
   pdl_wait();
   pdl_trigger();
-  const int per = cols / 8;
-  const int64_t idx = (int64_t)blockIdx.x * 256 + threadIdx.x;
-  if (idx >= R * per) return;
-  const int64_t row = idx / per;
-  if (row >= counts[kCntRows]) return;
-  const int c = (int)(idx % per) * 8;
-  const int64_t t = row_pair[row] / k;
-  if (t < 0 || t >= T) return;
-  *reinterpret_cast<uint4*>(dst + row * cols + c) = *reinterpret_cast<const uint4*>(X + t * cols + c);
+  const int per = cols / 8;  // 16-byte pieces per row
+  const int64_t nrow = min(R, (int64_t)counts[kCntRows]);
+  const int lane = threadIdx.x & 31;
+  const int64_t nwarps = (int64_t)gridDim.x * (blockDim.x >> 5);
+  for (int64_t row = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; row < nrow; row += nwarps) {
+    const int64_t t = row_pair[row] / k;
+    if (t < 0 || t >= T) continue;
+    const uint4* __restrict__ src = reinterpret_cast<const uint4*>(X + t * cols);
+    uint4* __restrict__ out = reinterpret_cast<uint4*>(dst + row * cols);
+    for (int c0 = 0; c0 < per; c0 += 8 * 32) {
+      uint4 v[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int c = c0 + i * 32 + lane;
+        if (c < per) v[i] = src[c];
+      }
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int c = c0 + i * 32 + lane;
+        if (c < per) out[c] = v[i];
+      }
+    }
+  }
 }
 
 // h = SiLU(v) * u elementwise (bf16 in, fp32 arithmetic, bf16 out), 8 a thread
@@ -339,11 +354,11 @@ cudaError_t launch_expert_gemm(const void* in, const void* W, const int32_t* exp
 }
 
 cudaError_t launch_gather_tokens(const int32_t* row_pair, const int32_t* counts, int k, int T, const uint16_t* X,
-                                 uint16_t* dst, int64_t R, int cols, cudaStream_t st) {
-  const int64_t n = R * (cols / 8);
-  if (n == 0) return cudaSuccess;
-  return launch_k(k_gather_tokens, (unsigned)((n + 255) / 256), 256, 0, st, row_pair, counts, k, T, X, dst, R,
-                  cols);
+                                 uint16_t* dst, int64_t R, int cols, int nsm, cudaStream_t st) {
+  if (R == 0) return cudaSuccess;
+  // a warp per row, eight warps a block, up to 16 blocks per SM
+  const int64_t blocks = std::min<int64_t>((R + 7) / 8, (int64_t)nsm * 16);
+  return launch_k(k_gather_tokens, (unsigned)blocks, 256, 0, st, row_pair, counts, k, T, X, dst, R, cols);
 }
 
 cudaError_t launch_swiglu(const uint16_t* u, const uint16_t* v, uint16_t* h, int64_t n, cudaStream_t st) {
@@ -407,7 +422,7 @@ ace_status ace_ffn_fwd(const ace_plan* plan, const ace_perm* perm, const uint16_
   // 2. the token rows in row order, then u, v (base + adapter) and
   // h = SiLU(v) u in one kernel
   uint16_t* Xr = static_cast<uint16_t*>(ws);
-  st = cuda(launch_gather_tokens(perm->row_pair, perm->counts, pt.k, perm->T, X, Xr, R, pt.d, cs),
+  st = cuda(launch_gather_tokens(perm->row_pair, perm->counts, pt.k, perm->T, X, Xr, R, pt.d, plan->num_sms, cs),
             "ace_ffn_fwd: gather launch");
   if (st != ACE_OK) return st;
   FfnFusedLaunch g{};

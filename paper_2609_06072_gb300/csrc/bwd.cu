@@ -639,14 +639,40 @@ __global__ void __launch_bounds__(256) k_splitk_reduce(const __grid_constant__ P
   int g = 0;
   while (pt.rank_off[g + 1] <= i) ++g;
   const int kk = i - pt.rank_off[g];
+  const int n = counts[slot];
+  // the split table lists the splits group by group (ascending g): find the
+  // range of group g in one pass of the block over the table
+  __shared__ int s_lo, s_hi;
+  if (threadIdx.x == 0) s_lo = s_hi = 0;
+  __syncthreads();
+  for (int t = threadIdx.x; t < n; t += blockDim.x)
+    if (splits[t].g == g) {
+      if (t == 0 || splits[t - 1].g != g) s_lo = t;
+      if (t == n - 1 || splits[t + 1].g != g) s_hi = t + 1;
+    }
+  __syncthreads();
+  const int lo = s_lo, hi = s_hi;
   const int c = (blockIdx.y * 256 + threadIdx.x) * 4;
   if (c >= width) return;
-  const int n = counts[slot];
+  const float* base = part + (int64_t)kk * width + c;
+  const int64_t stride = (int64_t)RP * width;  // one split's partial
   float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-  for (int sidx = 0; sidx < n; ++sidx) {
-    const Tile sp = splits[sidx];
-    if (sp.g != g) continue;
-    const float4 v = *reinterpret_cast<const float4*>(part + ((int64_t)sp.id * RP + kk) * width + c);
+  // in split order, four partials in flight at a time
+  int sidx = lo;
+  for (; sidx + 4 <= hi; sidx += 4) {
+    float4 v[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) v[q] = *reinterpret_cast<const float4*>(base + (int64_t)splits[sidx + q].id * stride);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      acc.x += v[q].x;
+      acc.y += v[q].y;
+      acc.z += v[q].z;
+      acc.w += v[q].w;
+    }
+  }
+  for (; sidx < hi; ++sidx) {
+    const float4 v = *reinterpret_cast<const float4*>(base + (int64_t)splits[sidx].id * stride);
     acc.x += v.x;
     acc.y += v.y;
     acc.z += v.z;

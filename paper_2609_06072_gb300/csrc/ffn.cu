@@ -179,17 +179,34 @@ __global__ void __launch_bounds__(kFThreads, 1) k_expert_gemm(const __grid_const
       for (int c16 = 0; c16 < 8; ++c16) {
         const int col = n0 + ehalf * 128 + c16 * 16;
         if (col >= a.N) break;  // warp-uniform
+        // out[row] += the product (fp32 sum, one rounding): the old values of
+        // a whole 16-column piece come in two 16-byte loads, issued before the
+        // accumulator is read
+        const bool whole = col + 16 <= a.N;
+        uint4 o0 = make_uint4(0u, 0u, 0u, 0u), o1 = o0;
+        if (a.accumulate && whole && m < cnt) {
+          o0 = *reinterpret_cast<const uint4*>(orow + col);
+          o1 = *reinterpret_cast<const uint4*>(orow + col + 8);
+        }
         uint32_t r[16];
         tmem_ld16(tmem + lane_base + b * kFN + ehalf * 128 + c16 * 16, r);
         tmem_ld_wait();
         if (m < cnt) {
-          if (a.accumulate) {  // out[row] += the product (fp32 sum, one rounding)
+          if (a.accumulate && whole) {
+            const uint32_t ow[8] = {o0.x, o0.y, o0.z, o0.w, o1.x, o1.y, o1.z, o1.w};
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+              const float2 f = unpack_bf16x2(ow[q]);
+              r[2 * q] = __float_as_uint(f.x + __uint_as_float(r[2 * q]));
+              r[2 * q + 1] = __float_as_uint(f.y + __uint_as_float(r[2 * q + 1]));
+            }
+          } else if (a.accumulate) {
             for (int q = 0; q < 16 && col + q < a.N; ++q) {
               const float old = __uint_as_float((uint32_t)orow[col + q] << 16);
               r[q] = __float_as_uint(old + __uint_as_float(r[q]));
             }
           }
-          if (col + 16 <= a.N) {
+          if (whole) {
             uint4 v0, v1;
             v0.x = pack_bf16x2(__uint_as_float(r[0]), __uint_as_float(r[1]));
             v0.y = pack_bf16x2(__uint_as_float(r[2]), __uint_as_float(r[3]));

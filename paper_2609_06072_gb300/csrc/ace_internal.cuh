@@ -345,9 +345,12 @@ cudaError_t launch_comb_reduce(const PlanTables& pt, const CombReduceLaunch& a, 
 // Expert FFN pieces (ffn.cu).
 // out[row] (+)= in[row] . W_e^T over the rows of each expert e; W is [E * N, K]
 // (W_e^T rows), or with w_kn [E * K, N] (W_e itself: the input gradient).
+// With in2 and W2 (same shapes) the second product is added in the same
+// accumulator: out[row] (+)= in[row] . W_e^T + in2[row] . W2_e^T.
 cudaError_t launch_expert_gemm(const void* in, const void* W, const int32_t* expert_off, const int32_t* expert_cnt,
                                uint16_t* out, int E, int64_t R, int N, int K, int grid, int32_t* err,
-                               cudaStream_t st, bool w_kn = false, bool accumulate = false);
+                               cudaStream_t st, bool w_kn = false, bool accumulate = false,
+                               const void* in2 = nullptr, const void* W2 = nullptr);
 // Expert FFN forward with the adapters fused into the base GEMMs
 // (ffn_fused.cu): gate/up writes u, v, h = SiLU(v) u; down writes y.
 struct FfnFusedLaunch {

@@ -11,7 +11,8 @@
 //   one expert x 256 output columns] tiles; both operands K-major by TMA
 //   (128-byte swizzle), four 48 KB stages, tcgen05 M = 128, N = 256 into one
 //   of two TMEM accumulators, eight epilogue warps (thread = row, 128 columns
-//   each) storing bf16.
+//   each) storing bf16.  A second product over the same rows (the backward's
+//   dv . W_gate beside du . W_up) can follow in the same accumulator.
 #include <algorithm>
 #include <cstdint>
 
@@ -31,6 +32,10 @@ constexpr int kFSmem = kFS * kFStage + 1024;
 struct ExpertGemmLaunch {
   CUtensorMap tm_in;   // in [R, K] bf16, box 64 x 128
   CUtensorMap tm_w;    // W_e^T rows: [E * N, K] bf16, box 64 x 256; or (B_MN) W_e: [E * K, N], box 64 x 64
+  // optional second product over the same rows, summed into the same
+  // accumulator (its K steps follow the first's): out = in . W + in2 . W2
+  CUtensorMap tm_in2, tm_w2;
+  int32_t two;
   const int32_t* expert_off;
   const int32_t* expert_cnt;
   uint16_t* out;       // [R, N] bf16
@@ -64,7 +69,7 @@ __global__ void __launch_bounds__(kFThreads, 1) k_expert_gemm(const __grid_const
   __shared__ int32_t tpre[ACE_MAX_EXPERTS + 1];  // row tiles before expert e
   __shared__ int32_t eoff[ACE_MAX_EXPERTS], ecnt[ACE_MAX_EXPERTS];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int E = a.E, nchunk = (a.N + kFN - 1) / kFN, NK = (a.K + 63) / 64;
+  const int E = a.E, nchunk = (a.N + kFN - 1) / kFN, NK1 = (a.K + 63) / 64, NK = a.two ? 2 * NK1 : NK1;
   const uint32_t s0 = smem_u32(smem);
   if (tid == 0) {
     for (int i = 0; i < kFS; ++i) {
@@ -118,13 +123,17 @@ __global__ void __launch_bounds__(kFThreads, 1) k_expert_gemm(const __grid_const
             break;
           }
           const uint32_t base = s0 + s * kFStage;
+          const bool second = kb >= NK1;
+          const int kq = second ? kb - NK1 : kb;
+          const CUtensorMap* tin = second ? &a.tm_in2 : &a.tm_in;
+          const CUtensorMap* tw = second ? &a.tm_w2 : &a.tm_w;
           mbar_arrive_expect_tx(&full[s], kFStage);
-          tma_load_2d(base, &a.tm_in, kb * 64, row0, &full[s]);
+          tma_load_2d(base, tin, kq * 64, row0, &full[s]);
           if (B_MN) {
             for (int q = 0; q < kFN / 64; ++q)
-              tma_load_2d(base + kFBlk + q * (kFBlk / 2), &a.tm_w, n0 + q * 64, e * a.K + kb * 64, &full[s]);
+              tma_load_2d(base + kFBlk + q * (kFBlk / 2), tw, n0 + q * 64, e * a.K + kq * 64, &full[s]);
           } else {
-            tma_load_2d(base + kFBlk, &a.tm_w, kb * 64, e * a.N + n0, &full[s]);
+            tma_load_2d(base + kFBlk, tw, kq * 64, e * a.N + n0, &full[s]);
           }
         }
       }
@@ -349,11 +358,16 @@ __global__ void __launch_bounds__(256) k_token_sum(const uint16_t* __restrict__ 
 
 cudaError_t launch_expert_gemm(const void* in, const void* W, const int32_t* expert_off, const int32_t* expert_cnt,
                                uint16_t* out, int E, int64_t R, int N, int K, int grid, int32_t* err,
-                               cudaStream_t st, bool w_kn, bool accumulate) {
+                               cudaStream_t st, bool w_kn, bool accumulate, const void* in2, const void* W2) {
   ExpertGemmLaunch a{};
-  const bool ok = make_tmap_bf16(&a.tm_in, in, (uint64_t)R, (uint64_t)K, 128) &&
-                  (w_kn ? make_tmap_bf16(&a.tm_w, W, (uint64_t)E * K, (uint64_t)N, 64)
-                        : make_tmap_bf16(&a.tm_w, W, (uint64_t)E * N, (uint64_t)K, 256));
+  auto maps = [&](CUtensorMap* ti, CUtensorMap* tw, const void* x, const void* w) {
+    return make_tmap_bf16(ti, x, (uint64_t)R, (uint64_t)K, 128) &&
+           (w_kn ? make_tmap_bf16(tw, w, (uint64_t)E * K, (uint64_t)N, 64)
+                 : make_tmap_bf16(tw, w, (uint64_t)E * N, (uint64_t)K, 256));
+  };
+  bool ok = maps(&a.tm_in, &a.tm_w, in, W);
+  a.two = in2 != nullptr && W2 != nullptr;
+  if (a.two) ok = ok && maps(&a.tm_in2, &a.tm_w2, in2, W2);
   if (!ok) return cudaErrorInvalidValue;
   a.accumulate = accumulate ? 1 : 0;
   a.expert_off = expert_off;
@@ -555,12 +569,12 @@ ace_status ace_ffn_bwd(const ace_plan* plan, const ace_perm* perm, const uint16_
   st = cuda(launch_k(k_swiglu_bwd, (unsigned)((n8 + 255) / 256), 256, 0, cs, (const uint16_t*)dh, U, V, du, dv, n8),
             "ace_ffn_bwd: SiLU gating backward launch");
   if (st != ACE_OK) return st;
-  // base input gradient per row: du . W_up + dv . W_gate, then summed per token
+  // base input gradient per row: du . W_up + dv . W_gate in one GEMM (the
+  // gate product's K steps follow the up product's in the same accumulator),
+  // then summed per token
   st = cuda(launch_expert_gemm(du, W_up, perm->expert_off, perm->expert_cnt, dxr, pt.E, R, pt.d, pt.f, plan->num_sms,
-                               err, cs, true, false), "ace_ffn_bwd: up input-gradient GEMM launch");
-  if (st != ACE_OK) return st;
-  st = cuda(launch_expert_gemm(dv, W_gate, perm->expert_off, perm->expert_cnt, dxr, pt.E, R, pt.d, pt.f,
-                               plan->num_sms, err, cs, true, true), "ace_ffn_bwd: gate input-gradient GEMM launch");
+                               err, cs, true, false, dv, W_gate),
+            "ace_ffn_bwd: up and gate input-gradient GEMM launch");
   if (st != ACE_OK) return st;
   const int64_t nt = (int64_t)perm->T * (pt.d / 8);
   st = cuda(launch_k(k_token_sum, (unsigned)((nt + 255) / 256), 256, 0, cs, (const uint16_t*)dxr,

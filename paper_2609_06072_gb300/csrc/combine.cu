@@ -22,32 +22,61 @@ constexpr int kReduceThreads = 256;  // one warp per token
 
 // Hx[t] for one token per warp: lane l owns the 8-column blocks
 // c = 8 (l + 32 i) of the row; for each of the token's pairs (ascending j)
-// the block's columns inside the pair's group add w * H_row.
+// the block's columns inside the pair's group add w * H_row.  Lane j < k
+// first reads pair j's group, row and weight, and the warp shares them by
+// shuffles; a block inside one group whose H row piece is 16-byte aligned is
+// read in two 16-byte loads.
 __global__ void __launch_bounds__(kReduceThreads) k_comb_reduce(const __grid_constant__ PlanTables pt,
                                                                 const __grid_constant__ CombReduceLaunch a) {
   pdl_wait();
   pdl_trigger();
   const int t = blockIdx.x * (kReduceThreads / 32) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
-  if (t >= a.T) return;
+  if (t >= a.T) return;  // warp-uniform
   const int k = pt.k;
-  for (int c = 8 * lane; c < a.n_rank_pad; c += 8 * 32) {
+  int g_l = -1, row_l = 0;
+  float w_l = 0.f;
+  if (lane < k) {
+    const int64_t p = (int64_t)t * k + lane;
+    g_l = ACE_CHK(a.pair_g[p], -1, pt.G, -1, a.err);
+    if (g_l >= 0) {  // an invalid token has no rows (the error flag is set)
+      row_l = ACE_CHK(a.pair_row[p], 0, a.T * k, 0, a.err);
+      w_l = a.w[p];
+      if (!isfinite(w_l)) atomicOr(a.err, kErrValue);
+    }
+  }
+  const bool vec = (pt.rank_max & 3) == 0;
+  for (int c0 = 0; c0 < a.n_rank_pad; c0 += 8 * 32) {  // warp-uniform trips
+    const int c = c0 + 8 * lane;
     float acc[8];
 #pragma unroll
     for (int q = 0; q < 8; ++q) acc[q] = 0.f;
     for (int j = 0; j < k; ++j) {
-      const int64_t p = (int64_t)t * k + j;
-      const int g = ACE_CHK(a.pair_g[p], -1, pt.G, -1, a.err);
-      if (g < 0) continue;  // invalid token: no rows (the error flag is set)
+      const int g = __shfl_sync(0xffffffffu, g_l, j);
+      const int row = __shfl_sync(0xffffffffu, row_l, j);
+      const float wv = __shfl_sync(0xffffffffu, w_l, j);
+      if (g < 0 || c >= a.n_rank_pad) continue;
       const int r0 = pt.rank_off[g], r1 = pt.rank_off[g + 1];
       if (c + 8 <= r0 || c >= r1) continue;
-      const float wv = a.w[p];
-      if (!isfinite(wv)) atomicOr(a.err, kErrValue);
-      const float* h = a.H + (int64_t)ACE_CHK(a.pair_row[p], 0, a.T * k, 0, a.err) * pt.rank_max - r0;
+      const float* h = a.H + (int64_t)row * pt.rank_max - r0;
+      if (vec && c >= r0 && c + 8 <= r1 && (r0 & 3) == 0) {
+        const float4 x0 = *reinterpret_cast<const float4*>(h + c);
+        const float4 x1 = *reinterpret_cast<const float4*>(h + c + 4);
+        acc[0] += wv * x0.x;
+        acc[1] += wv * x0.y;
+        acc[2] += wv * x0.z;
+        acc[3] += wv * x0.w;
+        acc[4] += wv * x1.x;
+        acc[5] += wv * x1.y;
+        acc[6] += wv * x1.z;
+        acc[7] += wv * x1.w;
+      } else {
 #pragma unroll
-      for (int q = 0; q < 8; ++q)
-        if (c + q >= r0 && c + q < r1) acc[q] += wv * h[c + q];
+        for (int q = 0; q < 8; ++q)
+          if (c + q >= r0 && c + q < r1) acc[q] += wv * h[c + q];
+      }
     }
+    if (c >= a.n_rank_pad) continue;
     uint4 o;
     o.x = pack_bf16x2(a.s * acc[0], a.s * acc[1]);
     o.y = pack_bf16x2(a.s * acc[2], a.s * acc[3]);

@@ -318,6 +318,13 @@ struct DenseBwdLaunch {
   int32_t T, d, n_rank, n_rank_pad, nproj;
   int32_t grid;  // persistent CTAs of the dX GEMM (the SM count)
   int32_t* err;
+  // dX then dA in one call (launch_dense_bwd): dA reads nothing dX writes,
+  // so dX signals its dependents as soon as its own inputs are ready and dA
+  // waits on the grid dependency only at its end; dA's CTAs then fill the
+  // SMs that dX's last round leaves idle.  (dA's inputs were complete before
+  // dX's wait returned, and dX's CTAs signal only after it; the late wait
+  // keeps dA from completing before dX.)
+  int32_t early_signal, no_wait;
 };
 // dA must be zero on entry (the GEMM adds its tiles into it).
 cudaError_t launch_dense_bwd(const DenseBwdLaunch& a, cudaStream_t st);

@@ -299,6 +299,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   cluster_sync();  // the peer's barriers exist before anything arrives on them
   tc_fence_after();
   pdl_wait();
+  if (a.early_signal) pdl_trigger();  // the dA GEMM that follows does not read dX
   const uint32_t tmem = tslot;
   bool bad = false;
   if (warp == 0) {
@@ -490,7 +491,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemm_da(const __grid_constant__
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  pdl_wait();
+  // no_wait (launch_dense_bwd): the inputs were complete before the dX GEMM's
+  // own wait returned, so the wait moves to the end (below), where it keeps
+  // this grid from completing before the dX GEMM
+  if (!a.no_wait) pdl_wait();
   const uint32_t tmem = tslot;
   bool bad = false;
   if (warp == 0) {
@@ -568,6 +572,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemm_da(const __grid_constant__
   __syncwarp();
   tc_fence_before();
   if (__syncthreads_or(bad) && tid == 0) atomicOr(a.err, kErrTimeout);
+  if (a.no_wait) pdl_wait();
   // signal dependents only as this CTA finishes: an earlier launch of the
   // next kernel (a whole SM per CTA) measured slower
   pdl_trigger();
@@ -788,8 +793,13 @@ cudaError_t launch_dense_da(const DenseBwdLaunch& a, cudaStream_t st) {
 }
 
 cudaError_t launch_dense_bwd(const DenseBwdLaunch& a, cudaStream_t st) {
-  cudaError_t e = launch_dense_dx(a, st);
-  return e != cudaSuccess ? e : launch_dense_da(a, st);
+  DenseBwdLaunch x = a, d = a;
+  // the pair kernel signals early; the one-CTA dX kernel (T < 256) keeps the
+  // plain chain
+  x.early_signal = a.T >= 256 && a.grid >= 2;
+  d.no_wait = x.early_signal;
+  cudaError_t e = launch_dense_dx(x, st);
+  return e != cudaSuccess ? e : launch_dense_da(d, st);
 }
 
 }  // namespace ace

@@ -53,6 +53,23 @@ def test_byte_model_counts_each_tensor_once():
     assert b["bwd_row"] == 2 * R * d + 2 * R * f + 4 * int((R_g * 8).sum()) + 4 * R * f + 6 * Pw
 
 
+def test_olmoe_byte_model_is_the_reported_one():
+    # the algorithmic bytes the benchmark's roofline divides by, for the
+    # OLMoE-shaped layer at seed 0 (the bench's default), from the realised
+    # routing: per-group row and unique-pair counts of the oracle permutation
+    import oracle
+    L = W.Layer(W.get_config("olmoe"), seed=0)
+    c = L.cfg
+    O = oracle.permute(L.topk_idx, L.e2g, L.G)
+    b, fl = bench.model(c.T, c.k, c.d, c.f, L.rank_off, np.diff(O["uniq_off"]), np.diff(O["group_off"]))
+    assert b["fwd_row"] == 682622976
+    assert b["bwd_row"] == 688914432
+    # every routed row moves its Y / dY / h / dh bytes once: the row traffic
+    # alone is most of each down call
+    R = c.T * c.k
+    assert 2 * R * c.f + 4 * R * c.d > 0.95 * b["fwd_row"]
+
+
 def test_source_hash_ignores_comments(tmp_path, monkeypatch):
     src = tmp_path / "paper_2609_06072_gb300" / "csrc"
     src.mkdir(parents=True)
